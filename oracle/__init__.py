@@ -1,0 +1,39 @@
+"""CPU oracle for per-group 3/4-bit weight quantization fused into matmul.
+
+TEST INFRASTRUCTURE ONLY.  This package is a plain, slow, obviously-correct
+restatement of what the quantized-matmul path computes, written in numpy with
+float64 wherever the definition does not fix another precision.  Only the test
+suite, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py`` may
+import it; the product path (the CUDA library and its Python binding) never does
+and shares no code with it.
+
+Modules
+-------
+``quant``   uniform asymmetric RTN quantizer and the non-uniform Lloyd-Max LUT
+            quantizer, per group of g consecutive weights along K
+            (paper Section 2.2, Section 3.2 "Q4_0"/"Q4_K", Table 1 "G128").
+``pack``    the packed byte layout of codes and zero-points (the paper fixes none;
+            Section 2.4 says only that packing/unpacking kernels set decode time).
+``matmul``  dequantize + float64 matvec / matmul and the parity tolerance.
+
+Every function names the passage (section, table or figure of the paper) it
+follows; where the paper is silent the docstring states the reading taken.
+"""
+from .quant import (  # noqa: F401
+    quantize_uniform,
+    dequant_uniform,
+    quantize_lut,
+    dequant_lut,
+    lloyd_max_trace,
+)
+from .pack import (  # noqa: F401
+    Recipe,
+    pack_codes,
+    unpack_codes,
+    pack_zeros,
+    unpack_zeros,
+    packed_sizes,
+    quantize,
+    dequant,
+)
+from .matmul import gemv, gemm, tolerance, max_abs_err  # noqa: F401
