@@ -1,0 +1,444 @@
+"""Benchmark of the quantized-matmul hot path on GB300.
+
+Workload (default): one Llama-7B-shaped decoder layer (q, k, v, o 4096x4096;
+gate, up 11008x4096; down 4096x11008), Student-t(4) weights with sigma 0.01
+(q, k), 0.02 (v, o), 0.04 (MLP), quantized to 3-bit non-uniform codes with a
+per-group 8-entry fp16 LUT (Lloyd-Max, group 128 along k).  One step = one
+decode token through all seven matrices (seven qx_gemv calls at batch 1).
+Metric: HBM GB/s of the packed weights (+ x, y) per step.
+
+Also reported on the same line: the prefill GEMM (M = 2048 tokens against the
+11008x4096 and 4096x11008 3-bit LUT matrices, tcgen05), the roofline of the
+dominant kernel, the CPU oracle as a baseline, SM clocks during the timed
+region and an end-to-end number with host buffers.
+
+Launch: python bench.py [--gpus N --steps K --warmup W] [--impl reference];
+for N > 1 under torch.distributed.run (one rank per GPU, weak scaling: every
+rank decodes its own copy of the layer; no collective on the data path).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "3/4-bit dequant-GEMV HBM GB/s (% of 8 TB/s); prefill dequant-GEMM TFLOP/s"
+NOMINAL_HBM_GBS = 8000.0
+LAYER = [  # name, n, k, sigma, stream id
+    ("q_proj", 4096, 4096, 0.01, 0),
+    ("k_proj", 4096, 4096, 0.01, 1),
+    ("v_proj", 4096, 4096, 0.02, 2),
+    ("o_proj", 4096, 4096, 0.02, 3),
+    ("gate_proj", 11008, 4096, 0.04, 4),
+    ("up_proj", 11008, 4096, 0.04, 5),
+    ("down_proj", 4096, 11008, 0.04, 6),
+]
+GEMM_M = 2048
+GEMM_MATS = [("gate_proj", 11008, 4096, 0.04, 4), ("down_proj", 4096, 11008, 0.04, 6)]
+REF_BUDGET_S = 150.0  # wall time of the whole reference (oracle) arm
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), float(d["bf16_tflops"]), float(d["bf16_tflops_sustained"]), "measured"
+    except Exception:
+        return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _src_sha(name: str) -> str:
+    with open(os.path.join(ROOT, "paper_2505_07531_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def _traffic(kernel_file: str, key: str):
+    """DRAM bytes per launch from a committed ncu summary, if taken on this source."""
+    path = os.path.join(ROOT, "profiles", "traffic.txt")
+    if not os.path.exists(path):
+        return None
+    sha = _src_sha(kernel_file)
+    with open(path) as f:
+        for line in f:
+            parts = line.split()
+            if len(parts) >= 4 and parts[0] == key and parts[1] == sha:
+                return float(parts[2])
+    return None
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons sampled every 200 ms."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+         "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.index}", f"--query-gpu={self.Q}", "--format=csv,noheader,nounits",
+                 "-lms", "200"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def _dist():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    if ws > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+        return dist, dist.get_rank(), ws, int(os.environ.get("LOCAL_RANK", "0"))
+    return None, 0, 1, 0
+
+
+# --------------------------------------------------------------- CPU oracle leg
+def _oracle_sample(rows_per_matrix: int, seed: int = 0):
+    """Oracle-quantized samples of the layer's matrices (first rows of each)."""
+    import oracle
+    import synth
+    from oracle.pack import Recipe as ORecipe
+
+    rec = ORecipe(3, 128, "lut", 25)
+    mats = []
+    for name, n, k, sigma, sid in LAYER:
+        W = synth.student_t_weights(rows_per_matrix, k, sigma, seed=seed, stream=100 + sid)
+        p = oracle.quantize(W, rec)
+        x = synth.activations(1, k, seed=seed, stream=200 + sid)
+        nbytes = p["codes"].nbytes + p["luts"].nbytes + x.nbytes + 2 * rows_per_matrix
+        mats.append((p, x, k, nbytes))
+    return rec, mats
+
+
+def _oracle_pass(rec, mats):
+    import oracle
+
+    for p, x, k, _ in mats:
+        oracle.gemv(p, rec, x, k)
+
+
+def cpu_baseline_child(seconds: float):
+    """Run in a single-threaded subprocess: oracle GB/s on a bounded sample."""
+    rec, mats = _oracle_sample(64)
+    nbytes = sum(m[3] for m in mats)
+    _oracle_pass(rec, mats)
+    t0 = time.perf_counter()
+    reps = 0
+    while True:
+        _oracle_pass(rec, mats)
+        reps += 1
+        if time.perf_counter() - t0 >= seconds:
+            break
+    dt = time.perf_counter() - t0
+    print(json.dumps({"value": nbytes * reps / dt / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                      "sample": f"{reps} passes over the first 64 rows of each of the 7 layer matrices "
+                                f"({nbytes / 1e6:.2f} MB packed per pass), numpy float64, 1 thread, {dt:.1f} s"}))
+
+
+def run_cpu_baseline(seconds: float = 12.0):
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-baseline-child", str(seconds)],
+                       capture_output=True, text=True, env=env, timeout=600)
+    try:
+        return json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception:
+        return {"value": None, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": "failed: " + r.stderr[-200:]}
+
+
+def run_reference(args):
+    """The oracle as the reference arm: same metric and config, bounded samples per step."""
+    dist, rank, ws, _ = _dist()
+    if rank != 0:
+        return
+    steps, warmup = args.steps, args.warmup
+    per_step = REF_BUDGET_S / max(1, steps + warmup)
+    rec, mats = _oracle_sample(16)
+    t0 = time.perf_counter()
+    _oracle_pass(rec, mats)
+    t16 = max(time.perf_counter() - t0, 1e-6)
+    rows = int(max(1, min(2048, 16 * per_step / t16 * 0.8)))
+    rec, mats = _oracle_sample(rows)
+    nbytes = sum(m[3] for m in mats)
+    for _ in range(warmup):
+        _oracle_pass(rec, mats)
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        _oracle_pass(rec, mats)
+    dt = time.perf_counter() - t0
+    v = nbytes * steps / dt / 1e9
+    cores = os.cpu_count() or 1
+    line = {
+        "impl": "reference", "metric": METRIC, "value": v, "unit": "GB/s", "n_gpus": ws, "steps": steps,
+        "warmup": warmup, "ms_per_step": dt / steps * 1e3, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": "llama7b_layer_decode_L3g128_b1", "sample_rows_per_matrix": rows},
+        "cpu_baseline": {"value": v, "unit": "GB/s", "cores": cores, "kind": "oracle",
+                         "sample": f"first {rows} rows of each of the 7 layer matrices per step "
+                                   f"({nbytes / 1e6:.2f} MB packed), numpy float64"},
+        "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+
+
+# --------------------------------------------------------------- GPU arm
+def _quantize_layer(qx, torch, dev, mats, recipe, seed=0):
+    import synth
+
+    out = []
+    for name, n, k, sigma, sid in mats:
+        W = synth.student_t_weights_torch(n, k, sigma, seed=seed, stream=sid, device=dev)
+        out.append((name, qx.quantize(W, recipe)))
+        del W
+    if qx.device_status() != 0:
+        raise RuntimeError("quantize reported a device error")
+    return out
+
+
+def _clone(qx, P):
+    c = lambda t: None if t is None else t.clone()
+    return qx.PackedMatrix(P.n, P.k, P.recipe, c(P.codes), c(P.scales), c(P.zeros), c(P.luts))
+
+
+def run_ours(args):
+    import torch
+
+    import synth
+    import paper_2505_07531_gb300.qx as qx
+
+    dist, rank, ws, local = _dist()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    qx._lib()  # fails loudly when the library is missing
+    hbm, tf_burst, tf_sust, peak_src = _peaks()
+    props = torch.cuda.get_device_properties(dev)
+    l2 = getattr(props, "L2_cache_size", 0) or 126 * 2 ** 20
+
+    recipe = qx.Recipe(3, 128, qx.LUT, 25)
+    base = _quantize_layer(qx, torch, dev, LAYER, recipe)
+    layer_bytes = sum(P.nbytes() for _, P in base)
+    copies = max(2, math.ceil(4 * l2 / layer_bytes))
+    layers = [base] + [[(nm, _clone(qx, P)) for nm, P in base] for _ in range(copies - 1)]
+    xs = [synth.activations_torch(1, k, seed=0, stream=50 + sid, device=dev) for _, n, k, _, sid in LAYER]
+    ys = [torch.empty((1, n), dtype=torch.float16, device=dev) for _, n, k, _, _ in LAYER]
+    io_bytes = sum(x.numel() * 2 for x in xs) + sum(y.numel() * 2 for y in ys)
+    step_bytes = layer_bytes + io_bytes
+
+    stream = torch.cuda.Stream(dev)
+
+    def step(c):
+        for (name, P), x, y in zip(layers[c], xs, ys):
+            qx.gemv(P, x, out=y)
+
+    with torch.cuda.stream(stream):
+        for c in range(copies):
+            step(c)
+    torch.cuda.synchronize(dev)
+    graphs = []
+    for c in range(copies):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            step(c)
+        graphs.append(g)
+    torch.cuda.synchronize(dev)
+
+    sampler = ClockSampler(dev.index if dev.index is not None else 0)
+    sampler.start()
+    with torch.cuda.stream(stream):
+        for i in range(args.warmup):
+            graphs[i % copies].replay()
+        # soak ~1.5 s so the clocks are sampled under this load, then time exactly K steps
+        t_end = time.time() + 1.5
+        i = 0
+        while time.time() < t_end:
+            for _ in range(64):
+                graphs[i % copies].replay()
+                i += 1
+            stream.synchronize()
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize(dev)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(stream):
+        ev0.record(stream)
+        for i in range(args.steps):
+            graphs[i % copies].replay()
+        ev1.record(stream)
+    torch.cuda.synchronize(dev)
+    clocks = sampler.stop()
+    ms = ev0.elapsed_time(ev1) / args.steps
+    if dist is not None:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    value = step_bytes * ws / (ms * 1e-3) / 1e9
+
+    # per-launch kernel durations (events on the launching stream) for the roofline
+    reps = max(3, min(args.steps, 200))
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in LAYER]
+           for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        for r in range(reps):
+            c = r % copies
+            for j, ((name, P), x, y) in enumerate(zip(layers[c], xs, ys)):
+                evs[r][j][0].record(stream)
+                qx.gemv(P, x, out=y)
+                evs[r][j][1].record(stream)
+    torch.cuda.synchronize(dev)
+    kern_ms = sum(a.elapsed_time(b) for row in evs for a, b in row) / reps
+    per_matrix_us = {LAYER[j][0]: 1e3 * sum(evs[r][j][0].elapsed_time(evs[r][j][1]) for r in range(reps)) / reps
+                     for j in range(len(LAYER))}
+    achieved = step_bytes / (kern_ms * 1e-3) / 1e9
+
+    # end to end through the public API with host buffers: pinned x in, y out, per step
+    hx = [x.cpu().pin_memory() for x in xs]
+    hy = [torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in ys]
+    e2e_steps = max(3, min(args.steps, 2000))
+    torch.cuda.synchronize(dev)
+    t0 = time.perf_counter()
+    with torch.cuda.stream(stream):
+        for i in range(e2e_steps):
+            c = i % copies
+            for j, ((name, P), x, y) in enumerate(zip(layers[c], xs, ys)):
+                x.copy_(hx[j], non_blocking=True)
+                qx.gemv(P, x, out=y)
+                hy[j].copy_(y, non_blocking=True)
+            stream.synchronize()
+    e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
+    e2e_value = step_bytes * ws / (e2e_ms * 1e-3) / 1e9
+
+    gemm = run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
+    del layers, graphs
+
+    if rank == 0:
+        cpu = run_cpu_baseline() if not args.skip_cpu_baseline else None
+        line = {
+            "metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f16", "data": "synthetic",
+            "pct_of_8TBs": 100.0 * value / ws / NOMINAL_HBM_GBS,
+            "config": {"workload": "llama7b_layer_decode_L3g128_b1",
+                       "matrices": {nm: [n, k] for nm, n, k, _, _ in LAYER},
+                       "recipe": "3-bit LUT (8 fp16 levels, Lloyd-Max) group 128",
+                       "batch": 1, "bytes_per_step": step_bytes,
+                       "l2": f"{copies} rotating weight copies ({copies * layer_bytes / 1e6:.0f} MB) > "
+                             f"4x L2 ({l2 / 1e6:.0f} MB)",
+                       "graph": "one CUDA graph per step (7 launches)"},
+            "per_matrix_us": per_matrix_us,
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                         "frac": achieved / hbm, "peak_source": f"{peak_src} hbm_gbs",
+                         "kernel": "gemv_kernel<3,LUT,1,2>",
+                         "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
+            "gemm": gemm,
+            "cpu_baseline": cpu,
+            "clocks": clocks,
+            "e2e": {"value": e2e_value, "unit": "GB/s", "ms_per_step": e2e_ms,
+                    "h2d_bytes_per_step": sum(x.numel() * 2 for x in hx),
+                    "d2h_bytes_per_step": sum(y.numel() * 2 for y in hy)},
+            "gpu_launches": args.steps * len(LAYER),
+        }
+        print(json.dumps(line))
+    if dist is not None:
+        dist.destroy_process_group()
+
+
+def run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src):
+    """Prefill GEMM, M = 2048, 3-bit LUT g128 11008x4096 and 4096x11008."""
+    import synth
+
+    recipe = qx.Recipe(3, 128, qx.LUT, 25)
+    mats = _quantize_layer(qx, torch, dev, GEMM_MATS, recipe, seed=1)
+    Xs = [synth.activations_torch(GEMM_M, P.k, seed=1, stream=70 + i, device=dev) for i, (_, P) in enumerate(mats)]
+    Ys = [torch.empty((GEMM_M, P.n), dtype=torch.float16, device=dev) for _, P in mats]
+    flops = sum(2.0 * GEMM_M * P.n * P.k for _, P in mats)
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            for (nm, P), X, Y in zip(mats, Xs, Ys):
+                qx.gemm(P, X, out=Y)
+    torch.cuda.synchronize(dev)
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("gemm reported a device error")
+    reps = 20
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in mats]
+           for _ in range(reps)]
+    with torch.cuda.stream(stream):
+        for r in range(reps):
+            for j, ((nm, P), X, Y) in enumerate(zip(mats, Xs, Ys)):
+                evs[r][j][0].record(stream)
+                qx.gemm(P, X, out=Y)
+                evs[r][j][1].record(stream)
+    torch.cuda.synchronize(dev)
+    ms = sum(a.elapsed_time(b) for row in evs for a, b in row) / reps
+    per = {mats[j][0]: 1e3 * sum(evs[r][j][0].elapsed_time(evs[r][j][1]) for r in range(reps)) / reps
+           for j in range(len(mats))}
+    tflops = flops / (ms * 1e-3) / 1e12
+    return {"value": tflops, "unit": "TFLOP/s", "ms_per_step": ms, "per_matrix_us": per,
+            "config": {"workload": "prefill_M2048_L3g128", "m": GEMM_M,
+                       "matrices": {nm: [P.n, P.k] for nm, P in mats}, "mma": "tcgen05 kind::f16, fp32 accumulate",
+                       "l2": "weights 22.5 MB and X 16-22 MB are L2-resident (compute-bound kernel)"},
+            "roofline": {"bound": "tensor", "achieved": tflops, "peak": tf_burst, "unit": "TFLOP/s",
+                         "frac": tflops / tf_burst,
+                         "peak_source": f"{peak_src} bf16_tflops (burst) x 1.0 nominal fp16/bf16 ratio",
+                         "kernel": "gemm_kernel<3,LUT>", "traffic": _traffic("qx_gemm.cu", "gemm_L3g128_m2048")}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=50)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--skip-gemm", action="store_true")
+    ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-baseline-child", type=float, default=None, help=argparse.SUPPRESS)
+    args = ap.parse_args()
+    if args.cpu_baseline_child is not None:
+        cpu_baseline_child(args.cpu_baseline_child)
+        return
+    if args.warmup < 3:
+        args.warmup = 3
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

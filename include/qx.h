@@ -1,0 +1,151 @@
+/*
+ * qx.h -- C ABI of the GB300 (sm_103a) library for per-group 3/4-bit weight
+ * quantization fused into matrix multiplication.
+ *
+ * The method: a weight matrix W [n][k] (fp16, row n = output feature) is split
+ * into groups of g consecutive weights along k, and every group is coded with
+ * 3 or 4 bits per weight, either uniformly (equally spaced points, per-group fp16
+ * scale and zero-point; paper Section 2.2 and Section 3.2, Q4_0 / Q4_K) or
+ * non-uniformly (a per-group codebook, a LUT of 2^b fp16 levels placed where the
+ * weights' probability mass is, fit by Lloyd-Max; Section 2.2, Fig. 2a).  The
+ * recipe (bits, group size, uniform vs non-uniform) is chosen per matrix
+ * (Sections 2.1 and 2.3: per-layer and per-sub-model choices).  Inference
+ * dequantizes inside the matrix multiply: decode is memory-bound, so the
+ * packing and the unpacking kernels decide its run time (Section 2.4); prefill
+ * is a dense contraction (Table 2, "Prefill").
+ *
+ * Conventions for every entry point
+ *   - Buffers are caller-owned.  "device" pointers are CUDA global memory of the
+ *     current device; "host" pointers are CPU memory.  The library keeps no
+ *     pointer after a call returns.
+ *   - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
+ *     stream.  Device work is asynchronous on that stream.
+ *   - Arguments are validated on the host before anything is launched; on a
+ *     validation failure nothing is launched and a non-zero qx_status returns.
+ *   - Errors the device can only detect while running (non-finite weights, a
+ *     bounded wait that gave up) set a per-device status word that
+ *     qx_get_device_status() reads and clears.
+ *   - fp16 values are IEEE binary16 stored as uint16_t; bf16 is not used.
+ *
+ * Packed layout (the paper prints none; this library fixes it).  k must be a
+ * multiple of 128 and of g; rows are stored one after another.
+ *   codes, 4-bit : k/2 bytes per row.  Little-endian 32-bit word t holds the
+ *                  codes of k = 8t..8t+7; the code of k = 8t+j sits in nibble
+ *                  j/2 + 4*(j%2).
+ *   codes, 3-bit : 3k/8 bytes per row, three planes of k/8 bytes.  Superblock s
+ *                  (k = 128s..128s+127) owns bytes 16s..16s+15 of each plane;
+ *                  word i (bytes 4i..4i+3 of those 16) of planes 0/1/2, called
+ *                  A_i/B_i/C_i, code k = 128s+32i+m (m = 0..31): bits 0-2 of
+ *                  nibble t (t = 0..7) of A_i, B_i, C_i hold the codes of
+ *                  m = t, 8+t, 16+t; bit 3 of nibble t of A_i, B_i, C_i holds
+ *                  bit 0, 1, 2 of the code of m = 24+t.
+ *   scales       : fp16 [n][k/g]                    (uniform only)
+ *   zeros        : uint8 [n][ceil(k/g/2)], group j in the low nibble of byte
+ *                  j/2 when j is even, else the high nibble (uniform only)
+ *   luts         : fp16 [n][k/g][2^bits], ascending (non-uniform only)
+ *
+ * Dequantized weight (bit-exact contract shared with the CPU oracle):
+ *   uniform: w_hat = fp16_rn((float)(q - z) * (float)s)
+ *   LUT    : w_hat = luts[n][group][q]
+ */
+#ifndef QX_H
+#define QX_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum qx_status {
+    QX_OK = 0,
+    QX_ERR_INVALID_ARG = 1,  /* NULL pointer, non-positive size, bad enum value   */
+    QX_ERR_UNSUPPORTED = 2,  /* well-formed but not built: bits/group/kind/batch   */
+    QX_ERR_ALIGNMENT = 3,    /* a pointer breaks the alignment stated below       */
+    QX_ERR_CUDA = 4,         /* a CUDA runtime call or a kernel launch failed     */
+    QX_ERR_TIMEOUT = 5,      /* device: a bounded wait gave up (device status)    */
+    QX_ERR_NONFINITE = 6     /* device: qx_quantize met NaN or Inf (device status) */
+} qx_status;
+
+typedef enum qx_kind {
+    QX_UNIFORM = 0, /* per-group fp16 scale + 4-bit zero-point, RTN (Section 3.2)   */
+    QX_LUT = 1      /* per-group 2^bits-entry fp16 codebook, Lloyd-Max (Section 2.2) */
+} qx_kind;
+
+typedef enum qx_dtype { QX_F16 = 0, QX_F32 = 1 } qx_dtype;
+
+/* Per-matrix recipe (Sections 2.1-2.3).  Built: uniform bits 3/4 with
+ * group_size 32/64/128/256; LUT bits 3 with group_size 32/64/128/256.
+ * lloyd_iters (LUT only): Lloyd-Max iteration limit, 0..1000. */
+typedef struct qx_recipe {
+    int32_t bits;
+    int32_t group_size;
+    int32_t kind;        /* qx_kind */
+    int32_t lloyd_iters;
+} qx_recipe;
+
+/* Byte sizes of the packed buffers; 0 for a buffer the recipe does not use. */
+typedef struct qx_sizes {
+    uint64_t codes, scales, zeros, luts;
+} qx_sizes;
+
+/* A packed matrix.  All four pointers are device memory, 16-byte aligned
+ * (unused ones may be NULL). */
+typedef struct qx_packed {
+    int64_t n, k;
+    qx_recipe recipe;
+    void *codes;
+    void *scales;
+    void *zeros;
+    void *luts;
+} qx_packed;
+
+/* Host only: byte sizes of the packed buffers of an n x k matrix.
+ * Errors: INVALID_ARG (NULL, n < 1, k < 1), UNSUPPORTED (recipe not built or
+ * k not a multiple of 128 and of g). */
+qx_status qx_packed_size(int64_t n, int64_t k, const qx_recipe *recipe, qx_sizes *out);
+
+/* Quantize and pack W (device fp16 [n][k], row-major, 16-byte aligned) into
+ * the caller-allocated buffers of *out (out->n, out->k, out->recipe must equal
+ * n, k, *recipe).  Uniform: Section 2.2 / 3.2 RTN with per-group scale and
+ * zero-point.  LUT: per-group Lloyd-Max codebook (Section 2.2, Fig. 2a).  Codes,
+ * scales, zeros and LUTs are bit-identical to the CPU oracle's.  A non-finite
+ * weight sets QX_ERR_NONFINITE in the device status; its group's output is
+ * unspecified. */
+qx_status qx_quantize(const void *W, int64_t n, int64_t k, const qx_recipe *recipe,
+                      const qx_packed *out, void *stream);
+
+/* Dequantize a packed matrix into W_out (device fp16 [n][k], 16-byte aligned),
+ * bit-exact with the formula in the header comment (Section 2.4 unpacking). */
+qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream);
+
+/* Decode matmul y = x W_hat^T (Section 2.4: memory-bound decoding; Table 2
+ * "Decode").  x: device fp16 [batch][k], row-major, 16-byte aligned;
+ * y: device [batch][n] of y_dtype (QX_F16 or QX_F32), 4-byte aligned.
+ * batch in 1..16.  fp32 accumulation across groups. */
+qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y,
+                  int32_t y_dtype, void *stream);
+
+/* Prefill matmul Y = X W_hat^T (Table 2 "Prefill") on the tcgen05 tensor cores:
+ * W_hat tiles are dequantized into shared memory and multiplied in fp16 with
+ * fp32 accumulation in tensor memory.  X: device fp16 [m][k] row-major,
+ * 16-byte aligned; Y: device fp16 [m][n] row-major, 4-byte aligned; m >= 1. */
+qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream);
+
+/* Synchronize `stream`, then return and clear the current device's status word
+ * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
+ * synchronization itself fails. */
+qx_status qx_get_device_status(void *stream);
+
+/* Static, NUL-terminated description of a status code. */
+const char *qx_status_string(qx_status s);
+
+/* Library version as major*10000 + minor*100 + patch. */
+int32_t qx_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* QX_H */

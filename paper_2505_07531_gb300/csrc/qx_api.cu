@@ -1,0 +1,268 @@
+// C ABI of the qx library: argument validation, dispatch, device status.
+// The declarations, with the meaning, layout, ownership and error behaviour of
+// every argument, are in include/qx.h.
+#include <cstdlib>
+#include <cstring>
+#include <mutex>
+
+#include "qx.h"
+#include "qx_kernels.cuh"
+
+#define QX_API extern "C" __attribute__((visibility("default")))
+
+namespace {
+
+constexpr int kMaxDevices = 64;
+
+// One status word per device, in the library's own device memory (a file-scope
+// __device__ symbol; nothing is allocated).  Its device address is fetched
+// once per device with that device current.
+__device__ uint32_t g_status_word;
+
+struct DeviceInfo {
+    uint32_t *status = nullptr;
+    int num_sms = 0;
+    bool ready = false;
+};
+
+DeviceInfo g_dev[kMaxDevices];
+std::mutex g_mu;
+
+qx_status device_info(DeviceInfo **out) {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return QX_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_mu);
+    DeviceInfo &d = g_dev[dev];
+    if (!d.ready) {
+        void *p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return QX_ERR_CUDA;
+        int sms = 0;
+        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return QX_ERR_CUDA;
+        d.status = static_cast<uint32_t *>(p);
+        d.num_sms = sms;
+        d.ready = true;
+    }
+    *out = &d;
+    return QX_OK;
+}
+
+uint64_t wait_limit_ns() {
+    // bounded waits inside the tensor-core kernel; QX_WAIT_LIMIT_MS overrides
+    const char *s = std::getenv("QX_WAIT_LIMIT_MS");
+    uint64_t ms = 2000;
+    if (s != nullptr) {
+        const long long v = std::atoll(s);
+        if (v > 0 && v < 600000) ms = (uint64_t)v;
+    }
+    return ms * 1000000ull;
+}
+
+bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
+
+int ilog2(int v) {
+    int r = 0;
+    while ((1 << r) < v) ++r;
+    return r;
+}
+
+qx_status check_recipe(const qx_recipe *r) {
+    if (r == nullptr) return QX_ERR_INVALID_ARG;
+    if (r->kind != QX_UNIFORM && r->kind != QX_LUT) return QX_ERR_INVALID_ARG;
+    if (r->bits != 3 && r->bits != 4) return QX_ERR_UNSUPPORTED;
+    if (r->kind == QX_LUT && r->bits != 3) return QX_ERR_UNSUPPORTED;
+    const int g = r->group_size;
+    if (g != 32 && g != 64 && g != 128 && g != 256) return QX_ERR_UNSUPPORTED;
+    if (r->kind == QX_LUT && (r->lloyd_iters < 0 || r->lloyd_iters > 1000)) return QX_ERR_INVALID_ARG;
+    return QX_OK;
+}
+
+qx_status check_shape(int64_t n, int64_t k, const qx_recipe *r) {
+    if (n < 1 || k < 1) return QX_ERR_INVALID_ARG;
+    if (k % 128 != 0 || k % r->group_size != 0) return QX_ERR_UNSUPPORTED;
+    // grid and index limits of the kernels
+    if (n > (int64_t)1 << 22 || k > (int64_t)1 << 20) return QX_ERR_UNSUPPORTED;
+    return QX_OK;
+}
+
+qx_status check_packed(const qx_packed *p) {
+    if (p == nullptr) return QX_ERR_INVALID_ARG;
+    qx_status s = check_recipe(&p->recipe);
+    if (s != QX_OK) return s;
+    s = check_shape(p->n, p->k, &p->recipe);
+    if (s != QX_OK) return s;
+    if (p->codes == nullptr) return QX_ERR_INVALID_ARG;
+    if (!aligned(p->codes, 16)) return QX_ERR_ALIGNMENT;
+    if (p->recipe.kind == QX_UNIFORM) {
+        if (p->scales == nullptr || p->zeros == nullptr) return QX_ERR_INVALID_ARG;
+        if (!aligned(p->scales, 2)) return QX_ERR_ALIGNMENT;
+    } else {
+        if (p->luts == nullptr) return QX_ERR_INVALID_ARG;
+        if (!aligned(p->luts, 16)) return QX_ERR_ALIGNMENT;
+    }
+    return QX_OK;
+}
+
+qx_status from_cuda(cudaError_t e) { return e == cudaSuccess ? QX_OK : QX_ERR_CUDA; }
+
+}  // namespace
+
+QX_API int32_t qx_version(void) { return 100; }
+
+QX_API const char *qx_status_string(qx_status s) {
+    switch (s) {
+        case QX_OK: return "ok";
+        case QX_ERR_INVALID_ARG: return "invalid argument";
+        case QX_ERR_UNSUPPORTED: return "unsupported recipe, shape or batch";
+        case QX_ERR_ALIGNMENT: return "pointer alignment";
+        case QX_ERR_CUDA: return "CUDA error";
+        case QX_ERR_TIMEOUT: return "device wait timed out";
+        case QX_ERR_NONFINITE: return "non-finite weight";
+    }
+    return "unknown status";
+}
+
+QX_API qx_status qx_packed_size(int64_t n, int64_t k, const qx_recipe *recipe, qx_sizes *out) {
+    if (out == nullptr) return QX_ERR_INVALID_ARG;
+    qx_status s = check_recipe(recipe);
+    if (s != QX_OK) return s;
+    s = check_shape(n, k, recipe);
+    if (s != QX_OK) return s;
+    const int64_t G = k / recipe->group_size;
+    out->codes = (uint64_t)(n * k * recipe->bits / 8);
+    if (recipe->kind == QX_UNIFORM) {
+        out->scales = (uint64_t)(n * G * 2);
+        out->zeros = (uint64_t)(n * ((G + 1) / 2));
+        out->luts = 0;
+    } else {
+        out->scales = 0;
+        out->zeros = 0;
+        out->luts = (uint64_t)(n * G * (1 << recipe->bits) * 2);
+    }
+    return QX_OK;
+}
+
+QX_API qx_status qx_quantize(const void *W, int64_t n, int64_t k, const qx_recipe *recipe, const qx_packed *out,
+                             void *stream) {
+    if (W == nullptr || out == nullptr || recipe == nullptr) return QX_ERR_INVALID_ARG;
+    qx_status s = check_packed(out);
+    if (s != QX_OK) return s;
+    if (out->n != n || out->k != k || out->recipe.bits != recipe->bits ||
+        out->recipe.group_size != recipe->group_size || out->recipe.kind != recipe->kind)
+        return QX_ERR_INVALID_ARG;
+    if (!aligned(W, 16)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::QuantArgs a{};
+    a.W = static_cast<const __half *>(W);
+    a.n = n;
+    a.k = k;
+    a.bits = recipe->bits;
+    a.g = recipe->group_size;
+    a.kind = recipe->kind;
+    a.lloyd_iters = recipe->lloyd_iters;
+    a.G = (int)(k / a.g);
+    a.zbytes = (a.G + 1) / 2;
+    a.codes = static_cast<uint8_t *>(out->codes);
+    a.scales = static_cast<__half *>(out->scales);
+    a.zeros = static_cast<uint8_t *>(out->zeros);
+    a.luts = static_cast<__half *>(out->luts);
+    a.status = d->status;
+    return from_cuda(qx::launch_quantize(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream) {
+    qx_status s = check_packed(p);
+    if (s != QX_OK) return s;
+    if (W_out == nullptr) return QX_ERR_INVALID_ARG;
+    if (!aligned(W_out, 16)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::DequantArgs a{};
+    a.codes = static_cast<const uint8_t *>(p->codes);
+    a.scales = static_cast<const __half *>(p->scales);
+    a.zeros = static_cast<const uint8_t *>(p->zeros);
+    a.luts = static_cast<const __half *>(p->luts);
+    a.n = p->n;
+    a.k = p->k;
+    a.bits = p->recipe.bits;
+    a.g = p->recipe.group_size;
+    a.kind = p->recipe.kind;
+    a.G = (int)(p->k / a.g);
+    a.zbytes = (a.G + 1) / 2;
+    a.W = static_cast<__half *>(W_out);
+    return from_cuda(qx::launch_dequant(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y, int32_t y_dtype,
+                         void *stream) {
+    qx_status s = check_packed(p);
+    if (s != QX_OK) return s;
+    if (x == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
+    if (y_dtype != QX_F16 && y_dtype != QX_F32) return QX_ERR_INVALID_ARG;
+    if (batch < 1) return QX_ERR_INVALID_ARG;
+    if (batch > 16) return QX_ERR_UNSUPPORTED;
+    if (!aligned(x, 16)) return QX_ERR_ALIGNMENT;
+    if (!aligned(y, y_dtype == QX_F32 ? 4 : 2)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::GemvArgs a{};
+    a.codes = static_cast<const uint8_t *>(p->codes);
+    a.scales = static_cast<const __half *>(p->scales);
+    a.zeros = static_cast<const uint8_t *>(p->zeros);
+    a.luts = static_cast<const __half *>(p->luts);
+    a.n = p->n;
+    a.k = p->k;
+    a.bits = p->recipe.bits;
+    a.kind = p->recipe.kind;
+    a.log2g = ilog2(p->recipe.group_size);
+    a.G = (int)(p->k / p->recipe.group_size);
+    a.zbytes = (a.G + 1) / 2;
+    a.x = static_cast<const __half *>(x);
+    a.y = y;
+    a.batch = batch;
+    a.y_f32 = y_dtype == QX_F32;
+    return from_cuda(qx::launch_gemv(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream) {
+    qx_status s = check_packed(p);
+    if (s != QX_OK) return s;
+    if (X == nullptr || Y == nullptr || m < 1) return QX_ERR_INVALID_ARG;
+    if (m > ((int64_t)1 << 31) - 1) return QX_ERR_UNSUPPORTED;
+    if (!aligned(X, 16)) return QX_ERR_ALIGNMENT;
+    if (!aligned(Y, 2)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::GemmArgs a{};
+    a.codes = static_cast<const uint8_t *>(p->codes);
+    a.scales = static_cast<const __half *>(p->scales);
+    a.zeros = static_cast<const uint8_t *>(p->zeros);
+    a.luts = static_cast<const __half *>(p->luts);
+    a.n = p->n;
+    a.k = p->k;
+    a.m = m;
+    a.bits = p->recipe.bits;
+    a.kind = p->recipe.kind;
+    a.log2g = ilog2(p->recipe.group_size);
+    a.G = (int)(p->k / p->recipe.group_size);
+    a.zbytes = (a.G + 1) / 2;
+    a.X = static_cast<const __half *>(X);
+    a.Y = static_cast<__half *>(Y);
+    a.status = d->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_get_device_status(void *stream) {
+    DeviceInfo *d = nullptr;
+    qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return QX_ERR_CUDA;
+    uint32_t v = 0;
+    if (cudaMemcpy(&v, d->status, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return QX_ERR_CUDA;
+    const uint32_t zero = 0;
+    if (cudaMemcpy(d->status, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return QX_ERR_CUDA;
+    if (v & qx::kStatusNonfinite) return QX_ERR_NONFINITE;
+    if (v & qx::kStatusTimeout) return QX_ERR_TIMEOUT;
+    return QX_OK;
+}

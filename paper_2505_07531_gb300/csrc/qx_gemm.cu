@@ -1,0 +1,419 @@
+// Prefill matmul Y[m][n] = sum_k X[m][k] w_hat[n][k] on the 5th-generation
+// tensor cores (tcgen05), with the weights dequantized on chip.
+//
+// Prefill is the one dense contraction on the path (paper Table 2, "Prefill"),
+// so it runs on the tensor cores.  The kernel computes the transposed tile
+// D = W_hat_tile * X_tile^T: the MMA's M dimension is 128 rows of W, its N
+// dimension 128 tokens, and the contraction runs over k in stages of 64.
+//
+// Warp roles (320 threads):
+//   warp 0      TMA producer: 128 x 64 fp16 X tiles (128B swizzle) -> smem
+//   warp 1      allocates tensor memory; one thread issues tcgen05.mma
+//   warps 2-9   dequantize 128 x 64 W_hat tiles from the packed codes straight
+//               into the 128B-swizzled K-major shared-memory layout the MMA
+//               reads (the same unpack primitives as qx_dequant, so W_hat is
+//               exact), then read the fp32 accumulator out of tensor memory
+//               and store fp16 Y.
+// A 4-stage mbarrier ring connects producers and the MMA issuer; the MMA
+// releases a stage with tcgen05.commit.  Every wait is bounded in time: a wait
+// that gives up raises QX_ERR_TIMEOUT in the device status word, tells the
+// other roles to stop, lets in-flight copies and MMAs drain, frees tensor
+// memory and returns.
+#include <cuda.h>
+
+#include "qx_kernels.cuh"
+
+namespace qx {
+
+namespace {
+
+constexpr int BM = 128;  // W rows per tile (MMA M)
+constexpr int BN = 128;  // tokens per tile (MMA N)
+constexpr int BK = 64;   // k per stage (one 128-byte swizzle row of fp16)
+constexpr int STAGES = 4;
+constexpr int A_BYTES = BM * BK * 2;
+constexpr int B_BYTES = BN * BK * 2;
+constexpr int NUM_DQ_WARPS = 8;
+constexpr int THREADS = 64 + NUM_DQ_WARPS * 32;
+constexpr uint32_t TMEM_COLS = 128;
+
+struct SmemLayout {
+    uint8_t a[STAGES][A_BYTES];
+    uint8_t b[STAGES][B_BYTES];
+    uint64_t full_a[STAGES];
+    uint64_t full_b[STAGES];
+    uint64_t empty[STAGES];
+    uint64_t accum_full;
+    uint32_t tmem_base;
+    uint32_t abort_flag;
+};
+
+constexpr size_t kSmemBytes = sizeof(SmemLayout) + 1024;
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(b)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(b)), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Wait for the phase of parity `parity` to complete.  Gives up after
+// `limit_ns`, or as soon as another role has raised the abort flag (when
+// `abort_flag` is not null).  Returns false if it gave up.
+__device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, uint64_t limit_ns,
+                                       volatile uint32_t *abort_flag) {
+    if (mbar_try_wait(b, parity)) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (uint32_t i = 1;; ++i) {
+        if (mbar_try_wait(b, parity)) return true;
+        if ((i & 31u) == 0) {
+            if (abort_flag != nullptr && *abort_flag) return false;
+            if (globaltimer_ns() - t0 > limit_ns) return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void raise_abort(SmemLayout &s, uint32_t *status) {
+    *reinterpret_cast<volatile uint32_t *>(&s.abort_flag) = 1u;
+    atomicOr(status, kStatusTimeout);
+}
+
+__device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, uint64_t *bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::
+            "r"(smem_u32(dst)),
+        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, rows of
+// 128 bytes, 8-row (1024-byte) swizzle atoms stacked along M/N.
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+    uint64_t d = 0;
+    d |= (uint64_t)((saddr & 0x3FFFFu) >> 4);  // start address
+    d |= (uint64_t)1 << 16;                   // leading-dimension offset (unused here)
+    d |= (uint64_t)(1024 >> 4) << 32;          // stride-dimension offset: 8 rows
+    d |= (uint64_t)1 << 46;                   // descriptor version for tcgen05
+    d |= (uint64_t)2 << 61;                   // 128-byte swizzle
+    return d;
+}
+
+// Instruction descriptor, kind::f16: fp16 A and B, fp32 D, both K-major.
+constexpr uint32_t kIdesc = (1u << 4)                  // D format f32
+                            | (0u << 7) | (0u << 10)    // A, B format f16
+                            | ((uint32_t)(BN >> 3) << 17)  // N
+                            | ((uint32_t)(BM >> 4) << 24); // M
+
+__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t acc) {
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "setp.ne.b32 p, %4, 0;\n\t"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
+        "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(acc)
+        : "memory");
+}
+
+__device__ __forceinline__ void mma_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(
+                     smem_u32(bar))
+                 : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+          "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+          "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// Codes and metadata one dequant thread needs for one 32-weight unit.
+struct UnitRaw {
+    uint32_t w[4];   // 4-bit: 16 bytes of codes; 3-bit: A, B, C of the triple
+    uint4 lut;       // LUT entries (LUT kind)
+    uint32_t zero;   // zero-point (uniform)
+    __half scale;    // scale (uniform)
+};
+
+template <int BITS, int KIND>
+__device__ __forceinline__ void load_unit(const GemmArgs &a, int64_t row, int64_t k0, UnitRaw &u) {
+    const int grp = (int)(k0 >> a.log2g);
+    if (BITS == 4) {
+        const uint4 c = ldg_nc_v4(a.codes + row * (a.k / 2) + (k0 >> 1));
+        u.w[0] = c.x;
+        u.w[1] = c.y;
+        u.w[2] = c.z;
+        u.w[3] = c.w;
+    } else {
+        const uint8_t *rc = a.codes + row * (3 * a.k / 8) + 16 * (k0 >> 7) + 4 * ((k0 & 127) >> 5);
+        const int64_t plane = a.k >> 3;
+        u.w[0] = __ldg(reinterpret_cast<const unsigned int *>(rc));
+        u.w[1] = __ldg(reinterpret_cast<const unsigned int *>(rc + plane));
+        u.w[2] = __ldg(reinterpret_cast<const unsigned int *>(rc + 2 * plane));
+        u.w[3] = 0;
+    }
+    if (KIND == 1) {
+        u.lut = ldg_nc_v4(a.luts + (row * a.G + grp) * 8);
+    } else {
+        u.zero = zero_nibble(a.zeros + row * a.zbytes, grp);
+        u.scale = a.scales[row * a.G + grp];
+    }
+}
+
+template <int BITS, int KIND>
+__device__ __forceinline__ void dequant_unit(const UnitRaw &u, __half2 (&v)[16]) {
+    if (BITS == 4) {
+        const __half2 s2 = __halves2half2(u.scale, u.scale);
+        const __half2 zl = zlo_of(u.zero), zh = zhi_of(u.zero);
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            __half2 o[4];
+            unpack4_qz(u.w[t], zl, zh, o);
+#pragma unroll
+            for (int p = 0; p < 4; ++p) v[4 * t + p] = __hmul2(o[p], s2);
+        }
+    } else if (KIND == 1) {
+        const Table8 t = make_table8(u.lut.x, u.lut.y, u.lut.z, u.lut.w);
+        lookup_triple(t, u.w[0], u.w[1], u.w[2], v);
+    } else {
+        const Table8 t = table8_offsets(u.zero);
+        lookup_triple(t, u.w[0], u.w[1], u.w[2], v);
+        const __half2 s2 = __halves2half2(u.scale, u.scale);
+#pragma unroll
+        for (int p = 0; p < 16; ++p) v[p] = __hmul2(v[p], s2);
+    }
+}
+
+template <int BITS, int KIND>
+__global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, GemmArgs a) {
+    extern __shared__ uint8_t smem_raw[];
+    SmemLayout &s = *reinterpret_cast<SmemLayout *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    volatile uint32_t *abort_flag = &s.abort_flag;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const int64_t n0 = (int64_t)blockIdx.y * BM;  // W rows
+    const int64_t m0 = (int64_t)blockIdx.x * BN;  // tokens
+    const int nkb = (int)(a.k / BK);
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < STAGES; ++i) {
+            mbar_init(&s.full_a[i], NUM_DQ_WARPS);
+            mbar_init(&s.full_b[i], 1);
+            mbar_init(&s.empty[i], 1);
+        }
+        mbar_init(&s.accum_full, 1);
+        s.abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_x) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(&s.tmem_base)),
+                     "r"(TMEM_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem_d = s.tmem_base;
+
+    if (warp == 0) {
+        // ------------------------------------------------ TMA producer (X)
+        if (lane == 0) {
+            int issued = 0;
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int st = kb % STAGES;
+                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+                if (!mbar_wait(&s.empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag)) {
+                    raise_abort(s, a.status);
+                    break;
+                }
+                mbar_arrive_expect_tx(&s.full_b[st], B_BYTES);
+                tma_load_2d(s.b[st], &tmap_x, &s.full_b[st], kb * BK, (int)m0);
+                ++issued;
+            }
+            // drain: never leave the CTA with a bulk copy still writing smem
+            for (int kb = issued - STAGES < 0 ? 0 : issued - STAGES; kb < issued; ++kb)
+                mbar_wait(&s.full_b[kb % STAGES], (uint32_t)(kb / STAGES) & 1u, a.wait_limit_ns, nullptr);
+        }
+    } else if (warp == 1) {
+        // ------------------------------------------------ MMA issuer
+        if (lane == 0) {
+            for (int kb = 0; kb < nkb; ++kb) {
+                const int st = kb % STAGES;
+                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+                if (!mbar_wait(&s.full_b[st], ph, a.wait_limit_ns, abort_flag) ||
+                    !mbar_wait(&s.full_a[st], ph, a.wait_limit_ns, abort_flag)) {
+                    raise_abort(s, a.status);
+                    break;
+                }
+                tc_fence_after();
+                const uint64_t ad = sw128_desc(smem_u32(s.a[st]));
+                const uint64_t bd = sw128_desc(smem_u32(s.b[st]));
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along k per step
+                    mma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, (kb | kk) != 0 ? 1u : 0u);
+                mma_commit(&s.empty[st]);
+            }
+            // always signal the epilogue, and do not free tensor memory under
+            // running MMAs: wait for this commit before leaving
+            mma_commit(&s.accum_full);
+            mbar_wait(&s.accum_full, 0, a.wait_limit_ns, nullptr);
+        }
+        __syncwarp();
+    } else {
+        // ------------------------------------------------ dequant producers
+        const int d = threadIdx.x - 64;  // 0..255
+        const int r = d >> 1;            // tile row 0..127
+        const int half_id = d & 1;       // which 32-wide half of the stage
+        const int64_t row = n0 + r;
+        const bool valid = row < a.n;
+        UnitRaw cur{}, nxt{};
+        if (valid) load_unit<BITS, KIND>(a, row, 32 * half_id, nxt);
+        bool ok = true;
+        for (int kb = 0; kb < nkb; ++kb) {
+            cur = nxt;
+            if (valid && kb + 1 < nkb) load_unit<BITS, KIND>(a, row, (int64_t)(kb + 1) * BK + 32 * half_id, nxt);
+            const int st = kb % STAGES;
+            const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
+            if (!mbar_wait(&s.empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag)) {
+                raise_abort(s, a.status);
+                ok = false;
+            }
+            if (__any_sync(0xffffffffu, !ok)) break;
+            __half2 v[16];
+            if (valid) {
+                dequant_unit<BITS, KIND>(cur, v);
+            } else {
+#pragma unroll
+                for (int p = 0; p < 16; ++p) v[p] = __float2half2_rn(0.0f);
+            }
+            uint8_t *tile = s.a[st] + (r >> 3) * 1024 + (r & 7) * 128;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int chunk = 4 * half_id + q;
+                *reinterpret_cast<uint4 *>(tile + ((chunk ^ (r & 7)) << 4)) =
+                    make_uint4(h22u(v[4 * q]), h22u(v[4 * q + 1]), h22u(v[4 * q + 2]), h22u(v[4 * q + 3]));
+            }
+            fence_proxy_async_smem();  // generic-proxy writes -> visible to the tensor core
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.full_a[st]);
+        }
+        // ------------------------------------------------ epilogue
+        const bool have = mbar_wait(&s.accum_full, 0, a.wait_limit_ns, nullptr);
+        if (!have) raise_abort(s, a.status);
+        tc_fence_after();
+        // tcgen05.ld is warp-collective: decide for the whole warp at once
+        if (__all_sync(0xffffffffu, have && !*abort_flag)) {
+            const int quarter = warp & 3;          // TMEM lanes this warp may read
+            const int col0 = (warp < 6) ? 0 : 64;  // two warps per lane quarter
+            const int64_t n = n0 + 32 * quarter + lane;
+#pragma unroll
+            for (int cb = 0; cb < 2; ++cb) {
+                uint32_t rv[32];
+                const int c = col0 + 32 * cb;
+                tmem_ld32(tmem_d + ((uint32_t)(32 * quarter) << 16) + (uint32_t)c, rv);
+                if (n < a.n) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) {
+                        const int64_t m = m0 + c + j;
+                        if (m < a.m) a.Y[m * a.n + n] = __float2half_rn(__uint_as_float(rv[j]));
+                    }
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_d), "r"(TMEM_COLS)
+                     : "memory");
+    }
+}
+
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_fn() {
+    static EncodeTiledFn fn = nullptr;
+    if (fn == nullptr) {
+        void *p = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(p);
+    }
+    return fn;
+}
+
+template <int BITS, int KIND>
+cudaError_t launch_t(const CUtensorMap &map, const GemmArgs &a, cudaStream_t st) {
+    auto kern = gemm_kernel<BITS, KIND>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((a.m + BN - 1) / BN), (unsigned)((a.n + BM - 1) / BM));
+    kern<<<grid, THREADS, kSmemBytes, st>>>(map, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st) {
+    (void)num_sms;
+    EncodeTiledFn enc = encode_fn();
+    if (enc == nullptr) return cudaErrorNotSupported;
+    CUtensorMap map;
+    const cuuint64_t dims[2] = {(cuuint64_t)a.k, (cuuint64_t)a.m};
+    const cuuint64_t strides[1] = {(cuuint64_t)a.k * 2};
+    const cuuint32_t box[2] = {BK, BN};
+    const cuuint32_t estr[2] = {1, 1};
+    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(a.X), dims, strides, box, estr,
+                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
+    if (a.bits == 4) return launch_t<4, 0>(map, a, st);
+    if (a.kind == 1) return launch_t<3, 1>(map, a, st);
+    return launch_t<3, 0>(map, a, st);
+}
+
+}  // namespace qx

@@ -1,0 +1,66 @@
+// Internal launch interface between the C ABI (qx_api.cu) and the kernels.
+#pragma once
+
+#include <algorithm>
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "qx_common.cuh"
+
+namespace qx {
+
+struct QuantArgs {
+    const __half *W;
+    int64_t n, k;
+    int bits, g, kind, lloyd_iters;
+    int G;       // groups per row
+    int zbytes;  // zero-point bytes per row
+    uint8_t *codes;
+    __half *scales;
+    uint8_t *zeros;
+    __half *luts;
+    uint32_t *status;
+};
+
+struct DequantArgs {
+    const uint8_t *codes;
+    const __half *scales;
+    const uint8_t *zeros;
+    const __half *luts;
+    int64_t n, k;
+    int bits, g, kind, G, zbytes;
+    __half *W;
+};
+
+struct GemvArgs {
+    const uint8_t *codes;
+    const __half *scales;
+    const uint8_t *zeros;
+    const __half *luts;
+    int64_t n, k;
+    int bits, kind, log2g, G, zbytes;
+    const __half *x;  // [batch][k]
+    void *y;          // [batch][n]
+    int batch;
+    int y_f32;
+};
+
+struct GemmArgs {
+    const uint8_t *codes;
+    const __half *scales;
+    const uint8_t *zeros;
+    const __half *luts;
+    int64_t n, k, m;
+    int bits, kind, log2g, G, zbytes;
+    const __half *X;  // [m][k]
+    __half *Y;        // [m][n]
+    uint32_t *status;
+    uint64_t wait_limit_ns;
+};
+
+cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_gemv(const GemvArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st);
+
+}  // namespace qx

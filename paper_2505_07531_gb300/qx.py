@@ -1,0 +1,227 @@
+"""Python binding of libqx.so (ctypes): argument marshalling only.
+
+Every computation runs in the library's CUDA kernels.  PyTorch supplies device
+memory and the current CUDA stream; tensors are passed as raw pointers.  If
+the library has not been built, importing this module raises: there is no CPU
+or PyTorch fallback.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libqx.so")
+
+UNIFORM, LUT = 0, 1
+F16, F32 = 0, 1
+
+STATUS = {
+    0: "QX_OK",
+    1: "QX_ERR_INVALID_ARG",
+    2: "QX_ERR_UNSUPPORTED",
+    3: "QX_ERR_ALIGNMENT",
+    4: "QX_ERR_CUDA",
+    5: "QX_ERR_TIMEOUT",
+    6: "QX_ERR_NONFINITE",
+}
+
+
+class QxError(RuntimeError):
+    """A non-zero qx_status returned by the library."""
+
+    def __init__(self, code: int, where: str):
+        self.code = code
+        self.name = STATUS.get(code, str(code))
+        super().__init__(f"{where}: {self.name} ({_lib().qx_status_string(code).decode()})")
+
+
+class _Recipe(ctypes.Structure):
+    _fields_ = [("bits", ctypes.c_int32), ("group_size", ctypes.c_int32),
+                ("kind", ctypes.c_int32), ("lloyd_iters", ctypes.c_int32)]
+
+
+class _Sizes(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_uint64), ("scales", ctypes.c_uint64),
+                ("zeros", ctypes.c_uint64), ("luts", ctypes.c_uint64)]
+
+
+class _Packed(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int64), ("k", ctypes.c_int64), ("recipe", _Recipe),
+                ("codes", ctypes.c_void_p), ("scales", ctypes.c_void_p),
+                ("zeros", ctypes.c_void_p), ("luts", ctypes.c_void_p)]
+
+
+_LIB = None
+
+
+def library_path() -> str:
+    return _LIB_PATH
+
+
+def _lib():
+    global _LIB
+    if _LIB is None:
+        if not os.path.exists(_LIB_PATH):
+            raise RuntimeError(
+                f"{_LIB_PATH} is missing: build it with paper_2505_07531_gb300.build.build_library() "
+                "(there is no fallback path)")
+        lib = ctypes.CDLL(_LIB_PATH)
+        P, I32, I64, VP = ctypes.POINTER, ctypes.c_int32, ctypes.c_int64, ctypes.c_void_p
+        lib.qx_packed_size.argtypes = [I64, I64, P(_Recipe), P(_Sizes)]
+        lib.qx_quantize.argtypes = [VP, I64, I64, P(_Recipe), P(_Packed), VP]
+        lib.qx_dequant.argtypes = [P(_Packed), VP, VP]
+        lib.qx_gemv.argtypes = [P(_Packed), VP, I32, VP, I32, VP]
+        lib.qx_gemm.argtypes = [P(_Packed), VP, I64, VP, VP]
+        lib.qx_get_device_status.argtypes = [VP]
+        lib.qx_status_string.argtypes = [ctypes.c_int]
+        lib.qx_status_string.restype = ctypes.c_char_p
+        lib.qx_version.argtypes = []
+        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemm",
+                   "qx_get_device_status", "qx_version"):
+            getattr(lib, fn).restype = ctypes.c_int
+        _LIB = lib
+    return _LIB
+
+
+def _check(code: int, where: str):
+    if code != 0:
+        raise QxError(code, where)
+
+
+@dataclass(frozen=True)
+class Recipe:
+    """Per-matrix recipe: bit-width, group size along k, uniform (0) or LUT (1)."""
+
+    bits: int
+    group_size: int
+    kind: int = UNIFORM
+    lloyd_iters: int = 25
+
+    def c(self) -> _Recipe:
+        return _Recipe(self.bits, self.group_size, self.kind, self.lloyd_iters)
+
+
+def packed_size(n: int, k: int, recipe: Recipe) -> dict:
+    """Byte sizes of the packed buffers (host-only call)."""
+    s = _Sizes()
+    r = recipe.c()
+    _check(_lib().qx_packed_size(n, k, ctypes.byref(r), ctypes.byref(s)), "qx_packed_size")
+    return {"codes": s.codes, "scales": s.scales, "zeros": s.zeros, "luts": s.luts}
+
+
+def _stream(dev: torch.device) -> ctypes.c_void_p:
+    return ctypes.c_void_p(torch.cuda.current_stream(dev).cuda_stream)
+
+
+def _ptr(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+class PackedMatrix:
+    """Packed weights of one n x k matrix, held in torch device tensors."""
+
+    def __init__(self, n, k, recipe, codes, scales=None, zeros=None, luts=None):
+        self.n, self.k, self.recipe = int(n), int(k), recipe
+        self.codes, self.scales, self.zeros, self.luts = codes, scales, zeros, luts
+
+    @classmethod
+    def empty(cls, n: int, k: int, recipe: Recipe, device) -> "PackedMatrix":
+        sz = packed_size(n, k, recipe)
+        u8 = dict(dtype=torch.uint8, device=device)
+        codes = torch.empty(sz["codes"], **u8)
+        scales = torch.empty(sz["scales"] // 2, dtype=torch.float16, device=device) if sz["scales"] else None
+        zeros = torch.empty(sz["zeros"], **u8) if sz["zeros"] else None
+        luts = torch.empty(sz["luts"] // 2, dtype=torch.float16, device=device) if sz["luts"] else None
+        return cls(n, k, recipe, codes, scales, zeros, luts)
+
+    @property
+    def device(self):
+        return self.codes.device
+
+    def nbytes(self) -> int:
+        return sum(t.numel() * t.element_size() for t in (self.codes, self.scales, self.zeros, self.luts)
+                   if t is not None)
+
+    def c(self) -> _Packed:
+        return _Packed(self.n, self.k, self.recipe.c(), _ptr(self.codes), _ptr(self.scales),
+                       _ptr(self.zeros), _ptr(self.luts))
+
+    def to_numpy(self) -> dict:
+        """Host copies in the oracle's array shapes (for tests)."""
+        G = self.k // self.recipe.group_size
+        out = {"codes": self.codes.cpu().numpy().reshape(self.n, -1), "scales": None, "zeros": None, "luts": None}
+        if self.scales is not None:
+            out["scales"] = self.scales.cpu().numpy().reshape(self.n, G)
+            out["zeros"] = self.zeros.cpu().numpy().reshape(self.n, -1)
+        if self.luts is not None:
+            out["luts"] = self.luts.cpu().numpy().reshape(self.n, G, 1 << self.recipe.bits)
+        return out
+
+
+def _dev_tensor(t: torch.Tensor, name: str, dtype=torch.float16):
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise ValueError(f"{name} must be {dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+
+
+def quantize(W: torch.Tensor, recipe: Recipe, out: PackedMatrix | None = None) -> PackedMatrix:
+    """Quantize and pack fp16 W [n][k] on its device (qx_quantize)."""
+    _dev_tensor(W, "W")
+    n, k = W.shape
+    P = out if out is not None else PackedMatrix.empty(n, k, recipe, W.device)
+    r = recipe.c()
+    pc = P.c()
+    _check(_lib().qx_quantize(_ptr(W), n, k, ctypes.byref(r), ctypes.byref(pc), _stream(W.device)),
+           "qx_quantize")
+    return P
+
+
+def dequant(P: PackedMatrix, out: torch.Tensor | None = None) -> torch.Tensor:
+    """fp16 W_hat [n][k] (qx_dequant)."""
+    W = out if out is not None else torch.empty((P.n, P.k), dtype=torch.float16, device=P.device)
+    _dev_tensor(W, "out")
+    pc = P.c()
+    _check(_lib().qx_dequant(ctypes.byref(pc), _ptr(W), _stream(P.device)), "qx_dequant")
+    return W
+
+
+def gemv(P: PackedMatrix, x: torch.Tensor, out: torch.Tensor | None = None,
+         out_dtype=torch.float16) -> torch.Tensor:
+    """Decode y = x W_hat^T for x [batch][k] (qx_gemv); returns [batch][n]."""
+    _dev_tensor(x, "x")
+    x2 = x.view(-1, P.k)
+    b = x2.shape[0]
+    dt = out.dtype if out is not None else out_dtype
+    y = out if out is not None else torch.empty((b, P.n), dtype=dt, device=x.device)
+    _dev_tensor(y, "out", dt)
+    code = F32 if dt == torch.float32 else F16
+    pc = P.c()
+    _check(_lib().qx_gemv(ctypes.byref(pc), _ptr(x2), b, _ptr(y), code, _stream(x.device)), "qx_gemv")
+    return y
+
+
+def gemm(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+    """Prefill Y = X W_hat^T for X [m][k] (qx_gemm); returns fp16 [m][n]."""
+    _dev_tensor(X, "X")
+    m = X.shape[0]
+    Y = out if out is not None else torch.empty((m, P.n), dtype=torch.float16, device=X.device)
+    _dev_tensor(Y, "out")
+    pc = P.c()
+    _check(_lib().qx_gemm(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _stream(X.device)), "qx_gemm")
+    return Y
+
+
+def device_status(stream=None) -> int:
+    """Synchronize and return/clear the device status (0 = QX_OK)."""
+    s = ctypes.c_void_p(stream.cuda_stream) if stream is not None else _stream(torch.device("cuda"))
+    return _lib().qx_get_device_status(s)
+
+
+def version() -> int:
+    return _lib().qx_version()

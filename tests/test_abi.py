@@ -1,0 +1,94 @@
+"""The C-ABI library loads, exports every entry point include/qx.h declares, and its
+host-only logic (sizes, validation, status strings) behaves; no GPU needed."""
+import ctypes
+import os
+import re
+
+import pytest
+
+import oracle
+from oracle.pack import Recipe as ORecipe
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def qx():
+    from paper_2505_07531_gb300 import build
+
+    if not os.path.exists(build.LIB):
+        build.build_library()
+    import paper_2505_07531_gb300.qx as qx
+
+    return qx
+
+
+def _declared():
+    names = []
+    for fn in os.listdir(os.path.join(ROOT, "include")):
+        if fn.endswith(".h"):
+            src = open(os.path.join(ROOT, "include", fn)).read()
+            src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+            names += re.findall(r"\b(qx_[a-z0-9_]+)\s*\(", src)
+    return sorted(set(names))
+
+
+def test_every_declared_symbol_is_exported(qx):
+    names = _declared()
+    assert "qx_gemv" in names and "qx_gemm" in names and "qx_quantize" in names
+    lib = ctypes.CDLL(qx.library_path())
+    for n in names:
+        assert hasattr(lib, n), n
+
+
+@pytest.mark.parametrize("n,k,bits,g,kind", [
+    (1, 128, 4, 64, 0), (37, 384, 4, 128, 0), (5, 4096, 3, 64, 0), (3, 11008, 3, 128, 1),
+    (2, 256, 4, 32, 0), (4, 512, 3, 256, 1), (7, 640, 3, 32, 0)])
+def test_packed_size_matches_oracle(qx, n, k, bits, g, kind):
+    got = qx.packed_size(n, k, qx.Recipe(bits, g, kind))
+    want = oracle.packed_sizes(n, k, ORecipe(bits, g, "lut" if kind else "uniform"))
+    assert got == want
+
+
+@pytest.mark.parametrize("n,k,recipe,code", [
+    (0, 128, (4, 64, 0, 0), 1),      # n < 1
+    (4, 100, (4, 64, 0, 0), 2),      # k not a multiple of 128
+    (4, 192, (4, 128, 0, 0), 2),     # k not a multiple of g... and of 128
+    (4, 128, (5, 64, 0, 0), 2),      # bits
+    (4, 128, (4, 48, 0, 0), 2),      # group size
+    (4, 128, (4, 64, 1, 25), 2),     # 4-bit LUT not built
+    (4, 128, (3, 64, 7, 0), 1),      # kind
+    (4, 128, (3, 64, 1, -1), 1),     # lloyd iterations
+])
+def test_packed_size_rejects(qx, n, k, recipe, code):
+    lib = qx._lib()
+    s = qx._Sizes()
+    r = qx._Recipe(*recipe)
+    assert lib.qx_packed_size(n, k, ctypes.byref(r), ctypes.byref(s)) == code
+
+
+def test_entry_points_reject_bad_arguments_before_launching(qx):
+    """Validation happens on the host: these calls return without touching a GPU."""
+    lib = qx._lib()
+    P = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), None, None, None, None)
+    assert lib.qx_gemv(ctypes.byref(P), None, 1, None, 0, None) == 1
+    assert lib.qx_gemm(None, None, 1, None, None) == 1
+    assert lib.qx_dequant(ctypes.byref(P), None, None) == 1
+    # misaligned codes pointer
+    P2 = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), ctypes.c_void_p(0x1008), ctypes.c_void_p(0x2000),
+                    ctypes.c_void_p(0x3000), None)
+    assert lib.qx_dequant(ctypes.byref(P2), ctypes.c_void_p(0x4000), None) == 3
+    # batch outside 1..16
+    P3 = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), ctypes.c_void_p(0x1000), ctypes.c_void_p(0x2000),
+                    ctypes.c_void_p(0x3000), None)
+    assert lib.qx_gemv(ctypes.byref(P3), ctypes.c_void_p(0x4000), 17, ctypes.c_void_p(0x5000), 0, None) == 2
+    assert lib.qx_gemv(ctypes.byref(P3), ctypes.c_void_p(0x4000), 0, ctypes.c_void_p(0x5000), 0, None) == 1
+    assert lib.qx_gemv(ctypes.byref(P3), ctypes.c_void_p(0x4008), 1, ctypes.c_void_p(0x5000), 0, None) == 3
+    assert lib.qx_gemm(ctypes.byref(P3), ctypes.c_void_p(0x4000), 0, ctypes.c_void_p(0x5000), None) == 1
+
+
+def test_status_strings_and_version(qx):
+    lib = qx._lib()
+    for code in range(7):
+        assert len(lib.qx_status_string(code)) > 0
+    assert lib.qx_version() >= 100

@@ -1,0 +1,157 @@
+"""GPU parity through the C ABI: packed codes, scales, zeros, LUTs and dequantized
+weights bit-exact with the CPU oracle; GEMV and GEMM outputs within
+max_n |y - y_ref| <= 2e-3 * ||x_b||_2 * max_n ||w_hat_n||_2 for every row b."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from oracle.pack import Recipe as ORecipe
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def qx(cuda_dev):
+    import paper_2505_07531_gb300.qx as qx
+
+    qx._lib()
+    return qx
+
+
+def _orecipe(bits, g, kind, iters=25):
+    return ORecipe(bits, g, "lut" if kind else "uniform", iters)
+
+
+def _weights(n, k, seed, sigma=0.02, outliers=0.001):
+    return synth.student_t_weights(n, k, sigma, seed=seed, stream=n * 7 + k, outlier_frac=outliers)
+
+
+CASES = [  # n, k, bits, g, kind -- ragged n, several groups/superblocks per row
+    (64, 512, 4, 64, 0),
+    (37, 384, 4, 128, 0),
+    (130, 640, 3, 64, 0),
+    (96, 1024, 3, 128, 1),
+    (33, 256, 4, 32, 0),
+    (17, 512, 3, 256, 1),
+    (50, 768, 3, 32, 1),
+    (257, 256, 4, 256, 0),
+    (1, 128, 3, 128, 0),
+    (3, 128, 4, 128, 0),
+]
+
+
+def _ids(c):
+    return "n%d_k%d_b%d_g%d_%s" % (c[0], c[1], c[2], c[3], "lut" if c[4] else "u")
+
+
+@pytest.fixture(scope="module")
+def packed(qx):
+    """Quantize every case once on the GPU and once in the oracle."""
+    out = {}
+    for c in CASES:
+        n, k, bits, g, kind = c
+        W = _weights(n, k, seed=sum(c))
+        P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+        assert qx.device_status() == 0
+        out[c] = (W, P, oracle.quantize(W, _orecipe(bits, g, kind)))
+    return out
+
+
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_quantize_bit_exact(packed, case):
+    W, P, ref = packed[case]
+    got = P.to_numpy()
+    assert np.array_equal(got["codes"], ref["codes"])
+    for key in ("scales", "zeros", "luts"):
+        if ref[key] is None:
+            assert got[key] is None
+        else:
+            assert np.array_equal(got[key].view(np.uint16) if got[key].dtype == np.float16 else got[key],
+                                  ref[key].view(np.uint16) if ref[key].dtype == np.float16 else ref[key]), key
+
+
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_dequant_bit_exact(qx, packed, case):
+    W, P, ref = packed[case]
+    n, k, bits, g, kind = case
+    Wh = qx.dequant(P).cpu().numpy()
+    want = oracle.dequant(ref, _orecipe(bits, g, kind), k)
+    assert np.array_equal(Wh.view(np.uint16), want.view(np.uint16))
+
+
+def _check_matmul(y_gpu, y_ref, X, Wh):
+    tol = oracle.tolerance(X, Wh)
+    err = oracle.max_abs_err(y_gpu, y_ref)
+    assert np.all(err <= tol), (err, tol)
+    return err / np.maximum(tol, 1e-300)
+
+
+@pytest.mark.parametrize("batch", [1, 2, 3, 4, 5, 8, 16])
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_gemv_tolerance(qx, packed, case, batch):
+    W, P, ref = packed[case]
+    n, k, bits, g, kind = case
+    x = synth.activations(batch, k, seed=batch, stream=k)
+    y_ref = oracle.gemv(ref, _orecipe(bits, g, kind), x, k)
+    Wh = oracle.dequant(ref, _orecipe(bits, g, kind), k)
+    xd = torch.from_numpy(x).cuda()
+    for dt in (torch.float16, torch.float32):
+        y = qx.gemv(P, xd, out_dtype=dt).cpu().numpy()
+        assert y.shape == (batch, n)
+        _check_matmul(y, y_ref, x, Wh)
+
+
+@pytest.mark.parametrize("m", [1, 7, 128, 200])
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_gemm_tolerance(qx, packed, case, m):
+    W, P, ref = packed[case]
+    n, k, bits, g, kind = case
+    X = synth.activations(m, k, seed=m, stream=3 * k)
+    Y = qx.gemm(P, torch.from_numpy(X).cuda())
+    assert qx.device_status() == 0
+    Y = Y.cpu().numpy()
+    y_ref = oracle.gemm(ref, _orecipe(bits, g, kind), X, k)
+    _check_matmul(Y, y_ref, X, oracle.dequant(ref, _orecipe(bits, g, kind), k))
+
+
+def test_gemm_many_tiles(qx):
+    """Several W-row tiles and token tiles, ragged in both, k spanning > 4 stages."""
+    n, k, m = 300, 1280, 333
+    for bits, g, kind in ((4, 64, 0), (3, 128, 1), (3, 64, 0)):
+        W = _weights(n, k, seed=bits + g + kind)
+        ref = oracle.quantize(W, _orecipe(bits, g, kind))
+        P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+        X = synth.activations(m, k, seed=5, stream=k)
+        Y = qx.gemm(P, torch.from_numpy(X).cuda()).cpu().numpy()
+        assert qx.device_status() == 0
+        _check_matmul(Y, oracle.gemm(ref, _orecipe(bits, g, kind), X, k), X,
+                      oracle.dequant(ref, _orecipe(bits, g, kind), k))
+
+
+def test_config_single_layer_512(qx):
+    """512 x 512 Student-t(4), sigma 0.02, 0.1% outliers at 10 sigma, seed 0; U4 g64; x 1 x 512."""
+    W = synth.student_t_weights(512, 512, 0.02, seed=0, stream=0, outlier_frac=0.001)
+    x = synth.activations(1, 512, seed=0, stream=1)
+    rec = _orecipe(4, 64, 0)
+    ref = oracle.quantize(W, rec)
+    P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(4, 64, 0))
+    got = P.to_numpy()
+    assert np.array_equal(got["codes"], ref["codes"])
+    assert np.array_equal(got["scales"].view(np.uint16), ref["scales"].view(np.uint16))
+    assert np.array_equal(got["zeros"], ref["zeros"])
+    y = qx.gemv(P, torch.from_numpy(x).cuda(), out_dtype=torch.float32).cpu().numpy()
+    _check_matmul(y, oracle.gemv(ref, rec, x, 512), x, oracle.dequant(ref, rec, 512))
+
+
+def test_nonfinite_weight_sets_status(qx):
+    W = torch.zeros((4, 128), dtype=torch.float16, device="cuda")
+    W[2, 5] = float("nan")
+    qx.quantize(W, qx.Recipe(4, 64, 0))
+    assert qx.device_status() == 6
+    assert qx.device_status() == 0  # read clears it
+    W[2, 5] = float("inf")
+    qx.quantize(W, qx.Recipe(3, 128, 1))
+    assert qx.device_status() == 6
+    assert qx.device_status() == 0
