@@ -243,7 +243,7 @@ def run_reference(args):
 def _quantize_layer(qx, torch, dev, mats, recipe, seed=0):
     import synth
 
-    out = []
+    out = []  # [(name, PackedMatrix)]
     for name, n, k, sigma, sid in mats:
         W = synth.student_t_weights_torch(n, k, sigma, seed=seed, stream=sid, device=dev)
         out.append((name, qx.quantize(W, recipe)))
@@ -273,20 +273,32 @@ def run_ours(args):
     l2 = getattr(props, "L2_cache_size", 0) or 126 * 2 ** 20
 
     recipe = qx.Recipe(3, 128, qx.LUT, 25)
-    base = _quantize_layer(qx, torch, dev, LAYER, recipe)
-    layer_bytes = sum(P.nbytes() for _, P in base)
+    base = dict(_quantize_layer(qx, torch, dev, LAYER, recipe))
+    layer_bytes = sum(P.nbytes() for P in base.values())
     copies = max(2, math.ceil(4 * l2 / layer_bytes))
-    layers = [base] + [[(nm, _clone(qx, P)) for nm, P in base] for _ in range(copies - 1)]
-    xs = [synth.activations_torch(1, k, seed=0, stream=50 + sid, device=dev) for _, n, k, _, sid in LAYER]
-    ys = [torch.empty((1, n), dtype=torch.float16, device=dev) for _, n, k, _, _ in LAYER]
-    io_bytes = sum(x.numel() * 2 for x in xs) + sum(y.numel() * 2 for y in ys)
+    layers = [base] + [{nm: _clone(qx, P) for nm, P in base.items()} for _ in range(copies - 1)]
+    # decode dependency chain of one token through the layer: q, k, v share the
+    # attention input; o reads the attention output; gate, up share the MLP
+    # input; down reads act(gate) * up.  Activations are synthetic N(0, 1).
+    x_attn = synth.activations_torch(1, 4096, seed=0, stream=50, device=dev)
+    x_o = synth.activations_torch(1, 4096, seed=0, stream=51, device=dev)
+    x_mlp = synth.activations_torch(1, 4096, seed=0, stream=52, device=dev)
+    x_down = synth.activations_torch(1, 11008, seed=0, stream=53, device=dev)
+    ys = {nm: torch.empty((1, n), dtype=torch.float16, device=dev) for nm, n, k, _, _ in LAYER}
+    CHAIN = [(["q_proj", "k_proj", "v_proj"], x_attn), (["o_proj"], x_o),
+             (["gate_proj", "up_proj"], x_mlp), (["down_proj"], x_down)]
+    io_bytes = sum(x.numel() * 2 for x in (x_attn, x_o, x_mlp, x_down)) + sum(y.numel() * 2 for y in ys.values())
     step_bytes = layer_bytes + io_bytes
 
     stream = torch.cuda.Stream(dev)
 
+    def launch(c, j):
+        names, x = CHAIN[j]
+        qx.gemv_multi([layers[c][nm] for nm in names], [x] * len(names), outs=[ys[nm] for nm in names], pdl=True)
+
     def step(c):
-        for (name, P), x, y in zip(layers[c], xs, ys):
-            qx.gemv(P, x, out=y)
+        for j in range(len(CHAIN)):
+            launch(c, j)
 
     with torch.cuda.stream(stream):
         for c in range(copies):
@@ -334,34 +346,50 @@ def run_ours(args):
 
     # per-launch kernel durations (events on the launching stream) for the roofline
     reps = max(3, min(args.steps, 200))
-    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in LAYER]
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in CHAIN]
            for _ in range(reps)]
     with torch.cuda.stream(stream):
         for r in range(reps):
-            c = r % copies
-            for j, ((name, P), x, y) in enumerate(zip(layers[c], xs, ys)):
+            for j in range(len(CHAIN)):
                 evs[r][j][0].record(stream)
-                qx.gemv(P, x, out=y)
+                launch(r % copies, j)
                 evs[r][j][1].record(stream)
     torch.cuda.synchronize(dev)
     kern_ms = sum(a.elapsed_time(b) for row in evs for a, b in row) / reps
-    per_matrix_us = {LAYER[j][0]: 1e3 * sum(evs[r][j][0].elapsed_time(evs[r][j][1]) for r in range(reps)) / reps
-                     for j in range(len(LAYER))}
+    per_launch_us = {"+".join(CHAIN[j][0]): 1e3 * sum(evs[r][j][0].elapsed_time(evs[r][j][1])
+                                                      for r in range(reps)) / reps for j in range(len(CHAIN))}
     achieved = step_bytes / (kern_ms * 1e-3) / 1e9
 
+    # the seven matrices as independent problems in one launch (upper bound of the chain)
+    xs7 = {nm: (x_down if nm == "down_proj" else x_attn) for nm, _, _, _, _ in LAYER}
+    with torch.cuda.stream(stream):
+        for r in range(3):
+            qx.gemv_multi([layers[r % copies][nm] for nm, *_ in LAYER], [xs7[nm] for nm, *_ in LAYER],
+                          outs=[ys[nm] for nm, *_ in LAYER], pdl=True)
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for r in range(reps):
+            qx.gemv_multi([layers[r % copies][nm] for nm, *_ in LAYER], [xs7[nm] for nm, *_ in LAYER],
+                          outs=[ys[nm] for nm, *_ in LAYER], pdl=True)
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    one_launch_ms = e0.elapsed_time(e1) / reps
+
     # end to end through the public API with host buffers: pinned x in, y out, per step
-    hx = [x.cpu().pin_memory() for x in xs]
-    hy = [torch.empty(y.shape, dtype=y.dtype).pin_memory() for y in ys]
+    xs_dev = [x_attn, x_o, x_mlp, x_down]
+    hx = [x.cpu().pin_memory() for x in xs_dev]
+    hy = {nm: torch.empty(y.shape, dtype=y.dtype).pin_memory() for nm, y in ys.items()}
     e2e_steps = max(3, min(args.steps, 2000))
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
     with torch.cuda.stream(stream):
         for i in range(e2e_steps):
             c = i % copies
-            for j, ((name, P), x, y) in enumerate(zip(layers[c], xs, ys)):
-                x.copy_(hx[j], non_blocking=True)
-                qx.gemv(P, x, out=y)
-                hy[j].copy_(y, non_blocking=True)
+            for x, h in zip(xs_dev, hx):
+                x.copy_(h, non_blocking=True)
+            step(c)
+            for nm, y in ys.items():
+                hy[nm].copy_(y, non_blocking=True)
             stream.synchronize()
     e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
     e2e_value = step_bytes * ws / (e2e_ms * 1e-3) / 1e9
@@ -380,21 +408,23 @@ def run_ours(args):
                        "matrices": {nm: [n, k] for nm, n, k, _, _ in LAYER},
                        "recipe": "3-bit LUT (8 fp16 levels, Lloyd-Max) group 128",
                        "batch": 1, "bytes_per_step": step_bytes,
+                       "step": "qkv | o | gate+up | down: 4 qx_gemv_multi launches (PDL) in one CUDA graph",
                        "l2": f"{copies} rotating weight copies ({copies * layer_bytes / 1e6:.0f} MB) > "
-                             f"4x L2 ({l2 / 1e6:.0f} MB)",
-                       "graph": "one CUDA graph per step (7 launches)"},
-            "per_matrix_us": per_matrix_us,
+                             f"4x L2 ({l2 / 1e6:.0f} MB)"},
+            "per_launch_us": per_launch_us,
+            "one_launch_7_matrices": {"us": one_launch_ms * 1e3,
+                                      "GBps": step_bytes / (one_launch_ms * 1e-3) / 1e9},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                          "frac": achieved / hbm, "peak_source": f"{peak_src} hbm_gbs",
-                         "kernel": "gemv_kernel<3,LUT,1,2>",
+                         "kernel": "gemv_kernel<3,LUT,1,4>",
                          "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
             "gemm": gemm,
             "cpu_baseline": cpu,
             "clocks": clocks,
             "e2e": {"value": e2e_value, "unit": "GB/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": sum(x.numel() * 2 for x in hx),
-                    "d2h_bytes_per_step": sum(y.numel() * 2 for y in hy)},
-            "gpu_launches": args.steps * len(LAYER),
+                    "d2h_bytes_per_step": sum(y.numel() * 2 for y in hy.values())},
+            "gpu_launches": args.steps * len(CHAIN),
         }
         print(json.dumps(line))
     if dist is not None:

@@ -123,9 +123,31 @@ qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream);
 /* Decode matmul y = x W_hat^T (Section 2.4: memory-bound decoding; Table 2
  * "Decode").  x: device fp16 [batch][k], row-major, 16-byte aligned;
  * y: device [batch][n] of y_dtype (QX_F16 or QX_F32), 4-byte aligned.
- * batch in 1..16.  fp32 accumulation across groups. */
+ * batch in 1..16; k <= 32768.  fp16 products summed in fp32 per 32 weights
+ * and across groups.  Batches above four stream the weights once per four
+ * rows of x. */
 qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y,
                   int32_t y_dtype, void *stream);
+
+/* Flags of qx_gemv_multi. */
+enum {
+    /* Launch with programmatic dependent launch: the kernel may start, and
+     * stream this call's weights, while the previous kernel in the stream is
+     * still running; it waits for that kernel before reading x or writing y.
+     * Set it only when the previous kernel does not write this call's weights. */
+    QX_GEMV_PDL = 1
+};
+
+/* Several decode matmuls in one launch: y[i] = x[i] W_hat_i^T, i < count
+ * (count 1..8).  All matrices share bits and kind (the recipe's group size and
+ * the shapes may differ); x[i], y[i] are device pointers with the layout and
+ * alignment of qx_gemv, passed in host arrays of `count` pointers.  One
+ * persistent grid covers the rows of all matrices in byte-balanced slices, so
+ * the launch and HBM ramp-up are paid once for the whole group (e.g. the q, k,
+ * v or gate, up projections of a decoder layer, which share x).
+ * flags: 0 or QX_GEMV_PDL. */
+qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const *x, int32_t batch,
+                        void *const *y, int32_t y_dtype, int32_t flags, void *stream);
 
 /* Prefill matmul Y = X W_hat^T (Table 2 "Prefill") on the tcgen05 tensor cores:
  * W_hat tiles are dequantized into shared memory and multiplied in fp16 with

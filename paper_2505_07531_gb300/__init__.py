@@ -6,6 +6,7 @@ C ABI in ``include/qx.h``); :mod:`.qx` is its thin ctypes binding.
 from .qx import (  # noqa: F401
     F16,
     F32,
+    GEMV_PDL,
     LUT,
     UNIFORM,
     PackedMatrix,
@@ -15,6 +16,7 @@ from .qx import (  # noqa: F401
     device_status,
     gemm,
     gemv,
+    gemv_multi,
     library_path,
     packed_size,
     quantize,

@@ -1,6 +1,7 @@
 // C ABI of the qx library: argument validation, dispatch, device status.
 // The declarations, with the meaning, layout, ownership and error behaviour of
 // every argument, are in include/qx.h.
+#include <algorithm>
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
@@ -193,35 +194,104 @@ QX_API qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream) {
     return from_cuda(qx::launch_dequant(a, d->num_sms, static_cast<cudaStream_t>(stream)));
 }
 
-QX_API qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y, int32_t y_dtype,
-                         void *stream) {
+namespace {
+
+// One decode launch over `count` matrices for activation rows b0 .. b0+nb-1
+// (nb <= 4).  When the group's activations do not fit one CTA's shared
+// memory, the group is split per matrix, then the rows are halved.
+qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int b0, int nb, void *const *y,
+                     int y_dtype, int flags, cudaStream_t st, DeviceInfo *d) {
+    const int esz = y_dtype == QX_F32 ? 4 : 2;
+    qx::GemvMulti a{};
+    a.count = count;
+    a.bits = mats[0].recipe.bits;
+    a.kind = mats[0].recipe.kind;
+    a.batch = nb;
+    a.y_f32 = y_dtype == QX_F32;
+    a.status = d->status;
+    a.wait_limit_ns = wait_limit_ns();
+    for (int i = 0; i < count; ++i) {
+        const qx_packed &p = mats[i];
+        qx::GemvMat &M = a.mat[i];
+        M.codes = static_cast<const uint8_t *>(p.codes);
+        M.scales = static_cast<const __half *>(p.scales);
+        M.zeros = static_cast<const uint8_t *>(p.zeros);
+        M.luts = static_cast<const __half *>(p.luts);
+        M.x = static_cast<const __half *>(x[i]) + (int64_t)b0 * p.k;
+        M.y = static_cast<uint8_t *>(y[i]) + (int64_t)b0 * p.n * esz;
+        M.n = p.n;
+        M.k = p.k;
+        M.G = (int)(p.k / p.recipe.group_size);
+        M.zbytes = (M.G + 1) / 2;
+        M.log2g = ilog2(p.recipe.group_size);
+    }
+    if (qx::plan_gemv(a, d->num_sms))
+        return qx::launch_gemv_multi(a, st, (flags & QX_GEMV_PDL) != 0) == cudaSuccess ? QX_OK : QX_ERR_CUDA;
+    if (count > 1) {
+        for (int i = 0; i < count; ++i) {
+            qx_status s = gemv_chunk(&mats[i], 1, &x[i], b0, nb, &y[i], y_dtype, flags, st, d);
+            if (s != QX_OK) return s;
+        }
+        return QX_OK;
+    }
+    if (nb > 1) {
+        const int h = nb / 2;
+        qx_status s = gemv_chunk(mats, 1, x, b0, h, y, y_dtype, flags, st, d);
+        return s != QX_OK ? s : gemv_chunk(mats, 1, x, b0 + h, nb - h, y, y_dtype, flags, st, d);
+    }
+    return QX_ERR_UNSUPPORTED;
+}
+
+// Batches above four are processed four rows of x at a time; each chunk
+// streams the weights once.
+qx_status run_gemv(const qx_packed *mats, int count, const void *const *x, int batch, void *const *y,
+                   int y_dtype, int flags, cudaStream_t st, DeviceInfo *d) {
+    for (int b0 = 0; b0 < batch; b0 += 4) {
+        qx_status s = gemv_chunk(mats, count, x, b0, std::min(4, batch - b0), y, y_dtype, flags, st, d);
+        if (s != QX_OK) return s;
+    }
+    return QX_OK;
+}
+
+qx_status check_gemv_args(const qx_packed *p, const void *x, int32_t batch, const void *y, int32_t y_dtype) {
     qx_status s = check_packed(p);
     if (s != QX_OK) return s;
     if (x == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
     if (y_dtype != QX_F16 && y_dtype != QX_F32) return QX_ERR_INVALID_ARG;
     if (batch < 1) return QX_ERR_INVALID_ARG;
     if (batch > 16) return QX_ERR_UNSUPPORTED;
+    if (p->k > 32768) return QX_ERR_UNSUPPORTED;  // x and a row must fit shared memory
     if (!aligned(x, 16)) return QX_ERR_ALIGNMENT;
     if (!aligned(y, y_dtype == QX_F32 ? 4 : 2)) return QX_ERR_ALIGNMENT;
+    return QX_OK;
+}
+
+}  // namespace
+
+QX_API qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y, int32_t y_dtype,
+                         void *stream) {
+    qx_status s = check_gemv_args(p, x, batch, y, y_dtype);
+    if (s != QX_OK) return s;
     DeviceInfo *d = nullptr;
     if ((s = device_info(&d)) != QX_OK) return s;
-    qx::GemvArgs a{};
-    a.codes = static_cast<const uint8_t *>(p->codes);
-    a.scales = static_cast<const __half *>(p->scales);
-    a.zeros = static_cast<const uint8_t *>(p->zeros);
-    a.luts = static_cast<const __half *>(p->luts);
-    a.n = p->n;
-    a.k = p->k;
-    a.bits = p->recipe.bits;
-    a.kind = p->recipe.kind;
-    a.log2g = ilog2(p->recipe.group_size);
-    a.G = (int)(p->k / p->recipe.group_size);
-    a.zbytes = (a.G + 1) / 2;
-    a.x = static_cast<const __half *>(x);
-    a.y = y;
-    a.batch = batch;
-    a.y_f32 = y_dtype == QX_F32;
-    return from_cuda(qx::launch_gemv(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+    return run_gemv(p, 1, &x, batch, &y, y_dtype, 0, static_cast<cudaStream_t>(stream), d);
+}
+
+QX_API qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const *x, int32_t batch,
+                               void *const *y, int32_t y_dtype, int32_t flags, void *stream) {
+    if (mats == nullptr || x == nullptr || y == nullptr || count < 1) return QX_ERR_INVALID_ARG;
+    if (count > qx::kMaxGemvMats) return QX_ERR_UNSUPPORTED;
+    if ((flags & ~QX_GEMV_PDL) != 0) return QX_ERR_INVALID_ARG;
+    for (int i = 0; i < count; ++i) {
+        qx_status s = check_gemv_args(&mats[i], x[i], batch, y[i], y_dtype);
+        if (s != QX_OK) return s;
+        if (mats[i].recipe.bits != mats[0].recipe.bits || mats[i].recipe.kind != mats[0].recipe.kind)
+            return QX_ERR_INVALID_ARG;
+    }
+    DeviceInfo *d = nullptr;
+    qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    return run_gemv(mats, count, x, batch, y, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
 }
 
 QX_API qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream) {

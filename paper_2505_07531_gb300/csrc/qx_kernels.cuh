@@ -32,17 +32,30 @@ struct DequantArgs {
     __half *W;
 };
 
-struct GemvArgs {
+constexpr int kMaxGemvMats = 8;
+
+// One matrix of a (multi-matrix) decode launch.  The geometry fields after
+// log2g are filled by plan_gemv().
+struct GemvMat {
     const uint8_t *codes;
     const __half *scales;
     const uint8_t *zeros;
     const __half *luts;
-    int64_t n, k;
-    int bits, kind, log2g, G, zbytes;
     const __half *x;  // [batch][k]
     void *y;          // [batch][n]
-    int batch;
-    int y_f32;
+    int64_t n, k;
+    int G, zbytes, log2g;
+    int CB, LB, SB, ZB, row_bytes, RB;
+    int64_t byte_off;
+};
+
+struct GemvMulti {
+    GemvMat mat[kMaxGemvMats];
+    int count, bits, kind, batch, y_f32;
+    int grid, stages, stage_bytes, x_smem_bytes, smem_bytes;
+    int64_t total_bytes;
+    uint32_t *status;
+    uint64_t wait_limit_ns;
 };
 
 struct GemmArgs {
@@ -60,7 +73,8 @@ struct GemmArgs {
 
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
-cudaError_t launch_gemv(const GemvArgs &a, int num_sms, cudaStream_t st);
+bool plan_gemv(GemvMulti &a, int num_sms);
+cudaError_t launch_gemv_multi(const GemvMulti &a, cudaStream_t st, bool pdl);
 cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st);
 
 }  // namespace qx

@@ -17,6 +17,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "lib
 
 UNIFORM, LUT = 0, 1
 F16, F32 = 0, 1
+GEMV_PDL = 1
 
 STATUS = {
     0: "QX_OK",
@@ -75,11 +76,12 @@ def _lib():
         lib.qx_dequant.argtypes = [P(_Packed), VP, VP]
         lib.qx_gemv.argtypes = [P(_Packed), VP, I32, VP, I32, VP]
         lib.qx_gemm.argtypes = [P(_Packed), VP, I64, VP, VP]
+        lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
         lib.qx_status_string.restype = ctypes.c_char_p
         lib.qx_version.argtypes = []
-        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemm",
+        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
@@ -204,6 +206,32 @@ def gemv(P: PackedMatrix, x: torch.Tensor, out: torch.Tensor | None = None,
     pc = P.c()
     _check(_lib().qx_gemv(ctypes.byref(pc), _ptr(x2), b, _ptr(y), code, _stream(x.device)), "qx_gemv")
     return y
+
+
+def gemv_multi(mats, xs, outs=None, out_dtype=torch.float16, pdl: bool = False):
+    """Several decode matmuls in one launch (qx_gemv_multi); returns the outputs.
+
+    ``mats`` share bits and kind; ``xs[i]`` is [batch][k_i].  ``pdl`` lets the
+    kernel start while the previous kernel in the stream runs: set it only when
+    that kernel does not write these weights.
+    """
+    mats, xs = list(mats), list(xs)
+    if len(mats) != len(xs) or not mats:
+        raise ValueError("need one x per matrix")
+    for x in xs:
+        _dev_tensor(x, "x")
+    b = xs[0].numel() // mats[0].k
+    dt = outs[0].dtype if outs is not None else out_dtype
+    ys = list(outs) if outs is not None else [torch.empty((b, P.n), dtype=dt, device=xs[0].device) for P in mats]
+    for y in ys:
+        _dev_tensor(y, "out", dt)
+    arr = (_Packed * len(mats))(*[P.c() for P in mats])
+    xp = (ctypes.c_void_p * len(xs))(*[x.data_ptr() for x in xs])
+    yp = (ctypes.c_void_p * len(ys))(*[y.data_ptr() for y in ys])
+    code = F32 if dt == torch.float32 else F16
+    _check(_lib().qx_gemv_multi(arr, len(mats), xp, b, yp, code, GEMV_PDL if pdl else 0, _stream(xs[0].device)),
+           "qx_gemv_multi")
+    return ys
 
 
 def gemm(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:

@@ -155,3 +155,106 @@ def test_nonfinite_weight_sets_status(qx):
     qx.quantize(W, qx.Recipe(3, 128, 1))
     assert qx.device_status() == 6
     assert qx.device_status() == 0
+
+
+MULTI_GROUPS = [  # matrices of one launch share bits and kind
+    [(2048, 4096, 3, 128, 1), (512, 4096, 3, 128, 1), (256, 11008, 3, 64, 1)],
+    [(300, 512, 4, 64, 0), (77, 1024, 4, 128, 0), (5, 256, 4, 32, 0), (640, 384, 4, 64, 0)],
+    [(129, 640, 3, 64, 0), (3, 128, 3, 32, 0)],
+    [(1, 128, 4, 128, 0)] * 8,
+]
+
+
+@pytest.fixture(scope="module")
+def multi_packed(qx):
+    """Each group quantized once on the GPU and once in the oracle."""
+    out = []
+    for gi, group in enumerate(MULTI_GROUPS):
+        Ps, refs = [], []
+        for i, (n, k, bits, g, kind) in enumerate(group):
+            W = _weights(n, k, seed=97 + i + 10 * gi)
+            Ps.append(qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind)))
+            refs.append(oracle.quantize(W, _orecipe(bits, g, kind)))
+        out.append((Ps, refs))
+    return out
+
+
+@pytest.mark.parametrize("pdl", [False, True])
+@pytest.mark.parametrize("batch", [1, 3, 6])
+@pytest.mark.parametrize("gi", range(len(MULTI_GROUPS)))
+def test_gemv_multi(qx, multi_packed, gi, batch, pdl):
+    """One launch over several matrices (slices spanning matrix boundaries)."""
+    group = MULTI_GROUPS[gi]
+    Ps, refs = multi_packed[gi]
+    xs = [synth.activations(batch, k, seed=i, stream=gi) for i, (n, k, bits, g, kind) in enumerate(group)]
+    xds = [torch.from_numpy(x).cuda() for x in xs]
+    if pdl:  # the flag's contract: the previous kernel must not write these weights
+        torch.cuda.synchronize()
+    ys = qx.gemv_multi(Ps, xds, out_dtype=torch.float32, pdl=pdl)
+    for (n, k, bits, g, kind), ref, x, y in zip(group, refs, xs, ys):
+        rec = _orecipe(bits, g, kind)
+        _check_matmul(y.cpu().numpy(), oracle.gemv(ref, rec, x, k), x, oracle.dequant(ref, rec, k))
+
+
+def test_gemv_multi_rejects_mixed_kinds(qx):
+    a = qx.quantize(torch.zeros((4, 128), dtype=torch.float16, device="cuda"), qx.Recipe(4, 64, 0))
+    b = qx.quantize(torch.zeros((4, 128), dtype=torch.float16, device="cuda"), qx.Recipe(3, 128, 1))
+    x = torch.zeros((1, 128), dtype=torch.float16, device="cuda")
+    with pytest.raises(qx.QxError):
+        qx.gemv_multi([a, b], [x, x])
+
+
+def test_gemv_pdl_chain_orders_activations(qx):
+    """A decode that reads the previous decode's output under PDL sees the finished
+    output: the chained result equals the same chain run without PDL, bit for bit."""
+    W1 = _weights(4096, 4096, seed=1)
+    W2 = _weights(2048, 4096, seed=2)
+    P1 = qx.quantize(torch.from_numpy(W1).cuda(), qx.Recipe(3, 128, 1))
+    P2 = qx.quantize(torch.from_numpy(W2).cuda(), qx.Recipe(3, 128, 1))
+    x = torch.from_numpy(synth.activations(1, 4096, seed=3, stream=3)).cuda()
+    y1 = torch.empty((1, 4096), dtype=torch.float16, device="cuda")
+    outs = []
+    for pdl in (False, True):
+        torch.cuda.synchronize()
+        for _ in range(20):
+            qx.gemv_multi([P1], [x], outs=[y1], pdl=pdl)
+            (y2,) = qx.gemv_multi([P2], [y1], pdl=pdl)
+        outs.append(y2.clone())
+    torch.cuda.synchronize()
+    assert torch.equal(outs[0], outs[1])
+
+
+@pytest.mark.parametrize("bits,g,kind", [(4, 32, 0), (3, 32, 1)])
+def test_gemv_longest_rows(qx, bits, g, kind):
+    """k = 32768 (the largest k the decode kernel takes), batch 3: the host splits the batch."""
+    n, k = 40, 32768
+    W = _weights(n, k, seed=k + bits)
+    ref = oracle.quantize(W, _orecipe(bits, g, kind))
+    P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+    x = synth.activations(3, k, seed=1, stream=2)
+    y = qx.gemv(P, torch.from_numpy(x).cuda(), out_dtype=torch.float32).cpu().numpy()
+    rec = _orecipe(bits, g, kind)
+    _check_matmul(y, oracle.gemv(ref, rec, x, k), x, oracle.dequant(ref, rec, k))
+
+
+WRAP_CASES = [  # enough rows that every CTA cycles its shared-memory ring several times
+    (20000, 128, 3, 128, 1),
+    (20000, 256, 3, 64, 0),
+    (20000, 512, 4, 64, 0),
+    (6000, 4096, 3, 128, 0),
+]
+
+
+@pytest.mark.parametrize("batch", [1, 3, 4])
+@pytest.mark.parametrize("case", WRAP_CASES, ids=_ids)
+def test_gemv_ring_wraps(qx, case, batch):
+    n, k, bits, g, kind = case
+    W = _weights(n, k, seed=n + k)
+    rec = _orecipe(bits, g, kind)
+    ref = oracle.quantize(W, rec)
+    P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+    x = synth.activations(batch, k, seed=batch, stream=n)
+    y = torch.full((batch, n), float("nan"), dtype=torch.float32, device="cuda")
+    qx.gemv(P, torch.from_numpy(x).cuda(), out=y)
+    assert qx.device_status() == 0
+    _check_matmul(y.cpu().numpy(), oracle.gemv(ref, rec, x, k), x, oracle.dequant(ref, rec, k))
