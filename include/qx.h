@@ -163,6 +163,10 @@ qx_status qx_get_device_status(void *stream);
 /* Static, NUL-terminated description of a status code. */
 const char *qx_status_string(qx_status s);
 
+/* Name of the last CUDA error an entry point of this thread turned into
+ * QX_ERR_CUDA (a static string; "no error" if none). */
+const char *qx_last_error_string(void);
+
 /* Library version as major*10000 + minor*100 + patch. */
 int32_t qx_version(void);
 

@@ -103,11 +103,19 @@ qx_status check_packed(const qx_packed *p) {
     return QX_OK;
 }
 
-qx_status from_cuda(cudaError_t e) { return e == cudaSuccess ? QX_OK : QX_ERR_CUDA; }
+thread_local const char *t_last_error = "no error";
+
+qx_status from_cuda(cudaError_t e) {
+    if (e == cudaSuccess) return QX_OK;
+    t_last_error = cudaGetErrorName(e);
+    return QX_ERR_CUDA;
+}
 
 }  // namespace
 
 QX_API int32_t qx_version(void) { return 100; }
+
+QX_API const char *qx_last_error_string(void) { return t_last_error; }
 
 QX_API const char *qx_status_string(qx_status s) {
     switch (s) {
@@ -226,7 +234,7 @@ qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int
         M.log2g = ilog2(p.recipe.group_size);
     }
     if (qx::plan_gemv(a, d->num_sms))
-        return qx::launch_gemv_multi(a, st, (flags & QX_GEMV_PDL) != 0) == cudaSuccess ? QX_OK : QX_ERR_CUDA;
+        return from_cuda(qx::launch_gemv_multi(a, st, (flags & QX_GEMV_PDL) != 0));
     if (count > 1) {
         for (int i = 0; i < count; ++i) {
             qx_status s = gemv_chunk(&mats[i], 1, &x[i], b0, nb, &y[i], y_dtype, flags, st, d);

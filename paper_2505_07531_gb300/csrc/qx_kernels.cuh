@@ -49,8 +49,14 @@ struct GemvMat {
     int64_t byte_off;
 };
 
+constexpr int kMaxGemvCtas = 1024;
+
 struct GemvMulti {
     GemvMat mat[kMaxGemvMats];
+    // first row of every CTA in the concatenation of all matrices' rows
+    // (byte-balanced slices computed on the host); cta_row[grid] = total rows
+    int64_t cta_row[kMaxGemvCtas + 1];
+    int64_t row_off[kMaxGemvMats + 1];  // first concatenated row of each matrix
     int count, bits, kind, batch, y_f32;
     int grid, stages, stage_bytes, x_smem_bytes, smem_bytes;
     int64_t total_bytes;

@@ -36,7 +36,10 @@ class QxError(RuntimeError):
     def __init__(self, code: int, where: str):
         self.code = code
         self.name = STATUS.get(code, str(code))
-        super().__init__(f"{where}: {self.name} ({_lib().qx_status_string(code).decode()})")
+        detail = _lib().qx_status_string(code).decode()
+        if code == 4:
+            detail += ": " + _lib().qx_last_error_string().decode()
+        super().__init__(f"{where}: {self.name} ({detail})")
 
 
 class _Recipe(ctypes.Structure):
@@ -81,6 +84,8 @@ def _lib():
         lib.qx_status_string.argtypes = [ctypes.c_int]
         lib.qx_status_string.restype = ctypes.c_char_p
         lib.qx_version.argtypes = []
+        lib.qx_last_error_string.argtypes = []
+        lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
