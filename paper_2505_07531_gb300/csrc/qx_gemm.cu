@@ -369,9 +369,17 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
     }
 }
 
-using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
-                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
-                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+template <int BITS, int KIND>
+cudaError_t launch_t(const CUtensorMap &map, const GemmArgs &a, cudaStream_t st) {
+    auto kern = gemm_kernel<BITS, KIND>;
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    if (e != cudaSuccess) return e;
+    dim3 grid((unsigned)((a.m + BN - 1) / BN), (unsigned)((a.n + BM - 1) / BM));
+    kern<<<grid, THREADS, kSmemBytes, st>>>(map, a);
+    return cudaGetLastError();
+}
+
+}  // namespace
 
 EncodeTiledFn encode_fn() {
     static EncodeTiledFn fn = nullptr;
@@ -385,18 +393,6 @@ EncodeTiledFn encode_fn() {
     }
     return fn;
 }
-
-template <int BITS, int KIND>
-cudaError_t launch_t(const CUtensorMap &map, const GemmArgs &a, cudaStream_t st) {
-    auto kern = gemm_kernel<BITS, KIND>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
-    if (e != cudaSuccess) return e;
-    dim3 grid((unsigned)((a.m + BN - 1) / BN), (unsigned)((a.n + BM - 1) / BM));
-    kern<<<grid, THREADS, kSmemBytes, st>>>(map, a);
-    return cudaGetLastError();
-}
-
-}  // namespace
 
 cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st) {
     (void)num_sms;

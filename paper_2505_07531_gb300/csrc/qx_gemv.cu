@@ -1,137 +1,137 @@
 // Decode matmul y[b][n] = sum_k w_hat[n][k] x[b][k] on CUDA cores, fed by TMA.
 //
-// Decoding reads every weight once per token: it is bound by HBM bandwidth
-// and by the cost of unpacking the codes (paper Section 2.4).  To keep HBM
-// busy every SM needs tens of kilobytes of loads in flight from its first
-// cycle, and the launch itself must be amortised over as many bytes as
-// possible, so the kernel is built around the Blackwell bulk-copy engine and
-// serves several matrices in one launch:
+// Decoding reads every weight once per token, so it is bound by HBM bandwidth
+// and by the cost of unpacking the codes (paper Section 2.4).  On GB300 the
+// unpack of a 3-bit code through an 8-entry table costs about one byte-permute
+// per weight, which at HBM speed keeps the integer pipe nearly busy: the
+// kernel is built to spend as few issue slots as possible on anything else.
 //
-//   * one persistent CTA per SM owns a byte-balanced slice of the rows of all
-//     matrices of the call, taken in order (a slice may span matrices);
-//   * a producer warp streams whole rows of packed codes (and LUTs) into a
-//     ring of up to 8 shared-memory stages with cp.async.bulk, completing on
-//     mbarriers; the small uniform scales and zero-points are copied by its
-//     lanes.  Weight copies are issued before the programmatic-dependent-launch
-//     wait, so they overlap the tail of the previous kernel;
-//   * sixteen consumer warps decode 32-weight units out of shared memory with
-//     the magic-number / byte-permute primitives and multiply them with x,
-//     which is staged once per CTA in a padded (bank-conflict-free) layout and
-//     reused across a group of rows held in registers;
-//   * per 32-weight unit the products form two half2 FMA chains of 8, promoted
-//     to fp32; a warp-shuffle reduction per row group feeds fp32 shared-memory
-//     row accumulators, and the producer writes finished rows to y.
-// The uniform scale is folded out of the inner loop (a unit contributes
-// s * sum (q - z) x); the LUT family contributes sum LUT[q] x.  Every wait is
-// bounded in time and reports QX_ERR_TIMEOUT through the device status word.
+//   * Work unit: a 32-row block of one matrix.  Lane r of every warp owns row
+//     r of the block, so a row's dot product never needs a warp shuffle and
+//     the activations x are the same for all lanes (a broadcast load).
+//   * The rows are streamed in slices of 1024 weights: one stage of the
+//     shared-memory ring holds the codes (and LUTs) of 32 rows x 1024 k,
+//     fetched with 2-D/3-D TMA tensor copies in the 128-byte swizzled layout,
+//     which makes the per-lane 16-byte reads of 32 different rows free of bank
+//     conflicts.  Each of the eight warps decodes 128 k (one 3-bit superblock)
+//     of every stage.
+//   * No producer warp: the first stages are issued by thread 0 before the
+//     programmatic-dependent-launch wait (weights do not depend on the previous
+//     kernel), and afterwards the last warp to finish a stage refills it.
+//   * Partial sums of a row block stay in registers across its slices; at the
+//     end of the block each warp stores its partials and the last of the eight
+//     adds them in a fixed order (deterministic) and writes y.
+//   * Uniform scales and zero-points are read by each lane from global memory
+//     one stage ahead, after the refilling thread has pulled the block's
+//     metadata into L2 with a bulk prefetch.
+// One CTA of 256 threads per SM leaves room for a CTA of the next decode
+// kernel, which then streams its weights while this one finishes.  Every wait
+// is bounded in time and reports QX_ERR_TIMEOUT through the device status.
 #include "qx_kernels.cuh"
 
 namespace qx {
 
 namespace {
 
-constexpr int kMaxStages = 8;
-constexpr int kMaxRB = 16;
-constexpr int kSmemBudget = 210 * 1024;
-constexpr int kStageTarget = 24 * 1024;
-constexpr int kHeader = 2048;  // barriers, flags, stage descriptors, matrix table
-constexpr int kAccBytes = kMaxStages * kMaxRB * 4 * 4;
+constexpr int kGroups = 4;       // warp groups; group g takes the stages q with q % kGroups == g
+constexpr int kGroupWarps = 4;   // warps per group, one 256-weight part of a stage each
+constexpr int kWarps = kGroups * kGroupWarps;
+constexpr int kThreads = 32 * kWarps;
+constexpr int kRows = 32;           // rows per block (one per lane)
+constexpr int kSliceK = 1024;       // weights per row per stage
+constexpr int kPartK = kSliceK / kGroupWarps;  // weights per warp per stage
+constexpr int kBox = kRows * 128;   // one 32-row x 128-byte TMA box
+constexpr int kMaxRing = 8;
+// Stages issued at start.  Requesting the whole ring at once would make every
+// stage arrive late (the memory system serves them interleaved); the rest of
+// the ring is issued as the first stages land.
+#ifndef QX_GEMV_INITIAL_STAGES
+#define QX_GEMV_INITIAL_STAGES 8
+#endif
+constexpr int kInitialStages = QX_GEMV_INITIAL_STAGES;
+constexpr int kMaxRbSlots = 16;
+constexpr int kHeader = 1024;       // barriers, counters, per-matrix CTA plan
+constexpr int kSmemBudget = 200 * 1024;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
 }
 
-__device__ __forceinline__ void mbar_init(uint64_t *b, uint32_t count) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_u32(b)), "r"(count) : "memory");
+__device__ __forceinline__ void mbar_init(uint32_t b, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(b), "r"(count) : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive(uint64_t *b) {
-    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_u32(b)) : "memory");
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t b, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b), "r"(bytes) : "memory");
 }
 
-__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t *b, uint32_t bytes) {
-    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_u32(b)), "r"(bytes)
-                 : "memory");
-}
-
-__device__ __forceinline__ bool mbar_try_wait(uint64_t *b, uint32_t parity) {
+__device__ __forceinline__ bool mbar_try_wait(uint32_t b, uint32_t parity) {
     uint32_t ok;
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
         "selp.u32 %0, 1, 0, p;\n\t}"
         : "=r"(ok)
-        : "r"(smem_u32(b)), "r"(parity)
-        : "memory");
-    return ok != 0;
-}
-
-// try_wait with a suspend-time hint: a thread whose phase is not complete
-// sleeps in hardware (up to the hint) instead of spinning on issue slots.
-__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *b, uint32_t parity) {
-    uint32_t ok;
-    asm volatile(
-        "{\n\t.reg .pred p;\n\t"
-        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
-        "selp.u32 %0, 1, 0, p;\n\t}"
-        : "=r"(ok)
-        : "r"(smem_u32(b)), "r"(parity), "r"(100000u)
+        : "r"(b), "r"(parity)
         : "memory");
     return ok != 0;
 }
 
 // Bounded wait: false after `limit_ns`, or once another warp has raised the
 // abort flag (when `abort_flag` is not null).
-__device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, uint64_t limit_ns,
+__device__ __noinline__ bool mbar_wait(uint32_t b, uint32_t parity, uint64_t limit_ns,
                                        volatile uint32_t *abort_flag) {
     if (mbar_try_wait(b, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
-        if (mbar_try_wait_sleep(b, parity)) return true;
+        if (mbar_try_wait(b, parity)) return true;
         if (abort_flag != nullptr && *abort_flag) return false;
         if (globaltimer_ns() - t0 > limit_ns) return false;
     }
 }
 
-__device__ __forceinline__ void bulk_g2s(void *dst, const void *src, uint32_t bytes, uint64_t *bar) {
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
-                     smem_u32(dst)),
-                 "l"(src), "r"(bytes), "r"(smem_u32(bar))
-                 : "memory");
+// Bounded wait for a shared-memory word to reach `want`.
+__device__ __noinline__ bool wait_equal(uint32_t *p, uint32_t want, uint64_t limit_ns,
+                                        volatile uint32_t *abort_flag) {
+    volatile uint32_t *v = p;
+    if (*v == want) return true;
+    const uint64_t t0 = globaltimer_ns();
+    for (;;) {
+        if (*v == want) {
+            __threadfence_block();
+            return true;
+        }
+        if (*abort_flag) return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
+    }
+}
+
+__device__ __forceinline__ void tma_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::
+            "r"(dst),
+        "l"(map), "r"(bar), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_3d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y, int z) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], "
+        "[%2];" ::"r"(dst),
+        "l"(map), "r"(bar), "r"(x), "r"(y), "r"(z)
+        : "memory");
+}
+
+__device__ __forceinline__ void prefetch_l2_bulk(const void *p, uint32_t bytes) {
+    asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(p), "r"(bytes) : "memory");
 }
 
 // Shared-memory loads with 32-bit shared-window addresses.  The ring's
 // contents change between barrier phases, so these are volatile: they are
 // neither merged nor moved across the (volatile) barrier waits.
-__device__ __forceinline__ uint32_t lds32(uint32_t a) {
-    uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
-    return v;
-}
-__device__ __forceinline__ uint32_t lds8(uint32_t a) {
-    uint32_t v;
-    asm volatile("ld.shared.u8 %0, [%1];" : "=r"(v) : "r"(a));
-    return v;
-}
-__device__ __forceinline__ uint32_t lds16(uint32_t a) {
-    uint16_t v;
-    asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(a));
-    return v;
-}
 __device__ __forceinline__ uint4 lds128(uint32_t a) {
     uint4 v;
     asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
-    return v;
-}
-
-template <int CW>
-__device__ __forceinline__ void consumer_bar() {
-    asm volatile("bar.sync 1, %0;" ::"n"(32 * CW) : "memory");
-}
-
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
     return v;
 }
 
@@ -148,375 +148,497 @@ __device__ __forceinline__ float dot16(const __half2 (&w)[16], const __half2 (&x
     return (f0.x + f0.y) + (f1.x + f1.y);
 }
 
-// x is kept in shared memory with every 32-value unit padded to 80 bytes, so
-// that lanes reading consecutive units hit distinct banks.
-__device__ __forceinline__ int64_t xpad(int64_t k) { return (k >> 5) * 40 + (k & 31); }
-
-__device__ __forceinline__ void load_x16(uint32_t unit, __half2 (&x)[16]) {
+// 32 activations x[k .. k+31] from shared memory (the same address in every
+// lane: a broadcast).
+__device__ __forceinline__ void load_x32(uint32_t p, __half2 (&x)[16]) {
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-        const uint4 t = lds128(unit + 16 * q);
-        x[4 * q + 0] = u2h2(t.x);
-        x[4 * q + 1] = u2h2(t.y);
-        x[4 * q + 2] = u2h2(t.z);
-        x[4 * q + 3] = u2h2(t.w);
+    for (int i = 0; i < 4; ++i) {
+        const uint4 t = lds128(p + 16u * i);
+        x[4 * i + 0] = u2h2(t.x);
+        x[4 * i + 1] = u2h2(t.y);
+        x[4 * i + 2] = u2h2(t.z);
+        x[4 * i + 3] = u2h2(t.w);
     }
 }
 
-// Per-matrix fields and this CTA's row range, copied once from the (large)
-// parameter block into shared memory: the loops then never index the
-// parameter space with a runtime matrix number.
-struct MatS {
-    const uint8_t *codes;
-    const __half *scales;
-    const uint8_t *zeros;
-    const __half *luts;
-    const __half *x;
-    void *y;
-    int64_t n, first, end;
-    int k, CB, LB, SB, RB, G, zbytes, log2g;
-};
-
-struct StageDesc {
-    int mat;
-    int rb;
-    int64_t row0;
-};
-
-// Rows [first, end) of matrix `m` owned by this CTA (slices precomputed on
-// the host, so the kernel does no 64-bit division).
-__device__ __forceinline__ void cta_rows(const GemvMulti &a, int m, int64_t &first, int64_t &end) {
-    const int64_t lo = a.cta_row[blockIdx.x], hi = a.cta_row[blockIdx.x + 1];
-    const int64_t o = a.row_off[m], n = a.mat[m].n;
-    const int64_t f = lo - o, e = hi - o;
-    first = f < 0 ? 0 : (f > n ? n : f);
-    end = e < 0 ? 0 : (e > n ? n : e);
+// Offset of 16-byte chunk `c` of 128-byte box row `r` inside a 1024-byte-aligned
+// TMA box written with CU_TENSOR_MAP_SWIZZLE_128B (chunk index XOR row % 8).
+__device__ __forceinline__ uint32_t swz(int r, int c) {
+    return (uint32_t)(r * 128 + (((c ^ r) & 7) << 4));
 }
 
-// 12 consumer warps + 1 producer: registers are reserved per four warps, so
-// 13 warps cost 16 warp slots and leave 128 registers per thread.
-constexpr int kConsumerWarps = 12;
-constexpr int kGroupWarps = 4;  // consumer warps that share one stage
-constexpr int kThreads = 32 * (1 + kConsumerWarps);
+// Per-matrix fields of this CTA, built once in shared memory.
+struct MatS {
+    const uint8_t *zeros;
+    const __half *scales;
+    const __half *x;
+    void *y;
+    int n, K, G, zbytes, log2g, nks, nlb;
+    int xoff;   // shared-memory offset (halves) of this matrix's x
+    int q0;     // first CTA-local stage of this matrix
+    int rb0;    // first matrix-local row block of this CTA
+    int nrb;    // row blocks of this CTA in this matrix
+};
+
+struct Header {
+    uint64_t full[kMaxRing];
+    uint32_t rel[kMaxRing];        // warps done with the stage's current fill
+    uint32_t cnt[kMaxRbSlots];     // warps that stored their partials of a block
+    uint32_t gen[kMaxRbSlots];     // blocks finished in each partial-sum slot
+    uint32_t abort_flag;
+    uint32_t issued;               // stages issued so far
+    int nstages;
+    MatS mats[kMaxGemvMats];
+    int q_end[kMaxGemvMats];       // q0 of the next matrix (nstages for the last)
+};
+static_assert(sizeof(Header) <= kHeader, "header does not fit");
+
+// Matrices i and j of the launch read the same activations.
+__device__ __forceinline__ bool same_x(const Header &h, int i, int j) {
+    return h.mats[i].x == h.mats[j].x && h.mats[i].K == h.mats[j].K;
+}
+
+// Matrix i is the first matrix of this CTA with its activations: it owns
+// their shared-memory copy.
+__device__ __forceinline__ bool x_owner(const Header &h, int i) {
+    if (h.mats[i].nrb == 0) return false;
+    for (int j = 0; j < i; ++j)
+        if (h.mats[j].nrb > 0 && same_x(h, i, j)) return false;
+    return true;
+}
+
+// Stage q of this CTA: matrix, matrix-local row block, slice.
+__device__ __forceinline__ void stage_coords(const Header &h, int count, int q, int &m, int &rb, int &ks) {
+    m = 0;
+    while (m + 1 < count && q >= h.q_end[m]) ++m;
+    const int local = q - h.mats[m].q0;
+    const int nks = h.mats[m].nks;
+    const int rbl = local / nks;
+    rb = h.mats[m].rb0 + rbl;
+    ks = local - rbl * nks;
+}
+
+// Issue the TMA copies of stage q into its ring slot (one thread).
+template <int BITS, int KIND>
+__device__ void issue_stage(const GemvMulti &a, Header &h, uint32_t ring_s, int q) {
+    int m, rb, ks;
+    stage_coords(h, a.count, q, m, rb, ks);
+    const MatS &M = h.mats[m];
+    const int ring = a.ring;
+    const int slot = q % ring;
+    const uint32_t bar = smem_u32(&h.full[slot]);
+    const uint32_t base = ring_s + (uint32_t)(slot * a.stage_bytes);
+    const int row0 = rb * kRows;
+    uint32_t tx = 0;
+    int ncb = 0;
+    if (BITS == 3) {
+        tx += 3 * kBox;
+    } else {
+        const int rowb = M.K / 2;
+        for (int j = 0; j < 4; ++j)
+            if (ks * 512 + 128 * j < rowb) ++ncb;
+        tx += ncb * kBox;
+    }
+    int nlb = 0;
+    if (KIND == 1) {
+        const int gps = kSliceK >> M.log2g;  // groups per slice
+        for (int b = 0; b < M.nlb; ++b)
+            if (ks * gps + 8 * b < M.G) ++nlb;
+        tx += nlb * kBox;
+    }
+    mbar_arrive_expect_tx(bar, tx);
+    const CUtensorMap *tc = &a.tm_codes[m];
+    if (BITS == 3) {
+        tma_3d(base, tc, bar, ks * 128, 0, row0);
+    } else {
+        for (int j = 0; j < ncb; ++j) tma_2d(base + j * kBox, tc, bar, ks * 512 + 128 * j, row0);
+    }
+    if (KIND == 1) {
+        const CUtensorMap *tl = &a.tm_luts[m];
+        const int gps = kSliceK >> M.log2g;
+        const uint32_t lbase = base + 3 * kBox;
+        for (int b = 0; b < nlb; ++b) tma_2d(lbase + b * kBox, tl, bar, (ks * gps + 8 * b) * 16, row0);
+    } else if (ks == 0) {
+        // pull this block's scales and zero-points into L2; the lanes read
+        // them from there a stage ahead of use
+        const int rows = min(kRows, M.n - row0);
+        const uint32_t sb = (uint32_t)(rows * M.G * 2) & ~15u;
+        const uint32_t zb = (uint32_t)(rows * M.zbytes) & ~15u;
+        if (sb) prefetch_l2_bulk(M.scales + (int64_t)row0 * M.G, sb);
+        if (zb) prefetch_l2_bulk(M.zeros + (int64_t)row0 * M.zbytes, zb);
+    }
+}
+
+// Scales and zero-points of one lane's 256-weight part: up to eight fp16
+// scales and eight 4-bit zero-points (group order, lowest first).
+struct Meta {
+    uint32_t s0, s1, s2, s3;  // scales 0-1, 2-3, 4-5, 6-7
+    uint32_t z;
+};
+
+__device__ __forceinline__ Meta load_meta(const MatS &M, int row, int k0) {
+    Meta t{0u, 0u, 0u, 0u, 0u};
+    if (row >= M.n || k0 >= M.K) return t;
+    const int g0 = k0 >> M.log2g;
+    // groups in the part, within the row (a part may run past k: then only
+    // its first half is valid)
+    const int ng = min(M.log2g >= 8 ? 1 : kPartK >> M.log2g, M.G - g0);
+    const unsigned short *sp = reinterpret_cast<const unsigned short *>(M.scales) + (int64_t)row * M.G + g0;
+    const uint8_t *zp = M.zeros + (int64_t)row * M.zbytes;
+    uint32_t s[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        if (j < ng) {
+            s[j >> 1] |= (uint32_t)sp[j] << ((j & 1) * 16);
+            t.z |= (((uint32_t)zp[(g0 + j) >> 1] >> (((g0 + j) & 1) * 4)) & 15u) << (4 * j);
+        }
+    }
+    t.s0 = s[0];
+    t.s1 = s[1];
+    t.s2 = s[2];
+    t.s3 = s[3];
+    return t;
+}
+
+__device__ __forceinline__ float meta_scale(const Meta &t, int gl) {
+    uint32_t w = t.s0;
+    if (gl >= 2) w = t.s1;
+    if (gl >= 4) w = t.s2;
+    if (gl >= 6) w = t.s3;
+    return __half2float(__ushort_as_half((unsigned short)(w >> ((gl & 1) * 16))));
+}
+
+__device__ __forceinline__ uint32_t meta_zero(const Meta &t, int gl) { return (t.z >> (4 * gl)) & 15u; }
+
+// Stage cursor: matrix, row block (CTA-local), slice.
+struct Cursor {
+    int m, rbl, ks;
+};
+
+__device__ __forceinline__ void advance(const Header &h, int count, Cursor &c) {
+    if (++c.ks == h.mats[c.m].nks) {
+        c.ks = 0;
+        if (++c.rbl == h.mats[c.m].nrb) {
+            c.rbl = 0;
+            ++c.m;
+            while (c.m < count && h.mats[c.m].nrb == 0) ++c.m;
+        }
+    }
+}
 
 template <int BITS, int KIND, int BMAX>
 __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant__ GemvMulti a) {
-    constexpr int NG = kConsumerWarps / kGroupWarps;  // consumer groups
-    constexpr int RMAX = 8 / BMAX;                    // rows accumulated per pass
-    extern __shared__ __align__(128) uint8_t smem[];
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem);
-    uint64_t *empty = full + kMaxStages;
-    volatile uint32_t *abort_flag = reinterpret_cast<volatile uint32_t *>(empty + kMaxStages);
-    StageDesc *desc = reinterpret_cast<StageDesc *>(smem + 256);
-    MatS *mats = reinterpret_cast<MatS *>(smem + 512);
-    float *acc = reinterpret_cast<float *>(smem + kHeader);
-    __half *xs = reinterpret_cast<__half *>(smem + kHeader + kAccBytes);
-    uint8_t *stages = smem + kHeader + kAccBytes + a.x_smem_bytes;
+    extern __shared__ uint8_t smem_raw[];
+    // 1024-byte alignment for the swizzled TMA boxes
+    const uint32_t raw_s = smem_u32(smem_raw);
+    const uint32_t base_s = (raw_s + 1023u) & ~1023u;
+    uint8_t *base = smem_raw + (base_s - raw_s);
+    Header &h = *reinterpret_cast<Header *>(base);
+    float *red = reinterpret_cast<float *>(base + kHeader);
+    __half *xs = reinterpret_cast<__half *>(base + kHeader + a.red_bytes);
+    const uint32_t xs_s = base_s + (uint32_t)(kHeader + a.red_bytes);
+    const uint32_t ring_s = base_s + (uint32_t)(kHeader + a.red_bytes + a.x_smem_bytes);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int nb = a.batch;
-    const int count = a.count, nring = a.stages, stage_bytes = a.stage_bytes;
+    const int count = a.count, ring = a.ring, nb = a.batch;
 
-    if (threadIdx.x == 0) {
-        for (int i = 0; i < nring; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], kGroupWarps);
-        }
-        *abort_flag = 0;
+    // ---- set-up, spread over threads so that the first copies start early
+    if (threadIdx.x < count) {  // this CTA's row blocks of matrix t
+        const int t = threadIdx.x;
+        const int lo = a.cta_rb[blockIdx.x], hi = a.cta_rb[blockIdx.x + 1];
+        const GemvMat &G = a.mat[t];
+        MatS &S = h.mats[t];
+        const int f = max(lo, G.rb_off), e = min(hi, G.rb_off + G.nrb);
+        S.zeros = G.zeros;
+        S.scales = G.scales;
+        S.x = G.x;
+        S.y = G.y;
+        S.n = (int)G.n;
+        S.K = (int)G.k;
+        S.G = G.G;
+        S.zbytes = G.zbytes;
+        S.log2g = G.log2g;
+        S.nks = G.nks;
+        S.nlb = G.nlb;
+        S.rb0 = f - G.rb_off;
+        S.nrb = e > f ? e - f : 0;
+    } else if (threadIdx.x >= 32 && threadIdx.x < 32 + count) {
+        const int t = threadIdx.x - 32;
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_codes[t]) : "memory");
+        if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_luts[t]) : "memory");
+    } else if (threadIdx.x == 64) {
+        for (int i = 0; i < ring; ++i) mbar_init(smem_u32(&h.full[i]), 1);
+        h.abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
-    if (threadIdx.x < count) {  // per-matrix fields -> shared memory, once
-        const int m = threadIdx.x;
-        const GemvMat &M = a.mat[m];
-        MatS &S = mats[m];
-        S.codes = M.codes;
-        S.scales = M.scales;
-        S.zeros = M.zeros;
-        S.luts = M.luts;
-        S.x = M.x;
-        S.y = M.y;
-        S.n = M.n;
-        cta_rows(a, m, S.first, S.end);
-        S.k = (int)M.k;
-        S.CB = M.CB;
-        S.LB = M.LB;
-        S.SB = M.SB;
-        S.RB = M.RB;
-        S.G = M.G;
-        S.zbytes = M.zbytes;
-        S.log2g = M.log2g;
+    if (threadIdx.x >= 96 && threadIdx.x < 96 + kMaxRing) h.rel[threadIdx.x - 96] = 0;
+    if (threadIdx.x >= 128 && threadIdx.x < 128 + kMaxRbSlots) {
+        h.cnt[threadIdx.x - 128] = 0;
+        h.gen[threadIdx.x - 128] = 0;
     }
-    for (int i = threadIdx.x; i < kMaxStages * kMaxRB * BMAX; i += blockDim.x) acc[i] = 0.0f;
     __syncthreads();
-    // let the next kernel in the stream begin its own weight prefetch early;
-    // it still waits for this grid's completion before touching activations
+    if (warp == 0) {
+        // stage numbering per matrix, then one lane per initial stage
+        int q = 0, mine = 0, qend = 0;
+        for (int m = 0; m < count; ++m) {
+            if (m == lane) mine = q;
+            q += h.mats[m].nrb * h.mats[m].nks;
+            if (m == lane) qend = q;
+        }
+        if (lane < count) {
+            h.mats[lane].q0 = mine;
+            h.q_end[lane] = qend;
+            // activations in shared memory: one copy per distinct x of this CTA
+            int off = 0, xo = -1;
+            for (int m = 0; m < lane; ++m) {
+                if (!x_owner(h, m)) continue;
+                if (xo < 0 && same_x(h, m, lane)) xo = off;
+                off += nb * h.mats[m].K;
+            }
+            h.mats[lane].xoff = xo >= 0 ? xo : off;
+        }
+        if (lane == 0) {
+            h.nstages = q;
+            h.issued = (uint32_t)min(min(ring, kInitialStages), q);
+        }
+        __syncwarp();
+        if (lane < min(min(ring, kInitialStages), q)) issue_stage<BITS, KIND>(a, h, ring_s, lane);
+    }
+    __syncthreads();
+    // let the next kernel in the stream start streaming its own weights; it
+    // still waits for this grid's completion before it reads activations
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    if (warp == 0) {
-        // ------------------------------------------------------------ producer
-        int sq = 0, st = 0;
-        uint32_t ph = 0;
-        bool ok = true;
-        bool waited_dep = false;
-        for (int m = 0; m < count && ok; ++m) {
-            const MatS &M = mats[m];
-            const int64_t first = M.first, end = M.end;
-            const int RB = M.RB, CB = M.CB, LB = M.LB, G = M.G;
-            const uint8_t *codes = M.codes;
-            const __half *luts = M.luts;
-            for (int64_t r0 = first; r0 < end && ok; r0 += RB) {
-                bool got = true;
-                if (lane == 0 && sq >= nring) got = mbar_wait(&empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag);
-                if (!__shfl_sync(0xffffffffu, got, 0)) {
-                    ok = false;
-                    break;
-                }
-                if (sq >= nring) {  // retire the rows that last used this stage
-                    if (!waited_dep) {
-                        asm volatile("griddepcontrol.wait;" ::: "memory");
-                        waited_dep = true;
-                    }
-                    const StageDesc d = desc[st];
-                    __syncwarp();  // every lane holds d before lane 0 overwrites desc[st] below
-                    const MatS &P = mats[d.mat];
-                    float *pacc = acc + st * kMaxRB * BMAX;
-                    for (int i = lane; i < d.rb * nb; i += 32) {
-                        const int r = i / nb, b = i - r * nb;
-                        const float v = pacc[r * BMAX + b];
-                        pacc[r * BMAX + b] = 0.0f;
-                        if (a.y_f32)
-                            reinterpret_cast<float *>(P.y)[(int64_t)b * P.n + d.row0 + r] = v;
-                        else
-                            reinterpret_cast<__half *>(P.y)[(int64_t)b * P.n + d.row0 + r] = __float2half_rn(v);
-                    }
-                }
-                const int rb = (int)((end - r0) < RB ? (end - r0) : RB);
-                uint8_t *sbase = stages + st * stage_bytes;
-                if (KIND == 0) {  // scales and zero-points: lane copies (rows not 16-byte aligned)
-                    __half *ss = reinterpret_cast<__half *>(sbase + RB * CB);
-                    uint8_t *sz = sbase + RB * CB + RB * M.SB;
-                    const __half *gs = M.scales + r0 * G;
-                    const uint8_t *gz = M.zeros + r0 * M.zbytes;
-                    for (int i = lane; i < rb * G; i += 32) ss[i] = gs[i];
-                    for (int i = lane; i < rb * M.zbytes; i += 32) sz[i] = gz[i];
-                }
-                if (lane == 0) {
-                    desc[st].mat = m;
-                    desc[st].rb = rb;
-                    desc[st].row0 = r0;
-                }
-                __syncwarp();
-                if (lane == 0) {
-                    const uint32_t cbytes = (uint32_t)(rb * CB);
-                    const uint32_t lbytes = (uint32_t)(rb * LB);
-                    mbar_arrive_expect_tx(&full[st], cbytes + lbytes);
-                    bulk_g2s(sbase, codes + r0 * CB, cbytes, &full[st]);
-                    if (KIND == 1) bulk_g2s(sbase + RB * CB, luts + r0 * G * 8, lbytes, &full[st]);
-                }
-                ++sq;
-                if (++st == nring) {
-                    st = 0;
-                    ph ^= 1u;
-                }
-            }
-        }
-        if (!waited_dep) asm volatile("griddepcontrol.wait;" ::: "memory");
-        // retire the last stages (after an abort: let in-flight copies land)
-        for (int q = (sq - nring > 0 ? sq - nring : 0); q < sq; ++q) {
-            const int qs = q % nring;
-            const uint32_t qp = (uint32_t)(q / nring) & 1u;
-            bool got = ok;
-            if (lane == 0 && ok) got = mbar_wait(&empty[qs], qp, a.wait_limit_ns, abort_flag);
-            got = __shfl_sync(0xffffffffu, got, 0);
-            if (!got) {
-                ok = false;
-                if (lane == 0) mbar_wait(&full[qs], qp, a.wait_limit_ns, nullptr);
-                __syncwarp();
-                continue;
-            }
-            const StageDesc d = desc[qs];
-            __syncwarp();
-            const MatS &P = mats[d.mat];
-            const float *pacc = acc + qs * kMaxRB * BMAX;
-            for (int i = lane; i < d.rb * nb; i += 32) {
-                const int r = i / nb, b = i - r * nb;
-                const float v = pacc[r * BMAX + b];
-                if (a.y_f32)
-                    reinterpret_cast<float *>(P.y)[(int64_t)b * P.n + d.row0 + r] = v;
-                else
-                    reinterpret_cast<__half *>(P.y)[(int64_t)b * P.n + d.row0 + r] = __float2half_rn(v);
-            }
-        }
-        if (!ok && lane == 0) {
-            *abort_flag = 1u;
-            atomicOr(a.status, kStatusTimeout);
-        }
-    } else {
-        // ------------------------------------------------------------ consumers
-        const int cw = warp - 1;
-        const int grp_id = cw / kGroupWarps;  // stages sq with sq % NG == grp_id
-        const int j = cw % kGroupWarps;       // warp within the group
-        const int ct = threadIdx.x - 32;
-        asm volatile("griddepcontrol.wait;" ::: "memory");
-        {   // stage the x of every matrix this CTA touches, padded
-            int xoff = 0;
-            for (int m = 0; m < count; ++m) {
-                const MatS &M = mats[m];
-                if (M.first >= M.end) continue;
-                const int K = M.k;
-                const int vecs = nb * K / 8;
-                const __half *xg = M.x;
-                for (int i = ct; i < vecs; i += 32 * kConsumerWarps) {
-                    const int e = 8 * i, b = e / K, kk = e - b * K;
-                    *reinterpret_cast<uint4 *>(xs + xoff + b * (K / 32) * 40 + xpad(kk)) =
-                        *reinterpret_cast<const uint4 *>(xg + e);
-                }
-                xoff += nb * (K / 32) * 40;
-            }
-        }
-        consumer_bar<kConsumerWarps>();
-        bool ok = true;
-        int sq = 0, st = 0;
-        uint32_t ph = 0;
-        uint32_t xm = smem_u32(xs);  // shared address of this matrix's padded x
-        const uint32_t stages_s = smem_u32(stages);
-        for (int m = 0; m < count && ok; ++m) {
-            const MatS &M = mats[m];
-            const int64_t first = M.first, end = M.end;
-            if (first >= end) continue;
-            // per-matrix constants in 32-bit registers (k <= 32768, a stage < 64 KB)
-            const int K = M.k;
-            const int CB = M.CB, RB = M.RB, G = M.G;
-            const int SBb = M.SB, ZBb = M.zbytes, log2g = M.log2g;
-            const int U = K >> 5;      // 32-weight units per row
-            const int plane = K >> 3;  // bytes per 3-bit plane
-            const int nuc = (U + 31) >> 5;  // unit-chunks (32 units, one per lane) per row
-            const uint32_t xstride = (uint32_t)U * 80u;  // bytes per batch row of padded x
-            // split of a stage among the group's warps: unit-chunks when there
-            // are enough of them, otherwise unit-chunks x interleaved rows
-            int uc0, ucstep, rfirst, rmask;
-            bool idle = false;
-            if (nuc >= kGroupWarps) {
-                uc0 = j;
-                ucstep = kGroupWarps;
-                rfirst = 0;
-                rmask = 0;
-            } else {
-                const int rsplit = nuc == 1 ? 4 : (nuc == 2 ? 2 : 1);
-                uc0 = j % nuc;
-                ucstep = nuc;
-                rfirst = j / nuc;
-                rmask = rsplit - 1;
-                idle = j >= nuc * rsplit;
-            }
-            for (int64_t r0 = first; r0 < end && ok; r0 += RB) {
-                const int mysq = sq;
-                const int myst = st;
-                const uint32_t myph = ph;
-                ++sq;
-                if (++st == nring) {
-                    st = 0;
-                    ph ^= 1u;
-                }
-                if (mysq % NG != grp_id) continue;  // another group's stage
-                ok = mbar_wait(&full[myst], myph, a.wait_limit_ns, abort_flag);
-                if (!__all_sync(0xffffffffu, ok)) {
-                    ok = false;
-                    break;
-                }
-                const int rb = (int)((end - r0) < RB ? (end - r0) : RB);
-                const uint32_t sb = stages_s + (uint32_t)(myst * stage_bytes);
-                const uint32_t meta = sb + (uint32_t)(RB * CB);
-                float *sacc = acc + myst * (kMaxRB * BMAX);
-                if (!idle) {
-                    for (int rp = 0; rp < rb; rp += RMAX) {
-                        float p[RMAX][BMAX];
-#pragma unroll
-                        for (int r = 0; r < RMAX; ++r)
-#pragma unroll
-                            for (int b = 0; b < BMAX; ++b) p[r][b] = 0.0f;
-                        for (int uc = uc0; uc < nuc; uc += ucstep) {
-                            const int u = uc * 32 + lane;
-                            if (u >= U) continue;
-                            const int grp = (32 * u) >> log2g;
-                            __half2 xv[BMAX][16];
-#pragma unroll
-                            for (int b = 0; b < BMAX; ++b)
-                                if (b < nb) load_x16(xm + (uint32_t)b * xstride + 80u * (uint32_t)u, xv[b]);
-#pragma unroll
-                            for (int ri = 0; ri < RMAX; ++ri) {
-                                const int rl = rp + ri;
-                                if (rl < rb && (rl & rmask) == rfirst) {
-                                    const uint32_t rc = sb + (uint32_t)(rl * CB);
-                                    __half2 w[16];
-                                    float s = 1.0f;
-                                    if (BITS == 4) {
-                                        const uint4 cw4 = lds128(rc + 16u * (uint32_t)u);
-                                        s = __half2float(__ushort_as_half((unsigned short)lds16(meta + 2u * (uint32_t)(rl * G + grp))));
-                                        const uint32_t z = (lds8(meta + (uint32_t)(RB * SBb + rl * ZBb + (grp >> 1))) >> ((grp & 1) * 4)) & 15u;
-                                        const __half2 zl = zlo_of(z), zh = zhi_of(z);
-                                        const uint32_t wd[4] = {cw4.x, cw4.y, cw4.z, cw4.w};
-#pragma unroll
-                                        for (int t = 0; t < 4; ++t) {
-                                            __half2 o[4];
-                                            unpack4_qz(wd[t], zl, zh, o);
-#pragma unroll
-                                            for (int q = 0; q < 4; ++q) w[4 * t + q] = o[q];
-                                        }
-                                    } else {
-                                        const uint32_t cp = rc + 4u * (uint32_t)u;  // word u of each plane
-                                        const uint32_t A = lds32(cp);
-                                        const uint32_t B = lds32(cp + (uint32_t)plane);
-                                        const uint32_t C = lds32(cp + 2u * (uint32_t)plane);
-                                        Table8 tab;
-                                        if (KIND == 1) {
-                                            const uint4 l = lds128(meta + 16u * (uint32_t)(rl * G + grp));
-                                            tab = make_table8(l.x, l.y, l.z, l.w);
-                                        } else {
-                                            s = __half2float(__ushort_as_half((unsigned short)lds16(meta + 2u * (uint32_t)(rl * G + grp))));
-                                            tab = table8_offsets((lds8(meta + (uint32_t)(RB * SBb + rl * ZBb + (grp >> 1))) >> ((grp & 1) * 4)) & 15u);
-                                        }
-                                        lookup_triple(tab, A, B, C, w);
-                                    }
-#pragma unroll
-                                    for (int b = 0; b < BMAX; ++b)
-                                        if (b < nb) p[ri][b] += s * dot16(w, xv[b]);
-                                }
-                            }
-                        }
-#pragma unroll
-                        for (int ri = 0; ri < RMAX; ++ri) {
-                            const int rl = rp + ri;
-                            if (rl < rb && (rl & rmask) == rfirst) {
-#pragma unroll
-                                for (int b = 0; b < BMAX; ++b) {
-                                    if (b < nb) {
-                                        const float v = warp_sum(p[ri][b]);
-                                        if (lane == 0) atomicAdd(&sacc[rl * BMAX + b], v);
-                                    }
-                                }
-                            }
-                        }
-                    }
-                }
-                __syncwarp();
-                if (lane == 0) mbar_arrive(&empty[myst]);
-            }
-            xm += (uint32_t)nb * xstride;
-        }
-        if (!ok && lane == 0) {
-            *abort_flag = 1u;
-            atomicOr(a.status, kStatusTimeout);
-        }
+    const int nst = h.nstages;
+    const int r = lane;
+    const int grp = warp / kGroupWarps;   // stages q with q % kGroups == grp
+    const int part = warp % kGroupWarps;  // 128-weight part of each of those stages
+    bool ok = true;
+    int q = 0, slot = 0, rbseq = 0;
+    uint32_t par = 0;
+
+    Cursor c{0, 0, 0};
+    while (c.m < count && h.mats[c.m].nrb == 0) ++c.m;
+    // uniform metadata of this warp's next stage, loaded one stage ahead
+    Meta cur{}, nxt{};
+    Cursor pc = c;
+    for (int i = 0; i < grp && pc.m < count; ++i) advance(h, count, pc);
+    if (KIND == 0 && pc.m < count)
+        cur = load_meta(h.mats[pc.m], (h.mats[pc.m].rb0 + pc.rbl) * kRows + r, pc.ks * kSliceK + part * kPartK);
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    // activations -> shared memory (every lane of a warp then reads the same
+    // address: a broadcast)
+    for (int m = 0; m < count; ++m) {
+        if (!x_owner(h, m)) continue;
+        const int vecs = nb * h.mats[m].K / 8;
+        const uint4 *src = reinterpret_cast<const uint4 *>(h.mats[m].x);
+        uint4 *dst = reinterpret_cast<uint4 *>(xs + h.mats[m].xoff);
+        for (int i = threadIdx.x; i < vecs; i += kThreads) dst[i] = src[i];
     }
     __syncthreads();
+
+    float acc[BMAX];
+#pragma unroll
+    for (int b = 0; b < BMAX; ++b) acc[b] = 0.0f;
+    for (; q < nst && ok; ++q) {
+        const MatS &M = h.mats[c.m];
+        const int K = M.K, log2g = M.log2g;
+        const int k0 = c.ks * kSliceK + part * kPartK;
+        if (q % kGroups == grp) {
+            if (KIND == 0) {  // metadata of this warp's following stage
+                for (int i = 0; i < kGroups && pc.m < count; ++i) advance(h, count, pc);
+                if (pc.m < count) {
+                    const MatS &N = h.mats[pc.m];
+                    nxt = load_meta(N, (N.rb0 + pc.rbl) * kRows + r, pc.ks * kSliceK + part * kPartK);
+                }
+            }
+            ok = mbar_wait(smem_u32(&h.full[slot]), par, a.wait_limit_ns, &h.abort_flag);
+            if (!__all_sync(0xffffffffu, ok)) {
+                ok = false;
+                break;
+            }
+            if (part == 0 && lane == 0 && q + kInitialStages < min(ring, nst)) {
+                // ramp-up: a stage has landed, request one more of the ring
+                issue_stage<BITS, KIND>(a, h, ring_s, q + kInitialStages);
+                atomicMax(&h.issued, (uint32_t)(q + kInitialStages + 1));
+            }
+            if (k0 < K) {
+                const uint32_t sb = ring_s + (uint32_t)(slot * a.stage_bytes);
+                const uint32_t xk = xs_s + 2u * (uint32_t)(M.xoff + k0);
+                if (BITS == 3) {
+                    uint32_t Aw[4], Bw[4], Cw[4];
+                    Table8 tab{};
+                    float s = 1.0f;
+#pragma unroll
+                    for (int i = 0; i < kPartK / 32; ++i) {
+                        if (i == 4 && k0 + 128 >= K) break;  // k is a multiple of 128, not of 256
+                        if ((i & 3) == 0) {
+                            // superblock (128 k): planes 0/1/2 of row r are box rows 3r, 3r+1, 3r+2
+                            const int sbk = part * (kPartK / 128) + (i >> 2);
+                            const uint4 A = lds128(sb + swz(3 * r, sbk));
+                            const uint4 B = lds128(sb + swz(3 * r + 1, sbk));
+                            const uint4 C = lds128(sb + swz(3 * r + 2, sbk));
+                            Aw[0] = A.x; Aw[1] = A.y; Aw[2] = A.z; Aw[3] = A.w;
+                            Bw[0] = B.x; Bw[1] = B.y; Bw[2] = B.z; Bw[3] = B.w;
+                            Cw[0] = C.x; Cw[1] = C.y; Cw[2] = C.z; Cw[3] = C.w;
+                        }
+                        __half2 xv[BMAX][16];
+#pragma unroll
+                        for (int b = 0; b < BMAX; ++b)
+                            if (b < nb) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
+                        // a new table where unit i starts a group
+                        if (i == 0 || ((32 * i) & ((1 << log2g) - 1)) == 0) {
+                            const int gl = (32 * i) >> log2g;
+                            if (KIND == 1) {
+                                const int lg = (part * kPartK + 32 * i) >> log2g;
+                                const uint4 l = lds128(sb + 3 * kBox + (uint32_t)((lg >> 3) * kBox) + swz(r, lg & 7));
+                                tab = make_table8(l.x, l.y, l.z, l.w);
+                            } else {
+                                tab = table8_offsets(meta_zero(cur, gl));
+                                s = meta_scale(cur, gl);
+                            }
+                        }
+                        __half2 w[16];
+                        lookup_triple(tab, Aw[i & 3], Bw[i & 3], Cw[i & 3], w);
+#pragma unroll
+                        for (int b = 0; b < BMAX; ++b) {
+                            if (b < nb) {
+                                if (KIND == 1)
+                                    acc[b] += dot16(w, xv[b]);
+                                else
+                                    acc[b] += s * dot16(w, xv[b]);
+                            }
+                        }
+                    }
+                } else {
+                    // 4-bit: box `part` holds this part's 256 k, 16 bytes per 32 k
+                    const uint32_t cb = sb + (uint32_t)(part * kBox);
+                    float s = 1.0f;
+                    __half2 zl{}, zh{};
+#pragma unroll
+                    for (int i = 0; i < kPartK / 32; ++i) {
+                        if (i == 4 && k0 + 128 >= K) break;  // k is a multiple of 128, not of 256
+                        __half2 xv[BMAX][16];
+#pragma unroll
+                        for (int b = 0; b < BMAX; ++b)
+                            if (b < nb) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
+                        if (i == 0 || ((32 * i) & ((1 << log2g) - 1)) == 0) {
+                            const int gl = (32 * i) >> log2g;
+                            const uint32_t z = meta_zero(cur, gl);
+                            zl = zlo_of(z);
+                            zh = zhi_of(z);
+                            s = meta_scale(cur, gl);
+                        }
+                        const uint4 cw = lds128(cb + swz(r, i));
+                        const uint32_t wd[4] = {cw.x, cw.y, cw.z, cw.w};
+                        __half2 w[16];
+#pragma unroll
+                        for (int t = 0; t < 4; ++t) {
+                            __half2 o[4];
+                            unpack4_qz(wd[t], zl, zh, o);
+#pragma unroll
+                            for (int u = 0; u < 4; ++u) w[4 * t + u] = o[u];
+                        }
+#pragma unroll
+                        for (int b = 0; b < BMAX; ++b)
+                            if (b < nb) acc[b] += s * dot16(w, xv[b]);
+                    }
+                }
+            }
+            // release the stage; the last warp of the group refills it
+            __syncwarp();
+            if (lane == 0) {
+                __threadfence_block();
+                const uint32_t old = atomicAdd(&h.rel[slot], 1u);
+                if (old == kGroupWarps - 1) {
+                    h.rel[slot] = 0;
+                    __threadfence_block();
+                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                    if (q + ring < nst && !*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) {
+                        issue_stage<BITS, KIND>(a, h, ring_s, q + ring);
+                        atomicMax(&h.issued, (uint32_t)(q + ring + 1));
+                    }
+                }
+            }
+            if (KIND == 0) cur = nxt;
+        }
+        if (++slot == ring) {
+            slot = 0;
+            par ^= 1u;
+        }
+        if (c.ks + 1 == M.nks) {
+            // end of a row block: partials -> shared memory; the last of all
+            // warps sums them in a fixed order and writes y
+            const int rs = rbseq % a.rb_slots;
+            const uint32_t use = (uint32_t)(rbseq / a.rb_slots);
+            ++rbseq;
+            // the warp groups run independently: the slot's previous block
+            // must have been summed before this warp overwrites its partials
+            if (lane == 0) ok = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
+            if (!__shfl_sync(0xffffffffu, ok, 0)) {
+                ok = false;
+                break;
+            }
+            float *rp = red + (size_t)rs * (kWarps * BMAX * 32);
+#pragma unroll
+            for (int b = 0; b < BMAX; ++b) {
+                rp[(warp * BMAX + b) * 32 + r] = acc[b];
+                acc[b] = 0.0f;
+            }
+            __syncwarp();
+            uint32_t fin = 0;
+            if (lane == 0) {
+                __threadfence_block();
+                fin = atomicAdd(&h.cnt[rs], 1u) == kWarps - 1;
+                __threadfence_block();
+            }
+            fin = __shfl_sync(0xffffffffu, fin, 0);
+            if (fin) {
+                const int row = (M.rb0 + c.rbl) * kRows + r;
+                if (row < M.n) {
+#pragma unroll
+                    for (int b = 0; b < BMAX; ++b) {
+                        if (b < nb) {
+                            float v = 0.0f;
+#pragma unroll
+                            for (int w2 = 0; w2 < kWarps; ++w2) v += rp[(w2 * BMAX + b) * 32 + r];
+                            if (a.y_f32)
+                                reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v;
+                            else
+                                reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v);
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) {
+                    h.cnt[rs] = 0;
+                    __threadfence_block();
+                    *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
+                }
+            }
+        }
+        advance(h, count, c);
+    }
+    if (!ok && lane == 0) {
+        h.abort_flag = 1u;
+        atomicOr(a.status, kStatusTimeout);
+    }
+    if (lane == 0 && (!ok || *reinterpret_cast<volatile uint32_t *>(&h.abort_flag))) {
+        // a warp that gives up lets the copies still in flight land before
+        // it exits, so the CTA's shared memory outlives them
+        const int iss = (int)*reinterpret_cast<volatile uint32_t *>(&h.issued);
+        for (int qq = max(0, iss - ring); qq < iss; ++qq)
+            mbar_wait(smem_u32(&h.full[qq % ring]), (uint32_t)(qq / ring) & 1u, a.wait_limit_ns, nullptr);
+    }
 }
 
 template <int BITS, int KIND, int BMAX>
 cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
     auto kern = gemv_kernel<BITS, KIND, BMAX>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
+    if (e != cudaSuccess) return e;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)a.grid);
@@ -531,65 +653,116 @@ cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
     return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
+bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims, const cuuint64_t *strides,
+            const cuuint32_t *box) {
+    EncodeTiledFn enc = encode_fn();
+    if (enc == nullptr) return false;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    return enc(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, (cuuint32_t)rank, const_cast<void *>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+               CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 }  // namespace
 
-// Host-side plan: per-matrix stage geometry, the byte-balanced CTA slices and
-// the shared-memory budget (x of every matrix a CTA touches + the ring).
-// Returns false if the matrices cannot share one launch.
+// Host-side plan: tensor maps, byte-balanced CTA row-block ranges and the
+// shared-memory budget.  Returns false if the matrices cannot share one launch.
 bool plan_gemv(GemvMulti &a, int num_sms) {
-    int max_stage = 0;
-    int64_t total = 0;
+    const int bmax = a.batch <= 1 ? 1 : (a.batch <= 2 ? 2 : 4);
+    int nks_min = 1 << 30, nlb_max = 1;
+    int64_t total = 0, rbs = 0;
     for (int m = 0; m < a.count; ++m) {
         GemvMat &M = a.mat[m];
-        M.CB = (int)(M.k * a.bits / 8);
-        M.LB = a.kind == 1 ? M.G * 16 : 0;
-        M.SB = a.kind == 0 ? ((M.G * 2 + 15) / 16) * 16 : 0;
-        M.ZB = a.kind == 0 ? ((M.zbytes + 15) / 16) * 16 : 0;
-        M.row_bytes = M.CB + M.LB + M.SB + M.ZB;
-        M.RB = std::max(1, std::min(kMaxRB, kStageTarget / M.row_bytes));
-        M.byte_off = total;
-        total += M.n * M.row_bytes;
-        max_stage = std::max(max_stage, M.RB * M.row_bytes);
+        M.nks = (int)((M.k + kSliceK - 1) / kSliceK);
+        M.nlb = a.kind == 1 ? std::max(1, 128 >> M.log2g) : 0;
+        M.nrb = (int)((M.n + kRows - 1) / kRows);
+        M.rb_off = (int)rbs;
+        rbs += M.nrb;
+        nks_min = std::min(nks_min, M.nks);
+        nlb_max = std::max(nlb_max, M.nlb);
+        if (M.n > (int64_t)1 << 30 || rbs > (int64_t)1 << 30) return false;
+        const uint8_t *codes = M.codes;
+        if (a.bits == 3) {
+            // bytes within a plane, plane, row: box = [32 rows][3 planes][128 bytes]
+            const cuuint64_t dims[3] = {(cuuint64_t)(M.k / 8), 3, (cuuint64_t)M.n};
+            const cuuint64_t strides[2] = {(cuuint64_t)(M.k / 8), (cuuint64_t)(M.k * 3 / 8)};
+            const cuuint32_t box[3] = {128, 3, kRows};
+            if (!encode(&a.tm_codes[m], codes, 3, dims, strides, box)) return false;
+        } else {
+            const cuuint64_t dims[2] = {(cuuint64_t)(M.k / 2), (cuuint64_t)M.n};
+            const cuuint64_t strides[1] = {(cuuint64_t)(M.k / 2)};
+            const cuuint32_t box[2] = {128, kRows};
+            if (!encode(&a.tm_codes[m], codes, 2, dims, strides, box)) return false;
+        }
+        if (a.kind == 1) {
+            const cuuint64_t dims[2] = {(cuuint64_t)M.G * 16, (cuuint64_t)M.n};
+            const cuuint64_t strides[1] = {(cuuint64_t)M.G * 16};
+            const cuuint32_t box[2] = {128, kRows};
+            if (!encode(&a.tm_luts[m], M.luts, 2, dims, strides, box)) return false;
+        }
+    }
+    // bytes per row block (balancing only)
+    int64_t rb_bytes[kMaxGemvMats];
+    for (int m = 0; m < a.count; ++m) {
+        const GemvMat &M = a.mat[m];
+        const int64_t row = M.k * a.bits / 8 + (a.kind == 1 ? (int64_t)M.G * 16 : (int64_t)M.G * 2 + M.zbytes);
+        rb_bytes[m] = row * kRows;
+        total += rb_bytes[m] * M.nrb;
     }
     a.total_bytes = total;
-    int64_t rows = 0;
-    for (int m = 0; m < a.count; ++m) {
-        a.row_off[m] = rows;
-        rows += a.mat[m].n;
-    }
-    a.row_off[a.count] = rows;
-    a.grid = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), rows);
-    // CTA c owns the rows whose first byte lies in [c * total / grid, (c+1) * total / grid)
+    a.grid = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), rbs);
+    // CTA c owns the row blocks whose first byte lies in [c T / grid, (c+1) T / grid)
     for (int c = 0; c <= a.grid; ++c) {
         const int64_t b = (int64_t)((__int128)c * total / a.grid);
-        int64_t r = rows;
+        int64_t acc = 0, r = rbs;
         for (int m = 0; m < a.count; ++m) {
             const GemvMat &M = a.mat[m];
-            if (b < M.byte_off + M.n * M.row_bytes) {
-                const int64_t lr = b <= M.byte_off ? 0 : (b - M.byte_off + M.row_bytes - 1) / M.row_bytes;
-                r = a.row_off[m] + std::min(lr, M.n);
+            const int64_t mb = rb_bytes[m] * M.nrb;
+            if (b < acc + mb) {
+                r = M.rb_off + std::min<int64_t>((b - acc + rb_bytes[m] - 1) / rb_bytes[m], M.nrb);
                 break;
             }
+            acc += mb;
         }
-        a.cta_row[c] = r;
+        a.cta_rb[c] = (int32_t)r;
     }
-    // x bytes per CTA: simulate the slices
+    // activations of the matrices a CTA touches (one copy per distinct x)
     int64_t xmax = 0;
     for (int c = 0; c < a.grid; ++c) {
         int64_t xb = 0;
         for (int m = 0; m < a.count; ++m) {
-            const int64_t f = std::max(a.cta_row[c], a.row_off[m]);
-            const int64_t e = std::min(a.cta_row[c + 1], a.row_off[m + 1]);
-            if (f < e) xb += (int64_t)a.batch * (a.mat[m].k / 32) * 80;
+            const GemvMat &M = a.mat[m];
+            if (std::max<int64_t>(a.cta_rb[c], M.rb_off) >= std::min<int64_t>(a.cta_rb[c + 1], M.rb_off + M.nrb))
+                continue;
+            bool dup = false;
+            for (int j = 0; j < m && !dup; ++j) {
+                const GemvMat &P = a.mat[j];
+                const bool touched =
+                    std::max<int64_t>(a.cta_rb[c], P.rb_off) < std::min<int64_t>(a.cta_rb[c + 1], P.rb_off + P.nrb);
+                dup = touched && P.x == M.x && P.k == M.k;
+            }
+            if (!dup) xb += (int64_t)a.batch * M.k * 2;
         }
         xmax = std::max(xmax, xb);
     }
-    a.x_smem_bytes = (int)((xmax + 127) / 128 * 128);
-    a.stage_bytes = (max_stage + 127) / 128 * 128;
-    const int fixed = kHeader + kAccBytes + a.x_smem_bytes;
-    a.stages = std::min(kMaxStages, (kSmemBudget - fixed) / a.stage_bytes);
-    a.smem_bytes = fixed + a.stages * a.stage_bytes;
-    return a.stages >= 2;
+    a.x_smem_bytes = (int)((xmax + 1023) / 1024 * 1024);  // the ring after it stays 1024-aligned
+    a.stage_bytes = (a.bits == 3 ? 3 * kBox : 4 * kBox) + (a.kind == 1 ? nlb_max * kBox : 0);
+    // The ring is a multiple of the number of warp groups, so that every
+    // slot is only ever used by one group: a warp then never waits on a
+    // barrier phase more than one ahead of the slot's current one.
+    for (int ring = kMaxRing; ring >= kGroups; ring -= kGroups) {
+        const int slots = std::min(kMaxRbSlots, (ring + nks_min - 1) / nks_min + 2);
+        const int red = (slots * kWarps * bmax * 32 * 4 + 1023) / 1024 * 1024;
+        const int smem = 1024 + kHeader + red + a.x_smem_bytes + ring * a.stage_bytes;
+        if (smem <= kSmemBudget || ring == kGroups) {
+            a.ring = ring;
+            a.rb_slots = slots;
+            a.red_bytes = red;
+            a.smem_bytes = smem;
+            break;
+        }
+    }
+    return a.ring >= kGroups && a.smem_bytes <= 227 * 1024;
 }
 
 cudaError_t launch_gemv_multi(const GemvMulti &a, cudaStream_t st, bool pdl) {

@@ -3,6 +3,7 @@
 
 #include <algorithm>
 #include <cstdint>
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include "qx_common.cuh"
@@ -33,9 +34,10 @@ struct DequantArgs {
 };
 
 constexpr int kMaxGemvMats = 8;
+constexpr int kMaxGemvCtas = 512;
 
-// One matrix of a (multi-matrix) decode launch.  The geometry fields after
-// log2g are filled by plan_gemv().
+// One matrix of a (multi-matrix) decode launch.  The fields after log2g are
+// filled by plan_gemv().
 struct GemvMat {
     const uint8_t *codes;
     const __half *scales;
@@ -45,23 +47,25 @@ struct GemvMat {
     void *y;          // [batch][n]
     int64_t n, k;
     int G, zbytes, log2g;
-    int CB, LB, SB, ZB, row_bytes, RB;
-    int64_t byte_off;
+    int nks;         // 1024-weight slices per row
+    int nlb;         // LUT boxes (32 rows x 8 groups) per slice
+    int nrb;         // 32-row blocks
+    int rb_off;      // first row-block of this matrix in the launch's list
 };
 
-constexpr int kMaxGemvCtas = 1024;
-
 struct GemvMulti {
-    GemvMat mat[kMaxGemvMats];
-    // first row of every CTA in the concatenation of all matrices' rows
-    // (byte-balanced slices computed on the host); cta_row[grid] = total rows
-    int64_t cta_row[kMaxGemvCtas + 1];
-    int64_t row_off[kMaxGemvMats + 1];  // first concatenated row of each matrix
+    // scalars first: the kernel's set-up reads them before anything else
     int count, bits, kind, batch, y_f32;
-    int grid, stages, stage_bytes, x_smem_bytes, smem_bytes;
+    int grid, ring, rb_slots, stage_bytes, red_bytes, x_smem_bytes, smem_bytes;
     int64_t total_bytes;
     uint32_t *status;
     uint64_t wait_limit_ns;
+    GemvMat mat[kMaxGemvMats];
+    // first row-block of every CTA (byte-balanced, computed on the host);
+    // cta_rb[grid] = total row-blocks
+    int32_t cta_rb[kMaxGemvCtas + 1];
+    CUtensorMap tm_codes[kMaxGemvMats];  // packed codes, 32-row x 128-byte boxes
+    CUtensorMap tm_luts[kMaxGemvMats];   // LUTs, 32-row x 128-byte boxes (LUT kind)
 };
 
 struct GemmArgs {
@@ -82,5 +86,12 @@ cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
 bool plan_gemv(GemvMulti &a, int num_sms);
 cudaError_t launch_gemv_multi(const GemvMulti &a, cudaStream_t st, bool pdl);
 cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st);
+
+// cuTensorMapEncodeTiled, fetched once through the runtime's driver entry
+// point (null if the driver does not provide it).
+using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                                   const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeTiledFn encode_fn();
 
 }  // namespace qx
