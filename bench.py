@@ -344,24 +344,35 @@ def run_ours(args):
         ms = float(t.item())
     value = step_bytes * ws / (ms * 1e-3) / 1e9
 
-    # per-launch kernel durations (events on the launching stream) for the roofline
-    reps = max(3, min(args.steps, 200))
-    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in CHAIN]
-           for _ in range(reps)]
-    with torch.cuda.stream(stream):
-        for r in range(reps):
-            for j in range(len(CHAIN)):
-                evs[r][j][0].record(stream)
-                launch(r % copies, j)
-                evs[r][j][1].record(stream)
-    torch.cuda.synchronize(dev)
-    kern_ms = sum(a.elapsed_time(b) for row in evs for a, b in row) / reps
-    per_launch_us = {"+".join(CHAIN[j][0]): 1e3 * sum(evs[r][j][0].elapsed_time(evs[r][j][1])
-                                                      for r in range(reps)) / reps for j in range(len(CHAIN))}
-    achieved = step_bytes / (kern_ms * 1e-3) / 1e9
+    # The timed region holds only gemv_kernel<3,LUT,1> launches (four per step),
+    # so its average launch duration is ms / 4 and the algorithmic bytes of an
+    # average launch are step_bytes / 4: achieved = step_bytes / ms.
+    launch_us = ms * 1e3 / len(CHAIN)
+    achieved = step_bytes / (ms * 1e-3) / 1e9
+    # steady-state duration of each launch of the chain: one graph per launch
+    # kind, `copies` back-to-back launches (PDL) over rotating weight copies
+    reps = 20
+    per_launch_us = {}
+    for j in range(len(CHAIN)):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for c in range(copies):
+                launch(c, j)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                g.replay()
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(reps):
+                g.replay()
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        per_launch_us["+".join(CHAIN[j][0])] = 1e3 * e0.elapsed_time(e1) / (reps * copies)
+        del g
 
     # the seven matrices as independent problems in one launch (upper bound of the chain)
     xs7 = {nm: (x_down if nm == "down_proj" else x_attn) for nm, _, _, _, _ in LAYER}
+    reps = 200
     with torch.cuda.stream(stream):
         for r in range(3):
             qx.gemv_multi([layers[r % copies][nm] for nm, *_ in LAYER], [xs7[nm] for nm, *_ in LAYER],
@@ -416,7 +427,8 @@ def run_ours(args):
                                       "GBps": step_bytes / (one_launch_ms * 1e-3) / 1e9},
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                          "frac": achieved / hbm, "peak_source": f"{peak_src} hbm_gbs",
-                         "kernel": "gemv_kernel<3,LUT,1,4>",
+                         "kernel": "gemv_kernel<3,LUT,1>", "launches_per_step": len(CHAIN),
+                         "launch_us": launch_us, "bytes_per_launch": step_bytes / len(CHAIN),
                          "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
             "gemm": gemm,
             "cpu_baseline": cpu,

@@ -42,13 +42,12 @@ constexpr int kSliceK = 1024;       // weights per row per stage
 constexpr int kPartK = kSliceK / kGroupWarps;  // weights per warp per stage
 constexpr int kBox = kRows * 128;   // one 32-row x 128-byte TMA box
 constexpr int kMaxRing = 8;
-// Stages issued at start.  Requesting the whole ring at once would make every
-// stage arrive late (the memory system serves them interleaved); the rest of
-// the ring is issued as the first stages land.
-#ifndef QX_GEMV_INITIAL_STAGES
-#define QX_GEMV_INITIAL_STAGES 8
-#endif
-constexpr int kInitialStages = QX_GEMV_INITIAL_STAGES;
+// Stages issued at start (GemvMulti::initial): one per warp group for a
+// standalone launch -- requesting the whole ring at once makes every stage
+// land late, as the memory system serves them interleaved; the rest of the
+// ring is issued as the first stages land.  A launch that follows another
+// kernel under programmatic dependent launch requests the whole ring, whose
+// latency then hides behind the previous kernel.
 constexpr int kMaxRbSlots = 16;
 constexpr int kHeader = 1024;       // barriers, counters, per-matrix CTA plan
 constexpr int kSmemBudget = 200 * 1024;
@@ -176,6 +175,7 @@ struct MatS {
     int n, K, G, zbytes, log2g, nks, nlb;
     int xoff;   // shared-memory offset (halves) of this matrix's x
     int q0;     // first CTA-local stage of this matrix
+    int rbq0;   // first CTA-local row block of this matrix
     int rb0;    // first matrix-local row block of this CTA
     int nrb;    // row blocks of this CTA in this matrix
 };
@@ -310,14 +310,17 @@ __device__ __forceinline__ float meta_scale(const Meta &t, int gl) {
 
 __device__ __forceinline__ uint32_t meta_zero(const Meta &t, int gl) { return (t.z >> (4 * gl)) & 15u; }
 
-// Stage cursor: matrix, row block (CTA-local), slice.
+// Cursor over one warp's stages: matrix, CTA-local row block of that matrix,
+// slice, and the CTA-local stage number.
 struct Cursor {
-    int m, rbl, ks;
+    int m, rbl, ks, q;
 };
 
-__device__ __forceinline__ void advance(const Header &h, int count, Cursor &c) {
-    if (++c.ks == h.mats[c.m].nks) {
-        c.ks = 0;
+__device__ __forceinline__ void advance_by(const Header &h, int count, Cursor &c, int d) {
+    c.q += d;
+    c.ks += d;
+    while (c.m < count && c.ks >= h.mats[c.m].nks) {
+        c.ks -= h.mats[c.m].nks;
         if (++c.rbl == h.mats[c.m].nrb) {
             c.rbl = 0;
             ++c.m;
@@ -326,7 +329,89 @@ __device__ __forceinline__ void advance(const Header &h, int count, Cursor &c) {
     }
 }
 
-template <int BITS, int KIND, int BMAX>
+// Wait for a full-barrier phase: a try in line, the bounded loop out of line.
+__device__ __forceinline__ bool wait_full(uint32_t bar, uint32_t par, uint64_t limit_ns,
+                                          volatile uint32_t *abort_flag) {
+    bool ok = mbar_try_wait(bar, par);
+    if (!__all_sync(0xffffffffu, ok)) ok = __all_sync(0xffffffffu, mbar_wait(bar, par, limit_ns, abort_flag));
+    return ok;
+}
+
+// One 3-bit superblock (128 k = four 32-weight units) of one row: codes words
+// A/B/C, tables built TPS times (once per group), products with NB rows of x.
+template <int KIND, int NB, int TPS>
+__device__ __forceinline__ void superblock3(const uint4 &A, const uint4 &B, const uint4 &C, uint32_t lut_s,
+                                            int lg0, int r, const Meta &meta, int gl0, uint32_t xk, int K,
+                                            bool half_only, float (&acc)[NB]) {
+    const uint32_t Aw[4] = {A.x, A.y, A.z, A.w};
+    const uint32_t Bw[4] = {B.x, B.y, B.z, B.w};
+    const uint32_t Cw[4] = {C.x, C.y, C.z, C.w};
+    (void)half_only;
+    Table8 tab{};
+    float s = 1.0f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        __half2 xv[NB][16];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
+        if (i % (4 / TPS) == 0) {
+            const int t = i / (4 / TPS);
+            if (KIND == 1) {
+                const int lg = lg0 + t;
+                const uint4 l = lds128(lut_s + (uint32_t)((lg >> 3) * kBox) + swz(r, lg & 7));
+                tab = make_table8(l.x, l.y, l.z, l.w);
+            } else {
+                tab = table8_offsets(meta_zero(meta, gl0 + t));
+                s = meta_scale(meta, gl0 + t);
+            }
+        }
+        __half2 w[16];
+        lookup_triple(tab, Aw[i], Bw[i], Cw[i], w);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) {
+            if (KIND == 1)
+                acc[b] += dot16(w, xv[b]);
+            else
+                acc[b] += s * dot16(w, xv[b]);
+        }
+    }
+}
+
+// Eight 4-bit units (256 k) of one row, UPG units per group.
+template <int NB, int UPG>
+__device__ __forceinline__ void part4(uint32_t cb, int r, const Meta &meta, uint32_t xk, int K, bool half_only,
+                                      float (&acc)[NB]) {
+    float s = 1.0f;
+    __half2 zl{}, zh{};
+#pragma unroll
+    for (int i = 0; i < 8; ++i) {
+        if (i == 4 && half_only) break;  // k is a multiple of 128, not of 256
+        __half2 xv[NB][16];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
+        if (i % UPG == 0) {
+            const int gl = i / UPG;
+            const uint32_t z = meta_zero(meta, gl);
+            zl = zlo_of(z);
+            zh = zhi_of(z);
+            s = meta_scale(meta, gl);
+        }
+        const uint4 cw = lds128(cb + swz(r, i));
+        const uint32_t wd[4] = {cw.x, cw.y, cw.z, cw.w};
+        __half2 w[16];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+            __half2 o[4];
+            unpack4_qz(wd[t], zl, zh, o);
+#pragma unroll
+            for (int u = 0; u < 4; ++u) w[4 * t + u] = o[u];
+        }
+#pragma unroll
+        for (int b = 0; b < NB; ++b) acc[b] += s * dot16(w, xv[b]);
+    }
+}
+
+template <int BITS, int KIND, int NB>
 __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant__ GemvMulti a) {
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled TMA boxes
@@ -341,7 +426,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int count = a.count, ring = a.ring, nb = a.batch;
+    const int count = a.count, ring = a.ring;
 
     // ---- set-up, spread over threads so that the first copies start early
     if (threadIdx.x < count) {  // this CTA's row blocks of matrix t
@@ -379,31 +464,36 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     }
     __syncthreads();
     if (warp == 0) {
-        // stage numbering per matrix, then one lane per initial stage
-        int q = 0, mine = 0, qend = 0;
+        // stage and row-block numbering per matrix, then one lane per initial stage
+        int q = 0, rbq = 0, mine = 0, mrb = 0, qend = 0;
         for (int m = 0; m < count; ++m) {
-            if (m == lane) mine = q;
+            if (m == lane) {
+                mine = q;
+                mrb = rbq;
+            }
             q += h.mats[m].nrb * h.mats[m].nks;
+            rbq += h.mats[m].nrb;
             if (m == lane) qend = q;
         }
         if (lane < count) {
             h.mats[lane].q0 = mine;
+            h.mats[lane].rbq0 = mrb;
             h.q_end[lane] = qend;
             // activations in shared memory: one copy per distinct x of this CTA
             int off = 0, xo = -1;
             for (int m = 0; m < lane; ++m) {
                 if (!x_owner(h, m)) continue;
                 if (xo < 0 && same_x(h, m, lane)) xo = off;
-                off += nb * h.mats[m].K;
+                off += NB * h.mats[m].K;
             }
             h.mats[lane].xoff = xo >= 0 ? xo : off;
         }
         if (lane == 0) {
             h.nstages = q;
-            h.issued = (uint32_t)min(min(ring, kInitialStages), q);
+            h.issued = (uint32_t)min(a.initial, q);
         }
         __syncwarp();
-        if (lane < min(min(ring, kInitialStages), q)) issue_stage<BITS, KIND>(a, h, ring_s, lane);
+        if (lane < min(a.initial, q)) issue_stage<BITS, KIND>(a, h, ring_s, lane);
     }
     __syncthreads();
     // let the next kernel in the stream start streaming its own weights; it
@@ -413,213 +503,182 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     const int nst = h.nstages;
     const int r = lane;
     const int grp = warp / kGroupWarps;   // stages q with q % kGroups == grp
-    const int part = warp % kGroupWarps;  // 128-weight part of each of those stages
+    const int part = warp % kGroupWarps;  // 256-weight part of each of those stages
     bool ok = true;
-    int q = 0, slot = 0, rbseq = 0;
-    uint32_t par = 0;
 
-    Cursor c{0, 0, 0};
+    // this warp's first stage, and the one after it
+    Cursor c{0, 0, 0, 0};
     while (c.m < count && h.mats[c.m].nrb == 0) ++c.m;
-    // uniform metadata of this warp's next stage, loaded one stage ahead
+    advance_by(h, count, c, grp);
+    Cursor cn = c;
+    advance_by(h, count, cn, kGroups);
+    // uniform metadata of this warp's stages, loaded one stage ahead
     Meta cur{}, nxt{};
-    Cursor pc = c;
-    for (int i = 0; i < grp && pc.m < count; ++i) advance(h, count, pc);
-    if (KIND == 0 && pc.m < count)
-        cur = load_meta(h.mats[pc.m], (h.mats[pc.m].rb0 + pc.rbl) * kRows + r, pc.ks * kSliceK + part * kPartK);
+    if (KIND == 0 && c.m < count)
+        cur = load_meta(h.mats[c.m], (h.mats[c.m].rb0 + c.rbl) * kRows + r, c.ks * kSliceK + part * kPartK);
     asm volatile("griddepcontrol.wait;" ::: "memory");
     // activations -> shared memory (every lane of a warp then reads the same
     // address: a broadcast)
     for (int m = 0; m < count; ++m) {
         if (!x_owner(h, m)) continue;
-        const int vecs = nb * h.mats[m].K / 8;
+        const int vecs = NB * h.mats[m].K / 8;
         const uint4 *src = reinterpret_cast<const uint4 *>(h.mats[m].x);
         uint4 *dst = reinterpret_cast<uint4 *>(xs + h.mats[m].xoff);
         for (int i = threadIdx.x; i < vecs; i += kThreads) dst[i] = src[i];
     }
     __syncthreads();
 
-    float acc[BMAX];
+    // per-lane offsets of this warp's 3-bit code chunks in a stage (planes 0-2
+    // of row r are box rows 3r..3r+2; superblocks 2 part and 2 part + 1)
+    uint32_t co[2][3];
 #pragma unroll
-    for (int b = 0; b < BMAX; ++b) acc[b] = 0.0f;
-    for (; q < nst && ok; ++q) {
-        const MatS &M = h.mats[c.m];
-        const int K = M.K, log2g = M.log2g;
-        const int k0 = c.ks * kSliceK + part * kPartK;
-        if (q % kGroups == grp) {
-            if (KIND == 0) {  // metadata of this warp's following stage
-                for (int i = 0; i < kGroups && pc.m < count; ++i) advance(h, count, pc);
-                if (pc.m < count) {
-                    const MatS &N = h.mats[pc.m];
-                    nxt = load_meta(N, (N.rb0 + pc.rbl) * kRows + r, pc.ks * kSliceK + part * kPartK);
+    for (int hb = 0; hb < 2; ++hb)
+#pragma unroll
+        for (int p = 0; p < 3; ++p) co[hb][p] = swz(3 * r + p, part * 2 + hb);
+
+    float acc[NB];
+#pragma unroll
+    for (int b = 0; b < NB; ++b) acc[b] = 0.0f;
+    int slot = grp, fm = -1, frbl = 0;
+    uint32_t par = 0;
+
+    // partials of row block (m, rbl) -> shared memory; the last contributor
+    // sums them in a fixed order and writes y
+    auto flush = [&](int m, int rbl) -> bool {
+        const MatS &M = h.mats[m];
+        const int rbi = M.rbq0 + rbl;
+        const int rs = rbi % a.rb_slots;
+        const uint32_t use = (uint32_t)(rbi / a.rb_slots);
+        // the warp groups run independently: the slot's previous block must
+        // have been summed before this warp overwrites its partials
+        bool okf = true;
+        if (lane == 0) okf = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
+        if (!__shfl_sync(0xffffffffu, okf, 0)) return false;
+        float *rp = red + (size_t)rs * (kWarps * NB * 32);
+#pragma unroll
+        for (int b = 0; b < NB; ++b) rp[(warp * NB + b) * 32 + r] = acc[b];
+        __syncwarp();
+        const int ng = min(M.nks, kGroups);  // groups that worked on this block
+        uint32_t fin = 0;
+        if (lane == 0) {
+            __threadfence_block();
+            fin = atomicAdd(&h.cnt[rs], 1u) + 1u == (uint32_t)(ng * kGroupWarps);
+            __threadfence_block();
+        }
+        fin = __shfl_sync(0xffffffffu, fin, 0);
+        if (fin) {
+            const int q0 = M.q0 + rbl * M.nks;  // the block's first stage
+            const int row = (M.rb0 + rbl) * kRows + r;
+            if (row < M.n) {
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    float v = 0.0f;
+                    for (int j = 0; j < ng; ++j) {
+                        const int g = (q0 + j) % kGroups;
+#pragma unroll
+                        for (int p = 0; p < kGroupWarps; ++p) v += rp[((g * kGroupWarps + p) * NB + b) * 32 + r];
+                    }
+                    if (a.y_f32)
+                        reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v;
+                    else
+                        reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v);
                 }
             }
-            ok = mbar_wait(smem_u32(&h.full[slot]), par, a.wait_limit_ns, &h.abort_flag);
-            if (!__all_sync(0xffffffffu, ok)) {
-                ok = false;
-                break;
-            }
-            if (part == 0 && lane == 0 && q + kInitialStages < min(ring, nst)) {
-                // ramp-up: a stage has landed, request one more of the ring
-                issue_stage<BITS, KIND>(a, h, ring_s, q + kInitialStages);
-                atomicMax(&h.issued, (uint32_t)(q + kInitialStages + 1));
-            }
-            if (k0 < K) {
-                const uint32_t sb = ring_s + (uint32_t)(slot * a.stage_bytes);
-                const uint32_t xk = xs_s + 2u * (uint32_t)(M.xoff + k0);
-                if (BITS == 3) {
-                    uint32_t Aw[4], Bw[4], Cw[4];
-                    Table8 tab{};
-                    float s = 1.0f;
-#pragma unroll
-                    for (int i = 0; i < kPartK / 32; ++i) {
-                        if (i == 4 && k0 + 128 >= K) break;  // k is a multiple of 128, not of 256
-                        if ((i & 3) == 0) {
-                            // superblock (128 k): planes 0/1/2 of row r are box rows 3r, 3r+1, 3r+2
-                            const int sbk = part * (kPartK / 128) + (i >> 2);
-                            const uint4 A = lds128(sb + swz(3 * r, sbk));
-                            const uint4 B = lds128(sb + swz(3 * r + 1, sbk));
-                            const uint4 C = lds128(sb + swz(3 * r + 2, sbk));
-                            Aw[0] = A.x; Aw[1] = A.y; Aw[2] = A.z; Aw[3] = A.w;
-                            Bw[0] = B.x; Bw[1] = B.y; Bw[2] = B.z; Bw[3] = B.w;
-                            Cw[0] = C.x; Cw[1] = C.y; Cw[2] = C.z; Cw[3] = C.w;
-                        }
-                        __half2 xv[BMAX][16];
-#pragma unroll
-                        for (int b = 0; b < BMAX; ++b)
-                            if (b < nb) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
-                        // a new table where unit i starts a group
-                        if (i == 0 || ((32 * i) & ((1 << log2g) - 1)) == 0) {
-                            const int gl = (32 * i) >> log2g;
-                            if (KIND == 1) {
-                                const int lg = (part * kPartK + 32 * i) >> log2g;
-                                const uint4 l = lds128(sb + 3 * kBox + (uint32_t)((lg >> 3) * kBox) + swz(r, lg & 7));
-                                tab = make_table8(l.x, l.y, l.z, l.w);
-                            } else {
-                                tab = table8_offsets(meta_zero(cur, gl));
-                                s = meta_scale(cur, gl);
-                            }
-                        }
-                        __half2 w[16];
-                        lookup_triple(tab, Aw[i & 3], Bw[i & 3], Cw[i & 3], w);
-#pragma unroll
-                        for (int b = 0; b < BMAX; ++b) {
-                            if (b < nb) {
-                                if (KIND == 1)
-                                    acc[b] += dot16(w, xv[b]);
-                                else
-                                    acc[b] += s * dot16(w, xv[b]);
-                            }
-                        }
-                    }
-                } else {
-                    // 4-bit: box `part` holds this part's 256 k, 16 bytes per 32 k
-                    const uint32_t cb = sb + (uint32_t)(part * kBox);
-                    float s = 1.0f;
-                    __half2 zl{}, zh{};
-#pragma unroll
-                    for (int i = 0; i < kPartK / 32; ++i) {
-                        if (i == 4 && k0 + 128 >= K) break;  // k is a multiple of 128, not of 256
-                        __half2 xv[BMAX][16];
-#pragma unroll
-                        for (int b = 0; b < BMAX; ++b)
-                            if (b < nb) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
-                        if (i == 0 || ((32 * i) & ((1 << log2g) - 1)) == 0) {
-                            const int gl = (32 * i) >> log2g;
-                            const uint32_t z = meta_zero(cur, gl);
-                            zl = zlo_of(z);
-                            zh = zhi_of(z);
-                            s = meta_scale(cur, gl);
-                        }
-                        const uint4 cw = lds128(cb + swz(r, i));
-                        const uint32_t wd[4] = {cw.x, cw.y, cw.z, cw.w};
-                        __half2 w[16];
-#pragma unroll
-                        for (int t = 0; t < 4; ++t) {
-                            __half2 o[4];
-                            unpack4_qz(wd[t], zl, zh, o);
-#pragma unroll
-                            for (int u = 0; u < 4; ++u) w[4 * t + u] = o[u];
-                        }
-#pragma unroll
-                        for (int b = 0; b < BMAX; ++b)
-                            if (b < nb) acc[b] += s * dot16(w, xv[b]);
-                    }
-                }
-            }
-            // release the stage; the last warp of the group refills it
             __syncwarp();
             if (lane == 0) {
+                h.cnt[rs] = 0;
                 __threadfence_block();
-                const uint32_t old = atomicAdd(&h.rel[slot], 1u);
-                if (old == kGroupWarps - 1) {
-                    h.rel[slot] = 0;
-                    __threadfence_block();
-                    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                    if (q + ring < nst && !*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) {
-                        issue_stage<BITS, KIND>(a, h, ring_s, q + ring);
-                        atomicMax(&h.issued, (uint32_t)(q + ring + 1));
-                    }
+                *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
+            }
+        }
+        return true;
+    };
+
+    while (c.m < count) {
+        const MatS &M = h.mats[c.m];
+        if (fm >= 0 && (fm != c.m || frbl != c.rbl)) {  // left the previous row block
+            ok = flush(fm, frbl);
+            if (!ok) break;
+#pragma unroll
+            for (int b = 0; b < NB; ++b) acc[b] = 0.0f;
+        }
+        fm = c.m;
+        frbl = c.rbl;
+        if (KIND == 0 && cn.m < count) {
+            const MatS &N = h.mats[cn.m];
+            nxt = load_meta(N, (N.rb0 + cn.rbl) * kRows + r, cn.ks * kSliceK + part * kPartK);
+        }
+        ok = wait_full(smem_u32(&h.full[slot]), par, a.wait_limit_ns, &h.abort_flag);
+        if (!ok) break;
+        const int q = c.q;
+        if (part == 0 && lane == 0 && q + a.initial < min(ring, nst)) {
+            // ramp-up: a stage has landed, request one more of the ring
+            issue_stage<BITS, KIND>(a, h, ring_s, q + a.initial);
+            atomicMax(&h.issued, (uint32_t)(q + a.initial + 1));
+        }
+        const int K = M.K;
+        const int k0 = c.ks * kSliceK + part * kPartK;
+        if (k0 < K) {
+            const uint32_t sb = ring_s + (uint32_t)(slot * a.stage_bytes);
+            const uint32_t xk = xs_s + 2u * (uint32_t)(M.xoff + k0);
+            const bool half_only = k0 + 128 >= K;  // k is a multiple of 128, not of 256
+            const int log2g = M.log2g;
+            if (BITS == 3) {
+                const uint32_t lut_s = sb + 3 * kBox;
+#pragma unroll
+                for (int hb = 0; hb < 2; ++hb) {
+                    if (hb == 1 && half_only) break;
+                    const uint4 A = lds128(sb + co[hb][0]);
+                    const uint4 B = lds128(sb + co[hb][1]);
+                    const uint4 C = lds128(sb + co[hb][2]);
+                    const int kk = part * kPartK + 128 * hb;  // within the slice
+                    const int gl0 = (128 * hb) >> log2g;       // first group of the superblock in the part
+                    const int lg0 = kk >> log2g;               // ... in the slice (LUT boxes)
+                    if (log2g >= 7)
+                        superblock3<KIND, NB, 1>(A, B, C, lut_s, lg0, r, cur, gl0, xk + 256u * hb, K, half_only, acc);
+                    else if (log2g == 6)
+                        superblock3<KIND, NB, 2>(A, B, C, lut_s, lg0, r, cur, gl0, xk + 256u * hb, K, half_only, acc);
+                    else
+                        superblock3<KIND, NB, 4>(A, B, C, lut_s, lg0, r, cur, gl0, xk + 256u * hb, K, half_only, acc);
+                }
+            } else {
+                // 4-bit: box `part` holds this part's 256 k, 16 bytes per 32 k
+                const uint32_t cb = sb + (uint32_t)(part * kBox);
+                if (log2g >= 8)
+                    part4<NB, 8>(cb, r, cur, xk, K, half_only, acc);
+                else if (log2g == 7)
+                    part4<NB, 4>(cb, r, cur, xk, K, half_only, acc);
+                else if (log2g == 6)
+                    part4<NB, 2>(cb, r, cur, xk, K, half_only, acc);
+                else
+                    part4<NB, 1>(cb, r, cur, xk, K, half_only, acc);
+            }
+        }
+        // release the stage; the last warp of the group refills it
+        __syncwarp();
+        if (lane == 0) {
+            __threadfence_block();
+            const uint32_t old = atomicAdd(&h.rel[slot], 1u);
+            if (old == kGroupWarps - 1) {
+                h.rel[slot] = 0;
+                __threadfence_block();
+                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+                if (q + ring < nst && !*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) {
+                    issue_stage<BITS, KIND>(a, h, ring_s, q + ring);
+                    atomicMax(&h.issued, (uint32_t)(q + ring + 1));
                 }
             }
-            if (KIND == 0) cur = nxt;
         }
-        if (++slot == ring) {
-            slot = 0;
+        if (KIND == 0) cur = nxt;
+        c = cn;
+        advance_by(h, count, cn, kGroups);
+        slot += kGroups;
+        if (slot >= ring) {
+            slot -= ring;
             par ^= 1u;
         }
-        if (c.ks + 1 == M.nks) {
-            // end of a row block: partials -> shared memory; the last of all
-            // warps sums them in a fixed order and writes y
-            const int rs = rbseq % a.rb_slots;
-            const uint32_t use = (uint32_t)(rbseq / a.rb_slots);
-            ++rbseq;
-            // the warp groups run independently: the slot's previous block
-            // must have been summed before this warp overwrites its partials
-            if (lane == 0) ok = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
-            if (!__shfl_sync(0xffffffffu, ok, 0)) {
-                ok = false;
-                break;
-            }
-            float *rp = red + (size_t)rs * (kWarps * BMAX * 32);
-#pragma unroll
-            for (int b = 0; b < BMAX; ++b) {
-                rp[(warp * BMAX + b) * 32 + r] = acc[b];
-                acc[b] = 0.0f;
-            }
-            __syncwarp();
-            uint32_t fin = 0;
-            if (lane == 0) {
-                __threadfence_block();
-                fin = atomicAdd(&h.cnt[rs], 1u) == kWarps - 1;
-                __threadfence_block();
-            }
-            fin = __shfl_sync(0xffffffffu, fin, 0);
-            if (fin) {
-                const int row = (M.rb0 + c.rbl) * kRows + r;
-                if (row < M.n) {
-#pragma unroll
-                    for (int b = 0; b < BMAX; ++b) {
-                        if (b < nb) {
-                            float v = 0.0f;
-#pragma unroll
-                            for (int w2 = 0; w2 < kWarps; ++w2) v += rp[(w2 * BMAX + b) * 32 + r];
-                            if (a.y_f32)
-                                reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v;
-                            else
-                                reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v);
-                        }
-                    }
-                }
-                __syncwarp();
-                if (lane == 0) {
-                    h.cnt[rs] = 0;
-                    __threadfence_block();
-                    *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
-                }
-            }
-        }
-        advance(h, count, c);
     }
+    if (ok && fm >= 0) ok = flush(fm, frbl);
     if (!ok && lane == 0) {
         h.abort_flag = 1u;
         atomicOr(a.status, kStatusTimeout);
@@ -633,9 +692,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     }
 }
 
-template <int BITS, int KIND, int BMAX>
+template <int BITS, int KIND, int NB>
 cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
-    auto kern = gemv_kernel<BITS, KIND, BMAX>;
+    auto kern = gemv_kernel<BITS, KIND, NB>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
     if (e != cudaSuccess) return e;
     e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
@@ -668,7 +727,7 @@ bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims
 // Host-side plan: tensor maps, byte-balanced CTA row-block ranges and the
 // shared-memory budget.  Returns false if the matrices cannot share one launch.
 bool plan_gemv(GemvMulti &a, int num_sms) {
-    const int bmax = a.batch <= 1 ? 1 : (a.batch <= 2 ? 2 : 4);
+    const int bmax = a.batch;  // kernels are built for batch 1..4 exactly
     int nks_min = 1 << 30, nlb_max = 1;
     int64_t total = 0, rbs = 0;
     for (int m = 0; m < a.count; ++m) {
@@ -765,20 +824,21 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
     return a.ring >= kGroups && a.smem_bytes <= 227 * 1024;
 }
 
-cudaError_t launch_gemv_multi(const GemvMulti &a, cudaStream_t st, bool pdl) {
-    if (a.bits == 4) {
-        if (a.batch <= 1) return launch_one<4, 0, 1>(a, st, pdl);
-        if (a.batch <= 2) return launch_one<4, 0, 2>(a, st, pdl);
-        return launch_one<4, 0, 4>(a, st, pdl);
+template <int BITS, int KIND>
+cudaError_t launch_nb(const GemvMulti &a, cudaStream_t st, bool pdl) {
+    switch (a.batch) {
+        case 1: return launch_one<BITS, KIND, 1>(a, st, pdl);
+        case 2: return launch_one<BITS, KIND, 2>(a, st, pdl);
+        case 3: return launch_one<BITS, KIND, 3>(a, st, pdl);
+        default: return launch_one<BITS, KIND, 4>(a, st, pdl);
     }
-    if (a.kind == 1) {
-        if (a.batch <= 1) return launch_one<3, 1, 1>(a, st, pdl);
-        if (a.batch <= 2) return launch_one<3, 1, 2>(a, st, pdl);
-        return launch_one<3, 1, 4>(a, st, pdl);
-    }
-    if (a.batch <= 1) return launch_one<3, 0, 1>(a, st, pdl);
-    if (a.batch <= 2) return launch_one<3, 0, 2>(a, st, pdl);
-    return launch_one<3, 0, 4>(a, st, pdl);
+}
+
+cudaError_t launch_gemv_multi(GemvMulti &a, cudaStream_t st, bool pdl) {
+    a.initial = pdl ? a.ring : kGroups;
+    if (a.bits == 4) return launch_nb<4, 0>(a, st, pdl);
+    if (a.kind == 1) return launch_nb<3, 1>(a, st, pdl);
+    return launch_nb<3, 0>(a, st, pdl);
 }
 
 }  // namespace qx

@@ -56,7 +56,7 @@ struct GemvMat {
 struct GemvMulti {
     // scalars first: the kernel's set-up reads them before anything else
     int count, bits, kind, batch, y_f32;
-    int grid, ring, rb_slots, stage_bytes, red_bytes, x_smem_bytes, smem_bytes;
+    int grid, ring, initial, rb_slots, stage_bytes, red_bytes, x_smem_bytes, smem_bytes;
     int64_t total_bytes;
     uint32_t *status;
     uint64_t wait_limit_ns;
@@ -84,7 +84,7 @@ struct GemmArgs {
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
 bool plan_gemv(GemvMulti &a, int num_sms);
-cudaError_t launch_gemv_multi(const GemvMulti &a, cudaStream_t st, bool pdl);
+cudaError_t launch_gemv_multi(GemvMulti &a, cudaStream_t st, bool pdl);
 cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st);
 
 // cuTensorMapEncodeTiled, fetched once through the runtime's driver entry
