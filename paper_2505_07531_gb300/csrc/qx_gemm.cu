@@ -2,23 +2,27 @@
 // tensor cores (tcgen05), with the weights dequantized on chip.
 //
 // Prefill is the one dense contraction on the path (paper Table 2, "Prefill"),
-// so it runs on the tensor cores.  The kernel computes the transposed tile
+// so it runs on the tensor cores.  The kernel computes transposed tiles
 // D = W_hat_tile * X_tile^T: the MMA's M dimension is 128 rows of W, its N
-// dimension 128 tokens, and the contraction runs over k in stages of 64.
+// dimension 256 tokens (each dequantized W tile feeds 256 tokens, which keeps
+// the dequantization below the tensor-core time), and the contraction runs
+// over k in stages of 64.
 //
-// Warp roles (320 threads):
-//   warp 0      TMA producer: 128 x 64 fp16 X tiles (128B swizzle) -> smem
-//   warp 1      allocates tensor memory; one thread issues tcgen05.mma
-//   warps 2-9   dequantize 128 x 64 W_hat tiles from the packed codes straight
-//               into the 128B-swizzled K-major shared-memory layout the MMA
-//               reads (the same unpack primitives as qx_dequant, so W_hat is
-//               exact), then read the fp32 accumulator out of tensor memory
-//               and store fp16 Y.
-// A 4-stage mbarrier ring connects producers and the MMA issuer; the MMA
-// releases a stage with tcgen05.commit.  Every wait is bounded in time: a wait
-// that gives up raises QX_ERR_TIMEOUT in the device status word, tells the
-// other roles to stop, lets in-flight copies and MMAs drain, frees tensor
-// memory and returns.
+// Persistent: one CTA per SM walks the (W-row tile, token tile) pairs.  Warp
+// roles (448 threads):
+//   warp 0       TMA producer: 256 x 64 fp16 X tiles (128B swizzle) -> smem
+//   warp 1       allocates tensor memory; one thread issues tcgen05.mma
+//   warps 2-9    dequantize 128 x 64 W_hat tiles from the packed codes straight
+//                into the 128B-swizzled K-major shared-memory layout the MMA
+//                reads (the same unpack primitives as qx_dequant, so W_hat is
+//                exact)
+//   warps 10-13  epilogue: fp32 accumulator (tensor memory) -> fp16 Y
+// Two accumulators of 256 columns let the epilogue of one tile overlap the
+// main loop of the next.  A 4-stage mbarrier ring connects producers and the
+// MMA issuer; the MMA releases a stage with tcgen05.commit.  Every wait is
+// bounded in time: a wait that gives up raises QX_ERR_TIMEOUT in the device
+// status word, tells the other roles to stop, lets in-flight copies and MMAs
+// drain, frees tensor memory and returns.
 #include <cuda.h>
 
 #include "qx_kernels.cuh"
@@ -28,22 +32,32 @@ namespace qx {
 namespace {
 
 constexpr int BM = 128;  // W rows per tile (MMA M)
-constexpr int BN = 128;  // tokens per tile (MMA N)
+constexpr int BN = 256;  // tokens per tile (MMA N): each dequantized W tile feeds 256 tokens
 constexpr int BK = 64;   // k per stage (one 128-byte swizzle row of fp16)
+// X tiles (TMA) and dequantized W tiles use rings of STAGES and W_SLOTS
+// slots tracked by the same per-stage barriers: the dequant warps know W slot
+// q % W_SLOTS is free once the MMAs of stage q - W_SLOTS are done.  Equal
+// depths measured best (a deeper X ring at the cost of W slots lets the
+// dequantization fall behind).
 constexpr int STAGES = 4;
+constexpr int W_SLOTS = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int NUM_DQ_WARPS = 8;
-constexpr int THREADS = 64 + NUM_DQ_WARPS * 32;
-constexpr uint32_t TMEM_COLS = 128;
+constexpr int NUM_EPI_WARPS = 4;
+constexpr int THREADS = 64 + (NUM_DQ_WARPS + NUM_EPI_WARPS) * 32;
+constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 
 struct SmemLayout {
-    uint8_t a[STAGES][A_BYTES];
+    uint8_t a[W_SLOTS][A_BYTES];
     uint8_t b[STAGES][B_BYTES];
-    uint64_t full_a[STAGES];
-    uint64_t full_b[STAGES];
-    uint64_t empty[STAGES];
-    uint64_t accum_full;
+    // one barrier per direction and stage: the MMA thread waits once and
+    // commits once per stage (its per-stage overhead bounds the MMA rate)
+    uint64_t full[STAGES];   // 8 dequant-warp arrivals + the X copy's bytes
+    uint64_t empty[STAGES];  // tcgen05.commit of the stage's MMAs
+    uint64_t accum_full[2];
+    uint64_t accum_empty[2];
+    uint64_t done;
     uint32_t tmem_base;
     uint32_t abort_flag;
 };
@@ -79,6 +93,22 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t *b, uint32_t parity) {
     return ok != 0;
 }
 
+// try_wait with a suspend-time hint: a thread whose phase is not complete
+// sleeps in hardware (woken when the phase completes) instead of spinning,
+// which would take issue slots from the dequantizing warps that share its
+// scheduler.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t *b, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(smem_u32(b)), "r"(parity), "r"(1000000u)
+        : "memory");
+    return ok != 0;
+}
+
 // Wait for the phase of parity `parity` to complete.  Gives up after
 // `limit_ns`, or as soon as another role has raised the abort flag (when
 // `abort_flag` is not null).  Returns false if it gave up.
@@ -86,13 +116,18 @@ __device__ __noinline__ bool mbar_wait(uint64_t *b, uint32_t parity, uint64_t li
                                        volatile uint32_t *abort_flag) {
     if (mbar_try_wait(b, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
-    for (uint32_t i = 1;; ++i) {
-        if (mbar_try_wait(b, parity)) return true;
-        if ((i & 31u) == 0) {
-            if (abort_flag != nullptr && *abort_flag) return false;
-            if (globaltimer_ns() - t0 > limit_ns) return false;
-        }
+    for (;;) {
+        if (mbar_try_wait_sleep(b, parity)) return true;
+        if (abort_flag != nullptr && *abort_flag) return false;
+        if (globaltimer_ns() - t0 > limit_ns) return false;
     }
+}
+
+// Fast path in line (a phase that is already complete costs one try_wait),
+// the bounded loop out of line.
+__device__ __forceinline__ bool wait_phase(uint64_t *b, uint32_t parity, uint64_t limit_ns,
+                                           volatile uint32_t *abort_flag) {
+    return mbar_try_wait(b, parity) || mbar_wait(b, parity, limit_ns, abort_flag);
 }
 
 __device__ __forceinline__ void raise_abort(SmemLayout &s, uint32_t *status) {
@@ -227,17 +262,23 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
     volatile uint32_t *abort_flag = &s.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int64_t n0 = (int64_t)blockIdx.y * BM;  // W rows
-    const int64_t m0 = (int64_t)blockIdx.x * BN;  // tokens
     const int nkb = (int)(a.k / BK);
+    const int mt = (int)((a.m + BN - 1) / BN);  // token tiles
+    const int nt = (int)((a.n + BM - 1) / BM);  // W-row tiles
+    const int ntiles = mt * nt;
+    // tile t: W rows n0 = (t / mt) * BM, tokens m0 = (t % mt) * BN; consecutive
+    // CTAs share a W tile (L2 reuse of the packed codes)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
-            mbar_init(&s.full_a[i], NUM_DQ_WARPS);
-            mbar_init(&s.full_b[i], 1);
+            mbar_init(&s.full[i], NUM_DQ_WARPS + 1);
             mbar_init(&s.empty[i], 1);
         }
-        mbar_init(&s.accum_full, 1);
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&s.accum_full[i], 1);
+            mbar_init(&s.accum_empty[i], NUM_EPI_WARPS);
+        }
+        mbar_init(&s.done, 1);
         s.abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_x) : "memory");
@@ -257,99 +298,144 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
     if (warp == 0) {
         // ------------------------------------------------ TMA producer (X)
         if (lane == 0) {
-            int issued = 0;
-            for (int kb = 0; kb < nkb; ++kb) {
-                const int st = kb % STAGES;
-                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-                if (!mbar_wait(&s.empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag)) {
-                    raise_abort(s, a.status);
-                    break;
+            int it = 0;  // stage counter across tiles
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                const int m0 = (t % mt) * BN;
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int st = it % STAGES;
+                    const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+                    if (!wait_phase(&s.empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag)) {
+                        raise_abort(s, a.status);
+                        ok = false;
+                        break;
+                    }
+                    mbar_arrive_expect_tx(&s.full[st], B_BYTES);
+                    tma_load_2d(s.b[st], &tmap_x, &s.full[st], kb * BK, m0);
                 }
-                mbar_arrive_expect_tx(&s.full_b[st], B_BYTES);
-                tma_load_2d(s.b[st], &tmap_x, &s.full_b[st], kb * BK, (int)m0);
-                ++issued;
             }
             // drain: never leave the CTA with a bulk copy still writing smem
-            for (int kb = issued - STAGES < 0 ? 0 : issued - STAGES; kb < issued; ++kb)
-                mbar_wait(&s.full_b[kb % STAGES], (uint32_t)(kb / STAGES) & 1u, a.wait_limit_ns, nullptr);
+            // (after an abort the dequant arrivals may be missing: the bounded
+            // wait then outlasts the copies by far)
+            for (int q = it - STAGES < 0 ? 0 : it - STAGES; q < it; ++q)
+                mbar_wait(&s.full[q % STAGES], (uint32_t)(q / STAGES) & 1u, a.wait_limit_ns, nullptr);
         }
     } else if (warp == 1) {
         // ------------------------------------------------ MMA issuer
         if (lane == 0) {
-            for (int kb = 0; kb < nkb; ++kb) {
-                const int st = kb % STAGES;
-                const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-                if (!mbar_wait(&s.full_b[st], ph, a.wait_limit_ns, abort_flag) ||
-                    !mbar_wait(&s.full_a[st], ph, a.wait_limit_ns, abort_flag)) {
+            int it = 0, ti = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++ti) {
+                const int buf = ti & 1;
+                const uint32_t dcol = tmem_d + (uint32_t)(buf * BN);
+                if (ti >= 2 && !mbar_wait(&s.accum_empty[buf], (uint32_t)((ti >> 1) - 1) & 1u, a.wait_limit_ns,
+                                          abort_flag)) {
                     raise_abort(s, a.status);
                     break;
                 }
                 tc_fence_after();
-                const uint64_t ad = sw128_desc(smem_u32(s.a[st]));
-                const uint64_t bd = sw128_desc(smem_u32(s.b[st]));
+                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                    const int st = it % STAGES;
+                    const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
+                    if (!wait_phase(&s.full[st], ph, a.wait_limit_ns, abort_flag)) {
+                        raise_abort(s, a.status);
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint64_t ad = sw128_desc(smem_u32(s.a[it % W_SLOTS]));
+                    const uint64_t bd = sw128_desc(smem_u32(s.b[st]));
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along k per step
-                    mma_f16(tmem_d, ad + 2 * kk, bd + 2 * kk, (kb | kk) != 0 ? 1u : 0u);
-                mma_commit(&s.empty[st]);
+                    for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along k per step
+                        mma_f16(dcol, ad + 2 * kk, bd + 2 * kk, (kb | kk) != 0 ? 1u : 0u);
+                    mma_commit(&s.empty[st]);
+                }
+                if (ok) mma_commit(&s.accum_full[buf]);
             }
-            // always signal the epilogue, and do not free tensor memory under
-            // running MMAs: wait for this commit before leaving
-            mma_commit(&s.accum_full);
-            mbar_wait(&s.accum_full, 0, a.wait_limit_ns, nullptr);
+            // do not free tensor memory under running MMAs: wait for them
+            mma_commit(&s.done);
+            mbar_wait(&s.done, 0, a.wait_limit_ns, nullptr);
         }
         __syncwarp();
-    } else {
+    } else if (warp < 2 + NUM_DQ_WARPS) {
         // ------------------------------------------------ dequant producers
         const int d = threadIdx.x - 64;  // 0..255
         const int r = d >> 1;            // tile row 0..127
         const int half_id = d & 1;       // which 32-wide half of the stage
-        const int64_t row = n0 + r;
-        const bool valid = row < a.n;
-        UnitRaw cur{}, nxt{};
-        if (valid) load_unit<BITS, KIND>(a, row, 32 * half_id, nxt);
+        int it = 0;
         bool ok = true;
-        for (int kb = 0; kb < nkb; ++kb) {
-            cur = nxt;
-            if (valid && kb + 1 < nkb) load_unit<BITS, KIND>(a, row, (int64_t)(kb + 1) * BK + 32 * half_id, nxt);
-            const int st = kb % STAGES;
-            const uint32_t ph = (uint32_t)(kb / STAGES) & 1u;
-            if (!mbar_wait(&s.empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag)) {
-                raise_abort(s, a.status);
-                ok = false;
-            }
-            if (__any_sync(0xffffffffu, !ok)) break;
-            __half2 v[16];
-            if (valid) {
-                dequant_unit<BITS, KIND>(cur, v);
-            } else {
+        for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+            const int64_t row = (int64_t)(t / mt) * BM + r;
+            const bool valid = row < a.n;
+            constexpr int kAhead = 4;
+            // pre[j] holds the codes of stage kb with kb % kAhead == j: the loop
+            // is unrolled by kAhead so that no in-flight load is ever copied
+            // between registers (a copy would wait for the load)
+            UnitRaw pre[kAhead];
 #pragma unroll
-                for (int p = 0; p < 16; ++p) v[p] = __float2half2_rn(0.0f);
-            }
-            uint8_t *tile = s.a[st] + (r >> 3) * 1024 + (r & 7) * 128;
+            for (int i = 0; i < kAhead; ++i)
+                if (valid && i < nkb) load_unit<BITS, KIND>(a, row, (int64_t)i * BK + 32 * half_id, pre[i]);
+            for (int kb0 = 0; kb0 < nkb && ok; kb0 += kAhead) {
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int chunk = 4 * half_id + q;
-                *reinterpret_cast<uint4 *>(tile + ((chunk ^ (r & 7)) << 4)) =
-                    make_uint4(h22u(v[4 * q]), h22u(v[4 * q + 1]), h22u(v[4 * q + 2]), h22u(v[4 * q + 3]));
+                for (int j = 0; j < kAhead; ++j) {
+                    const int kb = kb0 + j;
+                    if (kb >= nkb) break;
+                    // stage q = it: its barriers are slot q % STAGES; its W slot
+                    // q % W_SLOTS is free once the MMAs of stage q - W_SLOTS are done
+                    const int q = it++;
+                    const int st = q % STAGES;
+                    const int qf = q - W_SLOTS;
+                    bool free_ok = true;
+                    if (qf >= 0)
+                        free_ok = wait_phase(&s.empty[qf % STAGES], (uint32_t)(qf / STAGES) & 1u, a.wait_limit_ns,
+                                             abort_flag);
+                    if (!free_ok) {
+                        raise_abort(s, a.status);
+                        ok = false;
+                    }
+                    if (__any_sync(0xffffffffu, !ok)) {
+                        ok = false;
+                        break;
+                    }
+                    __half2 v[16];
+                    if (valid) {
+                        dequant_unit<BITS, KIND>(pre[j], v);
+                    } else {
+#pragma unroll
+                        for (int p = 0; p < 16; ++p) v[p] = __float2half2_rn(0.0f);
+                    }
+                    if (valid && kb + kAhead < nkb)
+                        load_unit<BITS, KIND>(a, row, (int64_t)(kb + kAhead) * BK + 32 * half_id, pre[j]);
+                    uint8_t *tile = s.a[q % W_SLOTS] + (r >> 3) * 1024 + (r & 7) * 128;
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) {
+                        const int chunk = 4 * half_id + q;
+                        *reinterpret_cast<uint4 *>(tile + ((chunk ^ (r & 7)) << 4)) =
+                            make_uint4(h22u(v[4 * q]), h22u(v[4 * q + 1]), h22u(v[4 * q + 2]), h22u(v[4 * q + 3]));
+                    }
+                    fence_proxy_async_smem();  // generic-proxy writes -> visible to the tensor core
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(&s.full[st]);
+                }
             }
-            fence_proxy_async_smem();  // generic-proxy writes -> visible to the tensor core
-            __syncwarp();
-            if (lane == 0) mbar_arrive(&s.full_a[st]);
         }
+    } else {
         // ------------------------------------------------ epilogue
-        const bool have = mbar_wait(&s.accum_full, 0, a.wait_limit_ns, nullptr);
-        if (!have) raise_abort(s, a.status);
-        tc_fence_after();
-        // tcgen05.ld is warp-collective: decide for the whole warp at once
-        if (__all_sync(0xffffffffu, have && !*abort_flag)) {
-            const int quarter = warp & 3;          // TMEM lanes this warp may read
-            const int col0 = (warp < 6) ? 0 : 64;  // two warps per lane quarter
-            const int64_t n = n0 + 32 * quarter + lane;
-#pragma unroll
-            for (int cb = 0; cb < 2; ++cb) {
+        const int quarter = warp & 3;  // the TMEM lanes (W rows) this warp may read
+        int ti = 0;
+        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++ti) {
+            const int buf = ti & 1;
+            const bool have = mbar_wait(&s.accum_full[buf], (uint32_t)(ti >> 1) & 1u, a.wait_limit_ns, abort_flag);
+            if (!have) raise_abort(s, a.status);
+            tc_fence_after();
+            // tcgen05.ld is warp-collective: decide for the whole warp at once
+            if (!__all_sync(0xffffffffu, have && !*abort_flag)) break;
+            const int64_t n = (int64_t)(t / mt) * BM + 32 * quarter + lane;
+            const int64_t m0 = (int64_t)(t % mt) * BN;
+#pragma unroll 1
+            for (int c = 0; c < BN; c += 32) {
                 uint32_t rv[32];
-                const int c = col0 + 32 * cb;
-                tmem_ld32(tmem_d + ((uint32_t)(32 * quarter) << 16) + (uint32_t)c, rv);
+                tmem_ld32(tmem_d + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * BN + c), rv);
                 if (n < a.n) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j) {
@@ -358,6 +444,10 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
                     }
                 }
             }
+            // this warp's rows of the accumulator are read: free it for tile ti + 2
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.accum_empty[buf]);
         }
     }
     tc_fence_before();
@@ -370,11 +460,12 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
 }
 
 template <int BITS, int KIND>
-cudaError_t launch_t(const CUtensorMap &map, const GemmArgs &a, cudaStream_t st) {
+cudaError_t launch_t(const CUtensorMap &map, const GemmArgs &a, int num_sms, cudaStream_t st) {
     auto kern = gemm_kernel<BITS, KIND>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
     if (e != cudaSuccess) return e;
-    dim3 grid((unsigned)((a.m + BN - 1) / BN), (unsigned)((a.n + BM - 1) / BM));
+    const int64_t tiles = ((a.m + BN - 1) / BN) * ((a.n + BM - 1) / BM);
+    const unsigned grid = (unsigned)std::min<int64_t>(tiles, num_sms);
     kern<<<grid, THREADS, kSmemBytes, st>>>(map, a);
     return cudaGetLastError();
 }
@@ -395,7 +486,6 @@ EncodeTiledFn encode_fn() {
 }
 
 cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st) {
-    (void)num_sms;
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
     CUtensorMap map;
@@ -407,9 +497,9 @@ cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st) {
                      CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                      CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
     if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    if (a.bits == 4) return launch_t<4, 0>(map, a, st);
-    if (a.kind == 1) return launch_t<3, 1>(map, a, st);
-    return launch_t<3, 0>(map, a, st);
+    if (a.bits == 4) return launch_t<4, 0>(map, a, num_sms, st);
+    if (a.kind == 1) return launch_t<3, 1>(map, a, num_sms, st);
+    return launch_t<3, 0>(map, a, num_sms, st);
 }
 
 }  // namespace qx
