@@ -92,21 +92,30 @@ __device__ __forceinline__ void lookup4(const Table8 &t, uint32_t sel, __half2 &
     p23 = u2h2(prmt(l, h, 0x7362u));
 }
 
+// x >> n (n = 1..31) computed as the high word of x * 2^(32-n): an integer
+// multiply-add, which runs on the FMA pipe.  The 3-bit unpack is bound by the
+// (half-rate) integer ALU pipe, which its byte permutes already fill.
+__device__ __forceinline__ uint32_t shr_fma(uint32_t x, int n) {
+    uint32_t d;
+    asm("mul.hi.u32 %0, %1, %2;" : "=r"(d) : "r"(x), "r"(1u << (32 - n)));
+    return d;
+}
+
 // One triple (A, B, C) codes 32 consecutive k.  Returns 16 half2 = T[code]
 // for k = 0..31 of the triple in natural order.
 __device__ __forceinline__ void lookup_triple(const Table8 &t, uint32_t A, uint32_t B, uint32_t C,
                                               __half2 (&o)[16]) {
     const uint32_t m = 0x77777777u;
     uint32_t a = A & m, b = B & m, c = C & m;
-    uint32_t e = ((A >> 3) & 0x11111111u) | ((B >> 2) & 0x22222222u) | ((C >> 1) & 0x44444444u);
+    uint32_t e = (shr_fma(A, 3) & 0x11111111u) | (shr_fma(B, 2) & 0x22222222u) | (shr_fma(C, 1) & 0x44444444u);
     lookup4(t, a, o[0], o[1]);
-    lookup4(t, a >> 16, o[2], o[3]);
+    lookup4(t, shr_fma(a, 16), o[2], o[3]);
     lookup4(t, b, o[4], o[5]);
-    lookup4(t, b >> 16, o[6], o[7]);
+    lookup4(t, shr_fma(b, 16), o[6], o[7]);
     lookup4(t, c, o[8], o[9]);
-    lookup4(t, c >> 16, o[10], o[11]);
+    lookup4(t, shr_fma(c, 16), o[10], o[11]);
     lookup4(t, e, o[12], o[13]);
-    lookup4(t, e >> 16, o[14], o[15]);
+    lookup4(t, shr_fma(e, 16), o[14], o[15]);
 }
 
 // Table of the uniform 3-bit grid offsets (j - z), j = 0..7, exact in fp16.

@@ -219,15 +219,26 @@ __device__ __forceinline__ void stage_coords(const Header &h, int count, int q, 
 }
 
 // Issue the TMA copies of stage q into its ring slot (one thread).
+// Geometry a stage copy needs, from the shared-memory table or straight from
+// the kernel parameters (the first copy is issued before the table exists).
+struct Geom {
+    int K, log2g, nlb, G, n, zbytes;
+    const __half *scales;
+    const uint8_t *zeros;
+};
+
+__device__ __forceinline__ Geom geom_of(const MatS &M) {
+    return Geom{M.K, M.log2g, M.nlb, M.G, M.n, M.zbytes, M.scales, M.zeros};
+}
+
+__device__ __forceinline__ Geom geom_of(const GemvMat &M) {
+    return Geom{(int)M.k, M.log2g, M.nlb, M.G, (int)M.n, M.zbytes, M.scales, M.zeros};
+}
+
+// Issue the TMA copies of one stage (matrix m, matrix-local row block rb,
+// slice ks) into ring slot `slot` (one thread).
 template <int BITS, int KIND>
-__device__ void issue_stage(const GemvMulti &a, Header &h, uint32_t ring_s, int q) {
-    int m, rb, ks;
-    stage_coords(h, a.count, q, m, rb, ks);
-    const MatS &M = h.mats[m];
-    const int ring = a.ring;
-    const int slot = q % ring;
-    const uint32_t bar = smem_u32(&h.full[slot]);
-    const uint32_t base = ring_s + (uint32_t)(slot * a.stage_bytes);
+__device__ void issue_geom(const GemvMulti &a, const Geom &M, int m, uint32_t bar, uint32_t base, int rb, int ks) {
     const int row0 = rb * kRows;
     uint32_t tx = 0;
     int ncb = 0;
@@ -267,6 +278,21 @@ __device__ void issue_stage(const GemvMulti &a, Header &h, uint32_t ring_s, int 
         if (sb) prefetch_l2_bulk(M.scales + (int64_t)row0 * M.G, sb);
         if (zb) prefetch_l2_bulk(M.zeros + (int64_t)row0 * M.zbytes, zb);
     }
+}
+
+template <int BITS, int KIND>
+__device__ __forceinline__ void issue_at(const GemvMulti &a, Header &h, uint32_t ring_s, int m, int rb, int ks,
+                                         int slot) {
+    issue_geom<BITS, KIND>(a, geom_of(h.mats[m]), m, smem_u32(&h.full[slot]),
+                           ring_s + (uint32_t)(slot * a.stage_bytes), rb, ks);
+}
+
+// Issue stage q (set-up path: coordinates from the stage number).
+template <int BITS, int KIND>
+__device__ void issue_stage(const GemvMulti &a, Header &h, uint32_t ring_s, int q) {
+    int m, rb, ks;
+    stage_coords(h, a.count, q, m, rb, ks);
+    issue_at<BITS, KIND>(a, h, ring_s, m, rb, ks, q % a.ring);
 }
 
 // Scales and zero-points of one lane's 256-weight part: up to eight fp16
@@ -456,6 +482,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         for (int i = 0; i < ring; ++i) mbar_init(smem_u32(&h.full[i]), 1);
         h.abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        // the CTA's first stage straight from the parameters, so that its
+        // data is on the way while the rest of the set-up runs
+        const int lo = a.cta_rb[blockIdx.x], hi = a.cta_rb[blockIdx.x + 1];
+        if (lo < hi) {
+            int m = 0;
+            while (m + 1 < count && lo >= a.mat[m].rb_off + a.mat[m].nrb) ++m;
+            issue_geom<BITS, KIND>(a, geom_of(a.mat[m]), m, smem_u32(&h.full[0]), ring_s, lo - a.mat[m].rb_off, 0);
+        }
     }
     if (threadIdx.x >= 96 && threadIdx.x < 96 + kMaxRing) h.rel[threadIdx.x - 96] = 0;
     if (threadIdx.x >= 128 && threadIdx.x < 128 + kMaxRbSlots) {
@@ -493,7 +527,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             h.issued = (uint32_t)min(a.initial, q);
         }
         __syncwarp();
-        if (lane < min(a.initial, q)) issue_stage<BITS, KIND>(a, h, ring_s, lane);
+        if (lane >= 1 && lane < min(a.initial, q)) issue_stage<BITS, KIND>(a, h, ring_s, lane);
     }
     __syncthreads();
     // let the next kernel in the stream start streaming its own weights; it
@@ -512,6 +546,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     advance_by(h, count, c, grp);
     Cursor cn = c;
     advance_by(h, count, cn, kGroups);
+    // the stage that refills this warp's current slot, q + ring: ring is a
+    // multiple of kGroups, so it is one of this warp's own later stages
+    Cursor cr = c;
+    advance_by(h, count, cr, ring);
     // uniform metadata of this warp's stages, loaded one stage ahead
     Meta cur{}, nxt{};
     if (KIND == 0 && c.m < count)
@@ -552,7 +590,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         // the warp groups run independently: the slot's previous block must
         // have been summed before this warp overwrites its partials
         bool okf = true;
-        if (lane == 0) okf = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
+        if (lane == 0 && *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) != use)
+            okf = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
         if (!__shfl_sync(0xffffffffu, okf, 0)) return false;
         float *rp = red + (size_t)rs * (kWarps * NB * 32);
 #pragma unroll
@@ -569,26 +608,31 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         if (fin) {
             const int q0 = M.q0 + rbl * M.nks;  // the block's first stage
             const int row = (M.rb0 + rbl) * kRows + r;
-            if (row < M.n) {
+            float v[NB];
 #pragma unroll
-                for (int b = 0; b < NB; ++b) {
-                    float v = 0.0f;
-                    for (int j = 0; j < ng; ++j) {
-                        const int g = (q0 + j) % kGroups;
+            for (int b = 0; b < NB; ++b) {
+                v[b] = 0.0f;
+                for (int j = 0; j < ng; ++j) {
+                    const int g = (q0 + j) % kGroups;
 #pragma unroll
-                        for (int p = 0; p < kGroupWarps; ++p) v += rp[((g * kGroupWarps + p) * NB + b) * 32 + r];
-                    }
-                    if (a.y_f32)
-                        reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v;
-                    else
-                        reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v);
+                    for (int p = 0; p < kGroupWarps; ++p) v[b] += rp[((g * kGroupWarps + p) * NB + b) * 32 + r];
                 }
             }
+            // free the slot first: the fence must not wait for the y stores
             __syncwarp();
             if (lane == 0) {
                 h.cnt[rs] = 0;
                 __threadfence_block();
                 *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
+            }
+            if (row < M.n) {
+#pragma unroll
+                for (int b = 0; b < NB; ++b) {
+                    if (a.y_f32)
+                        reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v[b];
+                    else
+                        reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v[b]);
+                }
             }
         }
         return true;
@@ -663,8 +707,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 h.rel[slot] = 0;
                 __threadfence_block();
                 asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                if (q + ring < nst && !*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) {
-                    issue_stage<BITS, KIND>(a, h, ring_s, q + ring);
+                if (cr.m < count && !*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) {
+                    issue_at<BITS, KIND>(a, h, ring_s, cr.m, h.mats[cr.m].rb0 + cr.rbl, cr.ks, slot);
                     atomicMax(&h.issued, (uint32_t)(q + ring + 1));
                 }
             }
@@ -672,6 +716,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         if (KIND == 0) cur = nxt;
         c = cn;
         advance_by(h, count, cn, kGroups);
+        advance_by(h, count, cr, kGroups);
         slot += kGroups;
         if (slot >= ring) {
             slot -= ring;
