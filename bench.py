@@ -4,13 +4,17 @@ Workload (default): one Llama-7B-shaped decoder layer (q, k, v, o 4096x4096;
 gate, up 11008x4096; down 4096x11008), Student-t(4) weights with sigma 0.01
 (q, k), 0.02 (v, o), 0.04 (MLP), quantized to 3-bit non-uniform codes with a
 per-group 8-entry fp16 LUT (Lloyd-Max, group 128 along k).  One step = one
-decode token through all seven matrices (seven qx_gemv calls at batch 1).
-Metric: HBM GB/s of the packed weights (+ x, y) per step.
+decode token through all seven matrices: the decode dependency chain
+q,k,v | o | gate,up | down as four qx_gemv_multi launches at batch 1 (PDL,
+one CUDA graph).  Metric: HBM GB/s of the packed weights (+ x, y) per step.
 
 Also reported on the same line: the prefill GEMM (M = 2048 tokens against the
-11008x4096 and 4096x11008 3-bit LUT matrices, tcgen05), the roofline of the
-dominant kernel, the CPU oracle as a baseline, SM clocks during the timed
-region and an end-to-end number with host buffers.
+11008x4096 and 4096x11008 3-bit LUT matrices, tcgen05), the same layer with
+4-bit uniform g128 and 3-bit uniform g64 weights at batch 1, 4 and 16, the
+mixed-recipe LLaVA-shaped stack (32 language layers decoded, 24 vision layers
+prefilled), the roofline of the dominant kernel, the CPU oracle as a
+baseline, SM clocks during the timed region and an end-to-end number with
+host buffers.
 
 Launch: python bench.py [--gpus N --steps K --warmup W] [--impl reference];
 for N > 1 under torch.distributed.run (one rank per GPU, weak scaling: every
@@ -407,6 +411,12 @@ def run_ours(args):
 
     gemm = run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
     del layers, graphs
+    extra = {}
+    if not args.skip_configs:
+        torch.cuda.empty_cache()
+        extra["config3"] = run_config3(qx, torch, dev, stream, l2)
+        torch.cuda.empty_cache()
+        extra["config5"] = run_config5(qx, torch, dev, stream)
 
     if rank == 0:
         cpu = run_cpu_baseline() if not args.skip_cpu_baseline else None
@@ -431,6 +441,7 @@ def run_ours(args):
                          "launch_us": launch_us, "bytes_per_launch": step_bytes / len(CHAIN),
                          "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
             "gemm": gemm,
+            **extra,
             "cpu_baseline": cpu,
             "clocks": clocks,
             "e2e": {"value": e2e_value, "unit": "GB/s", "ms_per_step": e2e_ms,
@@ -483,6 +494,132 @@ def run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src):
                          "kernel": "gemm_kernel<3,LUT>", "traffic": _traffic("qx_gemm.cu", "gemm_L3g128_m2048")}}
 
 
+def _chain_graph(qx, torch, stream, layers, chain, outs, pdl=True):
+    """One CUDA graph of the decode chain over every layer copy in `layers`."""
+    def body():
+        for L in layers:
+            for names, x in chain:
+                qx.gemv_multi([L[nm] for nm in names], [x] * len(names), outs=[outs[nm] for nm in names], pdl=pdl)
+
+    with torch.cuda.stream(stream):
+        body()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        body()
+    return g
+
+
+def _time_graph(torch, stream, g, reps):
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            g.replay()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1) / reps  # ms per replay
+
+
+def run_config3(qx, torch, dev, stream, l2):
+    """Llama-7B layer, 4-bit uniform g128 and 3-bit uniform g64, batch 1 / 4 / 16."""
+    import synth
+
+    out = {}
+    for bits, g in ((4, 128), (3, 64)):
+        recipe = qx.Recipe(bits, g, qx.UNIFORM)
+        base = dict(_quantize_layer(qx, torch, dev, LAYER, recipe))
+        layer_bytes = sum(P.nbytes() for P in base.values())
+        copies = max(2, math.ceil(4 * l2 / layer_bytes))
+        layers = [base] + [{nm: _clone(qx, P) for nm, P in base.items()} for _ in range(copies - 1)]
+        for batch in (1, 4, 16):
+            xs = [synth.activations_torch(batch, k, seed=batch, stream=60 + i, device=dev)
+                  for i, k in enumerate((4096, 4096, 4096, 11008))]
+            ys = {nm: torch.empty((batch, n), dtype=torch.float16, device=dev) for nm, n, *_ in LAYER}
+            chain = [(["q_proj", "k_proj", "v_proj"], xs[0]), (["o_proj"], xs[1]),
+                     (["gate_proj", "up_proj"], xs[2]), (["down_proj"], xs[3])]
+            gr = _chain_graph(qx, torch, stream, layers, chain, ys)
+            ms = _time_graph(torch, stream, gr, 20) / copies
+            del gr
+            io = sum(x.numel() * 2 for x in xs) + sum(y.numel() * 2 for y in ys.values())
+            out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}"] = {
+                "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
+                "weight_bytes": layer_bytes, "launches_per_layer": 4 * ((batch + 3) // 4)}
+        del layers, base
+    return out
+
+
+LLAVA_LANG = [  # Q/K 3-bit LUT g128; V/O and the MLP 4-bit uniform g64
+    ("q_proj", 4096, 4096, 0.01, 0, (3, 128, 1)), ("k_proj", 4096, 4096, 0.01, 1, (3, 128, 1)),
+    ("v_proj", 4096, 4096, 0.02, 2, (4, 64, 0)), ("o_proj", 4096, 4096, 0.02, 3, (4, 64, 0)),
+    ("gate_proj", 11008, 4096, 0.04, 4, (4, 64, 0)), ("up_proj", 11008, 4096, 0.04, 5, (4, 64, 0)),
+    ("down_proj", 4096, 11008, 0.04, 6, (4, 64, 0)),
+]
+LLAVA_VISION = [  # CLIP ViT-L/14: hidden 1024, MLP 4096; 4-bit uniform g128
+    ("q_proj", 1024, 1024, 0.02, 10), ("k_proj", 1024, 1024, 0.02, 11), ("v_proj", 1024, 1024, 0.02, 12),
+    ("o_proj", 1024, 1024, 0.02, 13), ("fc1", 4096, 1024, 0.04, 14), ("fc2", 1024, 4096, 0.04, 15),
+]
+
+
+def run_config5(qx, torch, dev, stream):
+    """LLaVA-v1.6-7B-shaped stack with the mixed per-layer recipe.
+
+    Decode: one token through the seven GEMVs of each of 32 language layers
+    (q,k | v | o | gate,up | down: launches group matrices that share the
+    activations and the recipe), PDL, one CUDA graph.  Prefill: 576 image
+    tokens through the six GEMMs of each of 24 vision layers.
+    """
+    import synth
+
+    base = {}
+    for nm, n, k, sigma, sid, (bits, g, kind) in LLAVA_LANG:
+        W = synth.student_t_weights_torch(n, k, sigma, seed=5, stream=sid, device=dev)
+        base[nm] = qx.quantize(W, qx.Recipe(bits, g, kind))
+        del W
+    lang = [base] + [{nm: _clone(qx, P) for nm, P in base.items()} for _ in range(31)]
+    lang_bytes = 32 * sum(P.nbytes() for P in base.values())
+    xs = {k: synth.activations_torch(1, k, seed=5, stream=80 + i, device=dev) for i, k in enumerate((4096, 11008))}
+    xa, xo, xm = (synth.activations_torch(1, 4096, seed=5, stream=90 + i, device=dev) for i in range(3))
+    ys = {nm: torch.empty((1, n), dtype=torch.float16, device=dev) for nm, n, *_ in LLAVA_LANG}
+    chain = [(["q_proj", "k_proj"], xa), (["v_proj"], xa), (["o_proj"], xo),
+             (["gate_proj", "up_proj"], xm), (["down_proj"], xs[11008])]
+    gr = _chain_graph(qx, torch, stream, lang, chain, ys)
+    dec_ms = _time_graph(torch, stream, gr, 10)
+    del gr, lang
+
+    vbase = dict(_quantize_layer(qx, torch, dev, LLAVA_VISION, qx.Recipe(4, 128, qx.UNIFORM), seed=5))
+    vis = [vbase] + [{nm: _clone(qx, P) for nm, P in vbase.items()} for _ in range(23)]
+    M = 576
+    X1 = synth.activations_torch(M, 1024, seed=5, stream=95, device=dev)
+    X4 = synth.activations_torch(M, 4096, seed=5, stream=96, device=dev)
+    Ys = {nm: torch.empty((M, n), dtype=torch.float16, device=dev) for nm, n, *_ in LLAVA_VISION}
+
+    def vision_pass():
+        for L in vis:
+            for nm, n, k, *_ in LLAVA_VISION:
+                qx.gemm(L[nm], X4 if k == 4096 else X1, out=Ys[nm])
+
+    with torch.cuda.stream(stream):
+        vision_pass()
+    torch.cuda.synchronize()
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("vision gemm reported a device error")
+    gv = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(gv, stream=stream):
+        vision_pass()
+    pre_ms = _time_graph(torch, stream, gv, 10)
+    flops = 24 * sum(2.0 * M * n * k for _, n, k, *_ in LLAVA_VISION)
+    del gv, vis
+    return {"workload": "llava16_7b_mixed_recipe",
+            "recipe": {"language": "q,k L3g128; v,o,gate,up,down U4g64", "vision": "all U4g128"},
+            "decode_token_us": dec_ms * 1e3, "decode_GBps": lang_bytes / (dec_ms * 1e-3) / 1e9,
+            "decode_launches": 32 * len(chain), "language_weight_bytes": lang_bytes,
+            "vision_prefill_us": pre_ms * 1e3, "vision_prefill_TFLOPs": flops / (pre_ms * 1e-3) / 1e12,
+            "vision_tokens": M, "vision_gemm_launches": 24 * len(LLAVA_VISION)}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -491,6 +628,7 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--skip-gemm", action="store_true")
     ap.add_argument("--skip-cpu-baseline", action="store_true")
+    ap.add_argument("--skip-configs", action="store_true", help="skip the config-3 / config-5 sections")
     ap.add_argument("--cpu-baseline-child", type=float, default=None, help=argparse.SUPPRESS)
     args = ap.parse_args()
     if args.cpu_baseline_child is not None:

@@ -258,3 +258,73 @@ def test_gemv_ring_wraps(qx, case, batch):
     qx.gemv(P, torch.from_numpy(x).cuda(), out=y)
     assert qx.device_status() == 0
     _check_matmul(y.cpu().numpy(), oracle.gemv(ref, rec, x, k), x, oracle.dequant(ref, rec, k))
+
+
+# Mixed per-layer recipe (paper Sections 2.1 and 2.3): each matrix carries its
+# own recipe.  A two-layer stack shaped like the LLaVA language layers (Q/K
+# 3-bit LUT g128, V/O and MLP 4-bit uniform g64) is decoded through the
+# launch sequence q,k | v | o | gate,up | down captured in one CUDA graph
+# with programmatic dependent launch, and a vision-shaped set of matrices
+# (4-bit uniform g128) is prefilled with qx_gemm.
+STACK = [("q", 256, 256, (3, 128, 1)), ("k", 256, 256, (3, 128, 1)), ("v", 256, 256, (4, 64, 0)),
+         ("o", 256, 256, (4, 64, 0)), ("gate", 640, 256, (4, 64, 0)), ("up", 640, 256, (4, 64, 0)),
+         ("down", 256, 640, (4, 64, 0))]
+
+
+@pytest.mark.gpu
+def test_mixed_recipe_stack_decode_graph(qx):
+    layers = []
+    for li in range(2):
+        L = {}
+        for i, (nm, n, k, (bits, g, kind)) in enumerate(STACK):
+            W = _weights(n, k, seed=300 + 10 * li + i)
+            L[nm] = (qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind)),
+                     oracle.quantize(W, _orecipe(bits, g, kind)), (bits, g, kind))
+        layers.append(L)
+    xa = synth.activations(1, 256, seed=1, stream=41)
+    xo = synth.activations(1, 256, seed=1, stream=42)
+    xm = synth.activations(1, 256, seed=1, stream=43)
+    xd = synth.activations(1, 640, seed=1, stream=44)
+    dx = {nm: torch.from_numpy(x).cuda() for nm, x in (("a", xa), ("o", xo), ("m", xm), ("d", xd))}
+    ys = [{nm: torch.empty((1, n), dtype=torch.float32, device="cuda") for nm, n, _, _ in STACK} for _ in layers]
+    chain = [(["q", "k"], "a"), (["v"], "a"), (["o"], "o"), (["gate", "up"], "m"), (["down"], "d")]
+    s = torch.cuda.Stream()
+
+    def body():
+        for L, Y in zip(layers, ys):
+            for names, xn in chain:
+                qx.gemv_multi([L[nm][0] for nm in names], [dx[xn]] * len(names), outs=[Y[nm] for nm in names],
+                              pdl=True)
+
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        body()
+    for Y in ys:
+        for y in Y.values():
+            y.fill_(float("nan"))
+    g.replay()
+    torch.cuda.synchronize()
+    assert qx.device_status() == 0
+    xs = {"a": xa, "o": xo, "m": xm, "d": xd}
+    for L, Y in zip(layers, ys):
+        for names, xn in chain:
+            for nm in names:
+                P, ref, (bits, g_, kind) = L[nm]
+                k = P.k
+                rec = _orecipe(bits, g_, kind)
+                _check_matmul(Y[nm].cpu().numpy(), oracle.gemv(ref, rec, xs[xn], k), xs[xn], oracle.dequant(ref, rec, k))
+
+
+@pytest.mark.gpu
+def test_mixed_recipe_vision_prefill(qx):
+    M = 300  # two token tiles, ragged
+    for i, (n, k) in enumerate(((256, 256), (1024, 256), (256, 1024))):
+        W = _weights(n, k, seed=400 + i)
+        P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(4, 128, 0))
+        ref = oracle.quantize(W, _orecipe(4, 128, 0))
+        X = synth.activations(M, k, seed=4, stream=50 + i)
+        Y = qx.gemm(P, torch.from_numpy(X).cuda())
+        assert qx.device_status() == 0
+        rec = _orecipe(4, 128, 0)
+        _check_matmul(Y.cpu().numpy(), oracle.gemm(ref, rec, X, k), X, oracle.dequant(ref, rec, k))
