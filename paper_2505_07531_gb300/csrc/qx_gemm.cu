@@ -41,11 +41,14 @@ constexpr int BK = 64;   // k per stage (one 128-byte swizzle row of fp16)
 // dequantization fall behind).
 constexpr int STAGES = 4;
 constexpr int W_SLOTS = 4;
+static_assert(W_SLOTS <= STAGES, "a W slot's release is read from the stage barrier W_SLOTS back");
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = BN * BK * 2;
 constexpr int NUM_DQ_WARPS = 8;
 constexpr int NUM_EPI_WARPS = 4;
-constexpr int THREADS = 64 + (NUM_DQ_WARPS + NUM_EPI_WARPS) * 32;
+constexpr int PK_WARP = 2 + NUM_DQ_WARPS + NUM_EPI_WARPS;  // packed-code producer
+constexpr int THREADS = (PK_WARP + 1) * 32;
+constexpr int kMaxPSlots = 8;
 constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
 
 struct SmemLayout {
@@ -57,12 +60,15 @@ struct SmemLayout {
     uint64_t empty[STAGES];  // tcgen05.commit of the stage's MMAs
     uint64_t accum_full[2];
     uint64_t accum_empty[2];
+    uint64_t pfull[kMaxPSlots];   // a packed superblock has landed (TMA bytes)
+    uint64_t pempty[kMaxPSlots];  // the 8 dequant warps have read it
     uint64_t done;
     uint32_t tmem_base;
     uint32_t abort_flag;
 };
 
-constexpr size_t kSmemBytes = sizeof(SmemLayout) + 1024;
+// The packed-code ring follows the layout (its size depends on the recipe).
+constexpr size_t kLayoutBytes = (sizeof(SmemLayout) + 1023) / 1024 * 1024;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -143,6 +149,34 @@ __device__ __forceinline__ void tma_load_2d(void *dst, const CUtensorMap *map, u
         : "memory");
 }
 
+__device__ __forceinline__ void tma_load_3d(uint32_t dst, const CUtensorMap *map, uint64_t *bar, int x, int y, int z) {
+    asm volatile(
+        "cp.async.bulk.tensor.3d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4, %5}], "
+        "[%2];" ::"r"(dst),
+        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y), "r"(z)
+        : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d_s(uint32_t dst, const CUtensorMap *map, uint64_t *bar, int x, int y) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%3, %4}], [%2];" ::
+            "r"(dst),
+        "l"(map), "r"(smem_u32(bar)), "r"(x), "r"(y)
+        : "memory");
+}
+
+__device__ __forceinline__ uint32_t lds32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds128(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
@@ -206,28 +240,34 @@ struct UnitRaw {
     __half scale;    // scale (uniform)
 };
 
-template <int BITS, int KIND>
-__device__ __forceinline__ void load_unit(const GemmArgs &a, int64_t row, int64_t k0, UnitRaw &u) {
-    const int grp = (int)(k0 >> a.log2g);
-    if (BITS == 4) {
-        const uint4 c = ldg_nc_v4(a.codes + row * (a.k / 2) + (k0 >> 1));
-        u.w[0] = c.x;
-        u.w[1] = c.y;
-        u.w[2] = c.z;
-        u.w[3] = c.w;
-    } else {
-        const uint8_t *rc = a.codes + row * (3 * a.k / 8) + 16 * (k0 >> 7) + 4 * ((k0 & 127) >> 5);
-        const int64_t plane = a.k >> 3;
-        u.w[0] = __ldg(reinterpret_cast<const unsigned int *>(rc));
-        u.w[1] = __ldg(reinterpret_cast<const unsigned int *>(rc + plane));
-        u.w[2] = __ldg(reinterpret_cast<const unsigned int *>(rc + 2 * plane));
-        u.w[3] = 0;
-    }
-    if (KIND == 1) {
-        u.lut = ldg_nc_v4(a.luts + (row * a.G + grp) * 8);
-    } else {
+// Uniform metadata of one unit, from global memory (read ahead of use).
+template <int KIND>
+__device__ __forceinline__ void load_meta(const GemmArgs &a, int64_t row, int64_t k0, UnitRaw &u) {
+    if (KIND == 0) {
+        const int grp = (int)(k0 >> a.log2g);
         u.zero = zero_nibble(a.zeros + row * a.zbytes, grp);
         u.scale = a.scales[row * a.G + grp];
+    }
+}
+
+// Codes (and the LUT) of one unit from the packed-code ring: slot `ps` holds
+// one superblock of 128 rows -- 3-bit: [row][plane][16 bytes] then the LUTs
+// [row][lut_box bytes]; 4-bit: [row][64 bytes].  u = unit in the superblock.
+template <int BITS, int KIND>
+__device__ __forceinline__ void read_codes(uint32_t ps, int r, int u, int gl, int lut_box, UnitRaw &w) {
+    if (BITS == 4) {
+        const uint4 c = lds128(ps + (uint32_t)(r * 64 + 16 * u));
+        w.w[0] = c.x;
+        w.w[1] = c.y;
+        w.w[2] = c.z;
+        w.w[3] = c.w;
+    } else {
+        const uint32_t rc = ps + (uint32_t)(r * 48 + 4 * u);
+        w.w[0] = lds32(rc);
+        w.w[1] = lds32(rc + 16);
+        w.w[2] = lds32(rc + 32);
+        w.w[3] = 0;
+        if (KIND == 1) w.lut = lds128(ps + (uint32_t)(BM * 48 + r * lut_box + 16 * gl));
     }
 }
 
@@ -256,9 +296,13 @@ __device__ __forceinline__ void dequant_unit(const UnitRaw &u, __half2 (&v)[16])
 }
 
 template <int BITS, int KIND>
-__global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, GemmArgs a) {
+__global__ void __launch_bounds__(THREADS, 1)
+    gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_c,
+                const __grid_constant__ CUtensorMap tmap_l, const __grid_constant__ GemmArgs a) {
     extern __shared__ uint8_t smem_raw[];
-    SmemLayout &s = *reinterpret_cast<SmemLayout *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
+    SmemLayout &s = *reinterpret_cast<SmemLayout *>(base);
+    const uint32_t pk_s = smem_u32(base + kLayoutBytes);  // packed-code ring
     volatile uint32_t *abort_flag = &s.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -278,10 +322,16 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
             mbar_init(&s.accum_full[i], 1);
             mbar_init(&s.accum_empty[i], NUM_EPI_WARPS);
         }
+        for (int i = 0; i < a.pslots; ++i) {
+            mbar_init(&s.pfull[i], 1);
+            mbar_init(&s.pempty[i], NUM_DQ_WARPS);
+        }
         mbar_init(&s.done, 1);
         s.abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_x) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_c) : "memory");
+        if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_l) : "memory");
     }
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
@@ -361,35 +411,52 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
         // ------------------------------------------------ dequant producers
         const int d = threadIdx.x - 64;  // 0..255
         const int r = d >> 1;            // tile row 0..127
-        const int half_id = d & 1;       // which 32-wide half of the stage
-        int it = 0;
+        const int half_id = d & 1;       // which 32-wide half of a stage
+        const int P = a.pslots;
+        const int nsb = nkb / 2;         // superblocks (128 k = 2 stages) per tile
+        int q = 0;                       // stage counter across tiles
+        int sbi = 0;                     // superblock counter across tiles
         bool ok = true;
+        // codes of one superblock for this thread: its unit of each of the two stages
+        auto read_sb = [&](int sb_global, int sbl, int64_t row, UnitRaw (&w)[2]) -> bool {
+            const int ps = sb_global % P;
+            if (!wait_phase(&s.pfull[ps], (uint32_t)(sb_global / P) & 1u, a.wait_limit_ns, abort_flag)) return false;
+            const uint32_t base_ps = pk_s + (uint32_t)(ps * a.pslot_bytes);
+#pragma unroll
+            for (int h2 = 0; h2 < 2; ++h2) {
+                const int u = 2 * h2 + half_id;
+                read_codes<BITS, KIND>(base_ps, r, u, (32 * u) >> a.log2g, a.lut_box, w[h2]);
+                if (KIND == 0 && row < a.n) load_meta<KIND>(a, row, (int64_t)sbl * 128 + 32 * u, w[h2]);
+            }
+            // every lane has its codes in registers: release the slot
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&s.pempty[ps]);
+            return true;
+        };
         for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
             const int64_t row = (int64_t)(t / mt) * BM + r;
             const bool valid = row < a.n;
-            constexpr int kAhead = 4;
-            // pre[j] holds the codes of stage kb with kb % kAhead == j: the loop
-            // is unrolled by kAhead so that no in-flight load is ever copied
-            // between registers (a copy would wait for the load)
-            UnitRaw pre[kAhead];
+            UnitRaw cur[2], nxt[2];
+            ok = read_sb(sbi, 0, row, cur);
+            for (int sbl = 0; sbl < nsb && ok; ++sbl, ++sbi) {
+                // the next superblock's codes are read while this one is dequantized
+                if (sbl + 1 < nsb && !read_sb(sbi + 1, sbl + 1, row, nxt)) {
+                    raise_abort(s, a.status);
+                    ok = false;
+                }
+                // both stages of the superblock are dequantized and stored, then
+                // one proxy fence (its cost is per fence, not per byte) and one
+                // arrival on each stage's full barrier
 #pragma unroll
-            for (int i = 0; i < kAhead; ++i)
-                if (valid && i < nkb) load_unit<BITS, KIND>(a, row, (int64_t)i * BK + 32 * half_id, pre[i]);
-            for (int kb0 = 0; kb0 < nkb && ok; kb0 += kAhead) {
-#pragma unroll
-                for (int j = 0; j < kAhead; ++j) {
-                    const int kb = kb0 + j;
-                    if (kb >= nkb) break;
-                    // stage q = it: its barriers are slot q % STAGES; its W slot
-                    // q % W_SLOTS is free once the MMAs of stage q - W_SLOTS are done
-                    const int q = it++;
-                    const int st = q % STAGES;
-                    const int qf = q - W_SLOTS;
-                    bool free_ok = true;
-                    if (qf >= 0)
-                        free_ok = wait_phase(&s.empty[qf % STAGES], (uint32_t)(qf / STAGES) & 1u, a.wait_limit_ns,
-                                             abort_flag);
-                    if (!free_ok) {
+                for (int h2 = 0; h2 < 2; ++h2) {
+                    // stage q + h2: W slot (q + h2) % W_SLOTS is free once the MMAs
+                    // of stage q + h2 - W_SLOTS are done
+                    const int qf = q + h2 - W_SLOTS;
+                    bool got = ok;
+                    if (got && qf >= 0)
+                        got = wait_phase(&s.empty[qf % STAGES], (uint32_t)(qf / STAGES) & 1u, a.wait_limit_ns,
+                                         abort_flag);
+                    if (!got) {
                         raise_abort(s, a.status);
                         ok = false;
                     }
@@ -399,26 +466,64 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
                     }
                     __half2 v[16];
                     if (valid) {
-                        dequant_unit<BITS, KIND>(pre[j], v);
+                        dequant_unit<BITS, KIND>(cur[h2], v);
                     } else {
 #pragma unroll
                         for (int p = 0; p < 16; ++p) v[p] = __float2half2_rn(0.0f);
                     }
-                    if (valid && kb + kAhead < nkb)
-                        load_unit<BITS, KIND>(a, row, (int64_t)(kb + kAhead) * BK + 32 * half_id, pre[j]);
-                    uint8_t *tile = s.a[q % W_SLOTS] + (r >> 3) * 1024 + (r & 7) * 128;
+                    uint8_t *tile = s.a[(q + h2) % W_SLOTS] + (r >> 3) * 1024 + (r & 7) * 128;
 #pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int chunk = 4 * half_id + q;
+                    for (int qq = 0; qq < 4; ++qq) {
+                        const int chunk = 4 * half_id + qq;
                         *reinterpret_cast<uint4 *>(tile + ((chunk ^ (r & 7)) << 4)) =
-                            make_uint4(h22u(v[4 * q]), h22u(v[4 * q + 1]), h22u(v[4 * q + 2]), h22u(v[4 * q + 3]));
+                            make_uint4(h22u(v[4 * qq]), h22u(v[4 * qq + 1]), h22u(v[4 * qq + 2]), h22u(v[4 * qq + 3]));
                     }
-                    fence_proxy_async_smem();  // generic-proxy writes -> visible to the tensor core
-                    __syncwarp();
-                    if (lane == 0) mbar_arrive(&s.full[st]);
+                }
+                if (!ok) break;
+                fence_proxy_async_smem();  // generic-proxy writes -> visible to the tensor core
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(&s.full[q % STAGES]);
+                    mbar_arrive(&s.full[(q + 1) % STAGES]);
+                }
+                q += 2;
+                cur[0] = nxt[0];
+                cur[1] = nxt[1];
+            }
+            if (!ok) break;
+        }
+    } else if (warp == PK_WARP) {
+        // ------------------------------------------------ TMA producer (packed codes)
+        if (lane == 0) {
+            const int P = a.pslots;
+            const uint32_t bytes = (uint32_t)(BITS == 3 ? BM * 48 + (KIND == 1 ? BM * a.lut_box : 0) : BM * 64);
+            int sbi = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
+                const int row0 = (t / mt) * BM;
+                for (int sb = 0; sb < nkb / 2; ++sb, ++sbi) {
+                    const int ps = sbi % P;
+                    if (!wait_phase(&s.pempty[ps], ((uint32_t)(sbi / P) & 1u) ^ 1u, a.wait_limit_ns, abort_flag)) {
+                        raise_abort(s, a.status);
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t dst = pk_s + (uint32_t)(ps * a.pslot_bytes);
+                    mbar_arrive_expect_tx(&s.pfull[ps], bytes);
+                    if (BITS == 3) {
+                        tma_load_3d(dst, &tmap_c, &s.pfull[ps], sb * 16, 0, row0);
+                        if (KIND == 1)
+                            tma_load_2d_s(dst + BM * 48, &tmap_l, &s.pfull[ps], ((sb * 128) >> a.log2g) * 16, row0);
+                    } else {
+                        tma_load_2d_s(dst, &tmap_c, &s.pfull[ps], sb * 64, row0);
+                    }
                 }
             }
+            // drain: never leave the CTA with a bulk copy still writing smem
+            for (int q = sbi - P < 0 ? 0 : sbi - P; q < sbi; ++q)
+                mbar_wait(&s.pfull[q % P], (uint32_t)(q / P) & 1u, a.wait_limit_ns, nullptr);
         }
+        __syncwarp();
     } else {
         // ------------------------------------------------ epilogue
         const int quarter = warp & 3;  // the TMEM lanes (W rows) this warp may read
@@ -460,13 +565,14 @@ __global__ void __launch_bounds__(THREADS, 1) gemm_kernel(const __grid_constant_
 }
 
 template <int BITS, int KIND>
-cudaError_t launch_t(const CUtensorMap &map, const GemmArgs &a, int num_sms, cudaStream_t st) {
+cudaError_t launch_t(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &ml, const GemmArgs &a,
+                     int num_sms, cudaStream_t st) {
     auto kern = gemm_kernel<BITS, KIND>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)kSmemBytes);
+    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
     if (e != cudaSuccess) return e;
     const int64_t tiles = ((a.m + BN - 1) / BN) * ((a.n + BM - 1) / BM);
     const unsigned grid = (unsigned)std::min<int64_t>(tiles, num_sms);
-    kern<<<grid, THREADS, kSmemBytes, st>>>(map, a);
+    kern<<<grid, THREADS, a.smem_bytes, st>>>(mx, mc, ml, a);
     return cudaGetLastError();
 }
 
@@ -485,21 +591,62 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
-cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st) {
+cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
-    CUtensorMap map;
-    const cuuint64_t dims[2] = {(cuuint64_t)a.k, (cuuint64_t)a.m};
-    const cuuint64_t strides[1] = {(cuuint64_t)a.k * 2};
-    const cuuint32_t box[2] = {BK, BN};
-    const cuuint32_t estr[2] = {1, 1};
-    CUresult r = enc(&map, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(a.X), dims, strides, box, estr,
-                     CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-                     CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
-    if (r != CUDA_SUCCESS) return cudaErrorInvalidValue;
-    if (a.bits == 4) return launch_t<4, 0>(map, a, num_sms, st);
-    if (a.kind == 1) return launch_t<3, 1>(map, a, num_sms, st);
-    return launch_t<3, 0>(map, a, num_sms, st);
+    GemmArgs a = args;
+    const cuuint32_t estr[3] = {1, 1, 1};
+    CUtensorMap mx{}, mc{}, ml{};
+    {
+        const cuuint64_t dims[2] = {(cuuint64_t)a.k, (cuuint64_t)a.m};
+        const cuuint64_t strides[1] = {(cuuint64_t)a.k * 2};
+        const cuuint32_t box[2] = {BK, BN};
+        if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(a.X), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    // packed codes: one box = one 128-weight superblock of 128 rows
+    if (a.bits == 3) {
+        const cuuint64_t dims[3] = {(cuuint64_t)(a.k / 8), 3, (cuuint64_t)a.n};
+        const cuuint64_t strides[2] = {(cuuint64_t)(a.k / 8), (cuuint64_t)(a.k * 3 / 8)};
+        const cuuint32_t box[3] = {16, 3, BM};
+        if (enc(&mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 3, const_cast<uint8_t *>(a.codes), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    } else {
+        const cuuint64_t dims[2] = {(cuuint64_t)(a.k / 2), (cuuint64_t)a.n};
+        const cuuint64_t strides[1] = {(cuuint64_t)(a.k / 2)};
+        const cuuint32_t box[2] = {64, BM};
+        if (enc(&mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t *>(a.codes), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    }
+    a.lut_box = 0;
+    if (a.kind == 1) {
+        // the LUTs of the groups one superblock spans (one group for g >= 128)
+        a.lut_box = 16 * std::max(1, 128 >> a.log2g);
+        const cuuint64_t dims[2] = {(cuuint64_t)a.G * 16, (cuuint64_t)a.n};
+        const cuuint64_t strides[1] = {(cuuint64_t)a.G * 16};
+        const cuuint32_t box[2] = {(cuuint32_t)a.lut_box, BM};
+        if (enc(&ml, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<__half *>(a.luts), dims, strides, box, estr,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
+            return cudaErrorInvalidValue;
+    } else {
+        ml = mc;  // unused
+    }
+    a.pslot_bytes = (a.bits == 3 ? BM * 48 + BM * a.lut_box : BM * 64 + 0);
+    a.pslot_bytes = (a.pslot_bytes + 1023) / 1024 * 1024;
+    const int budget = 227 * 1024 - (int)kLayoutBytes - 1024;
+    a.pslots = std::min(kMaxPSlots, budget / a.pslot_bytes);
+    if (a.pslots < 2) return cudaErrorInvalidConfiguration;
+    a.smem_bytes = (int)kLayoutBytes + 1024 + a.pslots * a.pslot_bytes;
+    if (a.bits == 4) return launch_t<4, 0>(mx, mc, ml, a, num_sms, st);
+    if (a.kind == 1) return launch_t<3, 1>(mx, mc, ml, a, num_sms, st);
+    return launch_t<3, 0>(mx, mc, ml, a, num_sms, st);
 }
 
 }  // namespace qx

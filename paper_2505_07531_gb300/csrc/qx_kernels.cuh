@@ -79,6 +79,10 @@ struct GemmArgs {
     __half *Y;        // [m][n]
     uint32_t *status;
     uint64_t wait_limit_ns;
+    // packed-code ring (filled by launch_gemm): slots of one 128-weight
+    // superblock of a 128-row W tile
+    int pslots, pslot_bytes, lut_box;
+    int smem_bytes;
 };
 
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
