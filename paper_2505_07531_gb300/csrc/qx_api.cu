@@ -205,7 +205,7 @@ QX_API qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream) {
 namespace {
 
 // One decode launch over `count` matrices for activation rows b0 .. b0+nb-1
-// (nb <= 4).  When the group's activations do not fit one CTA's shared
+// (nb <= 4, or 8).  When the group's activations do not fit one CTA's shared
 // memory, the group is split per matrix, then the rows are halved.
 qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int b0, int nb, void *const *y,
                      int y_dtype, int flags, cudaStream_t st, DeviceInfo *d) {
@@ -250,13 +250,16 @@ qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int
     return QX_ERR_UNSUPPORTED;
 }
 
-// Batches above four are processed four rows of x at a time; each chunk
+// Kernels exist for 1..4 and 8 rows of x: a batch is processed eight rows at
+// a time while at least eight remain, then four at a time; each chunk
 // streams the weights once.
 qx_status run_gemv(const qx_packed *mats, int count, const void *const *x, int batch, void *const *y,
                    int y_dtype, int flags, cudaStream_t st, DeviceInfo *d) {
-    for (int b0 = 0; b0 < batch; b0 += 4) {
-        qx_status s = gemv_chunk(mats, count, x, b0, std::min(4, batch - b0), y, y_dtype, flags, st, d);
+    for (int b0 = 0; b0 < batch;) {
+        const int nb = batch - b0 >= 8 ? 8 : std::min(4, batch - b0);
+        qx_status s = gemv_chunk(mats, count, x, b0, nb, y, y_dtype, flags, st, d);
         if (s != QX_OK) return s;
+        b0 += nb;
     }
     return QX_OK;
 }

@@ -50,7 +50,7 @@ constexpr int kMaxRing = 8;
 // latency then hides behind the previous kernel.
 constexpr int kMaxRbSlots = 16;
 constexpr int kHeader = 1024;       // barriers, counters, per-matrix CTA plan
-constexpr int kSmemBudget = 200 * 1024;
+constexpr int kSmemBudget = 220 * 1024;
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -193,20 +193,6 @@ struct Header {
 };
 static_assert(sizeof(Header) <= kHeader, "header does not fit");
 
-// Matrices i and j of the launch read the same activations.
-__device__ __forceinline__ bool same_x(const Header &h, int i, int j) {
-    return h.mats[i].x == h.mats[j].x && h.mats[i].K == h.mats[j].K;
-}
-
-// Matrix i is the first matrix of this CTA with its activations: it owns
-// their shared-memory copy.
-__device__ __forceinline__ bool x_owner(const Header &h, int i) {
-    if (h.mats[i].nrb == 0) return false;
-    for (int j = 0; j < i; ++j)
-        if (h.mats[j].nrb > 0 && same_x(h, i, j)) return false;
-    return true;
-}
-
 // Stage q of this CTA: matrix, matrix-local row block, slice.
 __device__ __forceinline__ void stage_coords(const Header &h, int count, int q, int &m, int &rb, int &ks) {
     m = 0;
@@ -336,6 +322,33 @@ __device__ __forceinline__ float meta_scale(const Meta &t, int gl) {
 
 __device__ __forceinline__ uint32_t meta_zero(const Meta &t, int gl) { return (t.z >> (4 * gl)) & 15u; }
 
+// Row blocks of matrix m in this CTA's range [lo, hi) of the launch's list.
+__device__ __forceinline__ int cta_nrb(const GemvMulti &a, int m, int lo, int hi) {
+    const int f = max(lo, a.mat[m].rb_off), e = min(hi, a.mat[m].rb_off + a.mat[m].nrb);
+    return e > f ? e - f : 0;
+}
+
+// Matrix m is the first matrix of this CTA with its activations: it owns
+// their shared-memory copy (matrices of a launch may share one x).
+__device__ __forceinline__ bool x_owner_p(const GemvMulti &a, int m, int lo, int hi) {
+    if (cta_nrb(a, m, lo, hi) == 0) return false;
+    for (int j = 0; j < m; ++j)
+        if (cta_nrb(a, j, lo, hi) > 0 && a.mat[j].x == a.mat[m].x && a.mat[j].k == a.mat[m].k) return false;
+    return true;
+}
+
+// Offset (halves) of matrix m's activations in the shared-memory copy.
+template <int NB>
+__device__ __forceinline__ int x_offset(const GemvMulti &a, int m, int lo, int hi) {
+    int off = 0;
+    for (int j = 0; j < m; ++j) {
+        if (!x_owner_p(a, j, lo, hi)) continue;
+        if (a.mat[j].x == a.mat[m].x && a.mat[j].k == a.mat[m].k) return off;
+        off += NB * (int)a.mat[j].k;
+    }
+    return off;
+}
+
 // Cursor over one warp's stages: matrix, CTA-local row block of that matrix,
 // slice, and the CTA-local stage number.
 struct Cursor {
@@ -377,9 +390,11 @@ __device__ __forceinline__ void superblock3(const uint4 &A, const uint4 &B, cons
     float s = 1.0f;
 #pragma unroll
     for (int i = 0; i < 4; ++i) {
-        __half2 xv[NB][16];
+        // up to four rows of x are held at once (batch 8 takes them one by one)
+        constexpr int XB = NB <= 4 ? NB : 1;
+        __half2 xv[XB][16];
 #pragma unroll
-        for (int b = 0; b < NB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
+        for (int b = 0; b < XB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
         if (i % (4 / TPS) == 0) {
             const int t = i / (4 / TPS);
             if (KIND == 1) {
@@ -395,10 +410,12 @@ __device__ __forceinline__ void superblock3(const uint4 &A, const uint4 &B, cons
         lookup_triple(tab, Aw[i], Bw[i], Cw[i], w);
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
+            const __half2(&xb)[16] = xv[XB == NB ? b : 0];
+            if (XB != NB && b > 0) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[0]);
             if (KIND == 1)
-                acc[b] += dot16(w, xv[b]);
+                acc[b] += dot16(w, xb);
             else
-                acc[b] += s * dot16(w, xv[b]);
+                acc[b] += s * dot16(w, xb);
         }
     }
 }
@@ -412,9 +429,10 @@ __device__ __forceinline__ void part4(uint32_t cb, int r, const Meta &meta, uint
 #pragma unroll
     for (int i = 0; i < 8; ++i) {
         if (i == 4 && half_only) break;  // k is a multiple of 128, not of 256
-        __half2 xv[NB][16];
+        constexpr int XB = NB <= 4 ? NB : 1;
+        __half2 xv[XB][16];
 #pragma unroll
-        for (int b = 0; b < NB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
+        for (int b = 0; b < XB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
         if (i % UPG == 0) {
             const int gl = i / UPG;
             const uint32_t z = meta_zero(meta, gl);
@@ -433,7 +451,11 @@ __device__ __forceinline__ void part4(uint32_t cb, int r, const Meta &meta, uint
             for (int u = 0; u < 4; ++u) w[4 * t + u] = o[u];
         }
 #pragma unroll
-        for (int b = 0; b < NB; ++b) acc[b] += s * dot16(w, xv[b]);
+        for (int b = 0; b < NB; ++b) {
+            const __half2(&xb)[16] = xv[XB == NB ? b : 0];
+            if (XB != NB && b > 0) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[0]);
+            acc[b] += s * dot16(w, xb);
+        }
     }
 }
 
@@ -454,85 +476,93 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     const int lane = threadIdx.x & 31;
     const int count = a.count, ring = a.ring;
 
-    // ---- set-up, spread over threads so that the first copies start early
-    if (threadIdx.x < count) {  // this CTA's row blocks of matrix t
-        const int t = threadIdx.x;
-        const int lo = a.cta_rb[blockIdx.x], hi = a.cta_rb[blockIdx.x + 1];
-        const GemvMat &G = a.mat[t];
-        MatS &S = h.mats[t];
-        const int f = max(lo, G.rb_off), e = min(hi, G.rb_off + G.nrb);
-        S.zeros = G.zeros;
-        S.scales = G.scales;
-        S.x = G.x;
-        S.y = G.y;
-        S.n = (int)G.n;
-        S.K = (int)G.k;
-        S.G = G.G;
-        S.zbytes = G.zbytes;
-        S.log2g = G.log2g;
-        S.nks = G.nks;
-        S.nlb = G.nlb;
-        S.rb0 = f - G.rb_off;
-        S.nrb = e > f ? e - f : 0;
-    } else if (threadIdx.x >= 32 && threadIdx.x < 32 + count) {
-        const int t = threadIdx.x - 32;
-        asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_codes[t]) : "memory");
-        if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_luts[t]) : "memory");
-    } else if (threadIdx.x == 64) {
-        for (int i = 0; i < ring; ++i) mbar_init(smem_u32(&h.full[i]), 1);
-        h.abort_flag = 0;
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        // the CTA's first stage straight from the parameters, so that its
-        // data is on the way while the rest of the set-up runs
-        const int lo = a.cta_rb[blockIdx.x], hi = a.cta_rb[blockIdx.x + 1];
-        if (lo < hi) {
-            int m = 0;
-            while (m + 1 < count && lo >= a.mat[m].rb_off + a.mat[m].nrb) ++m;
-            issue_geom<BITS, KIND>(a, geom_of(a.mat[m]), m, smem_u32(&h.full[0]), ring_s, lo - a.mat[m].rb_off, 0);
-        }
-    }
-    if (threadIdx.x >= 96 && threadIdx.x < 96 + kMaxRing) h.rel[threadIdx.x - 96] = 0;
-    if (threadIdx.x >= 128 && threadIdx.x < 128 + kMaxRbSlots) {
-        h.cnt[threadIdx.x - 128] = 0;
-        h.gen[threadIdx.x - 128] = 0;
-    }
-    __syncthreads();
-    if (warp == 0) {
-        // stage and row-block numbering per matrix, then one lane per initial stage
-        int q = 0, rbq = 0, mine = 0, mrb = 0, qend = 0;
-        for (int m = 0; m < count; ++m) {
-            if (m == lane) {
-                mine = q;
-                mrb = rbq;
-            }
-            q += h.mats[m].nrb * h.mats[m].nks;
-            rbq += h.mats[m].nrb;
-            if (m == lane) qend = q;
-        }
-        if (lane < count) {
-            h.mats[lane].q0 = mine;
-            h.mats[lane].rbq0 = mrb;
-            h.q_end[lane] = qend;
-            // activations in shared memory: one copy per distinct x of this CTA
-            int off = 0, xo = -1;
-            for (int m = 0; m < lane; ++m) {
-                if (!x_owner(h, m)) continue;
-                if (xo < 0 && same_x(h, m, lane)) xo = off;
-                off += NB * h.mats[m].K;
-            }
-            h.mats[lane].xoff = xo >= 0 ? xo : off;
-        }
-        if (lane == 0) {
-            h.nstages = q;
-            h.issued = (uint32_t)min(a.initial, q);
-        }
-        __syncwarp();
-        if (lane >= 1 && lane < min(a.initial, q)) issue_stage<BITS, KIND>(a, h, ring_s, lane);
-    }
-    __syncthreads();
     // let the next kernel in the stream start streaming its own weights; it
     // still waits for this grid's completion before it reads activations
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+
+    // ---- set-up from the kernel parameters, spread over threads, with a
+    // single barrier before the main loop: the first copies start at once and
+    // the activations are staged while the tables are built
+    const int lo = a.cta_rb[blockIdx.x], hi = a.cta_rb[blockIdx.x + 1];
+    if (warp == 0) {
+        if (lane < count) {  // matrix `lane`: this CTA's row blocks, stage numbering, x offset
+            const int t = lane;
+            const GemvMat &G = a.mat[t];
+            MatS &S = h.mats[t];
+            const int f = max(lo, G.rb_off);
+            S.zeros = G.zeros;
+            S.scales = G.scales;
+            S.x = G.x;
+            S.y = G.y;
+            S.n = (int)G.n;
+            S.K = (int)G.k;
+            S.G = G.G;
+            S.zbytes = G.zbytes;
+            S.log2g = G.log2g;
+            S.nks = G.nks;
+            S.nlb = G.nlb;
+            S.rb0 = f - G.rb_off;
+            S.nrb = cta_nrb(a, t, lo, hi);
+            int q = 0, rbq = 0;
+            for (int m = 0; m < t; ++m) {
+                const int nr = cta_nrb(a, m, lo, hi);
+                q += nr * a.mat[m].nks;
+                rbq += nr;
+            }
+            S.q0 = q;
+            S.rbq0 = rbq;
+            h.q_end[t] = q + S.nrb * G.nks;
+            S.xoff = x_offset<NB>(a, t, lo, hi);
+        }
+        if (lane == 0) {
+            int q = 0;
+            for (int m = 0; m < count; ++m) q += cta_nrb(a, m, lo, hi) * a.mat[m].nks;
+            h.nstages = q;
+        }
+    } else if (warp == 1) {
+        if (lane < count) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_codes[lane]) : "memory");
+            if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_luts[lane]) : "memory");
+        }
+    } else if (warp == 2) {
+        if (lane == 0) {
+            for (int i = 0; i < ring; ++i) mbar_init(smem_u32(&h.full[i]), 1);
+            h.abort_flag = 0;
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        __syncwarp();
+        // the CTA's first stages straight from the parameters, one per lane, so
+        // that their data is on the way while the rest of the set-up runs
+        int q = 0;
+        for (int m = 0; m < count; ++m) {
+            const GemvMat &G = a.mat[m];
+            const int nq = cta_nrb(a, m, lo, hi) * G.nks;
+            if (lane < a.initial && lane >= q && lane < q + nq) {
+                const int j = lane - q, rbl = j / G.nks, ks = j - rbl * G.nks;
+                const int rb0 = max(lo, G.rb_off) - G.rb_off;
+                issue_geom<BITS, KIND>(a, geom_of(G), m, smem_u32(&h.full[lane]),
+                                       ring_s + (uint32_t)(lane * a.stage_bytes), rb0 + rbl, ks);
+            }
+            q += nq;
+        }
+        if (lane == 0) h.issued = (uint32_t)min(a.initial, q);
+    } else if (threadIdx.x >= 96 && threadIdx.x < 96 + kMaxRing) {
+        h.rel[threadIdx.x - 96] = 0;
+    } else if (threadIdx.x >= 128 && threadIdx.x < 128 + kMaxRbSlots) {
+        h.cnt[threadIdx.x - 128] = 0;
+        h.gen[threadIdx.x - 128] = 0;
+    }
+    // activations -> shared memory (every lane of a warp then reads the same
+    // address: a broadcast), after the previous kernel in the stream is done
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    for (int m = 0; m < count; ++m) {
+        if (!x_owner_p(a, m, lo, hi)) continue;
+        const int vecs = NB * (int)a.mat[m].k / 8;
+        const uint4 *src = reinterpret_cast<const uint4 *>(a.mat[m].x);
+        uint4 *dst = reinterpret_cast<uint4 *>(xs + x_offset<NB>(a, m, lo, hi));
+        for (int i = threadIdx.x; i < vecs; i += kThreads) dst[i] = src[i];
+    }
+    __syncthreads();
 
     const int nst = h.nstages;
     const int r = lane;
@@ -554,17 +584,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     Meta cur{}, nxt{};
     if (KIND == 0 && c.m < count)
         cur = load_meta(h.mats[c.m], (h.mats[c.m].rb0 + c.rbl) * kRows + r, c.ks * kSliceK + part * kPartK);
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    // activations -> shared memory (every lane of a warp then reads the same
-    // address: a broadcast)
-    for (int m = 0; m < count; ++m) {
-        if (!x_owner(h, m)) continue;
-        const int vecs = NB * h.mats[m].K / 8;
-        const uint4 *src = reinterpret_cast<const uint4 *>(h.mats[m].x);
-        uint4 *dst = reinterpret_cast<uint4 *>(xs + h.mats[m].xoff);
-        for (int i = threadIdx.x; i < vecs; i += kThreads) dst[i] = src[i];
-    }
-    __syncthreads();
 
     // per-lane offsets of this warp's 3-bit code chunks in a stage (planes 0-2
     // of row r are box rows 3r..3r+2; superblocks 2 part and 2 part + 1)
@@ -855,7 +874,9 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
     // slot is only ever used by one group: a warp then never waits on a
     // barrier phase more than one ahead of the slot's current one.
     for (int ring = kMaxRing; ring >= kGroups; ring -= kGroups) {
-        const int slots = std::min(kMaxRbSlots, (ring + nks_min - 1) / nks_min + 2);
+        // partial-sum slots: any count is safe (a warp waits for the slot's
+        // previous block); enough of them keep the warp groups from waiting
+        const int slots = bmax > 4 ? 1 : std::min(kMaxRbSlots, (ring + nks_min - 1) / nks_min + 2);
         const int red = (slots * kWarps * bmax * 32 * 4 + 1023) / 1024 * 1024;
         const int smem = 1024 + kHeader + red + a.x_smem_bytes + ring * a.stage_bytes;
         if (smem <= kSmemBudget || ring == kGroups) {
@@ -875,7 +896,8 @@ cudaError_t launch_nb(const GemvMulti &a, cudaStream_t st, bool pdl) {
         case 1: return launch_one<BITS, KIND, 1>(a, st, pdl);
         case 2: return launch_one<BITS, KIND, 2>(a, st, pdl);
         case 3: return launch_one<BITS, KIND, 3>(a, st, pdl);
-        default: return launch_one<BITS, KIND, 4>(a, st, pdl);
+        case 4: return launch_one<BITS, KIND, 4>(a, st, pdl);
+        default: return launch_one<BITS, KIND, 8>(a, st, pdl);
     }
 }
 
