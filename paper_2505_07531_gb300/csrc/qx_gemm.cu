@@ -254,7 +254,8 @@ __device__ __forceinline__ void load_meta(const GemmArgs &a, int64_t row, int64_
 // one superblock of 128 rows -- 3-bit: [row][plane][16 bytes] then the LUTs
 // [row][lut_box bytes]; 4-bit: [row][64 bytes].  u = unit in the superblock.
 template <int BITS, int KIND>
-__device__ __forceinline__ void read_codes(uint32_t ps, int r, int u, int gl, int lut_box, UnitRaw &w) {
+__device__ __forceinline__ void read_codes(uint32_t ps, int r, int u, int gl, int lut_box, bool need_lut,
+                                           UnitRaw &w) {
     if (BITS == 4) {
         const uint4 c = lds128(ps + (uint32_t)(r * 64 + 16 * u));
         w.w[0] = c.x;
@@ -267,7 +268,7 @@ __device__ __forceinline__ void read_codes(uint32_t ps, int r, int u, int gl, in
         w.w[1] = lds32(rc + 16);
         w.w[2] = lds32(rc + 32);
         w.w[3] = 0;
-        if (KIND == 1) w.lut = lds128(ps + (uint32_t)(BM * 48 + r * lut_box + 16 * gl));
+        if (KIND == 1 && need_lut) w.lut = lds128(ps + (uint32_t)(BM * 48 + r * lut_box + 16 * gl));
     }
 }
 
@@ -425,7 +426,8 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
             for (int h2 = 0; h2 < 2; ++h2) {
                 const int u = 2 * h2 + half_id;
-                read_codes<BITS, KIND>(base_ps, r, u, (32 * u) >> a.log2g, a.lut_box, w[h2]);
+                // with g >= 128 both units use the first unit's table
+                read_codes<BITS, KIND>(base_ps, r, u, (32 * u) >> a.log2g, a.lut_box, h2 == 0 || a.log2g < 7, w[h2]);
                 if (KIND == 0 && row < a.n) load_meta<KIND>(a, row, (int64_t)sbl * 128 + 32 * u, w[h2]);
             }
             // every lane has its codes in registers: release the slot
@@ -444,39 +446,58 @@ __global__ void __launch_bounds__(THREADS, 1)
                     raise_abort(s, a.status);
                     ok = false;
                 }
-                // both stages of the superblock are dequantized and stored, then
-                // one proxy fence (its cost is per fence, not per byte) and one
-                // arrival on each stage's full barrier
+                // Both stages of the superblock: wait for both W slots, then
+                // dequantize the two units as one block of independent work (the
+                // two table lookups interleave: a dequant warp's latency, not the
+                // ALU, bounds the producer rate), store both, then one proxy
+                // fence (its cost is per fence, not per byte) and one arrival on
+                // each stage's full barrier.  W slot (q + h2) % W_SLOTS is free
+                // once the MMAs of stage q + h2 - W_SLOTS are done.
 #pragma unroll
                 for (int h2 = 0; h2 < 2; ++h2) {
-                    // stage q + h2: W slot (q + h2) % W_SLOTS is free once the MMAs
-                    // of stage q + h2 - W_SLOTS are done
                     const int qf = q + h2 - W_SLOTS;
-                    bool got = ok;
-                    if (got && qf >= 0)
-                        got = wait_phase(&s.empty[qf % STAGES], (uint32_t)(qf / STAGES) & 1u, a.wait_limit_ns,
-                                         abort_flag);
-                    if (!got) {
+                    if (ok && qf >= 0 &&
+                        !wait_phase(&s.empty[qf % STAGES], (uint32_t)(qf / STAGES) & 1u, a.wait_limit_ns, abort_flag)) {
                         raise_abort(s, a.status);
                         ok = false;
                     }
-                    if (__any_sync(0xffffffffu, !ok)) {
-                        ok = false;
-                        break;
-                    }
-                    __half2 v[16];
-                    if (valid) {
-                        dequant_unit<BITS, KIND>(cur[h2], v);
-                    } else {
+                }
+                if (__any_sync(0xffffffffu, !ok)) {
+                    ok = false;
+                    break;
+                }
+                __half2 v[2][16];
+                if (BITS == 3 && KIND == 1 && a.log2g >= 7) {
+                    // one group spans the superblock: one table for both units
+                    const Table8 t = make_table8(cur[0].lut.x, cur[0].lut.y, cur[0].lut.z, cur[0].lut.w);
 #pragma unroll
-                        for (int p = 0; p < 16; ++p) v[p] = __float2half2_rn(0.0f);
+                    for (int h2 = 0; h2 < 2; ++h2) lookup_triple(t, cur[h2].w[0], cur[h2].w[1], cur[h2].w[2], v[h2]);
+                    if (!valid) {
+#pragma unroll
+                        for (int h2 = 0; h2 < 2; ++h2)
+#pragma unroll
+                            for (int p = 0; p < 16; ++p) v[h2][p] = __float2half2_rn(0.0f);
                     }
+                } else {
+#pragma unroll
+                    for (int h2 = 0; h2 < 2; ++h2) {
+                        if (valid) {
+                            dequant_unit<BITS, KIND>(cur[h2], v[h2]);
+                        } else {
+#pragma unroll
+                            for (int p = 0; p < 16; ++p) v[h2][p] = __float2half2_rn(0.0f);
+                        }
+                    }
+                }
+#pragma unroll
+                for (int h2 = 0; h2 < 2; ++h2) {
                     uint8_t *tile = s.a[(q + h2) % W_SLOTS] + (r >> 3) * 1024 + (r & 7) * 128;
 #pragma unroll
                     for (int qq = 0; qq < 4; ++qq) {
                         const int chunk = 4 * half_id + qq;
                         *reinterpret_cast<uint4 *>(tile + ((chunk ^ (r & 7)) << 4)) =
-                            make_uint4(h22u(v[4 * qq]), h22u(v[4 * qq + 1]), h22u(v[4 * qq + 2]), h22u(v[4 * qq + 3]));
+                            make_uint4(h22u(v[h2][4 * qq]), h22u(v[h2][4 * qq + 1]), h22u(v[h2][4 * qq + 2]),
+                                       h22u(v[h2][4 * qq + 3]));
                     }
                 }
                 if (!ok) break;

@@ -13,20 +13,26 @@
 //     shared-memory ring holds the codes (and LUTs) of 32 rows x 1024 k,
 //     fetched with 2-D/3-D TMA tensor copies in the 128-byte swizzled layout,
 //     which makes the per-lane 16-byte reads of 32 different rows free of bank
-//     conflicts.  Each of the eight warps decodes 128 k (one 3-bit superblock)
-//     of every stage.
-//   * No producer warp: the first stages are issued by thread 0 before the
-//     programmatic-dependent-launch wait (weights do not depend on the previous
-//     kernel), and afterwards the last warp to finish a stage refills it.
+//     conflicts.
+//   * Sixteen warps in four groups of four: group g decodes the stages q with
+//     q % 4 == g, and each of its warps one 256-weight part of each of them
+//     (two 3-bit superblocks), so four stages are in decode at once.
+//   * No producer warp (a seventeenth warp puts five warps on one SM
+//     sub-partition, which caps every thread at 96 registers): the first
+//     stages are issued from the kernel parameters by one lane each before the
+//     programmatic-dependent-launch wait (weights do not depend on the
+//     previous kernel); the rest of the ring is requested as those land, and
+//     afterwards the last warp of a group to release a stage refills it.
 //   * Partial sums of a row block stay in registers across its slices; at the
-//     end of the block each warp stores its partials and the last of the eight
+//     end of the block each warp stores its partials and the last contributor
 //     adds them in a fixed order (deterministic) and writes y.
 //   * Uniform scales and zero-points are read by each lane from global memory
-//     one stage ahead, after the refilling thread has pulled the block's
-//     metadata into L2 with a bulk prefetch.
-// One CTA of 256 threads per SM leaves room for a CTA of the next decode
-// kernel, which then streams its weights while this one finishes.  Every wait
-// is bounded in time and reports QX_ERR_TIMEOUT through the device status.
+//     one stage ahead, after the block's first copy has pulled its metadata
+//     into L2 with a bulk prefetch.
+// One CTA of 512 threads per SM.  Under programmatic dependent launch the
+// next decode kernel's CTA takes an SM as soon as this kernel's CTA there has
+// exited and issues its weight copies before it waits.  Every wait is
+// bounded in time and reports QX_ERR_TIMEOUT through the device status.
 #include "qx_kernels.cuh"
 
 namespace qx {
