@@ -151,9 +151,34 @@ qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const 
 
 /* Prefill matmul Y = X W_hat^T (Table 2 "Prefill") on the tcgen05 tensor cores:
  * W_hat tiles are dequantized into shared memory and multiplied in fp16 with
- * fp32 accumulation in tensor memory.  X: device fp16 [m][k] row-major,
- * 16-byte aligned; Y: device fp16 [m][n] row-major, 4-byte aligned; m >= 1. */
+ * fp32 accumulation in tensor memory, 256 tokens per tile (16 when m <= 16).
+ * X: device fp16 [m][k] row-major, 16-byte aligned; Y: device fp16 [m][n]
+ * row-major, 4-byte aligned; m >= 1.  One CTA per tile: no workspace. */
 qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream);
+
+/* Bytes of workspace qx_gemm_splitk needs for an n x k matrix of `recipe` and
+ * m rows of X on the current device (host-only call; 0 when the call will not
+ * split k).  Same shape rules as qx_packed_size; m >= 1. */
+qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const qx_recipe *recipe,
+                                   size_t *bytes);
+
+/* qx_gemm with the contraction split along k (at 128-weight boundaries) when
+ * the tiles alone would leave SMs idle -- the decode case (m <= 16: 16-token
+ * tiles, so this is also the tensor-core decode matmul for batches of 1..16)
+ * and short prefills.  Each split stores an fp32 partial tile to `workspace`;
+ * the last split of a tile to finish sums the partials in split order (the
+ * result does not depend on timing) and writes Y.  Same X, Y, m rules as
+ * qx_gemm.
+ * workspace: caller-owned device memory, 256-byte aligned, of at least
+ * qx_gemm_splitk_workspace() bytes (may be null when that is 0).  Its first
+ * 64 KiB hold counters, which must be zero before the first call: fill the
+ * whole buffer with zeros once; every completed call, whatever its shape,
+ * leaves them zero again.  After a call that ends
+ * in QX_ERR_TIMEOUT, zero it again.  Calls that may run at the same time need
+ * separate workspaces.  Returns QX_ERR_INVALID_ARG if the workspace is
+ * missing or too small, QX_ERR_ALIGNMENT if it is misaligned. */
+qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, void *workspace,
+                         size_t workspace_bytes, void *stream);
 
 /* Synchronize `stream`, then return and clear the current device's status word
  * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the

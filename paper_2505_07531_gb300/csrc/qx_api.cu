@@ -305,15 +305,19 @@ QX_API qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void 
     return run_gemv(mats, count, x, batch, y, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
 }
 
-QX_API qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream) {
+namespace {
+
+qx_status check_gemm_args(const qx_packed *p, const void *X, int64_t m, const void *Y) {
     qx_status s = check_packed(p);
     if (s != QX_OK) return s;
     if (X == nullptr || Y == nullptr || m < 1) return QX_ERR_INVALID_ARG;
     if (m > ((int64_t)1 << 31) - 1) return QX_ERR_UNSUPPORTED;
     if (!aligned(X, 16)) return QX_ERR_ALIGNMENT;
     if (!aligned(Y, 2)) return QX_ERR_ALIGNMENT;
-    DeviceInfo *d = nullptr;
-    if ((s = device_info(&d)) != QX_OK) return s;
+    return QX_OK;
+}
+
+qx::GemmArgs gemm_args(const qx_packed *p, const void *X, int64_t m, void *Y, const DeviceInfo *d) {
     qx::GemmArgs a{};
     a.codes = static_cast<const uint8_t *>(p->codes);
     a.scales = static_cast<const __half *>(p->scales);
@@ -331,6 +335,52 @@ QX_API qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, 
     a.Y = static_cast<__half *>(Y);
     a.status = d->status;
     a.wait_limit_ns = wait_limit_ns();
+    return a;
+}
+
+}  // namespace
+
+QX_API qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream) {
+    qx_status s = check_gemm_args(p, X, m, Y);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::GemmArgs a = gemm_args(p, X, m, Y, d);
+    const qx::GemmPlan plan = qx::plan_gemm(p->n, p->k, m, d->num_sms, false);
+    a.bn = plan.bn;
+    a.splits = 1;
+    return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const qx_recipe *recipe,
+                                          size_t *bytes) {
+    if (bytes == nullptr || recipe == nullptr || m < 1) return QX_ERR_INVALID_ARG;
+    qx_status s = check_recipe(recipe);
+    if (s != QX_OK) return s;
+    if ((s = check_shape(n, k, recipe)) != QX_OK) return s;
+    if (m > ((int64_t)1 << 31) - 1) return QX_ERR_UNSUPPORTED;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    *bytes = qx::plan_gemm(n, k, m, d->num_sms, true).ws_bytes;
+    return QX_OK;
+}
+
+QX_API qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, void *workspace,
+                                size_t workspace_bytes, void *stream) {
+    qx_status s = check_gemm_args(p, X, m, Y);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    const qx::GemmPlan plan = qx::plan_gemm(p->n, p->k, m, d->num_sms, true);
+    qx::GemmArgs a = gemm_args(p, X, m, Y, d);
+    a.bn = plan.bn;
+    a.splits = plan.splits;
+    if (plan.splits > 1) {
+        if (workspace == nullptr || workspace_bytes < plan.ws_bytes) return QX_ERR_INVALID_ARG;
+        if (!aligned(workspace, 256)) return QX_ERR_ALIGNMENT;
+        a.ws_cnt = static_cast<uint32_t *>(workspace);
+        a.ws_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + qx::kSplitCounterBytes);
+    }
     return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
 }
 

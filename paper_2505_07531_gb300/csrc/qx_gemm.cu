@@ -4,22 +4,32 @@
 // Prefill is the one dense contraction on the path (paper Table 2, "Prefill"),
 // so it runs on the tensor cores.  The kernel computes transposed tiles
 // D = W_hat_tile * X_tile^T: the MMA's M dimension is 128 rows of W, its N
-// dimension 256 tokens (each dequantized W tile feeds 256 tokens, which keeps
-// the dequantization below the tensor-core time), and the contraction runs
-// over k in stages of 64.
+// dimension BN tokens, and the contraction runs over k in stages of 64.
+// BN = 256 for prefill (each dequantized W tile feeds 256 tokens, which keeps
+// the dequantization below the tensor-core time); BN = 16 for m <= 16, which
+// makes the same kernel a decode matmul for batches of up to 16 tokens: the
+// tensor cores then take the products, and the dequantization alone bounds
+// the rate.
 //
-// Persistent: one CTA per SM walks the (W-row tile, token tile) pairs.  Warp
-// roles (448 threads):
-//   warp 0       TMA producer: 256 x 64 fp16 X tiles (128B swizzle) -> smem
+// Persistent: one CTA per SM walks the work units -- (W-row tile, token tile,
+// k split).  A tile is split along k (at 128-weight superblock boundaries)
+// when the tiles alone would leave SMs idle, as a 4096-row decode matrix does
+// (32 W tiles for 152 SMs); each split then stores its fp32 partial tile to a
+// workspace, and the last of a tile's splits to finish sums them in split
+// order (deterministic) and writes Y.  Warp roles (480 threads):
+//   warp 0       TMA producer: BN x 64 fp16 X tiles (128B swizzle) -> smem
 //   warp 1       allocates tensor memory; one thread issues tcgen05.mma
 //   warps 2-9    dequantize 128 x 64 W_hat tiles from the packed codes straight
 //                into the 128B-swizzled K-major shared-memory layout the MMA
 //                reads (the same unpack primitives as qx_dequant, so W_hat is
 //                exact)
-//   warps 10-13  epilogue: fp32 accumulator (tensor memory) -> fp16 Y
-// Two accumulators of 256 columns let the epilogue of one tile overlap the
-// main loop of the next.  A 4-stage mbarrier ring connects producers and the
-// MMA issuer; the MMA releases a stage with tcgen05.commit.  Every wait is
+//   warps 10-13  epilogue: fp32 accumulator (tensor memory) -> fp16 Y, or
+//                the fp32 partial of a k split -> workspace
+//   warp 14      TMA producer: packed codes (and LUTs) of 128-weight
+//                superblocks -> a ring the dequant warps read a superblock ahead
+// Two accumulators of BN columns let the epilogue of one unit overlap the
+// main loop of the next.  An mbarrier ring connects producers and the MMA
+// issuer; the MMA releases a stage with tcgen05.commit.  Every wait is
 // bounded in time: a wait that gives up raises QX_ERR_TIMEOUT in the device
 // status word, tells the other roles to stop, lets in-flight copies and MMAs
 // drain, frees tensor memory and returns.
@@ -32,32 +42,46 @@ namespace qx {
 namespace {
 
 constexpr int BM = 128;  // W rows per tile (MMA M)
-constexpr int BN = 256;  // tokens per tile (MMA N): each dequantized W tile feeds 256 tokens
 constexpr int BK = 64;   // k per stage (one 128-byte swizzle row of fp16)
-// X tiles (TMA) and dequantized W tiles use rings of STAGES and W_SLOTS
-// slots tracked by the same per-stage barriers: the dequant warps know W slot
-// q % W_SLOTS is free once the MMAs of stage q - W_SLOTS are done.  Equal
-// depths measured best (a deeper X ring at the cost of W slots lets the
-// dequantization fall behind).
-constexpr int STAGES = 4;
-constexpr int W_SLOTS = 4;
-static_assert(W_SLOTS <= STAGES, "a W slot's release is read from the stage barrier W_SLOTS back");
 constexpr int A_BYTES = BM * BK * 2;
-constexpr int B_BYTES = BN * BK * 2;
 constexpr int NUM_DQ_WARPS = 8;
 constexpr int NUM_EPI_WARPS = 4;
 constexpr int PK_WARP = 2 + NUM_DQ_WARPS + NUM_EPI_WARPS;  // packed-code producer
 constexpr int THREADS = (PK_WARP + 1) * 32;
 constexpr int kMaxPSlots = 8;
-constexpr uint32_t TMEM_COLS = 2 * BN;  // two accumulators
+constexpr int kMaxSplits = 16;
 
+// Per token-tile constants.  X tiles (TMA) and dequantized W tiles use rings
+// of STAGES and W_SLOTS slots tracked by the same per-stage barriers: the
+// dequant warps know W slot q % W_SLOTS is free once the MMAs of stage
+// q - W_SLOTS are done.  Equal depths measured best for BN = 256 (a deeper X
+// ring at the cost of W slots lets the dequantization fall behind); the
+// 2 KB X tiles of BN = 16 leave room for six.
+template <int BN>
+struct Cfg {
+    static_assert(BN == 16 || BN == 256, "token tile");
+    static constexpr int STAGES = BN >= 128 ? 4 : 6;
+    static constexpr int W_SLOTS = STAGES;
+    static constexpr int B_BYTES = BN * BK * 2;
+    static constexpr uint32_t TMEM_COLS = 2 * BN < 32 ? 32 : 2 * BN;  // two accumulators
+    // instruction descriptor, kind::f16: fp16 A and B, fp32 D, both K-major
+    static constexpr uint32_t IDESC = (1u << 4)                        // D format f32
+                                      | (0u << 7) | (0u << 10)          // A, B format f16
+                                      | ((uint32_t)(BN >> 3) << 17)     // N
+                                      | ((uint32_t)(BM >> 4) << 24);    // M
+    static constexpr int CHUNK = BN < 32 ? BN : 32;  // accumulator columns per tcgen05.ld
+};
+static_assert(Cfg<256>::W_SLOTS <= Cfg<256>::STAGES && Cfg<16>::W_SLOTS <= Cfg<16>::STAGES,
+              "a W slot's release is read from the stage barrier W_SLOTS back");
+
+template <int BN>
 struct SmemLayout {
-    uint8_t a[W_SLOTS][A_BYTES];
-    uint8_t b[STAGES][B_BYTES];
+    uint8_t a[Cfg<BN>::W_SLOTS][A_BYTES];
+    uint8_t b[Cfg<BN>::STAGES][Cfg<BN>::B_BYTES];
     // one barrier per direction and stage: the MMA thread waits once and
     // commits once per stage (its per-stage overhead bounds the MMA rate)
-    uint64_t full[STAGES];   // 8 dequant-warp arrivals + the X copy's bytes
-    uint64_t empty[STAGES];  // tcgen05.commit of the stage's MMAs
+    uint64_t full[Cfg<BN>::STAGES];   // 8 dequant-warp arrivals + the X copy's bytes
+    uint64_t empty[Cfg<BN>::STAGES];  // tcgen05.commit of the stage's MMAs
     uint64_t accum_full[2];
     uint64_t accum_empty[2];
     uint64_t pfull[kMaxPSlots];   // a packed superblock has landed (TMA bytes)
@@ -68,7 +92,10 @@ struct SmemLayout {
 };
 
 // The packed-code ring follows the layout (its size depends on the recipe).
-constexpr size_t kLayoutBytes = (sizeof(SmemLayout) + 1023) / 1024 * 1024;
+template <int BN>
+__host__ __device__ constexpr size_t layout_bytes() {
+    return (sizeof(SmemLayout<BN>) + 1023) / 1024 * 1024;
+}
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -136,8 +163,8 @@ __device__ __forceinline__ bool wait_phase(uint64_t *b, uint32_t parity, uint64_
     return mbar_try_wait(b, parity) || mbar_wait(b, parity, limit_ns, abort_flag);
 }
 
-__device__ __forceinline__ void raise_abort(SmemLayout &s, uint32_t *status) {
-    *reinterpret_cast<volatile uint32_t *>(&s.abort_flag) = 1u;
+__device__ __forceinline__ void raise_abort(uint32_t *abort_flag, uint32_t *status) {
+    *reinterpret_cast<volatile uint32_t *>(abort_flag) = 1u;
     atomicOr(status, kStatusTimeout);
 }
 
@@ -196,18 +223,13 @@ __device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
     return d;
 }
 
-// Instruction descriptor, kind::f16: fp16 A and B, fp32 D, both K-major.
-constexpr uint32_t kIdesc = (1u << 4)                  // D format f32
-                            | (0u << 7) | (0u << 10)    // A, B format f16
-                            | ((uint32_t)(BN >> 3) << 17)  // N
-                            | ((uint32_t)(BM >> 4) << 24); // M
-
-__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t acc) {
+__device__ __forceinline__ void mma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                        uint32_t acc) {
     asm volatile(
         "{\n\t.reg .pred p;\n\t"
         "setp.ne.b32 p, %4, 0;\n\t"
         "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n\t}" ::"r"(d_tmem),
-        "l"(adesc), "l"(bdesc), "r"(kIdesc), "r"(acc)
+        "l"(adesc), "l"(bdesc), "r"(idesc), "r"(acc)
         : "memory");
 }
 
@@ -230,6 +252,39 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
         : "r"(taddr)
         : "memory");
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 "
+        "{%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15])
+        : "r"(taddr)
+        : "memory");
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+template <int N>
+__device__ __forceinline__ void tmem_ld(uint32_t taddr, uint32_t (&r)[N]) {
+    static_assert(N == 16 || N == 32, "columns per load");
+    if constexpr (N == 32)
+        tmem_ld32(taddr, r);
+    else
+        tmem_ld16(taddr, r);
+}
+
+// k range of one work unit: tile t = u / splits, split s = u % splits takes
+// superblocks [sb0, sb1) of the nsb in k (128 weights each), i.e. the
+// 64-wide k blocks [2 sb0, 2 sb1).
+struct Unit {
+    int t, sb0, sb1;
+};
+
+__device__ __forceinline__ Unit unit_of(int u, int splits, int nsb) {
+    const int t = u / splits, s = u - t * splits;
+    return Unit{t, (int)((int64_t)s * nsb / splits), (int)((int64_t)(s + 1) * nsb / splits)};
 }
 
 // Codes and metadata one dequant thread needs for one 32-weight unit.
@@ -296,23 +351,28 @@ __device__ __forceinline__ void dequant_unit(const UnitRaw &u, __half2 (&v)[16])
     }
 }
 
-template <int BITS, int KIND>
+template <int BITS, int KIND, int BN>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_c,
                 const __grid_constant__ CUtensorMap tmap_l, const __grid_constant__ GemmArgs a) {
+    using C = Cfg<BN>;
+    constexpr int STAGES = C::STAGES;
+    constexpr int W_SLOTS = C::W_SLOTS;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
-    SmemLayout &s = *reinterpret_cast<SmemLayout *>(base);
-    const uint32_t pk_s = smem_u32(base + kLayoutBytes);  // packed-code ring
+    SmemLayout<BN> &s = *reinterpret_cast<SmemLayout<BN> *>(base);
+    const uint32_t pk_s = smem_u32(base + layout_bytes<BN>());  // packed-code ring
     volatile uint32_t *abort_flag = &s.abort_flag;
+    uint32_t *abort_w = &s.abort_flag;
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int nkb = (int)(a.k / BK);
-    const int mt = (int)((a.m + BN - 1) / BN);  // token tiles
-    const int nt = (int)((a.n + BM - 1) / BM);  // W-row tiles
-    const int ntiles = mt * nt;
-    // tile t: W rows n0 = (t / mt) * BM, tokens m0 = (t % mt) * BN; consecutive
-    // CTAs share a W tile (L2 reuse of the packed codes)
+    const int nsb = (int)(a.k / 128);             // superblocks (two 64-k stages) in k
+    const int mt = (int)((a.m + BN - 1) / BN);    // token tiles
+    const int nt = (int)((a.n + BM - 1) / BM);    // W-row tiles
+    const int S = a.splits;
+    const int nunits = mt * nt * S;
+    // unit u: tile t = u / S, W rows n0 = (t / mt) * BM, tokens m0 = (t % mt) * BN;
+    // consecutive CTAs share a W tile (L2 reuse of the packed codes)
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
@@ -337,7 +397,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(&s.tmem_base)),
-                     "r"(TMEM_COLS)
+                     "r"(C::TMEM_COLS)
                      : "memory");
         asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
@@ -349,19 +409,20 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         // ------------------------------------------------ TMA producer (X)
         if (lane == 0) {
-            int it = 0;  // stage counter across tiles
+            int it = 0;  // stage counter across units
             bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-                const int m0 = (t % mt) * BN;
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+            for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x) {
+                const Unit w = unit_of(u, S, nsb);
+                const int m0 = (w.t % mt) * BN;
+                for (int kb = 2 * w.sb0; kb < 2 * w.sb1; ++kb, ++it) {
                     const int st = it % STAGES;
                     const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
                     if (!wait_phase(&s.empty[st], ph ^ 1u, a.wait_limit_ns, abort_flag)) {
-                        raise_abort(s, a.status);
+                        raise_abort(abort_w, a.status);
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(&s.full[st], B_BYTES);
+                    mbar_arrive_expect_tx(&s.full[st], C::B_BYTES);
                     tma_load_2d(s.b[st], &tmap_x, &s.full[st], kb * BK, m0);
                 }
             }
@@ -376,20 +437,21 @@ __global__ void __launch_bounds__(THREADS, 1)
         if (lane == 0) {
             int it = 0, ti = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x, ++ti) {
+            for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x, ++ti) {
+                const Unit w = unit_of(u, S, nsb);
                 const int buf = ti & 1;
                 const uint32_t dcol = tmem_d + (uint32_t)(buf * BN);
                 if (ti >= 2 && !mbar_wait(&s.accum_empty[buf], (uint32_t)((ti >> 1) - 1) & 1u, a.wait_limit_ns,
                                           abort_flag)) {
-                    raise_abort(s, a.status);
+                    raise_abort(abort_w, a.status);
                     break;
                 }
                 tc_fence_after();
-                for (int kb = 0; kb < nkb; ++kb, ++it) {
+                for (int kb = 2 * w.sb0; kb < 2 * w.sb1; ++kb, ++it) {
                     const int st = it % STAGES;
                     const uint32_t ph = (uint32_t)(it / STAGES) & 1u;
                     if (!wait_phase(&s.full[st], ph, a.wait_limit_ns, abort_flag)) {
-                        raise_abort(s, a.status);
+                        raise_abort(abort_w, a.status);
                         ok = false;
                         break;
                     }
@@ -398,7 +460,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const uint64_t bd = sw128_desc(smem_u32(s.b[st]));
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk)  // +32 bytes along k per step
-                        mma_f16(dcol, ad + 2 * kk, bd + 2 * kk, (kb | kk) != 0 ? 1u : 0u);
+                        mma_f16(dcol, ad + 2 * kk, bd + 2 * kk, C::IDESC, (kb > 2 * w.sb0 || kk > 0) ? 1u : 0u);
                     mma_commit(&s.empty[st]);
                 }
                 if (ok) mma_commit(&s.accum_full[buf]);
@@ -414,9 +476,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int r = d >> 1;            // tile row 0..127
         const int half_id = d & 1;       // which 32-wide half of a stage
         const int P = a.pslots;
-        const int nsb = nkb / 2;         // superblocks (128 k = 2 stages) per tile
-        int q = 0;                       // stage counter across tiles
-        int sbi = 0;                     // superblock counter across tiles
+        int q = 0;                       // stage counter across units
+        int sbi = 0;                     // superblock counter across units
         bool ok = true;
         // codes of one superblock for this thread: its unit of each of the two stages
         auto read_sb = [&](int sb_global, int sbl, int64_t row, UnitRaw (&w)[2]) -> bool {
@@ -435,15 +496,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             if (lane == 0) mbar_arrive(&s.pempty[ps]);
             return true;
         };
-        for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-            const int64_t row = (int64_t)(t / mt) * BM + r;
+        for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x) {
+            const Unit wu = unit_of(u, S, nsb);
+            const int64_t row = (int64_t)(wu.t / mt) * BM + r;
             const bool valid = row < a.n;
             UnitRaw cur[2], nxt[2];
-            ok = read_sb(sbi, 0, row, cur);
-            for (int sbl = 0; sbl < nsb && ok; ++sbl, ++sbi) {
+            ok = read_sb(sbi, wu.sb0, row, cur);
+            for (int sbl = wu.sb0; sbl < wu.sb1 && ok; ++sbl, ++sbi) {
                 // the next superblock's codes are read while this one is dequantized
-                if (sbl + 1 < nsb && !read_sb(sbi + 1, sbl + 1, row, nxt)) {
-                    raise_abort(s, a.status);
+                if (sbl + 1 < wu.sb1 && !read_sb(sbi + 1, sbl + 1, row, nxt)) {
+                    raise_abort(abort_w, a.status);
                     ok = false;
                 }
                 // Both stages of the superblock: wait for both W slots, then
@@ -458,7 +520,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const int qf = q + h2 - W_SLOTS;
                     if (ok && qf >= 0 &&
                         !wait_phase(&s.empty[qf % STAGES], (uint32_t)(qf / STAGES) & 1u, a.wait_limit_ns, abort_flag)) {
-                        raise_abort(s, a.status);
+                        raise_abort(abort_w, a.status);
                         ok = false;
                     }
                 }
@@ -520,12 +582,13 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint32_t bytes = (uint32_t)(BITS == 3 ? BM * 48 + (KIND == 1 ? BM * a.lut_box : 0) : BM * 64);
             int sbi = 0;
             bool ok = true;
-            for (int t = blockIdx.x; t < ntiles && ok; t += gridDim.x) {
-                const int row0 = (t / mt) * BM;
-                for (int sb = 0; sb < nkb / 2; ++sb, ++sbi) {
+            for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x) {
+                const Unit w = unit_of(u, S, nsb);
+                const int row0 = (w.t / mt) * BM;
+                for (int sb = w.sb0; sb < w.sb1; ++sb, ++sbi) {
                     const int ps = sbi % P;
                     if (!wait_phase(&s.pempty[ps], ((uint32_t)(sbi / P) & 1u) ^ 1u, a.wait_limit_ns, abort_flag)) {
-                        raise_abort(s, a.status);
+                        raise_abort(abort_w, a.status);
                         ok = false;
                         break;
                     }
@@ -547,54 +610,93 @@ __global__ void __launch_bounds__(THREADS, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------ epilogue
+        constexpr int CH = C::CHUNK;
         const int quarter = warp & 3;  // the TMEM lanes (W rows) this warp may read
         int ti = 0;
-        for (int t = blockIdx.x; t < ntiles; t += gridDim.x, ++ti) {
+        for (int u = blockIdx.x; u < nunits; u += gridDim.x, ++ti) {
+            const int t = u / S;
             const int buf = ti & 1;
             const bool have = mbar_wait(&s.accum_full[buf], (uint32_t)(ti >> 1) & 1u, a.wait_limit_ns, abort_flag);
-            if (!have) raise_abort(s, a.status);
+            if (!have) raise_abort(abort_w, a.status);
             tc_fence_after();
             // tcgen05.ld is warp-collective: decide for the whole warp at once
             if (!__all_sync(0xffffffffu, have && !*abort_flag)) break;
             const int64_t n = (int64_t)(t / mt) * BM + 32 * quarter + lane;
             const int64_t m0 = (int64_t)(t % mt) * BN;
+            // this unit's partial: [BN][BM] fp32, row n of the tile at column
+            // 32 quarter + lane (a warp's stores are 128 contiguous bytes)
+            float *part = S > 1 ? a.ws_part + (size_t)u * BN * BM + 32 * quarter + lane : nullptr;
 #pragma unroll 1
-            for (int c = 0; c < BN; c += 32) {
-                uint32_t rv[32];
-                tmem_ld32(tmem_d + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * BN + c), rv);
-                if (n < a.n) {
+            for (int c = 0; c < BN; c += CH) {
+                uint32_t rv[CH];
+                tmem_ld<CH>(tmem_d + ((uint32_t)(32 * quarter) << 16) + (uint32_t)(buf * BN + c), rv);
+                if (S > 1) {
 #pragma unroll
-                    for (int j = 0; j < 32; ++j) {
+                    for (int j = 0; j < CH; ++j) part[(size_t)(c + j) * BM] = __uint_as_float(rv[j]);
+                } else if (n < a.n) {
+#pragma unroll
+                    for (int j = 0; j < CH; ++j) {
                         const int64_t m = m0 + c + j;
                         if (m < a.m) a.Y[m * a.n + n] = __float2half_rn(__uint_as_float(rv[j]));
                     }
                 }
             }
-            // this warp's rows of the accumulator are read: free it for tile ti + 2
+            // this warp's rows of the accumulator are read: free it for unit ti + 2
             tc_fence_before();
             __syncwarp();
             if (lane == 0) mbar_arrive(&s.accum_empty[buf]);
+            if (S > 1) {
+                // the last split of the tile to store its quarter sums all of
+                // them in split order and writes Y, then re-arms the counter
+                __threadfence();
+                __syncwarp();
+                uint32_t last = 0;
+                if (lane == 0) last = atomicAdd(&a.ws_cnt[(size_t)t * 4 + quarter], 1u) == (uint32_t)(S - 1) ? 1u : 0u;
+                last = __shfl_sync(0xffffffffu, last, 0);
+                if (last) {
+                    __threadfence();
+                    const float *p0 = a.ws_part + (size_t)t * S * BN * BM + 32 * quarter + lane;
+                    if (n < a.n) {
+#pragma unroll 1
+                        for (int j = 0; j < BN; ++j) {
+                            const int64_t m = m0 + j;
+                            if (m >= a.m) break;
+                            float v = 0.0f;
+                            for (int sp = 0; sp < S; ++sp) v += __ldcg(p0 + ((size_t)sp * BN + j) * BM);
+                            a.Y[m * a.n + n] = __float2half_rn(v);
+                        }
+                    }
+                    __syncwarp();
+                    if (lane == 0) a.ws_cnt[(size_t)t * 4 + quarter] = 0u;
+                }
+            }
         }
     }
     tc_fence_before();
     __syncthreads();
     if (warp == 1) {
         tc_fence_after();
-        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_d), "r"(TMEM_COLS)
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem_d), "r"(C::TMEM_COLS)
                      : "memory");
     }
 }
 
-template <int BITS, int KIND>
+template <int BITS, int KIND, int BN>
 cudaError_t launch_t(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &ml, const GemmArgs &a,
-                     int num_sms, cudaStream_t st) {
-    auto kern = gemm_kernel<BITS, KIND>;
+                     int64_t units, int num_sms, cudaStream_t st) {
+    auto kern = gemm_kernel<BITS, KIND, BN>;
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
     if (e != cudaSuccess) return e;
-    const int64_t tiles = ((a.m + BN - 1) / BN) * ((a.n + BM - 1) / BM);
-    const unsigned grid = (unsigned)std::min<int64_t>(tiles, num_sms);
+    const unsigned grid = (unsigned)std::min<int64_t>(units, num_sms);
     kern<<<grid, THREADS, a.smem_bytes, st>>>(mx, mc, ml, a);
     return cudaGetLastError();
+}
+
+template <int BITS, int KIND>
+cudaError_t launch_bn(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &ml, const GemmArgs &a,
+                      int64_t units, int num_sms, cudaStream_t st) {
+    if (a.bn == 16) return launch_t<BITS, KIND, 16>(mx, mc, ml, a, units, num_sms, st);
+    return launch_t<BITS, KIND, 256>(mx, mc, ml, a, units, num_sms, st);
 }
 
 }  // namespace
@@ -612,16 +714,46 @@ EncodeTiledFn encode_fn() {
     return fn;
 }
 
+GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_split) {
+    GemmPlan p{};
+    p.bn = m <= 16 ? 16 : 256;
+    const int64_t mt = (m + p.bn - 1) / p.bn, nt = (n + BM - 1) / BM;
+    p.tiles = mt * nt;
+    const int nsb = (int)(k / 128);
+    p.splits = 1;
+    if (allow_split && p.bn == 16 && num_sms > 0 && p.tiles <= (int64_t)(kSplitCounterBytes / 16)) {
+        // time ~ rounds of units per CTA x (superblocks per unit + a fixed
+        // cost of about two superblocks per unit: pipeline fill, epilogue)
+        int64_t best = -1;
+        for (int sp = 1; sp <= std::min(nsb, kMaxSplits); ++sp) {
+            const int64_t rounds = (p.tiles * sp + num_sms - 1) / num_sms;
+            const int64_t cost = rounds * ((nsb + sp - 1) / sp + 2);
+            if (best < 0 || cost < best) {
+                best = cost;
+                p.splits = sp;
+            }
+        }
+    }
+    p.units = p.tiles * p.splits;
+    p.ws_bytes = p.splits > 1 ? kSplitCounterBytes + (size_t)p.units * p.bn * BM * sizeof(float) : 0;
+    return p;
+}
+
 cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
     GemmArgs a = args;
+    if (a.bn != 16 && a.bn != 256) return cudaErrorInvalidValue;
+    if (a.splits < 1 || a.splits > kMaxSplits || a.splits > a.k / 128) return cudaErrorInvalidValue;
+    if (a.splits > 1 && (a.ws_part == nullptr || a.ws_cnt == nullptr)) return cudaErrorInvalidValue;
+    const int64_t units = ((a.m + a.bn - 1) / a.bn) * ((a.n + BM - 1) / BM) * a.splits;
+    if (units > ((int64_t)1 << 31) - 1) return cudaErrorInvalidValue;
     const cuuint32_t estr[3] = {1, 1, 1};
     CUtensorMap mx{}, mc{}, ml{};
     {
         const cuuint64_t dims[2] = {(cuuint64_t)a.k, (cuuint64_t)a.m};
         const cuuint64_t strides[1] = {(cuuint64_t)a.k * 2};
-        const cuuint32_t box[2] = {BK, BN};
+        const cuuint32_t box[2] = {BK, (cuuint32_t)a.bn};
         if (enc(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<__half *>(a.X), dims, strides, box, estr,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
@@ -661,13 +793,14 @@ cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     }
     a.pslot_bytes = (a.bits == 3 ? BM * 48 + BM * a.lut_box : BM * 64 + 0);
     a.pslot_bytes = (a.pslot_bytes + 1023) / 1024 * 1024;
-    const int budget = 227 * 1024 - (int)kLayoutBytes - 1024;
+    const int layout = (int)(a.bn == 16 ? layout_bytes<16>() : layout_bytes<256>());
+    const int budget = 227 * 1024 - layout - 1024;
     a.pslots = std::min(kMaxPSlots, budget / a.pslot_bytes);
     if (a.pslots < 2) return cudaErrorInvalidConfiguration;
-    a.smem_bytes = (int)kLayoutBytes + 1024 + a.pslots * a.pslot_bytes;
-    if (a.bits == 4) return launch_t<4, 0>(mx, mc, ml, a, num_sms, st);
-    if (a.kind == 1) return launch_t<3, 1>(mx, mc, ml, a, num_sms, st);
-    return launch_t<3, 0>(mx, mc, ml, a, num_sms, st);
+    a.smem_bytes = layout + 1024 + a.pslots * a.pslot_bytes;
+    if (a.bits == 4) return launch_bn<4, 0>(mx, mc, ml, a, units, num_sms, st);
+    if (a.kind == 1) return launch_bn<3, 1>(mx, mc, ml, a, units, num_sms, st);
+    return launch_bn<3, 0>(mx, mc, ml, a, units, num_sms, st);
 }
 
 }  // namespace qx

@@ -83,7 +83,32 @@ struct GemmArgs {
     // superblock of a 128-row W tile
     int pslots, pslot_bytes, lut_box;
     int smem_bytes;
+    // token tile (16 or 256) and the number of k splits of every tile (from
+    // plan_gemm); with splits > 1, ws_cnt [tiles][4] counts the row quarters
+    // that have stored their fp32 partial tiles to ws_part [units][bn][128]
+    int bn, splits;
+    float *ws_part;
+    uint32_t *ws_cnt;
 };
+
+// A split-k workspace starts with a fixed region of counters (one word per
+// row quarter of a tile, so at most 4096 tiles split), which every completed
+// call leaves zero whatever the shapes of earlier calls; the fp32 partial
+// tiles follow it.
+constexpr size_t kSplitCounterBytes = 65536;
+
+// Tiling of one prefill/decode matmul on the tensor cores.
+struct GemmPlan {
+    int bn;            // tokens per tile: 16 for m <= 16, else 256
+    int splits;        // k splits per tile (1: no workspace)
+    int64_t tiles;     // token tiles x 128-row W tiles
+    int64_t units;     // tiles x splits
+    size_t ws_bytes;   // workspace the split needs (0 when splits == 1)
+};
+
+// allow_split = false: one CTA per tile (qx_gemm); true: k is split when the
+// tile grid leaves SMs idle (qx_gemm_splitk).
+GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_split);
 
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);

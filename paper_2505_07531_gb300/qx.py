@@ -79,6 +79,8 @@ def _lib():
         lib.qx_dequant.argtypes = [P(_Packed), VP, VP]
         lib.qx_gemv.argtypes = [P(_Packed), VP, I32, VP, I32, VP]
         lib.qx_gemm.argtypes = [P(_Packed), VP, I64, VP, VP]
+        lib.qx_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(_Recipe), P(ctypes.c_size_t)]
+        lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
@@ -87,7 +89,7 @@ def _lib():
         lib.qx_last_error_string.argtypes = []
         lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
-                   "qx_get_device_status", "qx_version"):
+                   "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -247,6 +249,49 @@ def gemm(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> t
     _dev_tensor(Y, "out")
     pc = P.c()
     _check(_lib().qx_gemm(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _stream(X.device)), "qx_gemm")
+    return Y
+
+
+def gemm_splitk_workspace_bytes(n: int, k: int, m: int, recipe: Recipe) -> int:
+    """Workspace bytes qx_gemm_splitk needs on the current device (0: no split)."""
+    b = ctypes.c_size_t(0)
+    r = recipe.c()
+    _check(_lib().qx_gemm_splitk_workspace(n, k, m, ctypes.byref(r), ctypes.byref(b)), "qx_gemm_splitk_workspace")
+    return int(b.value)
+
+
+_WORKSPACES: dict = {}
+
+
+def splitk_workspace(device, nbytes: int) -> torch.Tensor:
+    """A zero-filled workspace of at least `nbytes` for `device`, kept per
+    device and current stream (calls on one stream run one after another, so
+    they may share it; qx_gemm_splitk leaves it zero-filled)."""
+    dev = torch.device(device)
+    key = (dev.index, torch.cuda.current_stream(dev).cuda_stream)
+    ws = _WORKSPACES.get(key)
+    if ws is None or ws.numel() < nbytes:
+        ws = torch.zeros(max(nbytes, 256), dtype=torch.uint8, device=dev)
+        _WORKSPACES[key] = ws
+    return ws
+
+
+def gemm_splitk(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None,
+                workspace: torch.Tensor | None = None) -> torch.Tensor:
+    """Y = X W_hat^T with k split across CTAs when the tiles alone leave SMs
+    idle (qx_gemm_splitk): the tensor-core decode path for 1..16 rows of X and
+    the path for short prefills.  Returns fp16 [m][n]."""
+    _dev_tensor(X, "X")
+    m = X.shape[0]
+    Y = out if out is not None else torch.empty((m, P.n), dtype=torch.float16, device=X.device)
+    _dev_tensor(Y, "out")
+    need = gemm_splitk_workspace_bytes(P.n, P.k, m, P.recipe)
+    ws = workspace if workspace is not None else splitk_workspace(X.device, need)
+    if not ws.is_cuda or ws.dtype != torch.uint8:
+        raise ValueError("workspace must be a CUDA uint8 tensor")
+    pc = P.c()
+    _check(_lib().qx_gemm_splitk(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _ptr(ws), ws.numel(), _stream(X.device)),
+           "qx_gemm_splitk")
     return Y
 
 

@@ -328,3 +328,122 @@ def test_mixed_recipe_vision_prefill(qx):
         assert qx.device_status() == 0
         rec = _orecipe(4, 128, 0)
         _check_matmul(Y.cpu().numpy(), oracle.gemm(ref, rec, X, k), X, oracle.dequant(ref, rec, k))
+
+
+# ---------------------------------------------------------------- split-k tensor-core matmul
+@pytest.mark.parametrize("m", [1, 3, 16, 17, 200])
+@pytest.mark.parametrize("case", CASES, ids=_ids)
+def test_gemm_splitk_tolerance(qx, packed, case, m):
+    W, P, ref = packed[case]
+    n, k, bits, g, kind = case
+    X = synth.activations(m, k, seed=m + 1, stream=5 * k)
+    Y = qx.gemm_splitk(P, torch.from_numpy(X).cuda())
+    assert qx.device_status() == 0
+    rec = _orecipe(bits, g, kind)
+    _check_matmul(Y.cpu().numpy(), oracle.gemm(ref, rec, X, k), X, oracle.dequant(ref, rec, k))
+
+
+@pytest.mark.parametrize("bits,g,kind", [(3, 128, 1), (4, 64, 0), (3, 64, 0)])
+def test_gemm_splitk_deterministic_and_rearmed(qx, bits, g, kind):
+    """A ragged 1000-row matrix (8 W tiles) with k = 4096 split across CTAs: the
+    result does not depend on which split finishes last, every call leaves the
+    workspace counters at zero, and a short workspace is refused."""
+    n, k = 1000, 4096
+    rec = _orecipe(bits, g, kind)
+    W = _weights(n, k, seed=500 + bits + g)
+    ref = oracle.quantize(W, rec)
+    Wh = oracle.dequant(ref, rec, k)
+    P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+    for m in (1, 5, 16):
+        nbytes = qx.gemm_splitk_workspace_bytes(n, k, m, P.recipe)
+        assert nbytes > 0
+        ws = torch.zeros(nbytes, dtype=torch.uint8, device="cuda")
+        X = synth.activations(m, k, seed=m, stream=77)
+        Xd = torch.from_numpy(X).cuda()
+        Y1 = qx.gemm_splitk(P, Xd, workspace=ws)
+        Y2 = qx.gemm_splitk(P, Xd, workspace=ws)
+        assert qx.device_status() == 0
+        assert torch.equal(Y1, Y2)
+        assert int(ws[:65536].count_nonzero()) == 0  # the counter region
+        _check_matmul(Y1.cpu().numpy(), oracle.gemm(ref, rec, X, k), X, Wh)
+    with pytest.raises(qx.QxError) as e:
+        qx.gemm_splitk(P, Xd, workspace=torch.zeros(256, dtype=torch.uint8, device="cuda"))
+    assert e.value.code == 1
+
+
+# ---------------------------------------------------------------- full sizes, sampled rows
+# The Llama-7B-shaped layer of the decode benchmark in 3-bit LUT g128.  The
+# weights are drawn on the GPU and quantized there; for each matrix a seeded
+# sample of rows is also quantized by the oracle (quantization is row-local,
+# so those rows' codes and outputs are unique) and every output of those rows
+# is checked.
+LLAMA_LAYER = [("q_proj", 4096, 4096, 0.01), ("k_proj", 4096, 4096, 0.01), ("v_proj", 4096, 4096, 0.02),
+               ("o_proj", 4096, 4096, 0.02), ("gate_proj", 11008, 4096, 0.04), ("up_proj", 11008, 4096, 0.04),
+               ("down_proj", 4096, 11008, 0.04)]
+SAMPLE_ROWS = 48
+
+
+@pytest.fixture(scope="module")
+def llama_layer(qx):
+    rec = _orecipe(3, 128, 1)
+    out = {}
+    for i, (nm, n, k, sigma) in enumerate(LLAMA_LAYER):
+        W = synth.student_t_weights_torch(n, k, sigma, seed=7, stream=i, device="cuda")
+        P = qx.quantize(W, qx.Recipe(3, 128, 1))
+        rows = np.sort(np.random.default_rng(i).choice(n, size=SAMPLE_ROWS, replace=False))
+        ref = oracle.quantize(W[torch.from_numpy(rows).cuda()].cpu().numpy(), rec)
+        out[nm] = (P, rows, ref, oracle.dequant(ref, rec, k))
+        del W
+    assert qx.device_status() == 0
+    return out
+
+
+def test_full_size_decode_layer_sampled(qx, llama_layer):
+    """The decode benchmark's launch configuration: q,k,v | o | gate,up | down as
+    four qx_gemv_multi launches with programmatic dependent launch, captured in
+    one CUDA graph, batch 1."""
+    chain = [(["q_proj", "k_proj", "v_proj"], 4096), (["o_proj"], 4096), (["gate_proj", "up_proj"], 4096),
+             (["down_proj"], 11008)]
+    xs = [synth.activations(1, k, seed=0, stream=60 + j) for j, (_, k) in enumerate(chain)]
+    dx = [torch.from_numpy(x).cuda() for x in xs]
+    ys = {nm: torch.empty((1, n), dtype=torch.float16, device="cuda") for nm, n, _, _ in LLAMA_LAYER}
+    s = torch.cuda.Stream()
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        for (names, _), x in zip(chain, dx):
+            qx.gemv_multi([llama_layer[nm][0] for nm in names], [x] * len(names), outs=[ys[nm] for nm in names],
+                          pdl=True)
+    for y in ys.values():
+        y.fill_(float("nan"))
+    g.replay()
+    torch.cuda.synchronize()
+    assert qx.device_status() == 0
+    rec = _orecipe(3, 128, 1)
+    for (names, k), x in zip(chain, xs):
+        for nm in names:
+            P, rows, ref, Wh = llama_layer[nm]
+            _check_matmul(ys[nm].float().cpu().numpy()[:, rows], oracle.gemv(ref, rec, x, k), x, Wh)
+
+
+@pytest.mark.parametrize("m", [1, 4, 16])
+def test_full_size_tensor_core_decode_sampled(qx, llama_layer, m):
+    """qx_gemm_splitk as a decode matmul (16-token tiles, k split) on the layer's shapes."""
+    rec = _orecipe(3, 128, 1)
+    for nm in ("q_proj", "gate_proj", "down_proj"):
+        P, rows, ref, Wh = llama_layer[nm]
+        X = synth.activations(m, P.k, seed=m, stream=70)
+        Y = qx.gemm_splitk(P, torch.from_numpy(X).cuda())
+        assert qx.device_status() == 0
+        _check_matmul(Y.cpu().numpy()[:, rows], oracle.gemm(ref, rec, X, P.k), X, Wh)
+
+
+def test_full_size_prefill_sampled(qx, llama_layer):
+    """Prefill of 2048 tokens against 11008x4096 and 4096x11008 (the GEMM benchmark's shapes)."""
+    rec = _orecipe(3, 128, 1)
+    for nm in ("gate_proj", "down_proj"):
+        P, rows, ref, Wh = llama_layer[nm]
+        X = synth.activations(2048, P.k, seed=2, stream=80)
+        Y = qx.gemm(P, torch.from_numpy(X).cuda())
+        assert qx.device_status() == 0
+        _check_matmul(Y.cpu().numpy()[:, rows], oracle.gemm(ref, rec, X, P.k), X, Wh)
