@@ -510,6 +510,22 @@ def _chain_graph(qx, torch, stream, layers, chain, outs, pdl=True):
     return g
 
 
+def _splitk_graph(qx, torch, stream, layers, xs, outs):
+    """One CUDA graph of the seven tensor-core (split-k) matmuls over every layer copy."""
+    def body():
+        for L in layers:
+            for nm, P in L.items():
+                qx.gemm_splitk(P, xs[nm], out=outs[nm])
+
+    with torch.cuda.stream(stream):
+        body()  # also sizes the stream's workspace before capture
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=stream):
+        body()
+    return g
+
+
 def _time_graph(torch, stream, g, reps):
     with torch.cuda.stream(stream):
         for _ in range(3):
@@ -524,7 +540,9 @@ def _time_graph(torch, stream, g, reps):
 
 
 def run_config3(qx, torch, dev, stream, l2):
-    """Llama-7B layer, 4-bit uniform g128 and 3-bit uniform g64, batch 1 / 4 / 16."""
+    """Llama-7B layer, 4-bit uniform g128 and 3-bit uniform g64, batch 1 / 4 / 16:
+    the CUDA-core decode chain (qx_gemv_multi, PDL) and, for batch 4 and 16,
+    the tensor-core path (qx_gemm_splitk, one launch per matrix)."""
     import synth
 
     out = {}
@@ -546,8 +564,18 @@ def run_config3(qx, torch, dev, stream, l2):
             io = sum(x.numel() * 2 for x in xs) + sum(y.numel() * 2 for y in ys.values())
             out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}"] = {
                 "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
-                "weight_bytes": layer_bytes, "launches_per_layer": 4 * ((batch + 3) // 4)}
+                "weight_bytes": layer_bytes, "path": "qx_gemv_multi chain (CUDA cores)"}
+            if batch >= 4:
+                xn = {nm: xs[3] if nm == "down_proj" else xs[0] for nm, *_ in LAYER}
+                gr = _splitk_graph(qx, torch, stream, layers, xn, ys)
+                ms = _time_graph(torch, stream, gr, 20) / copies
+                del gr
+                out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}_tensorcore"] = {
+                    "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
+                    "weight_bytes": layer_bytes, "path": "qx_gemm_splitk per matrix (tcgen05, k split)"}
         del layers, base
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("config-3 decode reported a device error")
     return out
 
 
