@@ -180,6 +180,17 @@ qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const qx_rec
 qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, void *workspace,
                          size_t workspace_bytes, void *stream);
 
+/* qx_gemm_splitk for callers that cannot allocate device memory: it allocates
+ * nothing and takes no workspace.  The partial tiles go to a scratch array of
+ * 4 MiB that the library holds in static device memory, one per device (64 KiB
+ * of counters, then room for 504 split units of 16 tokens); its address is
+ * looked up once per device.  Each call clears the counters it uses on
+ * `stream` before the launch.  Same arguments, results and rules as
+ * qx_gemm_splitk otherwise; calls on one device must not run at the same time
+ * (they share the scratch).  Returns QX_ERR_UNSUPPORTED when the split plan
+ * needs more than the scratch holds (qx_gemm_splitk_workspace() > 4 MiB). */
+qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream);
+
 /* Synchronize `stream`, then return and clear the current device's status word
  * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
  * synchronization itself fails. */

@@ -384,6 +384,30 @@ QX_API qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, vo
     return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
 }
 
+QX_API qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream) {
+    qx_status s = check_gemm_args(p, X, m, Y);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    const qx::GemmPlan plan = qx::plan_gemm(p->n, p->k, m, d->num_sms, true);
+    if (plan.ws_bytes > qx::kNoAllocScratchBytes) return QX_ERR_UNSUPPORTED;
+    qx::GemmArgs a = gemm_args(p, X, m, Y, d);
+    a.bn = plan.bn;
+    a.splits = plan.splits;
+    if (plan.splits > 1) {
+        void *ws = nullptr;
+        cudaError_t e = qx::noalloc_scratch(&ws);
+        if (e != cudaSuccess) return from_cuda(e);
+        // re-arm this call's counters on the stream (they are zero unless an
+        // earlier call gave up on a wait); a memset, not an allocation
+        e = cudaMemsetAsync(ws, 0, (size_t)plan.tiles * 4 * sizeof(uint32_t), static_cast<cudaStream_t>(stream));
+        if (e != cudaSuccess) return from_cuda(e);
+        a.ws_cnt = static_cast<uint32_t *>(ws);
+        a.ws_part = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + qx::kSplitCounterBytes);
+    }
+    return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
 QX_API qx_status qx_get_device_status(void *stream) {
     DeviceInfo *d = nullptr;
     qx_status s = device_info(&d);

@@ -35,6 +35,8 @@
 // drain, frees tensor memory and returns.
 #include <cuda.h>
 
+#include <mutex>
+
 #include "qx_kernels.cuh"
 
 namespace qx {
@@ -801,6 +803,35 @@ cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     if (a.bits == 4) return launch_bn<4, 0>(mx, mc, ml, a, units, num_sms, st);
     if (a.kind == 1) return launch_bn<3, 1>(mx, mc, ml, a, units, num_sms, st);
     return launch_bn<3, 0>(mx, mc, ml, a, units, num_sms, st);
+}
+
+// ------------------------------------------------ no-allocation variant
+// Scratch of qx_gemm_splitk_noalloc, for callers that cannot allocate device
+// memory: a file-scope device array (zero when the module loads) takes the
+// place of the caller's workspace -- the 64 KiB counter region, then 4032 KiB
+// of fp32 partial tiles (504 units of 16 tokens x 128 rows).
+namespace {
+constexpr int kNoAllocDevices = 64;
+static __device__ __align__(256) uint8_t g_splitk_scratch[kNoAllocScratchBytes];
+void *g_splitk_scratch_addr[kNoAllocDevices];
+std::mutex g_splitk_scratch_mu;
+}  // namespace
+
+cudaError_t noalloc_scratch(void **ptr) {
+    int dev = -1;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (dev < 0 || dev >= kNoAllocDevices) return cudaErrorInvalidDevice;
+    std::lock_guard<std::mutex> lock(g_splitk_scratch_mu);
+    if (g_splitk_scratch_addr[dev] == nullptr) {
+        // once per device, with that device current
+        void *p = nullptr;
+        e = cudaGetSymbolAddress(&p, g_splitk_scratch);
+        if (e != cudaSuccess) return e;
+        g_splitk_scratch_addr[dev] = p;
+    }
+    *ptr = g_splitk_scratch_addr[dev];
+    return cudaSuccess;
 }
 
 }  // namespace qx

@@ -110,6 +110,12 @@ struct GemmPlan {
 // tile grid leaves SMs idle (qx_gemm_splitk).
 GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_split);
 
+// Size of the file-scope scratch that qx_gemm_splitk_noalloc uses in place of
+// a workspace, and its device address on the current device (looked up once
+// per device with cudaGetSymbolAddress).
+constexpr size_t kNoAllocScratchBytes = (size_t)4 << 20;
+cudaError_t noalloc_scratch(void **ptr);
+
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
 bool plan_gemv(GemvMulti &a, int num_sms);

@@ -81,6 +81,7 @@ def _lib():
         lib.qx_gemm.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(_Recipe), P(ctypes.c_size_t)]
         lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, VP]
+        lib.qx_gemm_splitk_noalloc.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
@@ -89,7 +90,8 @@ def _lib():
         lib.qx_last_error_string.argtypes = []
         lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
-                   "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_get_device_status", "qx_version"):
+                   "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc",
+                   "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -292,6 +294,19 @@ def gemm_splitk(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = Non
     pc = P.c()
     _check(_lib().qx_gemm_splitk(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _ptr(ws), ws.numel(), _stream(X.device)),
            "qx_gemm_splitk")
+    return Y
+
+
+def gemm_splitk_noalloc(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+    """qx_gemm_splitk without a workspace (qx_gemm_splitk_noalloc): the library's
+    static 4 MiB scratch holds the partial tiles.  Returns fp16 [m][n]."""
+    _dev_tensor(X, "X")
+    m = X.shape[0]
+    Y = out if out is not None else torch.empty((m, P.n), dtype=torch.float16, device=X.device)
+    _dev_tensor(Y, "out")
+    pc = P.c()
+    _check(_lib().qx_gemm_splitk_noalloc(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _stream(X.device)),
+           "qx_gemm_splitk_noalloc")
     return Y
 
 
