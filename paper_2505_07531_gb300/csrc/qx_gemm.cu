@@ -659,13 +659,25 @@ __global__ void __launch_bounds__(THREADS, 1)
                     __threadfence();
                     const float *p0 = a.ws_part + (size_t)t * S * BN * BM + 32 * quarter + lane;
                     if (n < a.n) {
+                        // a chunk of columns at a time, splits outer: the CH loads
+                        // of one split are independent (one round trip to L2 per
+                        // split, not per column); the sum order stays split order
 #pragma unroll 1
-                        for (int j = 0; j < BN; ++j) {
-                            const int64_t m = m0 + j;
-                            if (m >= a.m) break;
-                            float v = 0.0f;
-                            for (int sp = 0; sp < S; ++sp) v += __ldcg(p0 + ((size_t)sp * BN + j) * BM);
-                            a.Y[m * a.n + n] = __float2half_rn(v);
+                        for (int c = 0; c < BN; c += CH) {
+                            float v[CH];
+#pragma unroll
+                            for (int j = 0; j < CH; ++j) v[j] = 0.0f;
+#pragma unroll 1
+                            for (int sp = 0; sp < S; ++sp) {
+                                const float *ps = p0 + ((size_t)sp * BN + c) * BM;
+#pragma unroll
+                                for (int j = 0; j < CH; ++j) v[j] += __ldcg(ps + (size_t)j * BM);
+                            }
+#pragma unroll
+                            for (int j = 0; j < CH; ++j) {
+                                const int64_t m = m0 + c + j;
+                                if (m < a.m) a.Y[m * a.n + n] = __float2half_rn(v[j]);
+                            }
                         }
                     }
                     __syncwarp();
