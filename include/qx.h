@@ -165,7 +165,8 @@ qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const qx_rec
 /* qx_gemm with the contraction split along k (at 128-weight boundaries) when
  * the tiles alone would leave SMs idle -- the decode case (m <= 16: 16-token
  * tiles, so this is also the tensor-core decode matmul for batches of 1..16)
- * and short prefills.  Each split stores an fp32 partial tile to `workspace`;
+ * and short prefills (64-token tiles split along k, or 256-token tiles,
+ * whichever the tile count favours).  Each split stores an fp32 partial tile to `workspace`;
  * the last split of a tile to finish sums the partials in split order (the
  * result does not depend on timing) and writes Y.  Same X, Y, m rules as
  * qx_gemm.

@@ -9,7 +9,8 @@
 // the dequantization below the tensor-core time); BN = 16 for m <= 16, which
 // makes the same kernel a decode matmul for batches of up to 16 tokens: the
 // tensor cores then take the products, and the dequantization alone bounds
-// the rate.
+// the rate; BN = 64 (split-k calls only) for short prefills whose 256-token
+// tiles would leave SMs idle.
 //
 // Persistent: one CTA per SM walks the work units -- (W-row tile, token tile,
 // k split).  A tile is split along k (at 128-weight superblock boundaries)
@@ -58,10 +59,10 @@ constexpr int kMaxSplits = 16;
 // dequant warps know W slot q % W_SLOTS is free once the MMAs of stage
 // q - W_SLOTS are done.  Equal depths measured best for BN = 256 (a deeper X
 // ring at the cost of W slots lets the dequantization fall behind); the
-// 2 KB X tiles of BN = 16 leave room for six.
+// 2 KB and 8 KB X tiles of BN = 16 and 64 leave room for six.
 template <int BN>
 struct Cfg {
-    static_assert(BN == 16 || BN == 256, "token tile");
+    static_assert(BN == 16 || BN == 64 || BN == 256, "token tile");
     static constexpr int STAGES = BN >= 128 ? 4 : 6;
     static constexpr int W_SLOTS = STAGES;
     static constexpr int B_BYTES = BN * BK * 2;
@@ -73,7 +74,8 @@ struct Cfg {
                                       | ((uint32_t)(BM >> 4) << 24);    // M
     static constexpr int CHUNK = BN < 32 ? BN : 32;  // accumulator columns per tcgen05.ld
 };
-static_assert(Cfg<256>::W_SLOTS <= Cfg<256>::STAGES && Cfg<16>::W_SLOTS <= Cfg<16>::STAGES,
+static_assert(Cfg<256>::W_SLOTS <= Cfg<256>::STAGES && Cfg<64>::W_SLOTS <= Cfg<64>::STAGES &&
+                  Cfg<16>::W_SLOTS <= Cfg<16>::STAGES,
               "a W slot's release is read from the stage barrier W_SLOTS back");
 
 template <int BN>
@@ -710,6 +712,7 @@ template <int BITS, int KIND>
 cudaError_t launch_bn(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &ml, const GemmArgs &a,
                       int64_t units, int num_sms, cudaStream_t st) {
     if (a.bn == 16) return launch_t<BITS, KIND, 16>(mx, mc, ml, a, units, num_sms, st);
+    if (a.bn == 64) return launch_t<BITS, KIND, 64>(mx, mc, ml, a, units, num_sms, st);
     return launch_t<BITS, KIND, 256>(mx, mc, ml, a, units, num_sms, st);
 }
 
@@ -729,22 +732,34 @@ EncodeTiledFn encode_fn() {
 }
 
 GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_split) {
+    const int nsb = (int)(k / 128);
+    const int64_t nt = (n + BM - 1) / BM;
     GemmPlan p{};
     p.bn = m <= 16 ? 16 : 256;
-    const int64_t mt = (m + p.bn - 1) / p.bn, nt = (n + BM - 1) / BM;
-    p.tiles = mt * nt;
-    const int nsb = (int)(k / 128);
     p.splits = 1;
-    if (allow_split && p.bn == 16 && num_sms > 0 && p.tiles <= (int64_t)(kSplitCounterBytes / 16)) {
-        // time ~ rounds of units per CTA x (superblocks per unit + a fixed
-        // cost of about two superblocks per unit: pipeline fill, epilogue)
-        int64_t best = -1;
-        for (int sp = 1; sp <= std::min(nsb, kMaxSplits); ++sp) {
-            const int64_t rounds = (p.tiles * sp + num_sms - 1) / num_sms;
-            const int64_t cost = rounds * ((nsb + sp - 1) / sp + 2);
-            if (best < 0 || cost < best) {
-                best = cost;
-                p.splits = sp;
+    p.tiles = ((m + p.bn - 1) / p.bn) * nt;
+    if (allow_split && num_sms > 0) {
+        // Time ~ rounds of units per CTA x (superblocks per unit + about two
+        // for pipeline fill and epilogue), plus the last split's reduction
+        // (one L2 round trip, about half a superblock, per split and 32
+        // columns).  Decode sizes take 16-token tiles; longer inputs choose
+        // between 64-token tiles, which may split k, and 256-token tiles.
+        const int cands[2] = {m <= 16 ? 16 : 64, 256};
+        double best = -1.0;
+        for (int ci = 0; ci < (m <= 16 ? 1 : 2); ++ci) {
+            const int bn = cands[ci];
+            const int64_t tiles = ((m + bn - 1) / bn) * nt;
+            const int smax = (bn == 256 || tiles > (int64_t)(kSplitCounterBytes / 16)) ? 1 : std::min(nsb, kMaxSplits);
+            for (int sp = 1; sp <= smax; ++sp) {
+                const int64_t rounds = (tiles * sp + num_sms - 1) / num_sms;
+                const double cost = (double)rounds * ((nsb + sp - 1) / sp + 2) +
+                                    (sp > 1 ? 0.5 * sp * ((bn + 31) / 32) : 0.0);
+                if (best < 0 || cost < best) {
+                    best = cost;
+                    p.bn = bn;
+                    p.splits = sp;
+                    p.tiles = tiles;
+                }
             }
         }
     }
@@ -757,7 +772,7 @@ cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     EncodeTiledFn enc = encode_fn();
     if (enc == nullptr) return cudaErrorNotSupported;
     GemmArgs a = args;
-    if (a.bn != 16 && a.bn != 256) return cudaErrorInvalidValue;
+    if (a.bn != 16 && a.bn != 64 && a.bn != 256) return cudaErrorInvalidValue;
     if (a.splits < 1 || a.splits > kMaxSplits || a.splits > a.k / 128) return cudaErrorInvalidValue;
     if (a.splits > 1 && (a.ws_part == nullptr || a.ws_cnt == nullptr)) return cudaErrorInvalidValue;
     const int64_t units = ((a.m + a.bn - 1) / a.bn) * ((a.n + BM - 1) / BM) * a.splits;
@@ -807,7 +822,7 @@ cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     }
     a.pslot_bytes = (a.bits == 3 ? BM * 48 + BM * a.lut_box : BM * 64 + 0);
     a.pslot_bytes = (a.pslot_bytes + 1023) / 1024 * 1024;
-    const int layout = (int)(a.bn == 16 ? layout_bytes<16>() : layout_bytes<256>());
+    const int layout = (int)(a.bn == 16 ? layout_bytes<16>() : a.bn == 64 ? layout_bytes<64>() : layout_bytes<256>());
     const int budget = 227 * 1024 - layout - 1024;
     a.pslots = std::min(kMaxPSlots, budget / a.pslot_bytes);
     if (a.pslots < 2) return cudaErrorInvalidConfiguration;

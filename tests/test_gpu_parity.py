@@ -324,10 +324,12 @@ def test_mixed_recipe_vision_prefill(qx):
         P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(4, 128, 0))
         ref = oracle.quantize(W, _orecipe(4, 128, 0))
         X = synth.activations(M, k, seed=4, stream=50 + i)
-        Y = qx.gemm(P, torch.from_numpy(X).cuda())
-        assert qx.device_status() == 0
         rec = _orecipe(4, 128, 0)
-        _check_matmul(Y.cpu().numpy(), oracle.gemm(ref, rec, X, k), X, oracle.dequant(ref, rec, k))
+        y_ref, Wh = oracle.gemm(ref, rec, X, k), oracle.dequant(ref, rec, k)
+        for gemm in (qx.gemm, qx.gemm_splitk):  # 256-token tiles; 64-token tiles split along k
+            Y = gemm(P, torch.from_numpy(X).cuda())
+            assert qx.device_status() == 0
+            _check_matmul(Y.cpu().numpy(), y_ref, X, Wh)
 
 
 # ---------------------------------------------------------------- split-k tensor-core matmul
