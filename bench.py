@@ -515,7 +515,7 @@ def _splitk_graph(qx, torch, stream, layers, xs, outs):
     def body():
         for L in layers:
             for nm, P in L.items():
-                qx.gemm_splitk(P, xs[nm], out=outs[nm])
+                qx.gemm_splitk(P, xs[nm], out=outs[nm], pdl=True)
 
     with torch.cuda.stream(stream):
         body()  # also sizes the stream's workspace before capture
@@ -572,7 +572,7 @@ def run_config3(qx, torch, dev, stream, l2):
                 del gr
                 out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}_tensorcore"] = {
                     "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
-                    "weight_bytes": layer_bytes, "path": "qx_gemm_splitk per matrix (tcgen05, k split)"}
+                    "weight_bytes": layer_bytes, "path": "qx_gemm_splitk per matrix with PDL (tcgen05, k split)"}
         del layers, base
     if qx.device_status(stream) != 0:
         raise RuntimeError("config-3 decode reported a device error")
@@ -643,7 +643,7 @@ def run_config5(qx, torch, dev, stream):
         del gv
         return ms
 
-    pre_ms = vision_ms(qx.gemm_splitk)
+    pre_ms = vision_ms(lambda P, X, out: qx.gemm_splitk(P, X, out=out, pdl=True))
     pre_ms_tile = vision_ms(qx.gemm)
     flops = 24 * sum(2.0 * M * n * k for _, n, k, *_ in LLAVA_VISION)
     del vis
@@ -652,7 +652,7 @@ def run_config5(qx, torch, dev, stream):
             "decode_token_us": dec_ms * 1e3, "decode_GBps": lang_bytes / (dec_ms * 1e-3) / 1e9,
             "decode_launches": 32 * len(chain), "language_weight_bytes": lang_bytes,
             "vision_prefill_us": pre_ms * 1e3, "vision_prefill_TFLOPs": flops / (pre_ms * 1e-3) / 1e12,
-            "vision_prefill_path": "qx_gemm_splitk (64- or 256-token tiles, k split where the tiles leave SMs idle)",
+            "vision_prefill_path": "qx_gemm_splitk with PDL (64- or 256-token tiles, k split where the tiles leave SMs idle)",
             "vision_prefill_us_one_cta_per_tile": pre_ms_tile * 1e3,
             "vision_tokens": M, "vision_gemm_launches": 24 * len(LLAVA_VISION)}
 

@@ -156,6 +156,16 @@ qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const 
  * row-major, 4-byte aligned; m >= 1.  One CTA per tile: no workspace. */
 qx_status qx_gemm(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream);
 
+/* Flags of qx_gemm_splitk. */
+enum {
+    /* Launch with programmatic dependent launch: the kernel may start, and
+     * stream and dequantize this call's weights, while the previous kernel in
+     * the stream is still running; it waits for that kernel before reading X
+     * or writing Y and the workspace.  Set it only when the previous kernel
+     * does not write this call's weights. */
+    QX_GEMM_PDL = 1
+};
+
 /* Bytes of workspace qx_gemm_splitk needs for an n x k matrix of `recipe` and
  * m rows of X on the current device (host-only call; 0 when the call will not
  * split k).  Same shape rules as qx_packed_size; m >= 1. */
@@ -177,9 +187,10 @@ qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const qx_rec
  * leaves them zero again.  After a call that ends
  * in QX_ERR_TIMEOUT, zero it again.  Calls that may run at the same time need
  * separate workspaces.  Returns QX_ERR_INVALID_ARG if the workspace is
- * missing or too small, QX_ERR_ALIGNMENT if it is misaligned. */
+ * missing or too small, QX_ERR_ALIGNMENT if it is misaligned.
+ * flags: 0 or QX_GEMM_PDL. */
 qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, void *workspace,
-                         size_t workspace_bytes, void *stream);
+                         size_t workspace_bytes, int32_t flags, void *stream);
 
 /* qx_gemm_splitk for callers that cannot allocate device memory: it allocates
  * nothing and takes no workspace.  The partial tiles go to a scratch array of

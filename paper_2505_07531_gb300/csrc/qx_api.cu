@@ -366,15 +366,17 @@ QX_API qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const
 }
 
 QX_API qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, void *workspace,
-                                size_t workspace_bytes, void *stream) {
+                                size_t workspace_bytes, int32_t flags, void *stream) {
     qx_status s = check_gemm_args(p, X, m, Y);
     if (s != QX_OK) return s;
+    if ((flags & ~QX_GEMM_PDL) != 0) return QX_ERR_INVALID_ARG;
     DeviceInfo *d = nullptr;
     if ((s = device_info(&d)) != QX_OK) return s;
     const qx::GemmPlan plan = qx::plan_gemm(p->n, p->k, m, d->num_sms, true);
     qx::GemmArgs a = gemm_args(p, X, m, Y, d);
     a.bn = plan.bn;
     a.splits = plan.splits;
+    a.pdl = (flags & QX_GEMM_PDL) ? 1 : 0;
     if (plan.splits > 1) {
         if (workspace == nullptr || workspace_bytes < plan.ws_bytes) return QX_ERR_INVALID_ARG;
         if (!aligned(workspace, 256)) return QX_ERR_ALIGNMENT;

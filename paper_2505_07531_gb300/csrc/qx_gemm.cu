@@ -378,6 +378,9 @@ __global__ void __launch_bounds__(THREADS, 1)
     // unit u: tile t = u / S, W rows n0 = (t / mt) * BM, tokens m0 = (t % mt) * BN;
     // consecutive CTAs share a W tile (L2 reuse of the packed codes)
 
+    // under programmatic dependent launch the next kernel in the stream may be
+    // scheduled now: it waits for this one before it reads what this one writes
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     if (threadIdx.x == 0) {
         for (int i = 0; i < STAGES; ++i) {
             mbar_init(&s.full[i], NUM_DQ_WARPS + 1);
@@ -413,6 +416,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         // ------------------------------------------------ TMA producer (X)
         if (lane == 0) {
+            // X may be the previous kernel's output (a no-op without PDL)
+            asm volatile("griddepcontrol.wait;" ::: "memory");
             int it = 0;  // stage counter across units
             bool ok = true;
             for (int u = blockIdx.x; u < nunits && ok; u += gridDim.x) {
@@ -614,6 +619,8 @@ __global__ void __launch_bounds__(THREADS, 1)
         __syncwarp();
     } else {
         // ------------------------------------------------ epilogue
+        // Y and the workspace may still be in use by the previous kernel
+        asm volatile("griddepcontrol.wait;" ::: "memory");
         constexpr int CH = C::CHUNK;
         const int quarter = warp & 3;  // the TMEM lanes (W rows) this warp may read
         int ti = 0;
@@ -704,8 +711,21 @@ cudaError_t launch_t(const CUtensorMap &mx, const CUtensorMap &mc, const CUtenso
     cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
     if (e != cudaSuccess) return e;
     const unsigned grid = (unsigned)std::min<int64_t>(units, num_sms);
-    kern<<<grid, THREADS, a.smem_bytes, st>>>(mx, mc, ml, a);
-    return cudaGetLastError();
+    if (!a.pdl) {
+        kern<<<grid, THREADS, a.smem_bytes, st>>>(mx, mc, ml, a);
+        return cudaGetLastError();
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(grid);
+    cfg.blockDim = dim3(THREADS);
+    cfg.dynamicSmemBytes = (size_t)a.smem_bytes;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, mx, mc, ml, a);
 }
 
 template <int BITS, int KIND>

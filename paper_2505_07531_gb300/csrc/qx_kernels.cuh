@@ -89,6 +89,10 @@ struct GemmArgs {
     int bn, splits;
     float *ws_part;
     uint32_t *ws_cnt;
+    // launched with programmatic dependent launch: the weight-side roles start
+    // while the previous kernel runs; X is read and Y / the workspace written
+    // only after it has finished
+    int pdl;
 };
 
 // A split-k workspace starts with a fixed region of counters (one word per

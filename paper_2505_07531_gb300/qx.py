@@ -18,6 +18,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "lib
 UNIFORM, LUT = 0, 1
 F16, F32 = 0, 1
 GEMV_PDL = 1
+GEMM_PDL = 1
 
 STATUS = {
     0: "QX_OK",
@@ -80,7 +81,7 @@ def _lib():
         lib.qx_gemv.argtypes = [P(_Packed), VP, I32, VP, I32, VP]
         lib.qx_gemm.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(_Recipe), P(ctypes.c_size_t)]
-        lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, VP]
+        lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, I32, VP]
         lib.qx_gemm_splitk_noalloc.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
@@ -279,10 +280,12 @@ def splitk_workspace(device, nbytes: int) -> torch.Tensor:
 
 
 def gemm_splitk(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None,
-                workspace: torch.Tensor | None = None) -> torch.Tensor:
+                workspace: torch.Tensor | None = None, pdl: bool = False) -> torch.Tensor:
     """Y = X W_hat^T with k split across CTAs when the tiles alone leave SMs
     idle (qx_gemm_splitk): the tensor-core decode path for 1..16 rows of X and
-    the path for short prefills.  Returns fp16 [m][n]."""
+    the path for short prefills.  ``pdl`` lets the kernel start while the
+    previous kernel in the stream runs: set it only when that kernel does not
+    write these weights.  Returns fp16 [m][n]."""
     _dev_tensor(X, "X")
     m = X.shape[0]
     Y = out if out is not None else torch.empty((m, P.n), dtype=torch.float16, device=X.device)
@@ -292,8 +295,8 @@ def gemm_splitk(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = Non
     if not ws.is_cuda or ws.dtype != torch.uint8:
         raise ValueError("workspace must be a CUDA uint8 tensor")
     pc = P.c()
-    _check(_lib().qx_gemm_splitk(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _ptr(ws), ws.numel(), _stream(X.device)),
-           "qx_gemm_splitk")
+    _check(_lib().qx_gemm_splitk(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _ptr(ws), ws.numel(),
+                                 GEMM_PDL if pdl else 0, _stream(X.device)), "qx_gemm_splitk")
     return Y
 
 

@@ -86,11 +86,13 @@ def test_entry_points_reject_bad_arguments_before_launching(qx):
     assert lib.qx_gemv(ctypes.byref(P3), ctypes.c_void_p(0x4008), 1, ctypes.c_void_p(0x5000), 0, None) == 3
     assert lib.qx_gemm(ctypes.byref(P3), ctypes.c_void_p(0x4000), 0, ctypes.c_void_p(0x5000), None) == 1
     # split-k matmul: the same argument checks, and the workspace query's own
-    assert lib.qx_gemm_splitk(None, None, 1, None, None, 0, None) == 1
-    assert lib.qx_gemm_splitk(ctypes.byref(P3), ctypes.c_void_p(0x4000), 0, ctypes.c_void_p(0x5000), None, 0,
+    assert lib.qx_gemm_splitk(None, None, 1, None, None, 0, 0, None) == 1
+    assert lib.qx_gemm_splitk(ctypes.byref(P3), ctypes.c_void_p(0x4000), 0, ctypes.c_void_p(0x5000), None, 0, 0,
                               None) == 1
-    assert lib.qx_gemm_splitk(ctypes.byref(P3), ctypes.c_void_p(0x4008), 1, ctypes.c_void_p(0x5000), None, 0,
+    assert lib.qx_gemm_splitk(ctypes.byref(P3), ctypes.c_void_p(0x4008), 1, ctypes.c_void_p(0x5000), None, 0, 0,
                               None) == 3
+    assert lib.qx_gemm_splitk(ctypes.byref(P3), ctypes.c_void_p(0x4000), 1, ctypes.c_void_p(0x5000), None, 0, 2,
+                              None) == 1  # unknown flag
     nbytes = ctypes.c_size_t(0)
     r = qx._Recipe(3, 128, 1, 0)
     assert lib.qx_gemm_splitk_workspace(4096, 4096, 1, ctypes.byref(r), None) == 1

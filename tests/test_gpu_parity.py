@@ -373,6 +373,26 @@ def test_gemm_splitk_deterministic_and_rearmed(qx, bits, g, kind):
     assert e.value.code == 1
 
 
+def test_gemm_splitk_pdl_chain_orders_inputs(qx):
+    """Under PDL a split-k call that reads the previous call's output (and shares
+    its workspace) sees the finished output: the chain equals the same chain run
+    without PDL, bit for bit."""
+    P1 = qx.quantize(torch.from_numpy(_weights(4096, 4096, seed=11)).cuda(), qx.Recipe(3, 128, 1))
+    P2 = qx.quantize(torch.from_numpy(_weights(1024, 4096, seed=12)).cuda(), qx.Recipe(4, 64, 0))
+    for m in (16, 300):
+        X = torch.from_numpy(synth.activations(m, 4096, seed=m, stream=13)).cuda()
+        outs = []
+        for pdl in (False, True):
+            torch.cuda.synchronize()
+            for _ in range(10):
+                Y1 = qx.gemm_splitk(P1, X, pdl=pdl)
+                Y2 = qx.gemm_splitk(P2, Y1, pdl=pdl)
+            outs.append(Y2.clone())
+        torch.cuda.synchronize()
+        assert qx.device_status() == 0
+        assert torch.equal(outs[0], outs[1])
+
+
 # ---------------------------------------------------------------- full sizes, sampled rows
 # The Llama-7B-shaped layer of the decode benchmark in 3-bit LUT g128.  The
 # weights are drawn on the GPU and quantized there; for each matrix a seeded
