@@ -15,6 +15,9 @@ Modules
 ``pack``    the packed byte layout of codes and zero-points (the paper fixes none;
             Section 2.4 says only that packing/unpacking kernels set decode time).
 ``matmul``  dequantize + float64 matvec / matmul and the parity tolerance.
+``q4x``     the Q4X shared-codebook quantizer (Section 3.2, Fig. 3a: groups of
+            64, per-group fp16 scale and 2-bit book index, 4 learned books of 16
+            centroids per matrix).
 
 Every function names the passage (section, table or figure of the paper) it
 follows; where the paper is silent the docstring states the reading taken.
@@ -37,3 +40,10 @@ from .pack import (  # noqa: F401
     dequant,
 )
 from .matmul import gemv, gemm, tolerance, max_abs_err  # noqa: F401
+from .q4x import (  # noqa: F401
+    quantize_q4x,
+    dequant_q4x,
+    pack_books,
+    unpack_books,
+    q4x_sizes,
+)
