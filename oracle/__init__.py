@@ -15,6 +15,8 @@ Modules
 ``pack``    the packed byte layout of codes and zero-points (the paper fixes none;
             Section 2.4 says only that packing/unpacking kernels set decode time).
 ``matmul``  dequantize + float64 matvec / matmul and the parity tolerance.
+``select``  per-matrix recipe selection by the exact Frobenius error under a
+            bits-per-weight budget (Sections 2.2-2.3).
 ``q4x``     the Q4X shared-codebook quantizer (Section 3.2, Fig. 3a: groups of
             64, per-group fp16 scale and 2-bit book index, 4 learned books of 16
             centroids per matrix).
@@ -47,3 +49,4 @@ from .q4x import (  # noqa: F401
     unpack_books,
     q4x_sizes,
 )
+from .select import select_recipe, sq_error_units, bits_per_weight  # noqa: F401
