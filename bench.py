@@ -415,6 +415,7 @@ def run_ours(args):
     if not args.skip_configs:
         torch.cuda.empty_cache()
         extra["config3"] = run_config3(qx, torch, dev, stream, l2)
+        extra["recipe_select"] = run_select(qx, torch, dev, stream)
         torch.cuda.empty_cache()
         extra["config5"] = run_config5(qx, torch, dev, stream)
 
@@ -589,6 +590,30 @@ LLAVA_VISION = [  # CLIP ViT-L/14: hidden 1024, MLP 4096; 4-bit uniform g128
     ("q_proj", 1024, 1024, 0.02, 10), ("k_proj", 1024, 1024, 0.02, 11), ("v_proj", 1024, 1024, 0.02, 12),
     ("o_proj", 1024, 1024, 0.02, 13), ("fc1", 4096, 1024, 0.04, 14), ("fc2", 1024, 4096, 0.04, 15),
 ]
+
+
+def run_select(qx, torch, dev, stream):
+    """Per-matrix recipe selection (qx_select_recipe) on one 4096x4096
+    Student-t matrix among 3-bit uniform g64, 3-bit LUT g128, 4-bit uniform
+    g64 and g128: quantize, dequantize and exact error per candidate."""
+    import synth
+
+    W = synth.student_t_weights_torch(4096, 4096, 0.02, seed=6, stream=0, device=dev)
+    cands = [qx.Recipe(3, 64, qx.UNIFORM), qx.Recipe(3, 128, qx.LUT), qx.Recipe(4, 64, qx.UNIFORM),
+             qx.Recipe(4, 128, qx.UNIFORM)]
+    with torch.cuda.stream(stream):
+        qx.select_recipe(W, cands)  # warm-up
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        best, errs, bpws = qx.select_recipe(W, cands)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    names = ["U3g64", "L3g128", "U4g64", "U4g128"]
+    return {"matrix": [4096, 4096], "candidates": names, "ms": e0.elapsed_time(e1),
+            "chosen": names[best] if best is not None else None,
+            "rel_frobenius_error": {nm: math.sqrt(e / float(1 << 48)) / float(W.float().norm())
+                                    for nm, e in zip(names, errs)},
+            "bpw": dict(zip(names, bpws))}
 
 
 def run_config5(qx, torch, dev, stream):

@@ -203,6 +203,26 @@ qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, 
  * needs more than the scratch holds (qx_gemm_splitk_workspace() > 4 MiB). */
 qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream);
 
+/* Per-matrix recipe selection (Sections 2.2-2.3: uniform or non-uniform per
+ * matrix by the Frobenius norm of the quantization error; bit-widths chosen
+ * per layer).  For each of the `count` candidate recipes (1..16) whose bits per
+ * weight (8 x packed bytes / (n k), returned in bpw[i]) are at most max_bpw
+ * (every candidate when max_bpw <= 0), W is quantized and dequantized on the
+ * device and E_i = sum (w - w_hat)^2 is taken exactly: sq_error[2i] (low word)
+ * and sq_error[2i+1] hold E_i * 2^48, an integer; both words are all ones for a
+ * candidate over the budget.  *chosen = the eligible candidate with the
+ * smallest E_i, ties to the smaller bpw, then to the earlier index; -1 when
+ * none is eligible.
+ * W: device fp16 [n][k], 16-byte aligned, as for qx_quantize.  candidates,
+ * chosen, sq_error (2 count words), bpw (count): host memory.  workspace:
+ * device memory, 256-byte aligned, of at least qx_select_workspace() bytes.
+ * The call synchronizes `stream`.  Returns QX_ERR_NONFINITE if W holds NaN or
+ * Inf (the device status word keeps the flag). */
+qx_status qx_select_workspace(int64_t n, int64_t k, const qx_recipe *candidates, int32_t count, size_t *bytes);
+qx_status qx_select_recipe(const void *W, int64_t n, int64_t k, const qx_recipe *candidates, int32_t count,
+                           double max_bpw, void *workspace, size_t workspace_bytes, int32_t *chosen,
+                           uint64_t *sq_error, double *bpw, void *stream);
+
 /* Synchronize `stream`, then return and clear the current device's status word
  * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
  * synchronization itself fails. */

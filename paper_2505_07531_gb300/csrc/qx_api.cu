@@ -410,6 +410,118 @@ QX_API qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64
     return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
 }
 
+namespace {
+
+// Workspace of qx_select_recipe: the largest candidate's packed buffers, the
+// dequantized matrix, the error partials and one 16-byte result per candidate.
+struct SelectLayout {
+    size_t packed, what, partials, results, total;
+};
+
+size_t round256(size_t x) { return (x + 255) / 256 * 256; }
+
+qx_status select_layout(int64_t n, int64_t k, const qx_recipe *cands, int32_t count, int num_sms, SelectLayout *L) {
+    if (cands == nullptr || count < 1 || count > 16) return QX_ERR_INVALID_ARG;
+    size_t packed = 0;
+    for (int i = 0; i < count; ++i) {
+        qx_sizes sz{};
+        qx_status s = qx_packed_size(n, k, &cands[i], &sz);
+        if (s != QX_OK) return s;
+        packed = std::max(packed, round256(sz.codes) + round256(sz.scales) + round256(sz.zeros) + round256(sz.luts));
+    }
+    L->packed = packed;
+    L->what = round256((size_t)n * k * 2);
+    L->partials = round256((size_t)qx::sq_error_blocks(num_sms) * 16);
+    L->results = round256((size_t)count * 16);
+    L->total = L->packed + L->what + L->partials + L->results;
+    return QX_OK;
+}
+
+}  // namespace
+
+QX_API qx_status qx_select_workspace(int64_t n, int64_t k, const qx_recipe *candidates, int32_t count,
+                                     size_t *bytes) {
+    if (bytes == nullptr) return QX_ERR_INVALID_ARG;
+    DeviceInfo *d = nullptr;
+    SelectLayout L{};
+    qx_status s = select_layout(n, k, candidates, count, 1, &L);  // validates first
+    if (s != QX_OK) return s;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    if ((s = select_layout(n, k, candidates, count, d->num_sms, &L)) != QX_OK) return s;
+    *bytes = L.total;
+    return QX_OK;
+}
+
+QX_API qx_status qx_select_recipe(const void *W, int64_t n, int64_t k, const qx_recipe *candidates, int32_t count,
+                                  double max_bpw, void *workspace, size_t workspace_bytes, int32_t *chosen,
+                                  uint64_t *sq_error, double *bpw, void *stream) {
+    if (W == nullptr || chosen == nullptr || sq_error == nullptr || bpw == nullptr) return QX_ERR_INVALID_ARG;
+    SelectLayout L{};
+    qx_status s = select_layout(n, k, candidates, count, 1, &L);
+    if (s != QX_OK) return s;
+    if (!aligned(W, 16)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    if ((s = select_layout(n, k, candidates, count, d->num_sms, &L)) != QX_OK) return s;
+    if (workspace == nullptr || workspace_bytes < L.total) return QX_ERR_INVALID_ARG;
+    if (!aligned(workspace, 256)) return QX_ERR_ALIGNMENT;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    uint8_t *ws = static_cast<uint8_t *>(workspace);
+    void *what = ws + L.packed;
+    auto *partials = reinterpret_cast<unsigned long long *>(ws + L.packed + L.what);
+    auto *results = reinterpret_cast<unsigned long long *>(ws + L.packed + L.what + L.partials);
+    bool eligible[16] = {};
+    for (int i = 0; i < count; ++i) {
+        qx_sizes sz{};
+        qx_packed_size(n, k, &candidates[i], &sz);
+        bpw[i] = 8.0 * (double)(sz.codes + sz.scales + sz.zeros + sz.luts) / ((double)n * (double)k);
+        eligible[i] = !(max_bpw > 0.0) || bpw[i] <= max_bpw;
+        if (!eligible[i]) continue;
+        // quantize into the workspace, dequantize, take the exact error
+        qx_packed p{};
+        p.n = n;
+        p.k = k;
+        p.recipe = candidates[i];
+        uint8_t *at = ws;
+        p.codes = at;
+        at += round256(sz.codes);
+        p.scales = sz.scales ? at : nullptr;
+        at += round256(sz.scales);
+        p.zeros = sz.zeros ? at : nullptr;
+        at += round256(sz.zeros);
+        p.luts = sz.luts ? at : nullptr;
+        if ((s = qx_quantize(W, n, k, &candidates[i], &p, stream)) != QX_OK) return s;
+        if ((s = qx_dequant(&p, what, stream)) != QX_OK) return s;
+        if ((s = from_cuda(qx::launch_sq_error(static_cast<const __half *>(W), static_cast<const __half *>(what),
+                                               n * k, partials, results + 2 * i, d->num_sms, st))) != QX_OK)
+            return s;
+    }
+    unsigned long long host[32] = {};
+    if ((s = from_cuda(cudaMemcpyAsync(host, results, (size_t)count * 16, cudaMemcpyDeviceToHost, st))) != QX_OK)
+        return s;
+    if ((s = from_cuda(cudaStreamSynchronize(st))) != QX_OK) return s;
+    uint32_t status = 0;
+    if ((s = from_cuda(cudaMemcpy(&status, d->status, sizeof(status), cudaMemcpyDeviceToHost))) != QX_OK) return s;
+    if (status & qx::kStatusNonfinite) return QX_ERR_NONFINITE;
+    // the smallest error, ties to fewer bits per weight, then to the earlier candidate
+    *chosen = -1;
+    unsigned __int128 best = 0;
+    for (int i = 0; i < count; ++i) {
+        if (!eligible[i]) {
+            sq_error[2 * i] = sq_error[2 * i + 1] = ~0ull;
+            continue;
+        }
+        sq_error[2 * i] = host[2 * i];
+        sq_error[2 * i + 1] = host[2 * i + 1];
+        const unsigned __int128 e = ((unsigned __int128)host[2 * i + 1] << 64) | host[2 * i];
+        if (*chosen < 0 || e < best || (e == best && bpw[i] < bpw[*chosen])) {
+            *chosen = i;
+            best = e;
+        }
+    }
+    return QX_OK;
+}
+
 QX_API qx_status qx_get_device_status(void *stream) {
     DeviceInfo *d = nullptr;
     qx_status s = device_info(&d);

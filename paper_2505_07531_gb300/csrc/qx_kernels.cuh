@@ -114,6 +114,13 @@ struct GemmPlan {
 // tile grid leaves SMs idle (qx_gemm_splitk).
 GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_split);
 
+// Exact sum of (W - W_hat)^2 2^48 over `count` fp16 elements (a multiple of 8,
+// 16-byte aligned): per-block partials (2 words per block, sq_error_blocks of
+// them) and the total in out[0] (low word), out[1].
+int sq_error_blocks(int num_sms);
+cudaError_t launch_sq_error(const __half *W, const __half *W_hat, int64_t count, unsigned long long *partials,
+                            unsigned long long *out, int num_sms, cudaStream_t st);
+
 // Size of the file-scope scratch that qx_gemm_splitk_noalloc uses in place of
 // a workspace, and its device address on the current device (looked up once
 // per device with cudaGetSymbolAddress).

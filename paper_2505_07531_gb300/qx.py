@@ -83,6 +83,9 @@ def _lib():
         lib.qx_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(_Recipe), P(ctypes.c_size_t)]
         lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, I32, VP]
         lib.qx_gemm_splitk_noalloc.argtypes = [P(_Packed), VP, I64, VP, VP]
+        lib.qx_select_workspace.argtypes = [I64, I64, P(_Recipe), I32, P(ctypes.c_size_t)]
+        lib.qx_select_recipe.argtypes = [VP, I64, I64, P(_Recipe), I32, ctypes.c_double, VP, ctypes.c_size_t,
+                                         P(I32), P(ctypes.c_uint64), P(ctypes.c_double), VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
@@ -92,7 +95,7 @@ def _lib():
         lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc",
-                   "qx_get_device_status", "qx_version"):
+                   "qx_select_workspace", "qx_select_recipe", "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -311,6 +314,28 @@ def gemm_splitk_noalloc(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | No
     _check(_lib().qx_gemm_splitk_noalloc(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _stream(X.device)),
            "qx_gemm_splitk_noalloc")
     return Y
+
+
+def select_recipe(W: torch.Tensor, candidates, max_bpw: float | None = None):
+    """Per-matrix recipe choice by the exact Frobenius error (qx_select_recipe).
+
+    Returns ``(index or None, errors, bpws)``: errors[i] is sum (w - w_hat)^2 in
+    units of 2^-48 as an exact int (None over the budget)."""
+    _dev_tensor(W, "W")
+    n, k = W.shape
+    cands = list(candidates)
+    arr = (_Recipe * len(cands))(*[r.c() for r in cands])
+    nbytes = ctypes.c_size_t(0)
+    _check(_lib().qx_select_workspace(n, k, arr, len(cands), ctypes.byref(nbytes)), "qx_select_workspace")
+    ws = torch.empty(max(int(nbytes.value), 256), dtype=torch.uint8, device=W.device)
+    chosen = ctypes.c_int32(-1)
+    err = (ctypes.c_uint64 * (2 * len(cands)))()
+    bpw = (ctypes.c_double * len(cands))()
+    _check(_lib().qx_select_recipe(_ptr(W), n, k, arr, len(cands), float(max_bpw or 0.0), _ptr(ws), ws.numel(),
+                                   ctypes.byref(chosen), err, bpw, _stream(W.device)), "qx_select_recipe")
+    errors = [None if err[2 * i] == err[2 * i + 1] == 2 ** 64 - 1 else err[2 * i] | (err[2 * i + 1] << 64)
+              for i in range(len(cands))]
+    return (None if chosen.value < 0 else chosen.value), errors, list(bpw)
 
 
 def device_status(stream=None) -> int:

@@ -99,6 +99,17 @@ def test_entry_points_reject_bad_arguments_before_launching(qx):
     assert lib.qx_gemm_splitk_workspace(4096, 4096, 0, ctypes.byref(r), ctypes.byref(nbytes)) == 1
     assert lib.qx_gemm_splitk_workspace(4096, 4000, 1, ctypes.byref(r), ctypes.byref(nbytes)) == 2
     assert lib.qx_gemm_splitk_workspace(4096, 4096, 1, None, ctypes.byref(nbytes)) == 1
+    # recipe selection: candidate list and shape checks come first
+    cands = (qx._Recipe * 2)(qx._Recipe(3, 64, 0, 0), qx._Recipe(4, 64, 0, 0))
+    assert lib.qx_select_workspace(64, 256, cands, 0, ctypes.byref(nbytes)) == 1
+    assert lib.qx_select_workspace(64, 256, cands, 17, ctypes.byref(nbytes)) == 1
+    assert lib.qx_select_workspace(64, 200, cands, 2, ctypes.byref(nbytes)) == 2
+    bad = (qx._Recipe * 1)(qx._Recipe(4, 64, 1, 0))  # 4-bit LUT is not built
+    assert lib.qx_select_workspace(64, 256, bad, 1, ctypes.byref(nbytes)) == 2
+    ch, err, bpw = ctypes.c_int32(0), (ctypes.c_uint64 * 4)(), (ctypes.c_double * 2)()
+    assert lib.qx_select_recipe(None, 64, 256, cands, 2, 0.0, None, 0, ctypes.byref(ch), err, bpw, None) == 1
+    assert lib.qx_select_recipe(ctypes.c_void_p(0x4008), 64, 256, cands, 2, 0.0, None, 0, ctypes.byref(ch), err, bpw,
+                                None) == 3
 
 
 def test_status_strings_and_version(qx):

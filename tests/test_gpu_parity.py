@@ -469,3 +469,32 @@ def test_full_size_prefill_sampled(qx, llama_layer):
         Y = qx.gemm(P, torch.from_numpy(X).cuda())
         assert qx.device_status() == 0
         _check_matmul(Y.cpu().numpy()[:, rows], oracle.gemm(ref, rec, X, P.k), X, Wh)
+
+
+# ---------------------------------------------------------------- recipe selection
+SELECT_CANDIDATES = [(3, 64, 0), (3, 128, 1), (4, 64, 0), (4, 128, 0), (3, 64, 1)]
+
+
+@pytest.mark.parametrize("shape", [(96, 512), (130, 256)])
+def test_select_recipe_matches_oracle(qx, shape):
+    """Same choice and the same exact errors (integers in units of 2^-48) as the
+    oracle, with no budget and with budgets that exclude candidates or all."""
+    from oracle import select as oselect
+    n, k = shape
+    W = _weights(n, k, seed=600 + n)
+    cands = [qx.Recipe(b, g, kd) for b, g, kd in SELECT_CANDIDATES]
+    orecs = [_orecipe(b, g, kd) for b, g, kd in SELECT_CANDIDATES]
+    Wd = torch.from_numpy(W).cuda()
+    for max_bpw in (None, 4.2, 3.3):
+        got = qx.select_recipe(Wd, cands, max_bpw)
+        want = oselect.select_recipe(W, orecs, max_bpw)
+        assert got[0] == want[0] and got[1] == want[1] and got[2] == want[2], max_bpw
+
+
+def test_select_recipe_lossless_lut_closed_form(qx):
+    """Eight unequally spaced values per group: the 3-bit LUT is exact (error 0) and chosen."""
+    rng = np.random.default_rng(12)
+    levels = np.array([-0.05, -0.011, -0.002, 0.0, 0.0007, 0.003, 0.02, 0.07])
+    W = levels[rng.integers(0, 8, (64, 512))].astype(np.float16)
+    best, errs, _ = qx.select_recipe(torch.from_numpy(W).cuda(), [qx.Recipe(3, 64, 0), qx.Recipe(3, 64, 1)])
+    assert best == 1 and errs[1] == 0 and errs[0] > 0
