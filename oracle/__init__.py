@@ -15,6 +15,8 @@ Modules
 ``pack``    the packed byte layout of codes and zero-points (the paper fixes none;
             Section 2.4 says only that packing/unpacking kernels set decode time).
 ``matmul``  dequantize + float64 matvec / matmul and the parity tolerance.
+``act8``    W.A8 decode: per-token 8-bit RTN activations against uniform
+            weights with integer group sums (Tables 1-2: W3A8, W4A8).
 ``select``  per-matrix recipe selection by the exact Frobenius error under a
             bits-per-weight budget (Sections 2.2-2.3).
 ``q4x``     the Q4X shared-codebook quantizer (Section 3.2, Fig. 3a: groups of
@@ -50,3 +52,4 @@ from .q4x import (  # noqa: F401
     q4x_sizes,
 )
 from .select import select_recipe, sq_error_units, bits_per_weight  # noqa: F401
+from .act8 import quantize_act, gemv_a8, dequant_act  # noqa: F401
