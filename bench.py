@@ -566,6 +566,36 @@ def run_config3(qx, torch, dev, stream, l2):
             out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}"] = {
                 "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
                 "weight_bytes": layer_bytes, "path": "qx_gemv_multi chain (CUDA cores)"}
+            if batch in (1, 4):
+                # W.A8: the four distinct activations quantized per token to int8,
+                # then seven integer-dot matmuls (qx_quantize_act + qx_gemv_a8)
+                xd = {"attn": xs[0], "o": xs[1], "mlp": xs[2], "down": xs[3]}
+                src = {"q_proj": "attn", "k_proj": "attn", "v_proj": "attn", "o_proj": "o", "gate_proj": "mlp",
+                       "up_proj": "mlp", "down_proj": "down"}
+                qa = {key: (torch.empty(x.shape, dtype=torch.int8, device=dev),
+                            torch.empty((batch,), dtype=torch.float32, device=dev)) for key, x in xd.items()}
+
+                def a8_step(L):
+                    for key, x in xd.items():
+                        qx._check(qx._lib().qx_quantize_act(qx._ptr(x), batch, x.shape[1], qx._ptr(qa[key][0]),
+                                                            qx._ptr(qa[key][1]), qx._stream(dev)), "qx_quantize_act")
+                    for nm, *_ in LAYER:
+                        qx.gemv_a8(L[nm], qa[src[nm]][0], qa[src[nm]][1], out=ys[nm])
+
+                with torch.cuda.stream(stream):
+                    for L in layers:
+                        a8_step(L)
+                torch.cuda.synchronize()
+                gr = torch.cuda.CUDAGraph()
+                with torch.cuda.graph(gr, stream=stream):
+                    for L in layers:
+                        a8_step(L)
+                ms = _time_graph(torch, stream, gr, 20) / copies
+                del gr
+                out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}_a8"] = {
+                    "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
+                    "weight_bytes": layer_bytes,
+                    "path": "qx_quantize_act x4 + qx_gemv_a8 x7 (int8 activations, dp4a)"}
             if batch >= 4:
                 xn = {nm: xs[3] if nm == "down_proj" else xs[0] for nm, *_ in LAYER}
                 gr = _splitk_graph(qx, torch, stream, layers, xn, ys)

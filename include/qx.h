@@ -203,6 +203,22 @@ qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, 
  * needs more than the scratch holds (qx_gemm_splitk_workspace() > 4 MiB). */
 qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64_t m, void *Y, void *stream);
 
+/* 8-bit per-token activations (Table 2: "8-bit RTN per-token quantization for
+ * the activation tensors"; Table 1: W3A8), for qx_gemv_a8.  For each token b
+ * (row of x): s_b = fp32(max_k |x[b][k]| / 127) and q[b][k] = clamp(rint(x / s_b),
+ * -127, 127) in IEEE fp32 (q = 0 when s_b = 0); bit-exact with the CPU oracle.
+ * x: device fp16 [batch][k], finite; q: device int8 [batch][k], 16-byte
+ * aligned; scales: device fp32 [batch].  batch 1..16, k a multiple of 16. */
+qx_status qx_quantize_act(const void *x, int32_t batch, int64_t k, void *q, void *scales, void *stream);
+
+/* W.A8 decode matmul for uniform weights: y[b][n] = s_b * sum_g s_g *
+ * sum_{k in g} (q_w - z) q[b][k], the group sums exact integers (dp4a), the
+ * scales applied in fp32.  q, scales: the output of qx_quantize_act for this
+ * matrix's k; y: device [batch][n] of y_dtype, 4-byte aligned.  Non-uniform
+ * (LUT) recipes have no integer form: QX_ERR_UNSUPPORTED. */
+qx_status qx_gemv_a8(const qx_packed *p, const void *q, const void *scales, int32_t batch, void *y,
+                     int32_t y_dtype, void *stream);
+
 /* Per-matrix recipe selection (Sections 2.2-2.3: uniform or non-uniform per
  * matrix by the Frobenius norm of the quantization error; bit-widths chosen
  * per layer).  For each of the `count` candidate recipes (1..16) whose bits per

@@ -410,6 +410,46 @@ QX_API qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64
     return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
 }
 
+QX_API qx_status qx_quantize_act(const void *x, int32_t batch, int64_t k, void *q, void *scales, void *stream) {
+    if (x == nullptr || q == nullptr || scales == nullptr) return QX_ERR_INVALID_ARG;
+    if (batch < 1 || batch > 16 || k < 1) return QX_ERR_INVALID_ARG;
+    if (k % 16 != 0 || k > ((int64_t)1 << 20)) return QX_ERR_UNSUPPORTED;
+    if (!aligned(x, 2) || !aligned(q, 16) || !aligned(scales, 4)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    return from_cuda(qx::launch_quantize_act(static_cast<const __half *>(x), batch, k, static_cast<int8_t *>(q),
+                                             static_cast<float *>(scales), static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_gemv_a8(const qx_packed *p, const void *q, const void *scales, int32_t batch, void *y,
+                            int32_t y_dtype, void *stream) {
+    qx_status s = check_packed(p);
+    if (s != QX_OK) return s;
+    if (q == nullptr || scales == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
+    if (batch < 1 || batch > 16 || (y_dtype != QX_F16 && y_dtype != QX_F32)) return QX_ERR_INVALID_ARG;
+    if (p->recipe.kind != QX_UNIFORM) return QX_ERR_UNSUPPORTED;
+    if (!aligned(q, 16) || !aligned(scales, 4) || !aligned(y, 4)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::GemvA8Args a{};
+    a.codes = static_cast<const uint8_t *>(p->codes);
+    a.scales = static_cast<const __half *>(p->scales);
+    a.zeros = static_cast<const uint8_t *>(p->zeros);
+    a.n = p->n;
+    a.k = p->k;
+    a.bits = p->recipe.bits;
+    a.log2g = ilog2(p->recipe.group_size);
+    a.G = (int)(p->k / p->recipe.group_size);
+    a.zbytes = (a.G + 1) / 2;
+    a.q = static_cast<const int8_t *>(q);
+    a.act_scales = static_cast<const float *>(scales);
+    a.batch = batch;
+    a.y = y;
+    a.y_f32 = y_dtype == QX_F32;
+    return from_cuda(qx::launch_gemv_a8(a, static_cast<cudaStream_t>(stream)));
+}
+
 namespace {
 
 // Workspace of qx_select_recipe: the largest candidate's packed buffers, the

@@ -114,6 +114,22 @@ struct GemmPlan {
 // tile grid leaves SMs idle (qx_gemm_splitk).
 GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_split);
 
+// W.A8 decode (uniform weights, int8 per-token activations).
+struct GemvA8Args {
+    const uint8_t *codes;
+    const __half *scales;
+    const uint8_t *zeros;
+    int64_t n, k;
+    int bits, G, zbytes, log2g;
+    const int8_t *q;          // [batch][k]
+    const float *act_scales;  // [batch]
+    int batch;
+    void *y;                  // [batch][n]
+    int y_f32;
+};
+cudaError_t launch_quantize_act(const __half *x, int batch, int64_t k, int8_t *q, float *scales, cudaStream_t st);
+cudaError_t launch_gemv_a8(const GemvA8Args &a, cudaStream_t st);
+
 // Exact sum of (W - W_hat)^2 2^48 over `count` fp16 elements (a multiple of 8,
 // 16-byte aligned): per-block partials (2 words per block, sq_error_blocks of
 // them) and the total in out[0] (low word), out[1].

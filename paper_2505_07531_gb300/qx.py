@@ -83,6 +83,8 @@ def _lib():
         lib.qx_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(_Recipe), P(ctypes.c_size_t)]
         lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, I32, VP]
         lib.qx_gemm_splitk_noalloc.argtypes = [P(_Packed), VP, I64, VP, VP]
+        lib.qx_quantize_act.argtypes = [VP, I32, I64, VP, VP, VP]
+        lib.qx_gemv_a8.argtypes = [P(_Packed), VP, VP, I32, VP, I32, VP]
         lib.qx_select_workspace.argtypes = [I64, I64, P(_Recipe), I32, P(ctypes.c_size_t)]
         lib.qx_select_recipe.argtypes = [VP, I64, I64, P(_Recipe), I32, ctypes.c_double, VP, ctypes.c_size_t,
                                          P(I32), P(ctypes.c_uint64), P(ctypes.c_double), VP]
@@ -95,7 +97,8 @@ def _lib():
         lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc",
-                   "qx_select_workspace", "qx_select_recipe", "qx_get_device_status", "qx_version"):
+                   "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
+                   "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
     return _LIB
@@ -314,6 +317,33 @@ def gemm_splitk_noalloc(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | No
     _check(_lib().qx_gemm_splitk_noalloc(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _stream(X.device)),
            "qx_gemm_splitk_noalloc")
     return Y
+
+
+def quantize_act(x: torch.Tensor):
+    """Per-token int8 activations (qx_quantize_act): returns (q int8 [b][k], scales fp32 [b])."""
+    _dev_tensor(x, "x")
+    x2 = x.view(-1, x.shape[-1])
+    b, k = x2.shape
+    q = torch.empty((b, k), dtype=torch.int8, device=x.device)
+    s = torch.empty((b,), dtype=torch.float32, device=x.device)
+    _check(_lib().qx_quantize_act(_ptr(x2), b, k, _ptr(q), _ptr(s), _stream(x.device)), "qx_quantize_act")
+    return q, s
+
+
+def gemv_a8(P: PackedMatrix, q: torch.Tensor, scales: torch.Tensor, out: torch.Tensor | None = None,
+            out_dtype=torch.float16) -> torch.Tensor:
+    """W.A8 decode y = s_b x (q_w - z) q x s_g (qx_gemv_a8) for uniform weights; returns [batch][n]."""
+    if not q.is_cuda or q.dtype != torch.int8 or not q.is_contiguous():
+        raise ValueError("q must be a contiguous CUDA int8 tensor")
+    _dev_tensor(scales, "scales", torch.float32)
+    b = q.shape[0]
+    dt = out.dtype if out is not None else out_dtype
+    y = out if out is not None else torch.empty((b, P.n), dtype=dt, device=q.device)
+    _dev_tensor(y, "out", dt)
+    pc = P.c()
+    _check(_lib().qx_gemv_a8(ctypes.byref(pc), _ptr(q), _ptr(scales), b, _ptr(y), F32 if dt == torch.float32 else F16,
+                             _stream(q.device)), "qx_gemv_a8")
+    return y
 
 
 def select_recipe(W: torch.Tensor, candidates, max_bpw: float | None = None):

@@ -99,6 +99,19 @@ def test_entry_points_reject_bad_arguments_before_launching(qx):
     assert lib.qx_gemm_splitk_workspace(4096, 4096, 0, ctypes.byref(r), ctypes.byref(nbytes)) == 1
     assert lib.qx_gemm_splitk_workspace(4096, 4000, 1, ctypes.byref(r), ctypes.byref(nbytes)) == 2
     assert lib.qx_gemm_splitk_workspace(4096, 4096, 1, None, ctypes.byref(nbytes)) == 1
+    # W.A8: activation and matmul argument checks
+    assert lib.qx_quantize_act(None, 1, 128, None, None, None) == 1
+    assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 17, 128, ctypes.c_void_p(0x5000), ctypes.c_void_p(0x6000),
+                               None) == 1
+    assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 1, 120, ctypes.c_void_p(0x5000), ctypes.c_void_p(0x6000),
+                               None) == 2
+    assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 1, 128, ctypes.c_void_p(0x5008), ctypes.c_void_p(0x6000),
+                               None) == 3
+    PL = qx._Packed(64, 128, qx._Recipe(3, 64, 1, 0), ctypes.c_void_p(0x1000), None, None, ctypes.c_void_p(0x2000))
+    assert lib.qx_gemv_a8(ctypes.byref(PL), ctypes.c_void_p(0x4000), ctypes.c_void_p(0x5000), 1,
+                          ctypes.c_void_p(0x6000), 0, None) == 2  # LUT weights: no integer form
+    assert lib.qx_gemv_a8(ctypes.byref(P3), ctypes.c_void_p(0x4008), ctypes.c_void_p(0x5000), 1,
+                          ctypes.c_void_p(0x6000), 0, None) == 3
     # recipe selection: candidate list and shape checks come first
     cands = (qx._Recipe * 2)(qx._Recipe(3, 64, 0, 0), qx._Recipe(4, 64, 0, 0))
     assert lib.qx_select_workspace(64, 256, cands, 0, ctypes.byref(nbytes)) == 1

@@ -498,3 +498,59 @@ def test_select_recipe_lossless_lut_closed_form(qx):
     W = levels[rng.integers(0, 8, (64, 512))].astype(np.float16)
     best, errs, _ = qx.select_recipe(torch.from_numpy(W).cuda(), [qx.Recipe(3, 64, 0), qx.Recipe(3, 64, 1)])
     assert best == 1 and errs[1] == 0 and errs[0] > 0
+
+
+# ---------------------------------------------------------------- W.A8 decode
+@pytest.mark.parametrize("batch", [1, 3, 16])
+def test_quantize_act_bit_exact(qx, batch):
+    from oracle import act8
+    x = synth.activations(batch, 1280, seed=batch, stream=90)
+    x[0, 7] = 0  # a zero element
+    q, s = qx.quantize_act(torch.from_numpy(x).cuda())
+    qr, sr = act8.quantize_act(x)
+    assert np.array_equal(q.cpu().numpy(), qr) and np.array_equal(s.cpu().numpy().view(np.uint32), sr.view(np.uint32))
+
+
+A8_CASES = [c for c in CASES if c[4] == 0]  # uniform recipes only
+
+
+@pytest.mark.parametrize("batch", [1, 2, 5, 16])
+@pytest.mark.parametrize("case", A8_CASES, ids=_ids)
+def test_gemv_a8_tolerance(qx, packed, case, batch):
+    """Within 2e-3 ||x_hat_b|| max_n ||w_n|| of the oracle's W.A8 product, w the
+    unrounded (q - z) s the integer path multiplies."""
+    from oracle import act8
+    W, P, ref = packed[case]
+    n, k, bits, g, kind = case
+    rec = _orecipe(bits, g, kind)
+    x = synth.activations(batch, k, seed=batch, stream=91)
+    q, s = qx.quantize_act(torch.from_numpy(x).cuda())
+    for dt in (torch.float16, torch.float32):
+        y = qx.gemv_a8(P, q, s, out_dtype=dt)
+        assert qx.device_status() == 0
+        y_ref = act8.gemv_a8(ref, rec, x, k)
+        qw = oracle.unpack_codes(ref["codes"], bits, k).astype(np.float64)
+        z = np.repeat(oracle.unpack_zeros(ref["zeros"], k // g).astype(np.float64), g, axis=1)
+        w_exact = (qw - z) * np.repeat(ref["scales"].astype(np.float64), g, axis=1)
+        qr, sr = act8.quantize_act(x)
+        _check_matmul(y.float().cpu().numpy(), y_ref, act8.dequant_act(qr, sr), w_exact)
+
+
+def test_gemv_a8_full_size_sampled(qx, llama_layer):
+    """4-bit uniform g128 on the q_proj / down_proj shapes: sampled rows, batch 4."""
+    from oracle import act8
+    rec = _orecipe(4, 128, 0)
+    for nm, n, k in (("q", 4096, 4096), ("down", 4096, 11008)):
+        W = synth.student_t_weights_torch(n, k, 0.02, seed=9, stream=n + k, device="cuda")
+        P = qx.quantize(W, qx.Recipe(4, 128, 0))
+        rows = np.sort(np.random.default_rng(n + k).choice(n, size=SAMPLE_ROWS, replace=False))
+        ref = oracle.quantize(W[torch.from_numpy(rows).cuda()].cpu().numpy(), rec)
+        x = synth.activations(4, k, seed=4, stream=92)
+        q, s = qx.quantize_act(torch.from_numpy(x).cuda())
+        y = qx.gemv_a8(P, q, s, out_dtype=torch.float32).cpu().numpy()[:, rows]
+        assert qx.device_status() == 0
+        qw = oracle.unpack_codes(ref["codes"], 4, k).astype(np.float64)
+        z = np.repeat(oracle.unpack_zeros(ref["zeros"], k // 128).astype(np.float64), 128, axis=1)
+        w_exact = (qw - z) * np.repeat(ref["scales"].astype(np.float64), 128, axis=1)
+        qr, sr = act8.quantize_act(x)
+        _check_matmul(y, act8.gemv_a8(ref, rec, x, k), act8.dequant_act(qr, sr), w_exact)
