@@ -284,11 +284,19 @@ def run_ours(args):
     # decode dependency chain of one token through the layer: q, k, v share the
     # attention input; o reads the attention output; gate, up share the MLP
     # input; down reads act(gate) * up.  Activations are synthetic N(0, 1).
-    x_attn = synth.activations_torch(1, 4096, seed=0, stream=50, device=dev)
-    x_o = synth.activations_torch(1, 4096, seed=0, stream=51, device=dev)
-    x_mlp = synth.activations_torch(1, 4096, seed=0, stream=52, device=dev)
-    x_down = synth.activations_torch(1, 11008, seed=0, stream=53, device=dev)
-    ys = {nm: torch.empty((1, n), dtype=torch.float16, device=dev) for nm, n, k, _, _ in LAYER}
+    # the four activations and the seven outputs are views of one input and one
+    # output buffer, so that the end-to-end loop moves each with one copy
+    x_flat = torch.empty(3 * 4096 + 11008, dtype=torch.float16, device=dev)
+    x_attn, x_o, x_mlp = (x_flat[4096 * i:4096 * (i + 1)].view(1, 4096) for i in range(3))
+    x_down = x_flat[3 * 4096:].view(1, 11008)
+    for i, x in enumerate((x_attn, x_o, x_mlp)):
+        x.copy_(synth.activations_torch(1, 4096, seed=0, stream=50 + i, device=dev))
+    x_down.copy_(synth.activations_torch(1, 11008, seed=0, stream=53, device=dev))
+    y_flat = torch.empty(sum(n for _, n, *_ in LAYER), dtype=torch.float16, device=dev)
+    ys, off = {}, 0
+    for nm, n, *_ in LAYER:
+        ys[nm] = y_flat[off:off + n].view(1, n)
+        off += n
     CHAIN = [(["q_proj", "k_proj", "v_proj"], x_attn), (["o_proj"], x_o),
              (["gate_proj", "up_proj"], x_mlp), (["down_proj"], x_down)]
     io_bytes = sum(x.numel() * 2 for x in (x_attn, x_o, x_mlp, x_down)) + sum(y.numel() * 2 for y in ys.values())
@@ -390,21 +398,20 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     one_launch_ms = e0.elapsed_time(e1) / reps
 
-    # end to end through the public API with host buffers: pinned x in, y out, per step
-    xs_dev = [x_attn, x_o, x_mlp, x_down]
-    hx = [x.cpu().pin_memory() for x in xs_dev]
-    hy = {nm: torch.empty(y.shape, dtype=y.dtype).pin_memory() for nm, y in ys.items()}
+    # end to end through the public API with host buffers: the step's activations
+    # in from pinned host memory (one copy), the four decode calls, the outputs
+    # back (one copy), then a stream synchronisation, per step
+    hx = x_flat.cpu().pin_memory()
+    hy = torch.empty(y_flat.shape, dtype=y_flat.dtype).pin_memory()
     e2e_steps = max(3, min(args.steps, 2000))
     torch.cuda.synchronize(dev)
     t0 = time.perf_counter()
     with torch.cuda.stream(stream):
         for i in range(e2e_steps):
             c = i % copies
-            for x, h in zip(xs_dev, hx):
-                x.copy_(h, non_blocking=True)
+            x_flat.copy_(hx, non_blocking=True)
             step(c)
-            for nm, y in ys.items():
-                hy[nm].copy_(y, non_blocking=True)
+            hy.copy_(y_flat, non_blocking=True)
             stream.synchronize()
     e2e_ms = (time.perf_counter() - t0) * 1e3 / e2e_steps
     e2e_value = step_bytes * ws / (e2e_ms * 1e-3) / 1e9
@@ -446,8 +453,8 @@ def run_ours(args):
             "cpu_baseline": cpu,
             "clocks": clocks,
             "e2e": {"value": e2e_value, "unit": "GB/s", "ms_per_step": e2e_ms,
-                    "h2d_bytes_per_step": sum(x.numel() * 2 for x in hx),
-                    "d2h_bytes_per_step": sum(y.numel() * 2 for y in hy.values())},
+                    "h2d_bytes_per_step": hx.numel() * hx.element_size(),
+                    "d2h_bytes_per_step": hy.numel() * hy.element_size()},
             "gpu_launches": args.steps * len(CHAIN),
         }
         print(json.dumps(line))

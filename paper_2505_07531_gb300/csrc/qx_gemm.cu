@@ -708,7 +708,8 @@ template <int BITS, int KIND, int BN>
 cudaError_t launch_t(const CUtensorMap &mx, const CUtensorMap &mc, const CUtensorMap &ml, const GemmArgs &a,
                      int64_t units, int num_sms, cudaStream_t st) {
     auto kern = gemm_kernel<BITS, KIND, BN>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
+    static std::atomic<uint64_t> attrs_ready{0};
+    cudaError_t e = ensure_kernel_attrs(reinterpret_cast<const void *>(kern), attrs_ready, false);
     if (e != cudaSuccess) return e;
     const unsigned grid = (unsigned)std::min<int64_t>(units, num_sms);
     if (!a.pdl) {

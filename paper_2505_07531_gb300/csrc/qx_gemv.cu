@@ -765,9 +765,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
 template <int BITS, int KIND, int NB>
 cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
     auto kern = gemv_kernel<BITS, KIND, NB>;
-    cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, a.smem_bytes);
-    if (e != cudaSuccess) return e;
-    e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    static std::atomic<uint64_t> attrs_ready{0};
+    cudaError_t e = ensure_kernel_attrs(reinterpret_cast<const void *>(kern), attrs_ready, true);
     if (e != cudaSuccess) return e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)a.grid);

@@ -1,6 +1,8 @@
 // Internal launch interface between the C ABI (qx_api.cu) and the kernels.
 #pragma once
 
+#include <atomic>
+
 #include <algorithm>
 #include <cstdint>
 #include <cuda.h>
@@ -142,6 +144,22 @@ cudaError_t launch_sq_error(const __half *W, const __half *W_hat, int64_t count,
 // per device with cudaGetSymbolAddress).
 constexpr size_t kNoAllocScratchBytes = (size_t)4 << 20;
 cudaError_t noalloc_scratch(void **ptr);
+
+// Raise a kernel's dynamic shared-memory limit to the 227 KB maximum (and the
+// preferred carveout to all shared memory) once per device: a driver call per
+// launch would cost host time on every decode step.  `ready` holds one bit per
+// device (devices 0..63; others set the attributes every time).
+inline cudaError_t ensure_kernel_attrs(const void *kern, std::atomic<uint64_t> &ready, bool carveout) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const uint64_t bit = (dev >= 0 && dev < 64) ? (1ull << dev) : 0ull;
+    if (bit != 0 && (ready.load(std::memory_order_acquire) & bit) != 0) return cudaSuccess;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+    if (e == cudaSuccess && carveout) e = cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout, 100);
+    if (e == cudaSuccess && bit != 0) ready.fetch_or(bit, std::memory_order_acq_rel);
+    return e;
+}
 
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);

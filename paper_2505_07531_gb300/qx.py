@@ -144,6 +144,7 @@ class PackedMatrix:
     def __init__(self, n, k, recipe, codes, scales=None, zeros=None, luts=None):
         self.n, self.k, self.recipe = int(n), int(k), recipe
         self.codes, self.scales, self.zeros, self.luts = codes, scales, zeros, luts
+        self._c_key, self._c_struct = None, None
 
     @classmethod
     def empty(cls, n: int, k: int, recipe: Recipe, device) -> "PackedMatrix":
@@ -164,8 +165,13 @@ class PackedMatrix:
                    if t is not None)
 
     def c(self) -> _Packed:
-        return _Packed(self.n, self.k, self.recipe.c(), _ptr(self.codes), _ptr(self.scales),
-                       _ptr(self.zeros), _ptr(self.luts))
+        # the ctypes struct is kept while the buffers stay the same (decode calls
+        # it for every matrix of every step)
+        key = tuple(None if t is None else t.data_ptr() for t in (self.codes, self.scales, self.zeros, self.luts))
+        if key != self._c_key:
+            self._c_struct = _Packed(self.n, self.k, self.recipe.c(), *key)
+            self._c_key = key
+        return self._c_struct
 
     def to_numpy(self) -> dict:
         """Host copies in the oracle's array shapes (for tests)."""
