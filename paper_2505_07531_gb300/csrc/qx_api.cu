@@ -204,6 +204,57 @@ QX_API qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream) {
 
 namespace {
 
+// Decode plans (CTA slices, shared-memory split, TMA descriptors) depend only
+// on the device, the recipe, the shapes, the buffer addresses and the batch
+// slice.  A model decodes the same matrices into the same buffers every step,
+// so the last plans are kept and reused: planning and descriptor encoding
+// would otherwise cost host time on every launch.
+struct PlanEntry {
+    bool used = false;
+    int dev = -1;
+    qx::GemvMulti plan;
+};
+constexpr int kPlanCache = 32;
+PlanEntry g_plans[kPlanCache];
+int g_plan_next = 0;
+std::mutex g_plan_mu;
+
+bool same_inputs(const qx::GemvMulti &p, const qx::GemvMulti &a) {
+    if (p.count != a.count || p.bits != a.bits || p.kind != a.kind || p.batch != a.batch || p.y_f32 != a.y_f32 ||
+        p.status != a.status || p.wait_limit_ns != a.wait_limit_ns)
+        return false;
+    for (int i = 0; i < a.count; ++i) {
+        const qx::GemvMat &u = p.mat[i], &v = a.mat[i];
+        if (u.codes != v.codes || u.scales != v.scales || u.zeros != v.zeros || u.luts != v.luts || u.x != v.x ||
+            u.y != v.y || u.n != v.n || u.k != v.k || u.G != v.G || u.log2g != v.log2g)
+            return false;
+    }
+    return true;
+}
+
+// plan_gemv through the cache; `a` holds the inputs on entry, the plan on return.
+bool plan_cached(qx::GemvMulti &a, const DeviceInfo *d) {
+    int dev = -1;
+    cudaGetDevice(&dev);
+    {
+        std::lock_guard<std::mutex> lock(g_plan_mu);
+        for (int i = 0; i < kPlanCache; ++i) {
+            if (g_plans[i].used && g_plans[i].dev == dev && same_inputs(g_plans[i].plan, a)) {
+                a = g_plans[i].plan;
+                return true;
+            }
+        }
+    }
+    if (!qx::plan_gemv(a, d->num_sms)) return false;
+    std::lock_guard<std::mutex> lock(g_plan_mu);
+    PlanEntry &e = g_plans[g_plan_next];
+    g_plan_next = (g_plan_next + 1) % kPlanCache;
+    e.used = true;
+    e.dev = dev;
+    e.plan = a;
+    return true;
+}
+
 // One decode launch over `count` matrices for activation rows b0 .. b0+nb-1
 // (nb <= 4, or 8).  When the group's activations do not fit one CTA's shared
 // memory, the group is split per matrix, then the rows are halved.
@@ -233,7 +284,7 @@ qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int
         M.zbytes = (M.G + 1) / 2;
         M.log2g = ilog2(p.recipe.group_size);
     }
-    if (qx::plan_gemv(a, d->num_sms))
+    if (plan_cached(a, d))
         return from_cuda(qx::launch_gemv_multi(a, st, (flags & QX_GEMV_PDL) != 0));
     if (count > 1) {
         for (int i = 0; i < count; ++i) {

@@ -130,8 +130,17 @@ def packed_size(n: int, k: int, recipe: Recipe) -> dict:
     return {"codes": s.codes, "scales": s.scales, "zeros": s.zeros, "luts": s.luts}
 
 
-def _stream(dev: torch.device) -> ctypes.c_void_p:
-    return ctypes.c_void_p(torch.cuda.current_stream(dev).cuda_stream)
+_RAW_STREAM = getattr(torch._C, "_cuda_getCurrentRawStream", None)
+
+
+def _stream(dev) -> ctypes.c_void_p:
+    """The current CUDA stream of device `dev` (a torch.device or an index)."""
+    idx = dev.index if isinstance(dev, torch.device) else dev
+    if idx is None:
+        idx = torch.cuda.current_device()
+    if _RAW_STREAM is not None:  # the same handle, without building a Stream object
+        return ctypes.c_void_p(_RAW_STREAM(idx))
+    return ctypes.c_void_p(torch.cuda.current_stream(idx).cuda_stream)
 
 
 def _ptr(t):
@@ -251,7 +260,7 @@ def gemv_multi(mats, xs, outs=None, out_dtype=torch.float16, pdl: bool = False):
     xp = (ctypes.c_void_p * len(xs))(*[x.data_ptr() for x in xs])
     yp = (ctypes.c_void_p * len(ys))(*[y.data_ptr() for y in ys])
     code = F32 if dt == torch.float32 else F16
-    _check(_lib().qx_gemv_multi(arr, len(mats), xp, b, yp, code, GEMV_PDL if pdl else 0, _stream(xs[0].device)),
+    _check(_lib().qx_gemv_multi(arr, len(mats), xp, b, yp, code, GEMV_PDL if pdl else 0, _stream(xs[0].get_device())),
            "qx_gemv_multi")
     return ys
 
