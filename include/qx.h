@@ -16,8 +16,10 @@
  *
  * Conventions for every entry point
  *   - Buffers are caller-owned.  "device" pointers are CUDA global memory of the
- *     current device; "host" pointers are CPU memory.  The library keeps no
- *     pointer after a call returns.
+ *     current device; "host" pointers are CPU memory.  The library reads no
+ *     buffer after a call's work has run; the decode calls keep their recent
+ *     launch plans keyed by the buffer addresses and shapes, and reuse a plan
+ *     only when a later call passes the same addresses and shapes again.
  *   - `stream` is a cudaStream_t passed as void*; NULL means the legacy default
  *     stream.  Device work is asynchronous on that stream.
  *   - Arguments are validated on the host before anything is launched; on a
@@ -171,6 +173,14 @@ enum {
  * split k).  Same shape rules as qx_packed_size; m >= 1. */
 qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const qx_recipe *recipe,
                                    size_t *bytes);
+
+/* Host only: the plan qx_gemm_splitk takes for an n x k matrix and m rows of X
+ * on a GPU with num_sms SMs -- tokens per tile (16, 64 or 256), k splits per
+ * tile (1..16) and workspace bytes (0 when splits = 1).  The plan depends only
+ * on these numbers.  Errors: INVALID_ARG (NULL, a size < 1), UNSUPPORTED (k
+ * not a multiple of 128, or n, k, m beyond the library's limits). */
+qx_status qx_gemm_splitk_plan(int64_t n, int64_t k, int64_t m, int32_t num_sms, int32_t *token_tile,
+                              int32_t *splits, size_t *bytes);
 
 /* qx_gemm with the contraction split along k (at 128-weight boundaries) when
  * the tiles alone would leave SMs idle -- the decode case (m <= 16: 16-token

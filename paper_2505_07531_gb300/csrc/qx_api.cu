@@ -416,6 +416,19 @@ QX_API qx_status qx_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, const
     return QX_OK;
 }
 
+QX_API qx_status qx_gemm_splitk_plan(int64_t n, int64_t k, int64_t m, int32_t num_sms, int32_t *token_tile,
+                                     int32_t *splits, size_t *bytes) {
+    if (token_tile == nullptr || splits == nullptr || bytes == nullptr) return QX_ERR_INVALID_ARG;
+    if (n < 1 || k < 1 || m < 1 || num_sms < 1) return QX_ERR_INVALID_ARG;
+    if (k % 128 != 0 || n > (int64_t)1 << 22 || k > (int64_t)1 << 20 || m > ((int64_t)1 << 31) - 1)
+        return QX_ERR_UNSUPPORTED;
+    const qx::GemmPlan plan = qx::plan_gemm(n, k, m, num_sms, true);
+    *token_tile = plan.bn;
+    *splits = plan.splits;
+    *bytes = plan.ws_bytes;
+    return QX_OK;
+}
+
 QX_API qx_status qx_gemm_splitk(const qx_packed *p, const void *X, int64_t m, void *Y, void *workspace,
                                 size_t workspace_bytes, int32_t flags, void *stream) {
     qx_status s = check_gemm_args(p, X, m, Y);

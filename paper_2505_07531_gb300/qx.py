@@ -82,6 +82,7 @@ def _lib():
         lib.qx_gemm.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(_Recipe), P(ctypes.c_size_t)]
         lib.qx_gemm_splitk.argtypes = [P(_Packed), VP, I64, VP, VP, ctypes.c_size_t, I32, VP]
+        lib.qx_gemm_splitk_plan.argtypes = [I64, I64, I64, I32, P(I32), P(I32), P(ctypes.c_size_t)]
         lib.qx_gemm_splitk_noalloc.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_quantize_act.argtypes = [VP, I32, I64, VP, VP, VP]
         lib.qx_gemv_a8.argtypes = [P(_Packed), VP, VP, I32, VP, I32, VP]
@@ -96,7 +97,7 @@ def _lib():
         lib.qx_last_error_string.argtypes = []
         lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
-                   "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc",
+                   "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
@@ -282,6 +283,14 @@ def gemm_splitk_workspace_bytes(n: int, k: int, m: int, recipe: Recipe) -> int:
     r = recipe.c()
     _check(_lib().qx_gemm_splitk_workspace(n, k, m, ctypes.byref(r), ctypes.byref(b)), "qx_gemm_splitk_workspace")
     return int(b.value)
+
+
+def gemm_splitk_plan(n: int, k: int, m: int, num_sms: int) -> tuple:
+    """(tokens per tile, k splits, workspace bytes) of qx_gemm_splitk (host only)."""
+    bn, sp, nb = ctypes.c_int32(0), ctypes.c_int32(0), ctypes.c_size_t(0)
+    _check(_lib().qx_gemm_splitk_plan(n, k, m, num_sms, ctypes.byref(bn), ctypes.byref(sp), ctypes.byref(nb)),
+           "qx_gemm_splitk_plan")
+    return bn.value, sp.value, int(nb.value)
 
 
 _WORKSPACES: dict = {}
