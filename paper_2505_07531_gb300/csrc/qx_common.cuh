@@ -129,14 +129,6 @@ __device__ __forceinline__ Table8 table8_offsets(uint32_t z) {
 }
 
 // ------------------------------------------------------------- misc helpers
-__device__ __forceinline__ uint4 ldg_nc_v4(const void *p) {
-    uint4 v;
-    asm volatile("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-                 : "l"(p));
-    return v;
-}
-
 __device__ __forceinline__ uint32_t zero_nibble(const uint8_t *zrow, int grp) {
     return (zrow[grp >> 1] >> ((grp & 1) * 4)) & 15u;
 }
