@@ -126,7 +126,9 @@ qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream);
  * "Decode").  x: device fp16 [batch][k], row-major, 16-byte aligned;
  * y: device [batch][n] of y_dtype (QX_F16 or QX_F32), 4-byte aligned.
  * batch in 1..16; k <= 32768.  fp16 products summed in fp32 per 32 weights
- * and across groups.  Batches above four stream the weights once per eight
+ * and across groups; the products and their sums over 16 consecutive weight
+ * pairs are formed in fp16, so they must stay within its range (|.| < 65504),
+ * which LLM weights and activations satisfy by orders of magnitude.  Batches above four stream the weights once per eight
  * rows of x (once per four where eight rows of x do not fit on chip). */
 qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y,
                   int32_t y_dtype, void *stream);

@@ -554,3 +554,57 @@ def test_gemv_a8_full_size_sampled(qx, llama_layer):
         w_exact = (qw - z) * np.repeat(ref["scales"].astype(np.float64), 128, axis=1)
         qr, sr = act8.quantize_act(x)
         _check_matmul(y, act8.gemv_a8(ref, rec, x, k), act8.dequant_act(qr, sr), w_exact)
+
+
+# ---------------------------------------------------------------- degenerate groups
+def _degenerate_weights(g):
+    """Rows of groups that take the quantizers' special paths: all zero, one
+    constant (positive and negative), a few distinct values, subnormals whose
+    scale underflows, fp16 extremes, and a single outlier among zeros."""
+    k = 4 * g
+    rows = []
+    rows.append(np.zeros(k))
+    rows.append(np.full(k, 0.0371))
+    rows.append(np.full(k, -2.5))
+    rows.append(np.tile(np.array([-0.25, 0.0, 0.125, 0.5]), k // 4))
+    rows.append(np.tile(np.array([6e-8, -1.2e-7, 0.0, 3e-8]), k // 4))  # fp16 subnormals
+    ext = np.zeros(k)
+    ext[::3] = 65504.0
+    ext[1::3] = -65504.0
+    rows.append(ext)
+    one = np.zeros(k)
+    one[g // 2] = 7.0
+    one[g + 3] = -0.001
+    rows.append(one)
+    rng = np.random.default_rng(g)
+    rows.append(rng.choice([-1.0, -0.5, 0.0, 0.5, 1.0, 2.0, -3.0, 0.25, 9.0], k))  # nine distinct values
+    return np.stack(rows).astype(np.float16)
+
+
+@pytest.mark.parametrize("bits,g,kind", [(4, 64, 0), (3, 64, 0), (4, 128, 0), (3, 128, 1), (3, 32, 1)])
+def test_degenerate_groups_bit_exact(qx, bits, g, kind):
+    W = _degenerate_weights(g)
+    n, k = W.shape
+    k_pad = max(k, 128)  # k must be a multiple of 128
+    if k_pad != k:
+        W = np.concatenate([W, np.zeros((n, k_pad - k), dtype=np.float16)], axis=1)
+        k = k_pad
+    rec = _orecipe(bits, g, kind)
+    ref = oracle.quantize(W, rec)
+    P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+    assert qx.device_status() == 0
+    got = P.to_numpy()
+    assert np.array_equal(got["codes"], ref["codes"])
+    for key in ("scales", "luts"):
+        if ref[key] is not None:
+            assert np.array_equal(got[key].view(np.uint16), ref[key].view(np.uint16)), key
+    if ref["zeros"] is not None:
+        assert np.array_equal(got["zeros"], ref["zeros"])
+    Wh = oracle.dequant(ref, rec, k)
+    assert np.array_equal(qx.dequant(P).cpu().numpy().view(np.uint16), Wh.view(np.uint16))
+    # the decode forms its products and 16-pair sums in fp16: the row of fp16
+    # extremes (row 5) is outside that range by design and is left out here
+    x = synth.activations(2, k, seed=g, stream=93)
+    y = qx.gemv(P, torch.from_numpy(x).cuda(), out_dtype=torch.float32).cpu().numpy()
+    keep = [r for r in range(n) if r != 5]
+    _check_matmul(y[:, keep], oracle.gemv(ref, rec, x, k)[:, keep], x, Wh[keep])
