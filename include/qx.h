@@ -251,6 +251,65 @@ qx_status qx_select_recipe(const void *W, int64_t n, int64_t k, const qx_recipe 
                            double max_bpw, void *workspace, size_t workspace_bytes, int32_t *chosen,
                            uint64_t *sq_error, double *bpw, void *stream);
 
+/* Q4X shared-codebook matrices (Section 3.2, Fig. 3a/3b; Table 2 "Q4X
+ * W4A8G64", 4.28 bits per weight).  Groups of 64 consecutive weights along k;
+ * each group has an fp16 scale s = max|w| and a 2-bit index b naming one of
+ * four codebooks of 16 fp16 levels in [-1, 1], learned per matrix; every
+ * weight has a 4-bit code q.
+ *   codes     : uint8 [n][k/2], the 4-bit code layout of the header comment
+ *   scales    : fp16 [n][k/64]
+ *   books     : uint8 [n][ceil(k/256)]; group j's index in bits 2(j%4) and
+ *               2(j%4)+1 of byte j/4; a row's unused high bits are zero
+ *   codebooks : fp16 [4][16], each ascending
+ * Dequantized weight: w_hat = fp16_rn((float)s * (float)codebooks[b][q]).
+ * Shapes: n >= 1, k a multiple of 64, n*k at most 2^31.  All four pointers
+ * are device memory; codes 16-byte aligned, scales and codebooks 2-byte. */
+typedef struct qx_q4x {
+    int64_t n, k;
+    void *codes;
+    void *scales;
+    void *books;
+    void *codebooks;
+} qx_q4x;
+
+typedef struct qx_q4x_sizes {
+    uint64_t codes, scales, books, codebooks;
+} qx_q4x_sizes;
+
+/* Host only: byte sizes of the four Q4X buffers of an n x k matrix, and of the
+ * workspace qx_q4x_quantize needs (about 42 bytes per group plus 42 MB:
+ * per-group histograms, the value histograms of the four books).
+ * Errors: INVALID_ARG (NULL, n < 1, k < 1), UNSUPPORTED (k not a multiple of
+ * 64, n*k above 2^31). */
+qx_status qx_q4x_size(int64_t n, int64_t k, qx_q4x_sizes *out);
+qx_status qx_q4x_workspace(int64_t n, int64_t k, size_t *bytes);
+
+/* Learn the four codebooks of W (device fp16 [n][k] = out->n x out->k,
+ * 16-byte aligned) and code it into *out, bit-identical to the CPU oracle:
+ * s = max|w| per group; U = rint(w / s 2^20) (float64); a 32-bin histogram of
+ * U per group; k-means with 4 centres over the histograms (start: the groups
+ * at ranks floor((2j+1) L / 8) by sum U^2, then position; float64 distances
+ * in bin order, ties to the lower centre; exact integer means); each book's
+ * 16 levels by Lloyd-Max over its groups' U (quantile start, ties to the lower
+ * level, exact integer cell sums); codebook = fp16(level / 2^20); codes = the
+ * nearest of the 16 fp16 candidates (ties to the lower).  Both iterations stop
+ * when an assignment repeats, after at most `iters` (0..1000) steps.
+ * workspace: device memory, 256-byte aligned, of at least qx_q4x_workspace()
+ * bytes; the call zero-fills what it needs.  Asynchronous on `stream`; NaN or
+ * Inf in a group sets QX_ERR_NONFINITE in the device status and codes that
+ * group as all zero. */
+qx_status qx_q4x_quantize(const void *W, int32_t iters, const qx_q4x *out, void *workspace,
+                          size_t workspace_bytes, void *stream);
+
+/* Dequantize into W_out (device fp16 [n][k], 16-byte aligned), bit-exact with
+ * the formula above. */
+qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream);
+
+/* Decode matmul y = x W_hat^T for a Q4X matrix: x device fp16 [batch][k],
+ * 16-byte aligned; y device [batch][n] of y_dtype, 4-byte aligned; batch
+ * 1..16.  w_hat exactly as above, products and sums in fp32. */
+qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream);
+
 /* Synchronize `stream`, then return and clear the current device's status word
  * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
  * synchronization itself fails. */

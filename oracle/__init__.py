@@ -50,6 +50,10 @@ from .q4x import (  # noqa: F401
     pack_books,
     unpack_books,
     q4x_sizes,
+    pack_codes4,
+    unpack_codes4,
+    pack_q4x,
+    gemv_q4x,
 )
 from .select import select_recipe, sq_error_units, bits_per_weight  # noqa: F401
 from .act8 import quantize_act, gemv_a8, dequant_act  # noqa: F401

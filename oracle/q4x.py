@@ -219,6 +219,47 @@ def unpack_books(packed: np.ndarray, G: int) -> np.ndarray:
     return out
 
 
+_NIBBLE = [j // 2 + 4 * (j % 2) for j in range(8)]  # nibble of k = 8t + j in word t
+
+
+def pack_codes4(codes: np.ndarray) -> np.ndarray:
+    """4-bit codes uint8 [n][k] (k a multiple of 8) -> bytes [n][k/2] in the
+    library's 4-bit layout: little-endian word t holds k = 8t..8t+7, the code of
+    k = 8t + j in nibble j/2 + 4 (j % 2)."""
+    c = np.asarray(codes, dtype=np.uint32)
+    n, k = c.shape
+    if k % 8:
+        raise ValueError("k must be a multiple of 8")
+    c = c.reshape(n, k // 8, 8)
+    words = np.zeros((n, k // 8), dtype=np.uint32)
+    for j in range(8):
+        words |= (c[:, :, j] & np.uint32(15)) << np.uint32(4 * _NIBBLE[j])
+    return words.astype("<u4").view(np.uint8).reshape(n, k // 2)
+
+
+def unpack_codes4(packed: np.ndarray, k: int) -> np.ndarray:
+    """Inverse of :func:`pack_codes4`."""
+    n = packed.shape[0]
+    words = np.ascontiguousarray(packed, dtype=np.uint8).reshape(n, k // 2).view("<u4").astype(np.uint32)
+    out = np.zeros((n, k // 8, 8), dtype=np.uint8)
+    for j in range(8):
+        out[:, :, j] = (words >> np.uint32(4 * _NIBBLE[j])) & np.uint32(15)
+    return out.reshape(n, k)
+
+
+def pack_q4x(q: dict) -> dict:
+    """The packed buffers of a :func:`quantize_q4x` result: codes [n][k/2],
+    scales fp16 [n][k/64], books [n][ceil(k/256)], codebooks fp16 [4][16]."""
+    return {"codes": pack_codes4(q["codes"]), "scales": q["scales"], "books": pack_books(q["books"]),
+            "codebooks": q["codebooks"]}
+
+
+def gemv_q4x(q: dict, x: np.ndarray) -> np.ndarray:
+    """float64 y [batch][n] = x W_hat^T with W_hat from :func:`dequant_q4x`."""
+    Wh = dequant_q4x(q["codes"], q["scales"], q["books"], q["codebooks"]).astype(F64)
+    return np.atleast_2d(np.asarray(x, dtype=F16)).astype(F64) @ Wh.T
+
+
 def q4x_sizes(n: int, k: int, g: int = GROUP) -> dict:
     """Byte sizes of a packed Q4X matrix: 4-bit codes, fp16 scales, 2-bit book
     indices (padded per row to whole bytes), and the 4 x 16 fp16 codebook."""

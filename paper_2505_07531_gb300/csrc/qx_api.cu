@@ -626,6 +626,110 @@ QX_API qx_status qx_select_recipe(const void *W, int64_t n, int64_t k, const qx_
     return QX_OK;
 }
 
+namespace {
+
+qx_status check_q4x_shape(int64_t n, int64_t k) {
+    if (n < 1 || k < 1) return QX_ERR_INVALID_ARG;
+    if (k % qx::kQ4xGroup != 0) return QX_ERR_UNSUPPORTED;
+    // value-histogram counts are 32-bit, group indices below 2^32
+    if (n > ((int64_t)1 << 31) / k) return QX_ERR_UNSUPPORTED;
+    return QX_OK;
+}
+
+qx_status check_q4x(const qx_q4x *p) {
+    if (p == nullptr) return QX_ERR_INVALID_ARG;
+    const qx_status s = check_q4x_shape(p->n, p->k);
+    if (s != QX_OK) return s;
+    if (p->codes == nullptr || p->scales == nullptr || p->books == nullptr || p->codebooks == nullptr)
+        return QX_ERR_INVALID_ARG;
+    if (!aligned(p->codes, 16) || !aligned(p->scales, 2) || !aligned(p->codebooks, 2)) return QX_ERR_ALIGNMENT;
+    return QX_OK;
+}
+
+qx::Q4xMat q4x_mat(const qx_q4x *p) {
+    qx::Q4xMat m{};
+    m.codes = static_cast<const uint8_t *>(p->codes);
+    m.scales = static_cast<const __half *>(p->scales);
+    m.books = static_cast<const uint8_t *>(p->books);
+    m.codebooks = static_cast<const __half *>(p->codebooks);
+    m.n = p->n;
+    m.k = p->k;
+    m.G = (int)(p->k / qx::kQ4xGroup);
+    m.bbytes = (m.G + 3) / 4;
+    return m;
+}
+
+}  // namespace
+
+QX_API qx_status qx_q4x_size(int64_t n, int64_t k, qx_q4x_sizes *out) {
+    if (out == nullptr) return QX_ERR_INVALID_ARG;
+    const qx_status s = check_q4x_shape(n, k);
+    if (s != QX_OK) return s;
+    const int64_t G = k / qx::kQ4xGroup;
+    out->codes = (uint64_t)(n * k / 2);
+    out->scales = (uint64_t)(n * G * 2);
+    out->books = (uint64_t)(n * ((G + 3) / 4));
+    out->codebooks = 4 * 16 * 2;
+    return QX_OK;
+}
+
+QX_API qx_status qx_q4x_workspace(int64_t n, int64_t k, size_t *bytes) {
+    if (bytes == nullptr) return QX_ERR_INVALID_ARG;
+    const qx_status s = check_q4x_shape(n, k);
+    if (s != QX_OK) return s;
+    *bytes = qx::q4x_workspace_bytes(n, k);
+    return QX_OK;
+}
+
+QX_API qx_status qx_q4x_quantize(const void *W, int32_t iters, const qx_q4x *out, void *workspace,
+                                 size_t workspace_bytes, void *stream) {
+    if (W == nullptr) return QX_ERR_INVALID_ARG;
+    qx_status s = check_q4x(out);
+    if (s != QX_OK) return s;
+    if (iters < 0 || iters > 1000) return QX_ERR_INVALID_ARG;
+    if (workspace == nullptr || workspace_bytes < qx::q4x_workspace_bytes(out->n, out->k)) return QX_ERR_INVALID_ARG;
+    if (!aligned(W, 16) || !aligned(workspace, 256)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::Q4xQuantArgs a{};
+    a.W = static_cast<const __half *>(W);
+    a.n = out->n;
+    a.k = out->k;
+    a.G = (int)(out->k / qx::kQ4xGroup);
+    a.bbytes = (a.G + 3) / 4;
+    a.iters = iters;
+    a.codes = static_cast<uint8_t *>(out->codes);
+    a.scales = static_cast<__half *>(out->scales);
+    a.books = static_cast<uint8_t *>(out->books);
+    a.codebooks = static_cast<__half *>(out->codebooks);
+    a.ws = workspace;
+    a.status = d->status;
+    return from_cuda(qx::launch_q4x_quantize(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream) {
+    qx_status s = check_q4x(p);
+    if (s != QX_OK) return s;
+    if (W_out == nullptr) return QX_ERR_INVALID_ARG;
+    if (!aligned(W_out, 16)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    return from_cuda(qx::launch_q4x_dequant(q4x_mat(p), static_cast<__half *>(W_out), d->num_sms,
+                                            static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream) {
+    qx_status s = check_q4x(p);
+    if (s != QX_OK) return s;
+    if (x == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
+    if (y_dtype != QX_F16 && y_dtype != QX_F32) return QX_ERR_INVALID_ARG;
+    if (batch < 1) return QX_ERR_INVALID_ARG;
+    if (batch > 16) return QX_ERR_UNSUPPORTED;
+    if (!aligned(x, 16) || !aligned(y, 4)) return QX_ERR_ALIGNMENT;
+    return from_cuda(qx::launch_q4x_gemv(q4x_mat(p), static_cast<const __half *>(x), batch, y, y_dtype == QX_F32,
+                                         static_cast<cudaStream_t>(stream)));
+}
+
 QX_API qx_status qx_get_device_status(void *stream) {
     DeviceInfo *d = nullptr;
     qx_status s = device_info(&d);

@@ -161,6 +161,37 @@ inline cudaError_t ensure_kernel_attrs(const void *kern, std::atomic<uint64_t> &
     return e;
 }
 
+// Q4X shared-codebook matrices: groups of 64 weights with an fp16 scale and a
+// 2-bit book index (four per byte), 4-bit codes in the 4-bit layout, and four
+// codebooks of 16 fp16 levels per matrix.
+constexpr int kQ4xGroup = 64;
+
+struct Q4xMat {
+    const uint8_t *codes;     // [n][k/2]
+    const __half *scales;     // [n][G]
+    const uint8_t *books;     // [n][bbytes]
+    const __half *codebooks;  // [4][16]
+    int64_t n, k;
+    int G, bbytes;            // G = k/64, bbytes = ceil(G/4)
+};
+
+struct Q4xQuantArgs {
+    const __half *W;  // [n][k]
+    int64_t n, k;
+    int G, bbytes, iters;
+    uint8_t *codes;
+    __half *scales;
+    uint8_t *books;
+    __half *codebooks;
+    void *ws;  // q4x_workspace_bytes(n, k), 256-byte aligned
+    uint32_t *status;
+};
+
+size_t q4x_workspace_bytes(int64_t n, int64_t k);
+cudaError_t launch_q4x_quantize(const Q4xQuantArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_q4x_dequant(const Q4xMat &m, __half *W, int num_sms, cudaStream_t st);
+cudaError_t launch_q4x_gemv(const Q4xMat &m, const __half *x, int batch, void *y, int y_f32, cudaStream_t st);
+
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
 bool plan_gemv(GemvMulti &a, int num_sms);

@@ -59,6 +59,16 @@ class _Packed(ctypes.Structure):
                 ("zeros", ctypes.c_void_p), ("luts", ctypes.c_void_p)]
 
 
+class _Q4x(ctypes.Structure):
+    _fields_ = [("n", ctypes.c_int64), ("k", ctypes.c_int64), ("codes", ctypes.c_void_p),
+                ("scales", ctypes.c_void_p), ("books", ctypes.c_void_p), ("codebooks", ctypes.c_void_p)]
+
+
+class _Q4xSizes(ctypes.Structure):
+    _fields_ = [("codes", ctypes.c_uint64), ("scales", ctypes.c_uint64),
+                ("books", ctypes.c_uint64), ("codebooks", ctypes.c_uint64)]
+
+
 _LIB = None
 
 
@@ -90,6 +100,11 @@ def _lib():
         lib.qx_select_recipe.argtypes = [VP, I64, I64, P(_Recipe), I32, ctypes.c_double, VP, ctypes.c_size_t,
                                          P(I32), P(ctypes.c_uint64), P(ctypes.c_double), VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
+        lib.qx_q4x_size.argtypes = [I64, I64, P(_Q4xSizes)]
+        lib.qx_q4x_workspace.argtypes = [I64, I64, P(ctypes.c_size_t)]
+        lib.qx_q4x_quantize.argtypes = [VP, I32, P(_Q4x), VP, ctypes.c_size_t, VP]
+        lib.qx_q4x_dequant.argtypes = [P(_Q4x), VP, VP]
+        lib.qx_q4x_gemv.argtypes = [P(_Q4x), VP, I32, VP, I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
         lib.qx_status_string.restype = ctypes.c_char_p
@@ -99,6 +114,7 @@ def _lib():
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
+                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
@@ -390,6 +406,93 @@ def select_recipe(W: torch.Tensor, candidates, max_bpw: float | None = None):
     errors = [None if err[2 * i] == err[2 * i + 1] == 2 ** 64 - 1 else err[2 * i] | (err[2 * i + 1] << 64)
               for i in range(len(cands))]
     return (None if chosen.value < 0 else chosen.value), errors, list(bpw)
+
+
+Q4X_GROUP = 64
+
+
+def q4x_size(n: int, k: int) -> dict:
+    """Byte sizes of the Q4X buffers of an n x k matrix (host-only call)."""
+    s = _Q4xSizes()
+    _check(_lib().qx_q4x_size(n, k, ctypes.byref(s)), "qx_q4x_size")
+    return {"codes": s.codes, "scales": s.scales, "books": s.books, "codebooks": s.codebooks}
+
+
+def q4x_workspace_bytes(n: int, k: int) -> int:
+    nbytes = ctypes.c_size_t(0)
+    _check(_lib().qx_q4x_workspace(n, k, ctypes.byref(nbytes)), "qx_q4x_workspace")
+    return int(nbytes.value)
+
+
+class Q4xMatrix:
+    """A Q4X shared-codebook matrix (4-bit codes, fp16 scale and 2-bit book
+    index per group of 64, four 16-level codebooks), in torch device tensors."""
+
+    def __init__(self, n, k, codes, scales, books, codebooks):
+        self.n, self.k = int(n), int(k)
+        self.codes, self.scales, self.books, self.codebooks = codes, scales, books, codebooks
+
+    @classmethod
+    def empty(cls, n: int, k: int, device) -> "Q4xMatrix":
+        sz = q4x_size(n, k)
+        return cls(n, k, torch.empty(sz["codes"], dtype=torch.uint8, device=device),
+                   torch.empty(sz["scales"] // 2, dtype=torch.float16, device=device),
+                   torch.empty(sz["books"], dtype=torch.uint8, device=device),
+                   torch.empty(sz["codebooks"] // 2, dtype=torch.float16, device=device))
+
+    @property
+    def device(self):
+        return self.codes.device
+
+    def nbytes(self) -> int:
+        return sum(t.numel() * t.element_size() for t in (self.codes, self.scales, self.books, self.codebooks))
+
+    def c(self) -> _Q4x:
+        return _Q4x(self.n, self.k, *(t.data_ptr() for t in (self.codes, self.scales, self.books, self.codebooks)))
+
+    def to_numpy(self) -> dict:
+        """Host copies in the oracle's array shapes (for tests)."""
+        G = self.k // Q4X_GROUP
+        return {"codes": self.codes.cpu().numpy().reshape(self.n, -1),
+                "scales": self.scales.cpu().numpy().reshape(self.n, G),
+                "books": self.books.cpu().numpy().reshape(self.n, -1),
+                "codebooks": self.codebooks.cpu().numpy().reshape(4, 16)}
+
+
+def q4x_quantize(W: torch.Tensor, iters: int = 25, out: Q4xMatrix | None = None) -> Q4xMatrix:
+    """Learn the four codebooks of fp16 W [n][k] and code it (qx_q4x_quantize)."""
+    _dev_tensor(W, "W")
+    n, k = W.shape
+    P = out if out is not None else Q4xMatrix.empty(n, k, W.device)
+    ws = torch.empty(q4x_workspace_bytes(n, k), dtype=torch.uint8, device=W.device)
+    pc = P.c()
+    _check(_lib().qx_q4x_quantize(_ptr(W), iters, ctypes.byref(pc), _ptr(ws), ws.numel(), _stream(W.device)),
+           "qx_q4x_quantize")
+    return P
+
+
+def q4x_dequant(P: Q4xMatrix, out: torch.Tensor | None = None) -> torch.Tensor:
+    """fp16 W_hat [n][k] of a Q4X matrix (qx_q4x_dequant)."""
+    W = out if out is not None else torch.empty((P.n, P.k), dtype=torch.float16, device=P.device)
+    _dev_tensor(W, "out")
+    pc = P.c()
+    _check(_lib().qx_q4x_dequant(ctypes.byref(pc), _ptr(W), _stream(P.device)), "qx_q4x_dequant")
+    return W
+
+
+def q4x_gemv(P: Q4xMatrix, x: torch.Tensor, out: torch.Tensor | None = None,
+             out_dtype=torch.float16) -> torch.Tensor:
+    """Decode y = x W_hat^T for a Q4X matrix, x [batch][k] (qx_q4x_gemv)."""
+    _dev_tensor(x, "x")
+    x2 = x.view(-1, P.k)
+    b = x2.shape[0]
+    dt = out.dtype if out is not None else out_dtype
+    y = out if out is not None else torch.empty((b, P.n), dtype=dt, device=x.device)
+    _dev_tensor(y, "out", dt)
+    pc = P.c()
+    _check(_lib().qx_q4x_gemv(ctypes.byref(pc), _ptr(x2), b, _ptr(y), F32 if dt == torch.float32 else F16,
+                              _stream(x.device)), "qx_q4x_gemv")
+    return y
 
 
 def device_status(stream=None) -> int:

@@ -130,3 +130,57 @@ def test_status_strings_and_version(qx):
     for code in range(7):
         assert len(lib.qx_status_string(code)) > 0
     assert lib.qx_version() >= 100
+
+
+@pytest.mark.parametrize("n,k", [(1, 64), (37, 320), (64, 512), (4096, 4096), (11008, 4096), (4096, 11008)])
+def test_q4x_size_matches_oracle(qx, n, k):
+    assert qx.q4x_size(n, k) == oracle.q4x_sizes(n, k)
+
+
+def test_q4x_shape_limits_and_workspace(qx):
+    lib = qx._lib()
+    s = qx._Q4xSizes()
+    nbytes = ctypes.c_size_t(0)
+    assert lib.qx_q4x_size(0, 64, ctypes.byref(s)) == 1
+    assert lib.qx_q4x_size(4, 100, ctypes.byref(s)) == 2            # k not a multiple of 64
+    assert lib.qx_q4x_size(4, 64, None) == 1
+    assert lib.qx_q4x_size(1 << 19, 4096, ctypes.byref(s)) == 0     # n k = 2^31: the limit
+    assert lib.qx_q4x_size((1 << 19) + 1, 4096, ctypes.byref(s)) == 2
+    assert lib.qx_q4x_workspace(4, 64, None) == 1
+    assert lib.qx_q4x_workspace(4, 100, ctypes.byref(nbytes)) == 2
+    # per-group histograms, sums and assignments grow with the groups; the
+    # value histograms of the four books are a fixed 42 MB
+    a, b = qx.q4x_workspace_bytes(64, 4096), qx.q4x_workspace_bytes(4096, 4096)
+    assert 4 * (2 ** 21 + 1) * 5 < a < b
+    assert b - a >= (4096 - 64) * 64 * 42 - 1024
+
+
+def test_q4x_entry_points_reject_bad_arguments_before_launching(qx):
+    lib = qx._lib()
+    A = ctypes.c_void_p
+    good = qx._Q4x(64, 512, A(0x10000), A(0x20000), A(0x30000), A(0x40000))
+    ws = A(0x100000)
+    big = 1 << 40
+    assert lib.qx_q4x_quantize(None, 25, ctypes.byref(good), ws, big, None) == 1
+    assert lib.qx_q4x_quantize(A(0x1000), 25, None, ws, big, None) == 1
+    nul = qx._Q4x(64, 512, A(0x10000), None, A(0x30000), A(0x40000))
+    assert lib.qx_q4x_quantize(A(0x1000), 25, ctypes.byref(nul), ws, big, None) == 1
+    assert lib.qx_q4x_quantize(A(0x1000), -1, ctypes.byref(good), ws, big, None) == 1
+    assert lib.qx_q4x_quantize(A(0x1000), 1001, ctypes.byref(good), ws, big, None) == 1
+    assert lib.qx_q4x_quantize(A(0x1000), 25, ctypes.byref(good), ws, 1024, None) == 1  # workspace too small
+    assert lib.qx_q4x_quantize(A(0x1000), 25, ctypes.byref(good), None, big, None) == 1
+    assert lib.qx_q4x_quantize(A(0x1008), 25, ctypes.byref(good), ws, big, None) == 3   # W alignment
+    assert lib.qx_q4x_quantize(A(0x1000), 25, ctypes.byref(good), A(0x100080), big, None) == 3
+    mis = qx._Q4x(64, 512, A(0x10008), A(0x20000), A(0x30000), A(0x40000))
+    assert lib.qx_q4x_quantize(A(0x1000), 25, ctypes.byref(mis), ws, big, None) == 3
+    odd = qx._Q4x(64, 500, A(0x10000), A(0x20000), A(0x30000), A(0x40000))
+    assert lib.qx_q4x_quantize(A(0x1000), 25, ctypes.byref(odd), ws, big, None) == 2
+    assert lib.qx_q4x_dequant(ctypes.byref(good), None, None) == 1
+    assert lib.qx_q4x_dequant(ctypes.byref(good), A(0x5008), None) == 3
+    assert lib.qx_q4x_dequant(ctypes.byref(mis), A(0x5000), None) == 3
+    assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5000), 0, A(0x6000), 0, None) == 1
+    assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5000), 17, A(0x6000), 0, None) == 2
+    assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5000), 1, A(0x6000), 2, None) == 1   # y dtype
+    assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5008), 1, A(0x6000), 0, None) == 3
+    assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5000), 1, A(0x6002), 0, None) == 3
+    assert lib.qx_q4x_gemv(ctypes.byref(good), None, 1, A(0x6000), 0, None) == 1

@@ -9,6 +9,7 @@ import os
 import numpy as np
 import pytest
 
+import oracle
 from oracle import q4x
 import synth
 
@@ -209,3 +210,31 @@ def test_dead_groups_take_no_part_in_learning():
     a, b = q4x.quantize_q4x(W), q4x.quantize_q4x(Wd)
     assert np.array_equal(a["codebooks"].view(np.uint16), b["codebooks"].view(np.uint16))
     assert np.array_equal(a["codes"], b["codes"][:24]) and np.array_equal(a["books"], b["books"][:24])
+
+
+def test_code_packing_byte_image():
+    """Codes 0..7 of k = 0..7: code j sits in nibble j/2 + 4 (j % 2), so the
+    little-endian word is 0x75316420."""
+    codes = np.arange(8, dtype=np.uint8)[None, :]
+    assert list(q4x.pack_codes4(codes)[0]) == [0x20, 0x64, 0x31, 0x75]
+
+
+def test_code_packing_matches_the_4bit_format_and_round_trips():
+    rng = np.random.default_rng(12)
+    c = rng.integers(0, 16, (7, 256)).astype(np.uint8)
+    assert np.array_equal(q4x.pack_codes4(c), oracle.pack_codes(c, 4))
+    c = rng.integers(0, 16, (5, 320)).astype(np.uint8)  # k = 5 groups: not a multiple of 128
+    assert np.array_equal(q4x.unpack_codes4(q4x.pack_codes4(c), 320), c)
+
+
+def test_gemv_against_exact_rational_arithmetic():
+    from fractions import Fraction
+
+    r = q4x.quantize_q4x(_w(3, 128, 13))
+    x = synth.activations(2, 128, seed=13, stream=13)
+    y = q4x.gemv_q4x(r, x)
+    Wh = q4x.dequant_q4x(r["codes"], r["scales"], r["books"], r["codebooks"])
+    for b in range(2):
+        for n in range(3):
+            want = sum(Fraction(float(x[b, kk])) * Fraction(float(Wh[n, kk])) for kk in range(128))
+            assert abs(Fraction(y[b, n]) - want) <= abs(want) * Fraction(1, 10 ** 13) + Fraction(1, 10 ** 30)
