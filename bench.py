@@ -446,6 +446,11 @@ def run_ours(args):
         extra["recipe_select"] = run_select(qx, torch, dev, stream)
         torch.cuda.empty_cache()
         extra["config5"] = run_config5(qx, torch, dev, stream)
+        torch.cuda.empty_cache()
+        try:  # last: its result or its error is reported, the sections above stand
+            extra["q4x"] = run_q4x(qx, torch, dev, stream, l2, hbm)
+        except Exception as e:  # noqa: BLE001
+            extra["q4x"] = {"error": f"{type(e).__name__}: {e}"[:300]}
 
     if rank == 0:
         cpu = run_cpu_baseline() if not args.skip_cpu_baseline else None
@@ -635,6 +640,64 @@ def run_config3(qx, torch, dev, stream, l2):
         del layers, base
     if qx.device_status(stream) != 0:
         raise RuntimeError("config-3 decode reported a device error")
+    return out
+
+
+def run_q4x(qx, torch, dev, stream, l2, hbm):
+    """Q4X shared codebooks (groups of 64 with an fp16 scale and a 2-bit book
+    index, 4-bit codes, four 16-level codebooks learned per matrix): the
+    learner's device time per Llama-7B layer matrix, and the decode matmul over
+    the layer at batch 1 and 4 (seven qx_q4x_gemv launches per layer copy in
+    one CUDA graph, weights rotated over copies larger than 4x L2)."""
+    import synth
+
+    def learn(name, n, k, sigma, sid):
+        W = synth.student_t_weights_torch(n, k, sigma, seed=0, stream=sid, device=dev)
+        with torch.cuda.stream(stream):
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            P = qx.q4x_quantize(W)
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        return P, e0.elapsed_time(e1)
+
+    learn(*LAYER[0])  # sizes the caching allocator's workspace block
+    base, learn_ms = {}, {}
+    for spec in LAYER:
+        base[spec[0]], learn_ms[spec[0]] = learn(*spec)
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("q4x_quantize reported a device error")
+    layer_bytes = sum(P.nbytes() for P in base.values())
+    copies = max(2, math.ceil(4 * l2 / layer_bytes))
+    dup = lambda P: qx.Q4xMatrix(P.n, P.k, P.codes.clone(), P.scales.clone(), P.books.clone(), P.codebooks.clone())
+    layers = [base] + [{nm: dup(P) for nm, P in base.items()} for _ in range(copies - 1)]
+    out = {"learn_ms": learn_ms, "weight_bytes": layer_bytes,
+           "bits_per_weight": 8.0 * layer_bytes / sum(n * k for _, n, k, _, _ in LAYER)}
+    for batch in (1, 4):
+        xs = {k: synth.activations_torch(batch, k, seed=batch, stream=70 + i, device=dev)
+              for i, k in enumerate((4096, 11008))}
+        ys = {nm: torch.empty((batch, n), dtype=torch.float16, device=dev) for nm, n, *_ in LAYER}
+
+        def body():
+            for L in layers:
+                for nm, P in L.items():
+                    qx.q4x_gemv(P, xs[P.k], out=ys[nm])
+
+        with torch.cuda.stream(stream):
+            body()
+        torch.cuda.synchronize(dev)
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            body()
+        ms = _time_graph(torch, stream, g, 20) / copies
+        del g
+        io = sum(2 * batch * k for _, _, k, _, _ in LAYER) + sum(y.numel() * 2 for y in ys.values())
+        gbps = (layer_bytes + io) / (ms * 1e-3) / 1e9
+        out[f"llama7b_layer_decode_Q4X_b{batch}"] = {
+            "us_per_layer": ms * 1e3, "GBps": gbps, "frac_of_measured_hbm": gbps / hbm,
+            "path": "qx_q4x_gemv x7 (one warp per row, codebooks in shared memory)"}
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("q4x decode reported a device error")
     return out
 
 

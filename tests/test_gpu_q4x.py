@@ -9,8 +9,7 @@ import torch
 import oracle
 import synth
 
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skip(reason="the Q4X kernels have not yet run on a GB300; enabled once they have")]
+pytestmark = pytest.mark.gpu
 
 
 @pytest.fixture(scope="module")
