@@ -647,8 +647,9 @@ def run_q4x(qx, torch, dev, stream, l2, hbm):
     """Q4X shared codebooks (groups of 64 with an fp16 scale and a 2-bit book
     index, 4-bit codes, four 16-level codebooks learned per matrix): the
     learner's device time per Llama-7B layer matrix, and the decode matmul over
-    the layer at batch 1 and 4 (seven qx_q4x_gemv launches per layer copy in
-    one CUDA graph, weights rotated over copies larger than 4x L2)."""
+    the layer at batch 1 and 4 (q,k,v | o | gate,up | down: four
+    qx_q4x_gemv_multi launches per layer copy in one CUDA graph, weights
+    rotated over copies larger than 4x L2)."""
     import synth
 
     def learn(name, n, k, sigma, sid):
@@ -678,10 +679,13 @@ def run_q4x(qx, torch, dev, stream, l2, hbm):
               for i, k in enumerate((4096, 11008))}
         ys = {nm: torch.empty((batch, n), dtype=torch.float16, device=dev) for nm, n, *_ in LAYER}
 
+        chain = (["q_proj", "k_proj", "v_proj"], ["o_proj"], ["gate_proj", "up_proj"], ["down_proj"])
+
         def body():
             for L in layers:
-                for nm, P in L.items():
-                    qx.q4x_gemv(P, xs[P.k], out=ys[nm])
+                for names in chain:
+                    qx.q4x_gemv_multi([L[nm] for nm in names], [xs[L[nm].k] for nm in names],
+                                      outs=[ys[nm] for nm in names])
 
         with torch.cuda.stream(stream):
             body()
@@ -695,7 +699,7 @@ def run_q4x(qx, torch, dev, stream, l2, hbm):
         gbps = (layer_bytes + io) / (ms * 1e-3) / 1e9
         out[f"llama7b_layer_decode_Q4X_b{batch}"] = {
             "us_per_layer": ms * 1e3, "GBps": gbps, "frac_of_measured_hbm": gbps / hbm,
-            "path": "qx_q4x_gemv x7 (one warp per row, codebooks in shared memory)"}
+            "path": "4 qx_q4x_gemv_multi launches (persistent warps over the rows, codebooks in shared memory)"}
     if qx.device_status(stream) != 0:
         raise RuntimeError("q4x decode reported a device error")
     return out

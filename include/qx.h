@@ -310,6 +310,15 @@ qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream);
  * 1..16.  w_hat exactly as above, products and sums in fp32. */
 qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream);
 
+/* Several Q4X decode matmuls in one launch: y[i] = x[i] W_hat_i^T, i < count
+ * (count 1..8), each matrix with its own shape and codebooks; x[i], y[i] have
+ * the layout and alignment of qx_q4x_gemv and are passed in host arrays of
+ * `count` device pointers.  One persistent grid strides over the rows of all
+ * matrices (e.g. the q, k, v or gate, up projections of a decoder layer,
+ * which share x), so the launch cost is paid once for the group. */
+qx_status qx_q4x_gemv_multi(const qx_q4x *mats, int32_t count, const void *const *x, int32_t batch,
+                            void *const *y, int32_t y_dtype, void *stream);
+
 /* Synchronize `stream`, then return and clear the current device's status word
  * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
  * synchronization itself fails. */

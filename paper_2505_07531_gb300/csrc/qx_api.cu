@@ -718,16 +718,37 @@ QX_API qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream) {
                                             static_cast<cudaStream_t>(stream)));
 }
 
-QX_API qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream) {
-    qx_status s = check_q4x(p);
-    if (s != QX_OK) return s;
-    if (x == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
+QX_API qx_status qx_q4x_gemv_multi(const qx_q4x *mats, int32_t count, const void *const *x, int32_t batch,
+                                   void *const *y, int32_t y_dtype, void *stream) {
+    if (mats == nullptr || x == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
+    if (count < 1 || count > qx::kMaxQ4xMats) return QX_ERR_INVALID_ARG;
     if (y_dtype != QX_F16 && y_dtype != QX_F32) return QX_ERR_INVALID_ARG;
     if (batch < 1) return QX_ERR_INVALID_ARG;
     if (batch > 16) return QX_ERR_UNSUPPORTED;
-    if (!aligned(x, 16) || !aligned(y, 4)) return QX_ERR_ALIGNMENT;
-    return from_cuda(qx::launch_q4x_gemv(q4x_mat(p), static_cast<const __half *>(x), batch, y, y_dtype == QX_F32,
-                                         static_cast<cudaStream_t>(stream)));
+    qx::Q4xGemvMulti a{};
+    a.count = count;
+    a.batch = batch;
+    a.y_f32 = y_dtype == QX_F32;
+    a.row_off[0] = 0;
+    for (int i = 0; i < count; ++i) {
+        qx_status s = check_q4x(&mats[i]);
+        if (s != QX_OK) return s;
+        if (x[i] == nullptr || y[i] == nullptr) return QX_ERR_INVALID_ARG;
+        if (!aligned(x[i], 16) || !aligned(y[i], 4)) return QX_ERR_ALIGNMENT;
+        a.mat[i] = q4x_mat(&mats[i]);
+        a.x[i] = static_cast<const __half *>(x[i]);
+        a.y[i] = y[i];
+        a.row_off[i + 1] = a.row_off[i] + mats[i].n;
+    }
+    DeviceInfo *d = nullptr;
+    qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    return from_cuda(qx::launch_q4x_gemv(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream) {
+    if (p == nullptr) return QX_ERR_INVALID_ARG;
+    return qx_q4x_gemv_multi(p, 1, &x, batch, &y, y_dtype, stream);
 }
 
 QX_API qx_status qx_get_device_status(void *stream) {

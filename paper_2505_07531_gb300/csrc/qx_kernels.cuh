@@ -187,10 +187,20 @@ struct Q4xQuantArgs {
     uint32_t *status;
 };
 
+// Decode matmul over up to eight Q4X matrices in one launch: y[i] = x[i] W_i^T.
+constexpr int kMaxQ4xMats = 8;
+struct Q4xGemvMulti {
+    int count, batch, y_f32;
+    Q4xMat mat[kMaxQ4xMats];
+    const __half *x[kMaxQ4xMats];  // [batch][k_i]
+    void *y[kMaxQ4xMats];          // [batch][n_i]
+    int64_t row_off[kMaxQ4xMats + 1];  // first row of matrix i in the launch's row list
+};
+
 size_t q4x_workspace_bytes(int64_t n, int64_t k);
 cudaError_t launch_q4x_quantize(const Q4xQuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_q4x_dequant(const Q4xMat &m, __half *W, int num_sms, cudaStream_t st);
-cudaError_t launch_q4x_gemv(const Q4xMat &m, const __half *x, int batch, void *y, int y_f32, cudaStream_t st);
+cudaError_t launch_q4x_gemv(const Q4xGemvMulti &a, int num_sms, cudaStream_t st);
 
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);

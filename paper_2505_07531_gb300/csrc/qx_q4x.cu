@@ -652,80 +652,108 @@ __global__ void __launch_bounds__(kThreads) q4x_dequant_kernel(Q4xMat m, __half 
 }
 
 // ---------------------------------------------------------------- decode matmul
-constexpr int kGemvWarps = 8;  // rows per block
+constexpr int kGemvWarps = 8;  // warps per block
 
-// y[b][row] = sum_k w_hat[row][k] x[b][k], one warp per row; lane l takes the
-// 32-weight units l, l + 32, ... (16 code bytes each, half a group).  A unit's
-// w_hat are the codebook entries (shared memory) times s in fp16, which is
-// exactly fp16(fp32(s) fp32(CB)); products and sums in fp32.
-template <int NB>
-__global__ void __launch_bounds__(32 * kGemvWarps) q4x_gemv_kernel(Q4xMat m, const __half *x, int batch, void *y,
-                                                                   int y_f32) {
-    __shared__ __half cb[kBooks * kLevels];
-    if (threadIdx.x < kBooks * kLevels) cb[threadIdx.x] = m.codebooks[threadIdx.x];
-    __syncthreads();
-    const int lane = threadIdx.x & 31;
-    const int64_t row = (int64_t)blockIdx.x * kGemvWarps + (threadIdx.x >> 5);
-    if (row >= m.n) return;
-    const int units = (int)(m.k / 32);
-    const uint8_t *brow = m.books + row * m.bbytes;
-    const __half *srow = m.scales + row * m.G;
-    const uint4 *crow = reinterpret_cast<const uint4 *>(m.codes + row * (m.k / 2));
-    float acc[NB];
+// w_hat of one 32-weight unit (16 code bytes): half2 pairs (k = 2i, 2i + 1),
+// the codebook entries times s in fp16, which is exactly fp16(fp32(s) fp32(CB)).
+__device__ __forceinline__ void unit_weights(const uint4 &cw, const __half *tb, __half2 s2, float2 (&wf)[16]) {
+    const uint32_t ws[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
-    for (int b = 0; b < NB; ++b) acc[b] = 0.0f;
-    for (int u = lane; u < units; u += 32) {
-        const int j = u >> 1;
-        const __half s = srow[j];
-        const __half2 s2 = __halves2half2(s, s);
-        const __half *tb = cb + kLevels * book_index(brow, j);
-        const uint4 cw = __ldg(crow + u);
-        const uint32_t ws[4] = {cw.x, cw.y, cw.z, cw.w};
-        float2 wf[16];  // w_hat of k = 32u + 2i, 32u + 2i + 1
+    for (int t = 0; t < 4; ++t) {
 #pragma unroll
-        for (int t = 0; t < 4; ++t) {
-#pragma unroll
-            for (int i = 0; i < 4; ++i) {
-                const uint32_t sel = (ws[t] >> (4 * i)) & 0x000F000Fu;  // codes of k = 8t+2i, 8t+2i+1
-                const __half2 e = __halves2half2(tb[sel & 15u], tb[sel >> 16]);
-                wf[4 * t + i] = __half22float2(__hmul2(e, s2));
-            }
-        }
-#pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            if (b >= batch) break;
-            const uint4 *xr = reinterpret_cast<const uint4 *>(x + (int64_t)b * m.k + 32 * (int64_t)u);
-            float a = acc[b];
-#pragma unroll
-            for (int v = 0; v < 4; ++v) {
-                const uint4 xv = __ldg(xr + v);
-                const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-                for (int p = 0; p < 4; ++p) {
-                    const float2 xf = __half22float2(u2h2(xs[p]));
-                    const float2 w = wf[4 * v + p];
-                    a = fmaf(w.x, xf.x, a);
-                    a = fmaf(w.y, xf.y, a);
-                }
-            }
-            acc[b] = a;
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t sel = (ws[t] >> (4 * i)) & 0x000F000Fu;  // codes of k = 8t+2i, 8t+2i+1
+            const __half2 e = __halves2half2(tb[sel & 15u], tb[sel >> 16]);
+            wf[4 * t + i] = __half22float2(__hmul2(e, s2));
         }
     }
+}
+
+// acc[b] += the unit's 32 products with x[b][32u .. 32u+31], in fp32.
+template <int NB>
+__device__ __forceinline__ void unit_dot(const float2 (&wf)[16], const __half *x, int64_t k, int u, int batch,
+                                         float (&acc)[NB]) {
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
-        float v = acc[b];
+        if (b >= batch) break;
+        const uint4 *xr = reinterpret_cast<const uint4 *>(x + (int64_t)b * k + 32 * (int64_t)u);
+        float a = acc[b];
 #pragma unroll
-        for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-        acc[b] = v;
+        for (int v = 0; v < 4; ++v) {
+            const uint4 xv = __ldg(xr + v);
+            const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w};
+#pragma unroll
+            for (int p = 0; p < 4; ++p) {
+                const float2 xf = __half22float2(u2h2(xs[p]));
+                a = fmaf(wf[4 * v + p].x, xf.x, a);
+                a = fmaf(wf[4 * v + p].y, xf.y, a);
+            }
+        }
+        acc[b] = a;
     }
-    if (lane == 0) {
+}
+
+// y_i[b][row] = sum_k w_hat_i[row][k] x_i[b][k] for the rows of up to eight
+// matrices, taken as one list (matrix 0's rows, then matrix 1's, ...).  A
+// persistent grid of warps strides over the list, one row per warp at a time;
+// lane l takes the 32-weight units l, l + 32, ... of the row, two at a time so
+// that two code loads are in flight.  The matrices' codebooks sit in shared
+// memory (128 bytes each: one word per bank, so any lookup is conflict-free).
+template <int NB>
+__global__ void __launch_bounds__(32 * kGemvWarps) q4x_gemv_kernel(const __grid_constant__ Q4xGemvMulti a) {
+    __shared__ __half cb[kMaxQ4xMats * kBooks * kLevels];
+    for (int i = threadIdx.x; i < a.count * kBooks * kLevels; i += 32 * kGemvWarps)
+        cb[i] = a.mat[i / (kBooks * kLevels)].codebooks[i % (kBooks * kLevels)];
+    __syncthreads();
+    const int lane = threadIdx.x & 31;
+    const int64_t total = a.row_off[a.count];
+    const int64_t nwarps = (int64_t)gridDim.x * kGemvWarps;
+    for (int64_t gr = (int64_t)blockIdx.x * kGemvWarps + (threadIdx.x >> 5); gr < total; gr += nwarps) {
+        int mi = 0;
+        while (mi + 1 < a.count && gr >= a.row_off[mi + 1]) ++mi;
+        const Q4xMat &m = a.mat[mi];
+        const int64_t row = gr - a.row_off[mi];
+        const int units = (int)(m.k / 32);
+        const uint8_t *brow = m.books + row * m.bbytes;
+        const __half *srow = m.scales + row * m.G;
+        const uint4 *crow = reinterpret_cast<const uint4 *>(m.codes + row * (m.k / 2));
+        const __half *cbm = cb + mi * kBooks * kLevels;
+        const __half *x = a.x[mi];
+        float acc[NB];
+#pragma unroll
+        for (int b = 0; b < NB; ++b) acc[b] = 0.0f;
+        for (int u0 = lane; u0 < units; u0 += 64) {
+            const int u1 = u0 + 32;
+            const bool two = u1 < units;
+            // both units' codes and metadata first, then the arithmetic
+            const uint4 c0 = __ldg(crow + u0);
+            const uint4 c1 = two ? __ldg(crow + u1) : make_uint4(0u, 0u, 0u, 0u);
+            const __half s0 = srow[u0 >> 1], s1 = srow[(two ? u1 : u0) >> 1];
+            const uint32_t b0 = book_index(brow, u0 >> 1), b1 = book_index(brow, (two ? u1 : u0) >> 1);
+            float2 wf[16];
+            unit_weights(c0, cbm + kLevels * b0, __halves2half2(s0, s0), wf);
+            unit_dot<NB>(wf, x, m.k, u0, a.batch, acc);
+            if (two) {
+                unit_weights(c1, cbm + kLevels * b1, __halves2half2(s1, s1), wf);
+                unit_dot<NB>(wf, x, m.k, u1, a.batch, acc);
+            }
+        }
 #pragma unroll
         for (int b = 0; b < NB; ++b) {
-            if (b >= batch) break;
-            if (y_f32)
-                reinterpret_cast<float *>(y)[(int64_t)b * m.n + row] = acc[b];
-            else
-                reinterpret_cast<__half *>(y)[(int64_t)b * m.n + row] = __float2half_rn(acc[b]);
+            float v = acc[b];
+#pragma unroll
+            for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+            acc[b] = v;
+        }
+        if (lane == 0) {
+#pragma unroll
+            for (int b = 0; b < NB; ++b) {
+                if (b >= a.batch) break;
+                if (a.y_f32)
+                    reinterpret_cast<float *>(a.y[mi])[(int64_t)b * m.n + row] = acc[b];
+                else
+                    reinterpret_cast<__half *>(a.y[mi])[(int64_t)b * m.n + row] = __float2half_rn(acc[b]);
+            }
         }
     }
 }
@@ -784,15 +812,31 @@ cudaError_t launch_q4x_dequant(const Q4xMat &m, __half *W, int num_sms, cudaStre
     return cudaGetLastError();
 }
 
-cudaError_t launch_q4x_gemv(const Q4xMat &m, const __half *x, int batch, void *y, int y_f32, cudaStream_t st) {
-    const unsigned grid = (unsigned)((m.n + kGemvWarps - 1) / kGemvWarps);
-    const unsigned threads = 32 * kGemvWarps;
-    if (batch <= 1) q4x_gemv_kernel<1><<<grid, threads, 0, st>>>(m, x, batch, y, y_f32);
-    else if (batch <= 2) q4x_gemv_kernel<2><<<grid, threads, 0, st>>>(m, x, batch, y, y_f32);
-    else if (batch <= 4) q4x_gemv_kernel<4><<<grid, threads, 0, st>>>(m, x, batch, y, y_f32);
-    else if (batch <= 8) q4x_gemv_kernel<8><<<grid, threads, 0, st>>>(m, x, batch, y, y_f32);
-    else q4x_gemv_kernel<16><<<grid, threads, 0, st>>>(m, x, batch, y, y_f32);
+// Persistent grid: as many blocks as are resident at once (from the kernel's
+// occupancy, looked up once per instance), fewer when there are fewer rows.
+template <int NB>
+cudaError_t launch_gemv_nb(const Q4xGemvMulti &a, int num_sms, cudaStream_t st) {
+    static std::atomic<int> per_sm{0};
+    int bps = per_sm.load(std::memory_order_relaxed);
+    if (bps == 0) {
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&bps, q4x_gemv_kernel<NB>, 32 * kGemvWarps, 0) !=
+                cudaSuccess ||
+            bps < 1)
+            bps = 1;
+        per_sm.store(bps, std::memory_order_relaxed);
+    }
+    const int64_t blocks = (a.row_off[a.count] + kGemvWarps - 1) / kGemvWarps;
+    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(blocks, (int64_t)bps * num_sms));
+    q4x_gemv_kernel<NB><<<grid, 32 * kGemvWarps, 0, st>>>(a);
     return cudaGetLastError();
+}
+
+cudaError_t launch_q4x_gemv(const Q4xGemvMulti &a, int num_sms, cudaStream_t st) {
+    if (a.batch <= 1) return launch_gemv_nb<1>(a, num_sms, st);
+    if (a.batch <= 2) return launch_gemv_nb<2>(a, num_sms, st);
+    if (a.batch <= 4) return launch_gemv_nb<4>(a, num_sms, st);
+    if (a.batch <= 8) return launch_gemv_nb<8>(a, num_sms, st);
+    return launch_gemv_nb<16>(a, num_sms, st);
 }
 
 }  // namespace qx

@@ -105,6 +105,7 @@ def _lib():
         lib.qx_q4x_quantize.argtypes = [VP, I32, P(_Q4x), VP, ctypes.c_size_t, VP]
         lib.qx_q4x_dequant.argtypes = [P(_Q4x), VP, VP]
         lib.qx_q4x_gemv.argtypes = [P(_Q4x), VP, I32, VP, I32, VP]
+        lib.qx_q4x_gemv_multi.argtypes = [P(_Q4x), I32, P(VP), I32, P(VP), I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
         lib.qx_status_string.restype = ctypes.c_char_p
@@ -114,7 +115,7 @@ def _lib():
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
-                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv",
+                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
@@ -493,6 +494,31 @@ def q4x_gemv(P: Q4xMatrix, x: torch.Tensor, out: torch.Tensor | None = None,
     _check(_lib().qx_q4x_gemv(ctypes.byref(pc), _ptr(x2), b, _ptr(y), F32 if dt == torch.float32 else F16,
                               _stream(x.device)), "qx_q4x_gemv")
     return y
+
+
+def q4x_gemv_multi(mats, xs, outs=None, out_dtype=torch.float16):
+    """Several Q4X decode matmuls in one launch (qx_q4x_gemv_multi): y[i] =
+    xs[i] W_hat_i^T for up to eight matrices; returns the outputs."""
+    mats, xs = list(mats), list(xs)
+    if len(mats) != len(xs) or not 1 <= len(mats) <= 8:
+        raise ValueError("1..8 matrices, one x per matrix")
+    x2 = [x.view(-1, P.k) for P, x in zip(mats, xs)]
+    for x in x2:
+        _dev_tensor(x, "x")
+    b = x2[0].shape[0]
+    if any(x.shape[0] != b for x in x2):
+        raise ValueError("every x must have the same batch")
+    dt = outs[0].dtype if outs is not None else out_dtype
+    ys = list(outs) if outs is not None else [torch.empty((b, P.n), dtype=dt, device=x2[0].device) for P in mats]
+    for y in ys:
+        _dev_tensor(y, "out", dt)
+    cnt = len(mats)
+    arr = (_Q4x * cnt)(*[P.c() for P in mats])
+    xa = (ctypes.c_void_p * cnt)(*[x.data_ptr() for x in x2])
+    ya = (ctypes.c_void_p * cnt)(*[y.data_ptr() for y in ys])
+    _check(_lib().qx_q4x_gemv_multi(arr, cnt, xa, b, ya, F32 if dt == torch.float32 else F16,
+                                    _stream(x2[0].device)), "qx_q4x_gemv_multi")
+    return ys
 
 
 def device_status(stream=None) -> int:

@@ -184,3 +184,25 @@ def test_q4x_entry_points_reject_bad_arguments_before_launching(qx):
     assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5008), 1, A(0x6000), 0, None) == 3
     assert lib.qx_q4x_gemv(ctypes.byref(good), A(0x5000), 1, A(0x6002), 0, None) == 3
     assert lib.qx_q4x_gemv(ctypes.byref(good), None, 1, A(0x6000), 0, None) == 1
+
+
+def test_q4x_gemv_multi_rejects_bad_arguments_before_launching(qx):
+    lib = qx._lib()
+    A = ctypes.c_void_p
+    mats = (qx._Q4x * 2)(qx._Q4x(64, 512, A(0x10000), A(0x20000), A(0x30000), A(0x40000)),
+                         qx._Q4x(32, 256, A(0x50000), A(0x60000), A(0x70000), A(0x80000)))
+    xs = (A * 2)(A(0x1000), A(0x2000))
+    ys = (A * 2)(A(0x3000), A(0x4000))
+    assert lib.qx_q4x_gemv_multi(None, 1, xs, 1, ys, 0, None) == 1
+    assert lib.qx_q4x_gemv_multi(mats, 0, xs, 1, ys, 0, None) == 1
+    assert lib.qx_q4x_gemv_multi(mats, 9, xs, 1, ys, 0, None) == 1
+    assert lib.qx_q4x_gemv_multi(mats, 2, None, 1, ys, 0, None) == 1
+    assert lib.qx_q4x_gemv_multi(mats, 2, xs, 0, ys, 0, None) == 1
+    assert lib.qx_q4x_gemv_multi(mats, 2, xs, 17, ys, 0, None) == 2
+    assert lib.qx_q4x_gemv_multi(mats, 2, xs, 1, ys, 3, None) == 1
+    bad_x = (A * 2)(A(0x1000), A(0x2008))
+    assert lib.qx_q4x_gemv_multi(mats, 2, bad_x, 1, ys, 0, None) == 3
+    nul_y = (A * 2)(A(0x3000), None)
+    assert lib.qx_q4x_gemv_multi(mats, 2, xs, 1, nul_y, 0, None) == 1
+    odd = (qx._Q4x * 2)(mats[0], qx._Q4x(32, 200, A(0x50000), A(0x60000), A(0x70000), A(0x80000)))
+    assert lib.qx_q4x_gemv_multi(odd, 2, xs, 1, ys, 0, None) == 2

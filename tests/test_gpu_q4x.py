@@ -96,6 +96,25 @@ def test_gemv_fp16_output(qx, learned):
     assert np.all(oracle.max_abs_err(y, y_ref) <= tol)
 
 
+@pytest.mark.parametrize("batch", [1, 4, 16])
+def test_gemv_multi_over_mixed_shapes(qx, learned, batch):
+    """One launch over all eight parity matrices (different n, k and
+    codebooks): every output within tolerance, and equal to the one-matrix
+    call bit for bit (the same per-row arithmetic)."""
+    cs = CASES
+    mats = [learned[c][1] for c in cs]
+    xs = [torch.from_numpy(synth.activations(batch, c[1], seed=batch, stream=c[0] + 1)).cuda() for c in cs]
+    ys = qx.q4x_gemv_multi(mats, xs, out_dtype=torch.float32)
+    assert qx.device_status() == 0
+    for c, P, x, y in zip(cs, mats, xs, ys):
+        ref = learned[c][2]
+        Wh = oracle.dequant_q4x(ref["codes"], ref["scales"], ref["books"], ref["codebooks"])
+        xn = x.cpu().numpy()
+        assert np.all(oracle.max_abs_err(y.cpu().numpy(), oracle.gemv_q4x(ref, xn)) <= oracle.tolerance(xn, Wh))
+        one = qx.q4x_gemv(P, x, out_dtype=torch.float32)
+        assert torch.equal(one, y)
+
+
 def test_repeat_is_bit_identical(qx):
     """Every reduction of the learner is an integer reduction: the result does
     not depend on how the threads were scheduled."""
