@@ -319,6 +319,13 @@ qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, in
 qx_status qx_q4x_gemv_multi(const qx_q4x *mats, int32_t count, const void *const *x, int32_t batch,
                             void *const *y, int32_t y_dtype, void *stream);
 
+/* Failure-detection self-test.  Launches one CTA on `stream` whose bounded
+ * wait (the mbarrier wait of the decode and prefill pipelines) is for a phase
+ * that nothing completes.  After limit_us microseconds (1..1000000) it gives
+ * up, records QX_ERR_TIMEOUT in the device status word and returns, leaving
+ * the context usable; qx_get_device_status() then returns QX_ERR_TIMEOUT. */
+qx_status qx_selftest_wait_timeout(int32_t limit_us, void *stream);
+
 /* Synchronize `stream`, then return and clear the current device's status word
  * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
  * synchronization itself fails. */

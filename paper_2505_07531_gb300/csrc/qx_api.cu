@@ -29,16 +29,27 @@ struct DeviceInfo {
 DeviceInfo g_dev[kMaxDevices];
 std::mutex g_mu;
 
+// The name of the CUDA error behind this thread's last QX_ERR_CUDA.
+thread_local const char *t_last_error = "no error";
+
+qx_status from_cuda(cudaError_t e) {
+    if (e == cudaSuccess) return QX_OK;
+    t_last_error = cudaGetErrorName(e);
+    return QX_ERR_CUDA;
+}
+
 qx_status device_info(DeviceInfo **out) {
     int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return QX_ERR_CUDA;
+    qx_status s = from_cuda(cudaGetDevice(&dev));
+    if (s != QX_OK) return s;
+    if (dev < 0 || dev >= kMaxDevices) return QX_ERR_UNSUPPORTED;
     std::lock_guard<std::mutex> lock(g_mu);
     DeviceInfo &d = g_dev[dev];
     if (!d.ready) {
         void *p = nullptr;
-        if (cudaGetSymbolAddress(&p, g_status_word) != cudaSuccess) return QX_ERR_CUDA;
+        if ((s = from_cuda(cudaGetSymbolAddress(&p, g_status_word))) != QX_OK) return s;
         int sms = 0;
-        if (cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return QX_ERR_CUDA;
+        if ((s = from_cuda(cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev))) != QX_OK) return s;
         d.status = static_cast<uint32_t *>(p);
         d.num_sms = sms;
         d.ready = true;
@@ -101,14 +112,6 @@ qx_status check_packed(const qx_packed *p) {
         if (!aligned(p->luts, 16)) return QX_ERR_ALIGNMENT;
     }
     return QX_OK;
-}
-
-thread_local const char *t_last_error = "no error";
-
-qx_status from_cuda(cudaError_t e) {
-    if (e == cudaSuccess) return QX_OK;
-    t_last_error = cudaGetErrorName(e);
-    return QX_ERR_CUDA;
 }
 
 }  // namespace
@@ -751,15 +754,24 @@ QX_API qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void
     return qx_q4x_gemv_multi(p, 1, &x, batch, &y, y_dtype, stream);
 }
 
+QX_API qx_status qx_selftest_wait_timeout(int32_t limit_us, void *stream) {
+    if (limit_us < 1 || limit_us > 1000000) return QX_ERR_INVALID_ARG;
+    DeviceInfo *d = nullptr;
+    const qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    return from_cuda(qx::launch_wait_selftest((uint64_t)limit_us * 1000ull, d->status,
+                                              static_cast<cudaStream_t>(stream)));
+}
+
 QX_API qx_status qx_get_device_status(void *stream) {
     DeviceInfo *d = nullptr;
     qx_status s = device_info(&d);
     if (s != QX_OK) return s;
-    if (cudaStreamSynchronize(static_cast<cudaStream_t>(stream)) != cudaSuccess) return QX_ERR_CUDA;
+    if ((s = from_cuda(cudaStreamSynchronize(static_cast<cudaStream_t>(stream)))) != QX_OK) return s;
     uint32_t v = 0;
-    if (cudaMemcpy(&v, d->status, sizeof(v), cudaMemcpyDeviceToHost) != cudaSuccess) return QX_ERR_CUDA;
+    if ((s = from_cuda(cudaMemcpy(&v, d->status, sizeof(v), cudaMemcpyDeviceToHost))) != QX_OK) return s;
     const uint32_t zero = 0;
-    if (cudaMemcpy(d->status, &zero, sizeof(zero), cudaMemcpyHostToDevice) != cudaSuccess) return QX_ERR_CUDA;
+    if ((s = from_cuda(cudaMemcpy(d->status, &zero, sizeof(zero), cudaMemcpyHostToDevice))) != QX_OK) return s;
     if (v & qx::kStatusNonfinite) return QX_ERR_NONFINITE;
     if (v & qx::kStatusTimeout) return QX_ERR_TIMEOUT;
     return QX_OK;

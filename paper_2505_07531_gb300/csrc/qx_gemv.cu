@@ -906,6 +906,30 @@ cudaError_t launch_nb(const GemvMulti &a, cudaStream_t st, bool pdl) {
     }
 }
 
+namespace {
+
+// Failure-detection self-test: one thread waits, with the bounded mbarrier
+// wait of the decode and prefill rings, for a phase that nothing completes
+// (a barrier expecting one arrival that never comes).  The wait gives up after
+// limit_ns; the kernel records the timeout in the device status word and
+// returns, leaving the context usable.
+__global__ void __launch_bounds__(32) wait_selftest_kernel(uint64_t limit_ns, uint32_t *status) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !mbar_wait(smem_u32(&bar), 0, limit_ns, nullptr)) atomicOr(status, kStatusTimeout);
+}
+
+}  // namespace
+
+cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t *status, cudaStream_t st) {
+    wait_selftest_kernel<<<1, 32, 0, st>>>(limit_ns, status);
+    return cudaGetLastError();
+}
+
 cudaError_t launch_gemv_multi(GemvMulti &a, cudaStream_t st, bool pdl) {
     a.initial = pdl ? a.ring : kGroups;
     if (a.bits == 4) return launch_nb<4, 0>(a, st, pdl);

@@ -202,6 +202,10 @@ cudaError_t launch_q4x_quantize(const Q4xQuantArgs &a, int num_sms, cudaStream_t
 cudaError_t launch_q4x_dequant(const Q4xMat &m, __half *W, int num_sms, cudaStream_t st);
 cudaError_t launch_q4x_gemv(const Q4xGemvMulti &a, int num_sms, cudaStream_t st);
 
+// One CTA whose bounded mbarrier wait runs out (nothing arrives): records
+// kStatusTimeout in *status after limit_ns and returns.
+cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t *status, cudaStream_t st);
+
 cudaError_t launch_quantize(const QuantArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_dequant(const DequantArgs &a, int num_sms, cudaStream_t st);
 bool plan_gemv(GemvMulti &a, int num_sms);

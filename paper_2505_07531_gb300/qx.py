@@ -106,6 +106,7 @@ def _lib():
         lib.qx_q4x_dequant.argtypes = [P(_Q4x), VP, VP]
         lib.qx_q4x_gemv.argtypes = [P(_Q4x), VP, I32, VP, I32, VP]
         lib.qx_q4x_gemv_multi.argtypes = [P(_Q4x), I32, P(VP), I32, P(VP), I32, VP]
+        lib.qx_selftest_wait_timeout.argtypes = [I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
         lib.qx_status_string.restype = ctypes.c_char_p
@@ -115,7 +116,7 @@ def _lib():
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
-                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi",
+                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_selftest_wait_timeout",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
@@ -519,6 +520,13 @@ def q4x_gemv_multi(mats, xs, outs=None, out_dtype=torch.float16):
     _check(_lib().qx_q4x_gemv_multi(arr, cnt, xa, b, ya, F32 if dt == torch.float32 else F16,
                                     _stream(x2[0].device)), "qx_q4x_gemv_multi")
     return ys
+
+
+def selftest_wait_timeout(limit_us: int, device=None) -> None:
+    """Launch the failure-detection self-test (qx_selftest_wait_timeout): a
+    bounded wait that runs out; device_status() then returns 5 (QX_ERR_TIMEOUT)."""
+    dev = device if device is not None else torch.device("cuda", torch.cuda.current_device())
+    _check(_lib().qx_selftest_wait_timeout(int(limit_us), _stream(dev)), "qx_selftest_wait_timeout")
 
 
 def device_status(stream=None) -> int:

@@ -206,3 +206,26 @@ def test_q4x_gemv_multi_rejects_bad_arguments_before_launching(qx):
     assert lib.qx_q4x_gemv_multi(mats, 2, xs, 1, nul_y, 0, None) == 1
     odd = (qx._Q4x * 2)(mats[0], qx._Q4x(32, 200, A(0x50000), A(0x60000), A(0x70000), A(0x80000)))
     assert lib.qx_q4x_gemv_multi(odd, 2, xs, 1, ys, 0, None) == 2
+
+
+def test_cuda_errors_are_reported_with_their_name():
+    """With no visible device, an entry point that passes validation fails in
+    the CUDA runtime: QX_ERR_CUDA, and qx_last_error_string() names the error."""
+    import subprocess
+    import sys
+
+    code = (
+        "import ctypes, paper_2505_07531_gb300.qx as qx\n"
+        "lib = qx._lib(); A = ctypes.c_void_p\n"
+        "P = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), A(0x10000), A(0x20000), A(0x30000), None)\n"
+        "print(lib.qx_dequant(ctypes.byref(P), A(0x40000), None), lib.qx_last_error_string().decode())\n"
+        "print(lib.qx_get_device_status(None), lib.qx_last_error_string().decode())\n"
+        "print(lib.qx_selftest_wait_timeout(0, None), lib.qx_selftest_wait_timeout(2000000, None))\n")
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=ROOT, env=env, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    lines = r.stdout.split("\n")
+    for line in lines[:2]:
+        status, name = line.split(" ", 1)
+        assert status == "4" and name.startswith("cuda") and name != "cudaSuccess", line
+    assert lines[2] == "1 1"  # limit outside 1 us .. 1 s
