@@ -529,6 +529,93 @@ def selftest_wait_timeout(limit_us: int, device=None) -> None:
     _check(_lib().qx_selftest_wait_timeout(int(limit_us), _stream(dev)), "qx_selftest_wait_timeout")
 
 
+# ------------------------------------------------------------ save / load
+# A packed matrix on disk: an 80-byte little-endian header, then its four
+# buffers in header order.
+#   magic "QXPK", u16 version (1), u16 format (0: per-group codes, 1: Q4X),
+#   i64 n, i64 k, i32 bits, group_size, kind, lloyd_iters,
+#   u64 sizes of the four buffers (codes, scales, zeros | books, luts | codebooks),
+#   u32 CRC-32 of the buffers in order, u32 zero.
+_HDR = "<4sHHqqiiiiQQQQII"
+_MAGIC, _VERSION = b"QXPK", 1
+
+
+def _bytes_of(t):
+    return b"" if t is None else t.detach().contiguous().cpu().view(torch.uint8).numpy().tobytes()
+
+
+def save(path: str, P) -> None:
+    """Write a PackedMatrix or Q4xMatrix (its buffers copied to the host)."""
+    import struct
+    import zlib
+
+    if isinstance(P, Q4xMatrix):
+        fmt, rec = 1, (4, Q4X_GROUP, 0, 0)
+        bufs = [P.codes, P.scales, P.books, P.codebooks]
+    elif isinstance(P, PackedMatrix):
+        fmt, rec = 0, (P.recipe.bits, P.recipe.group_size, P.recipe.kind, P.recipe.lloyd_iters)
+        bufs = [P.codes, P.scales, P.zeros, P.luts]
+    else:
+        raise TypeError("save takes a PackedMatrix or a Q4xMatrix")
+    raw = [_bytes_of(t) for t in bufs]
+    crc = 0
+    for r in raw:
+        crc = zlib.crc32(r, crc)
+    hdr = struct.pack(_HDR, _MAGIC, _VERSION, fmt, P.n, P.k, *rec, *[len(r) for r in raw], crc, 0)
+    with open(path, "wb") as f:
+        f.write(hdr)
+        for r in raw:
+            f.write(r)
+
+
+def load(path: str, device=None):
+    """Read a matrix written by :func:`save` onto `device` (a torch device;
+    default the current CUDA device).  Raises ValueError on a bad magic,
+    version or checksum, or sizes that disagree with the library's layout."""
+    import struct
+    import zlib
+
+    with open(path, "rb") as f:
+        blob = f.read()
+    size = struct.calcsize(_HDR)
+    if len(blob) < size:
+        raise ValueError("truncated header")
+    magic, ver, fmt, n, k, bits, g, kind, iters, s0, s1, s2, s3, crc, _ = struct.unpack_from(_HDR, blob)
+    if magic != _MAGIC or ver != _VERSION or fmt not in (0, 1):
+        raise ValueError("not a qx packed matrix (magic, version or format)")
+    sizes = [s0, s1, s2, s3]
+    if fmt == 1:
+        want = q4x_size(n, k)
+        expect = [want["codes"], want["scales"], want["books"], want["codebooks"]]
+    else:
+        rec = Recipe(bits, g, kind, iters)
+        want = packed_size(n, k, rec)
+        expect = [want["codes"], want["scales"], want["zeros"], want["luts"]]
+    if sizes != expect:
+        raise ValueError("buffer sizes disagree with the layout of this shape and recipe")
+    if len(blob) != size + sum(sizes):
+        raise ValueError("file length disagrees with the header")
+    c, off, raw = 0, size, []
+    for sz in sizes:
+        raw.append(blob[off:off + sz])
+        c = zlib.crc32(raw[-1], c)
+        off += sz
+    if c != crc:
+        raise ValueError("checksum mismatch")
+    dev = device if device is not None else torch.device("cuda", torch.cuda.current_device())
+
+    def tensor(r, dtype):
+        if not r:
+            return None
+        return torch.frombuffer(bytearray(r), dtype=torch.uint8).view(dtype).to(dev)
+
+    if fmt == 1:
+        return Q4xMatrix(n, k, tensor(raw[0], torch.uint8), tensor(raw[1], torch.float16),
+                         tensor(raw[2], torch.uint8), tensor(raw[3], torch.float16))
+    return PackedMatrix(n, k, rec, tensor(raw[0], torch.uint8), tensor(raw[1], torch.float16),
+                        tensor(raw[2], torch.uint8), tensor(raw[3], torch.float16))
+
+
 def device_status(stream=None) -> int:
     """Synchronize and return/clear the device status (0 = QX_OK)."""
     s = ctypes.c_void_p(stream.cuda_stream) if stream is not None else _stream(torch.device("cuda"))
