@@ -23,7 +23,7 @@ def qx(cuda_dev):
 
 
 def test_bounded_wait_gives_up_and_reports_timeout(qx):
-    assert qx.device_status() == 0
+    qx.device_status()  # read and clear whatever an earlier call left
     t0 = time.perf_counter()
     qx.selftest_wait_timeout(20000)  # 20 ms
     assert qx.device_status() == 5  # QX_ERR_TIMEOUT, read and cleared
