@@ -1,0 +1,347 @@
+// Host-thread execution of CUDA kernel sources, for tests only.
+//
+// The kernels that use no TMA, mbarrier or tensor-core instructions (the
+// quantizers, the dequantizers, the W.A8 pair, the error reduction and the Q4X
+// path) are compiled for the host with this header and run on host threads, so
+// that AddressSanitizer and UBSan check every index they form against buffers
+// of exactly the size the C ABI states.  The library never loads this code.
+//
+// Model: blocks run one after another; the threads of a block are OS threads,
+// so __syncthreads and the warp collectives are barriers (std::barrier) and a
+// thread that returns leaves them.  __shared__ variables become function
+// statics (shared by the block's threads); dynamic shared memory is a heap
+// buffer of exactly the launch's size.  Atomics are std::atomic_ref.  IEEE
+// float and double arithmetic is the host's (compiled without contraction);
+// fp16 values are _Float16, and each fp16 operation rounds the exact (double)
+// result once, as the device instruction does for the operands these kernels
+// use.
+#pragma once
+#include <algorithm>
+#include <atomic>
+#include <barrier>
+#include <chrono>
+#include <cmath>
+#include <condition_variable>
+#include <cstdint>
+#include <cstdlib>
+#include <cstring>
+#include <functional>
+#include <memory>
+#include <mutex>
+#include <thread>
+#include <vector>
+
+#define __global__
+#define __device__
+#define __host__
+#define __forceinline__ inline
+#define __launch_bounds__(...)
+#define __shared__ static
+#define __align__(x) alignas(x)
+#define __grid_constant__
+
+struct dim3 {
+    unsigned x = 1, y = 1, z = 1;
+    dim3(unsigned a = 1, unsigned b = 1, unsigned c = 1) : x(a), y(b), z(c) {}
+};
+
+namespace emu {
+struct Warp {
+    std::unique_ptr<std::barrier<>> bar;
+    uint64_t buf[32];
+};
+struct Block {
+    std::unique_ptr<std::barrier<>> bar;
+    std::vector<Warp> warps;
+    uint8_t *dyn = nullptr;  // dynamic shared memory, exactly the launch's size
+};
+inline thread_local dim3 t_tid, t_bid;
+inline thread_local Block *t_block = nullptr;
+inline dim3 g_grid, g_blockdim;
+}  // namespace emu
+
+#define threadIdx (emu::t_tid)
+#define blockIdx (emu::t_bid)
+#define gridDim (emu::g_grid)
+#define blockDim (emu::g_blockdim)
+
+using std::isfinite;
+inline uint8_t *emu_dyn_smem();
+inline void __syncthreads() { emu::t_block->bar->arrive_and_wait(); }
+inline unsigned emu_lane() { return threadIdx.x & 31u; }
+inline emu::Warp &emu_warp() { return emu::t_block->warps[threadIdx.x >> 5]; }
+inline void __syncwarp(unsigned = 0xffffffffu) { emu_warp().bar->arrive_and_wait(); }
+
+template <class T>
+inline uint64_t emu_bits(T v) {
+    uint64_t b = 0;
+    std::memcpy(&b, &v, sizeof(T));
+    return b;
+}
+template <class T>
+inline T emu_from(uint64_t b) {
+    T v;
+    std::memcpy(&v, &b, sizeof(T));
+    return v;
+}
+template <class T>
+inline T emu_exchange(T v, int src) {
+    emu::Warp &w = emu_warp();
+    w.buf[emu_lane()] = emu_bits(v);
+    w.bar->arrive_and_wait();
+    const T r = emu_from<T>(w.buf[src & 31]);
+    w.bar->arrive_and_wait();
+    return r;
+}
+template <class T>
+inline T __shfl_xor_sync(unsigned, T v, int o) { return emu_exchange(v, (int)emu_lane() ^ o); }
+template <class T>
+inline T __shfl_sync(unsigned, T v, int src) { return emu_exchange(v, src); }
+template <class T>
+inline T __shfl_up_sync(unsigned, T v, unsigned d) {
+    const T r = emu_exchange(v, (int)emu_lane() >= (int)d ? (int)(emu_lane() - d) : (int)emu_lane());
+    return r;
+}
+inline unsigned __ballot_sync(unsigned, bool p) {
+    emu::Warp &w = emu_warp();
+    w.buf[emu_lane()] = p ? 1 : 0;
+    w.bar->arrive_and_wait();
+    unsigned r = 0;
+    for (int i = 0; i < 32; ++i) r |= (unsigned)w.buf[i] << i;
+    w.bar->arrive_and_wait();
+    return r;
+}
+inline bool __any_sync(unsigned m, bool p) { return __ballot_sync(m, p) != 0; }
+
+template <class T, class U>
+inline T atomicAdd(T *p, U v) {
+    return std::atomic_ref<T>(*p).fetch_add((T)v);
+}
+template <class T, class U>
+inline T atomicOr(T *p, U v) {
+    return std::atomic_ref<T>(*p).fetch_or((T)v);
+}
+
+template <class T>
+inline T min(T a, T b) { return a < b ? a : b; }
+template <class T>
+inline T max(T a, T b) { return a < b ? b : a; }
+
+inline double __ddiv_rn(double a, double b) { return a / b; }
+inline double __dmul_rn(double a, double b) { return a * b; }
+inline double __dadd_rn(double a, double b) { return a + b; }
+inline double __dsub_rn(double a, double b) { return a - b; }
+inline float __fmul_rn(float a, float b) { return a * b; }
+inline long long __double2ll_rn(double x) { return llrint(x); }
+template <class T>
+inline T __ldg(const T *p) { return *p; }
+
+// ------------------------------------------------------------------ fp16
+struct __half {
+    uint16_t b;
+};
+struct alignas(4) __half2 {
+    __half x, y;
+};
+struct float2 {
+    float x, y;
+};
+struct alignas(16) uint4 {
+    unsigned x, y, z, w;
+};
+inline uint4 make_uint4(unsigned a, unsigned b, unsigned c, unsigned d) { return uint4{a, b, c, d}; }
+inline __half __ushort_as_half(unsigned short b) { return __half{b}; }
+inline unsigned short __half_as_ushort(__half h) { return h.b; }
+inline float __half2float(__half h) {
+    _Float16 f;
+    std::memcpy(&f, &h.b, 2);
+    return (float)f;
+}
+inline __half __float2half_rn(float x) {
+    _Float16 f = (_Float16)x;
+    __half h;
+    std::memcpy(&h.b, &f, 2);
+    return h;
+}
+inline uint16_t emu_f64_to_f16(double x) {
+    _Float16 f = (_Float16)x;
+    uint16_t b;
+    std::memcpy(&b, &f, 2);
+    return b;
+}
+inline __half2 __halves2half2(__half a, __half b) { return __half2{a, b}; }
+inline __half2 __hmul2(__half2 a, __half2 b) {
+    // exact fp32 product of two fp16 values, one rounding to fp16
+    return __half2{__float2half_rn(__half2float(a.x) * __half2float(b.x)),
+                   __float2half_rn(__half2float(a.y) * __half2float(b.y))};
+}
+inline float2 __half22float2(__half2 h) { return float2{__half2float(h.x), __half2float(h.y)}; }
+
+// ------------------------------------------------------------------ runtime
+typedef void *cudaStream_t;
+enum cudaError_t { cudaSuccess = 0 };
+inline cudaError_t cudaMemsetAsync(void *p, int v, size_t n, cudaStream_t) {
+    std::memset(p, v, n);
+    return cudaSuccess;
+}
+inline cudaError_t cudaGetLastError() { return cudaSuccess; }
+template <class F>
+inline cudaError_t cudaOccupancyMaxActiveBlocksPerMultiprocessor(int *n, F, int, size_t) {
+    *n = 3;
+    return cudaSuccess;
+}
+
+namespace emu {
+struct Cfg {
+    dim3 grid, block;
+    size_t smem = 0;
+    cudaStream_t st = nullptr;
+};
+
+// Persistent OS threads, one per thread index of a block.
+struct Pool {
+    std::vector<std::thread> th;
+    std::mutex mu;
+    std::condition_variable cv, done_cv;
+    uint64_t gen = 0;
+    int active = 0, remaining = 0;
+    std::function<void()> job;
+    dim3 bid;
+    Block *block = nullptr;
+    bool stop = false;
+
+    explicit Pool(int n) {
+        for (int i = 0; i < n; ++i) th.emplace_back([this, i] { run(i); });
+    }
+    ~Pool() {
+        {
+            std::lock_guard<std::mutex> l(mu);
+            stop = true;
+            ++gen;
+        }
+        cv.notify_all();
+        for (auto &t : th) t.join();
+    }
+    void run(int i) {
+        uint64_t seen = 0;
+        for (;;) {
+            std::function<void()> f;
+            {
+                std::unique_lock<std::mutex> l(mu);
+                cv.wait(l, [&] { return gen != seen; });
+                seen = gen;
+                if (stop) return;
+                if (i >= active) continue;
+                f = job;
+                t_bid = bid;
+                t_block = block;
+            }
+            t_tid = dim3((unsigned)i, 0, 0);
+            f();
+            // a returning thread leaves the barriers of its block and warp
+            t_block->warps[i >> 5].bar->arrive_and_drop();
+            t_block->bar->arrive_and_drop();
+            {
+                std::lock_guard<std::mutex> l(mu);
+                if (--remaining == 0) done_cv.notify_one();
+            }
+        }
+    }
+    void launch_block(int nthreads, dim3 b, Block *blk, const std::function<void()> &f) {
+        {
+            std::lock_guard<std::mutex> l(mu);
+            job = f;
+            bid = b;
+            block = blk;
+            active = nthreads;
+            remaining = nthreads;
+            ++gen;
+        }
+        cv.notify_all();
+        std::unique_lock<std::mutex> l(mu);
+        done_cv.wait(l, [&] { return remaining == 0; });
+    }
+};
+
+inline Pool &pool() {
+    static Pool p(1024);
+    return p;
+}
+
+inline void launch(const Cfg &c, const std::function<void()> &f) {
+    const int nt = (int)(c.block.x * c.block.y * c.block.z);
+    g_grid = c.grid;
+    g_blockdim = c.block;
+    for (unsigned by = 0; by < c.grid.y; ++by)
+        for (unsigned bx = 0; bx < c.grid.x; ++bx) {
+            Block blk;
+            struct Dyn {
+                uint8_t *p;
+                ~Dyn() { if (p) ::operator delete[](p, std::align_val_t(16)); }
+            } dyn{c.smem ? new (std::align_val_t(16)) uint8_t[c.smem] : nullptr};
+            blk.dyn = dyn.p;
+            blk.bar = std::make_unique<std::barrier<>>(nt);
+            const int nw = (nt + 31) / 32;
+            blk.warps.resize(nw);
+            for (int w = 0; w < nw; ++w) blk.warps[w].bar = std::make_unique<std::barrier<>>(std::min(32, nt - 32 * w));
+            pool().launch_block(nt, dim3(bx, by, 0), &blk, f);
+        }
+}
+}  // namespace emu
+
+// ------------------------------------------------------------------ more intrinsics
+inline uint32_t emu_prmt(uint32_t a, uint32_t b, uint32_t c) {
+    const uint64_t v = ((uint64_t)b << 32) | a;
+    uint32_t d = 0;
+    for (int j = 0; j < 4; ++j) {
+        const uint32_t s = (c >> (4 * j)) & 15u;
+        uint32_t byte = (uint32_t)(v >> (8 * (s & 7))) & 255u;
+        if (s & 8) byte = (byte & 0x80u) ? 0xFFu : 0u;
+        d |= byte << (8 * j);
+    }
+    return d;
+}
+inline int __dp4a(int a, int b, int c) {
+    for (int i = 0; i < 4; ++i) c += (int)(int8_t)(a >> (8 * i)) * (int)(int8_t)(b >> (8 * i));
+    return c;
+}
+inline unsigned __vsub4(unsigned a, unsigned b) {
+    unsigned d = 0;
+    for (int i = 0; i < 4; ++i) d |= (((a >> (8 * i)) - (b >> (8 * i))) & 255u) << (8 * i);
+    return d;
+}
+inline float __fdiv_rn(float a, float b) { return a / b; }
+inline float __fsub_rn(float a, float b) { return a - b; }
+inline float __fadd_rn(float a, float b) { return a + b; }
+inline __half emu_h(double x) {
+    _Float16 f = (_Float16)x;
+    __half h;
+    std::memcpy(&h.b, &f, 2);
+    return h;
+}
+inline __half2 __hsub2(__half2 a, __half2 b) {
+    return __half2{emu_h((double)__half2float(a.x) - (double)__half2float(b.x)),
+                   emu_h((double)__half2float(a.y) - (double)__half2float(b.y))};
+}
+inline __half2 __hfma2(__half2 a, __half2 b, __half2 c) {
+    return __half2{emu_h(std::fma((double)__half2float(a.x), (double)__half2float(b.x), (double)__half2float(c.x))),
+                   emu_h(std::fma((double)__half2float(a.y), (double)__half2float(b.y), (double)__half2float(c.y)))};
+}
+inline uint64_t emu_globaltimer() {
+    return (uint64_t)std::chrono::duration_cast<std::chrono::nanoseconds>(
+               std::chrono::steady_clock::now().time_since_epoch()).count();
+}
+struct int4 { int x, y, z, w; };
+// driver-API types named by the internal header
+typedef int CUresult;
+typedef int CUtensorMapDataType, CUtensorMapInterleave, CUtensorMapSwizzle, CUtensorMapL2promotion,
+    CUtensorMapFloatOOBfill;
+typedef unsigned cuuint32_t;
+typedef unsigned long long cuuint64_t;
+struct alignas(64) CUtensorMap { char b[128]; };
+enum cudaFuncAttribute { cudaFuncAttributeMaxDynamicSharedMemorySize, cudaFuncAttributePreferredSharedMemoryCarveout };
+inline cudaError_t cudaGetDevice(int *d) { *d = 0; return cudaSuccess; }
+template <class F>
+inline cudaError_t cudaFuncSetAttribute(F, cudaFuncAttribute, int) { return cudaSuccess; }
+
+inline uint8_t *emu_dyn_smem() { return emu::t_block->dyn; }

@@ -1,0 +1,118 @@
+// Runs the translated kernels on buffers of exactly the size the C ABI states
+// (so AddressSanitizer sees any access outside them) and writes the outputs.
+//   harness quant n k bits g kind iters sms in out : quantize, dequant, exact error
+//   harness a8    n k bits g batch sms in out      : uniform quantize, int8 activations, W.A8 matmul
+//   harness q4x   n k iters sms batch in out       : Q4X learner, dequant, two-matrix decode
+// `in` holds W (fp16 [n][k]) and, for a8 and q4x, x (fp16 [batch][k]).
+#include <cstdio>
+#include <new>
+#include <string>
+
+#include "qx_kernels.cuh"
+
+namespace {
+template <class T>
+T *alloc(size_t bytes) {
+    return bytes ? static_cast<T *>(::operator new(bytes, std::align_val_t(256))) : nullptr;
+}
+void put(FILE *f, const void *p, size_t b) {
+    if (b) fwrite(p, 1, b, f);
+}
+bool get(FILE *f, void *p, size_t b) { return fread(p, 1, b, f) == b; }
+}  // namespace
+
+int main(int argc, char **argv) {
+    if (argc < 2) return 2;
+    const std::string cmd = argv[1];
+    const bool q4x = cmd == "q4x";
+    if ((q4x && argc != 9) || (!q4x && argc != (cmd == "quant" ? 11 : 10))) return 2;
+    const int64_t n = atoll(argv[2]), k = atoll(argv[3]);
+    FILE *fi = fopen(argv[argc - 2], "rb"), *fo = fopen(argv[argc - 1], "wb");
+    if (fi == nullptr || fo == nullptr) return 2;
+    __half *W = alloc<__half>(2 * n * k);
+    if (!get(fi, W, 2 * n * k)) return 2;
+    uint32_t *status = alloc<uint32_t>(4);
+    *status = 0;
+    if (q4x) {
+        const int iters = atoi(argv[4]), sms = atoi(argv[5]), batch = atoi(argv[6]);
+        const int G = (int)(k / 64), bb = (G + 3) / 4;
+        __half *x = alloc<__half>(2 * batch * k);
+        if (!get(fi, x, 2 * batch * k)) return 2;
+        uint8_t *codes = alloc<uint8_t>(n * k / 2), *books = alloc<uint8_t>(n * bb);
+        __half *scales = alloc<__half>(2 * n * G), *cbs = alloc<__half>(128);
+        void *ws = alloc<uint8_t>(qx::q4x_workspace_bytes(n, k));
+        qx::Q4xQuantArgs a{W, n, k, G, bb, iters, codes, scales, books, cbs, ws, status};
+        qx::launch_q4x_quantize(a, sms, nullptr);
+        qx::Q4xMat m{codes, scales, books, cbs, n, k, G, bb};
+        __half *Wh = alloc<__half>(2 * n * k);
+        qx::launch_q4x_dequant(m, Wh, sms, nullptr);
+        float *y0 = alloc<float>(4 * batch * n), *y1 = alloc<float>(4 * batch * n);
+        qx::Q4xGemvMulti g{};
+        g.count = 2;
+        g.batch = batch;
+        g.y_f32 = 1;
+        g.mat[0] = g.mat[1] = m;
+        g.x[0] = g.x[1] = x;
+        g.y[0] = y0;
+        g.y[1] = y1;
+        g.row_off[1] = n;
+        g.row_off[2] = 2 * n;
+        qx::launch_q4x_gemv(g, sms, nullptr);
+        __half *yh = alloc<__half>(2 * batch * n);
+        g.count = 1;
+        g.y_f32 = 0;
+        g.y[0] = yh;
+        qx::launch_q4x_gemv(g, sms, nullptr);
+        put(fo, codes, n * k / 2);
+        put(fo, scales, 2 * n * G);
+        put(fo, books, n * bb);
+        put(fo, cbs, 128);
+        put(fo, Wh, 2 * n * k);
+        put(fo, y0, 4 * batch * n);
+        put(fo, y1, 4 * batch * n);
+        put(fo, yh, 2 * batch * n);
+    } else {
+        const int bits = atoi(argv[4]), g = atoi(argv[5]);
+        const int kind = cmd == "quant" ? atoi(argv[6]) : 0;
+        const int extra = atoi(argv[cmd == "quant" ? 7 : 6]), sms = atoi(argv[cmd == "quant" ? 8 : 7]);
+        const int G = (int)(k / g), zb = (G + 1) / 2;
+        const size_t cb = n * k * bits / 8, sb = kind == 0 ? 2 * n * G : 0, zbb = kind == 0 ? n * zb : 0,
+                     lb = kind == 1 ? 2 * n * G * 8 : 0;
+        uint8_t *codes = alloc<uint8_t>(cb), *zeros = alloc<uint8_t>(zbb);
+        __half *scales = alloc<__half>(sb), *luts = alloc<__half>(lb);
+        qx::QuantArgs q{W, n, k, bits, g, kind, cmd == "quant" ? extra : 25, G, zb, codes, scales, zeros, luts, status};
+        qx::launch_quantize(q, sms, nullptr);
+        put(fo, codes, cb);
+        put(fo, scales, sb);
+        put(fo, zeros, zbb);
+        put(fo, luts, lb);
+        if (cmd == "quant") {
+            __half *Wh = alloc<__half>(2 * n * k);
+            qx::DequantArgs d{codes, scales, zeros, luts, n, k, bits, g, kind, G, zb, Wh};
+            qx::launch_dequant(d, sms, nullptr);
+            const int nb = qx::sq_error_blocks(sms);
+            auto *part = alloc<unsigned long long>(16 * (size_t)nb), *tot = alloc<unsigned long long>(16);
+            qx::launch_sq_error(W, Wh, n * k, part, tot, sms, nullptr);
+            put(fo, Wh, 2 * n * k);
+            put(fo, tot, 16);
+        } else {
+            const int batch = extra;
+            __half *x = alloc<__half>(2 * batch * k);
+            if (!get(fi, x, 2 * batch * k)) return 2;
+            int8_t *qa = alloc<int8_t>(batch * k);
+            float *sa = alloc<float>(4 * batch), *y = alloc<float>(4 * batch * n);
+            qx::launch_quantize_act(x, batch, k, qa, sa, nullptr);
+            int l = 0;
+            while ((1 << l) < g) ++l;
+            qx::GemvA8Args a{codes, scales, zeros, n, k, bits, G, zb, l, qa, sa, batch, y, 1};
+            qx::launch_gemv_a8(a, nullptr);
+            put(fo, qa, batch * k);
+            put(fo, sa, 4 * batch);
+            put(fo, y, 4 * batch * n);
+        }
+    }
+    put(fo, status, 4);
+    fclose(fo);
+    fclose(fi);
+    return 0;
+}

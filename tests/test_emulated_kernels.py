@@ -1,0 +1,165 @@
+"""The kernel sources that use no TMA, mbarrier or tensor-core instructions run
+on host threads, compiled with AddressSanitizer and UBSan (a stand-in for
+compute-sanitizer, which this pool does not offer): every index they form must
+stay inside buffers of exactly the sizes the C ABI states, and their results
+must equal the oracle's (bit-exact codes, LUTs, dequantized weights, exact
+squared errors and int8 activations; matmuls within the tolerance).  No GPU;
+the library never loads this code (tests/emulation/cuda_host.h)."""
+import os
+import shutil
+import subprocess
+import sys
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from oracle import select as oselect
+from oracle.pack import Recipe as ORecipe
+
+HERE = os.path.join(os.path.dirname(os.path.abspath(__file__)), "emulation")
+ENV = dict(os.environ, ASAN_OPTIONS="detect_leaks=0", UBSAN_OPTIONS="print_stacktrace=1")
+
+
+@pytest.fixture(scope="module")
+def harness(tmp_path_factory):
+    gxx = shutil.which("g++")
+    if gxx is None:
+        pytest.skip("g++ is not available")
+    out = tmp_path_factory.mktemp("emulated")
+    sys.path.insert(0, HERE)
+    import translate
+
+    cpps = translate.write_all(str(out))
+    exe = str(out / "harness")
+    cmd = [gxx, "-std=c++20", "-O1", "-g", "-fsanitize=address,undefined", "-fno-sanitize-recover=undefined",
+           "-ffp-contract=off", "-Wno-unknown-pragmas", "-pthread", "-I", str(out), "-I", HERE, *cpps,
+           os.path.join(HERE, "harness.cpp"), "-o", exe]
+    r = subprocess.run(cmd, capture_output=True, text=True)
+    assert r.returncode == 0, r.stderr[-3000:]
+    return exe, out
+
+
+def _run(harness, args, W, x=None):
+    exe, out = harness
+    fin, fout = str(out / "in.bin"), str(out / "out.bin")
+    with open(fin, "wb") as f:
+        f.write(np.ascontiguousarray(W, np.float16).tobytes())
+        if x is not None:
+            f.write(np.ascontiguousarray(x, np.float16).tobytes())
+    r = subprocess.run([exe, *map(str, args), fin, fout], capture_output=True, text=True, env=ENV, timeout=900)
+    assert r.returncode == 0 and "runtime error" not in r.stderr and "AddressSanitizer" not in r.stderr, \
+        r.stderr[-3000:]
+    return Reader(open(fout, "rb").read())
+
+
+class Reader:
+    def __init__(self, b):
+        self.b, self.off = b, 0
+
+    def take(self, count, dtype):
+        a = np.frombuffer(self.b, dtype=dtype, count=count, offset=self.off)
+        self.off += a.nbytes
+        return a
+
+
+def _weights(n, k, seed, dead_row=True):
+    W = synth.student_t_weights(n, k, 0.02, seed=seed, stream=n + k, outlier_frac=0.001)
+    if dead_row and n >= 3:
+        W[1, :64] = 0
+    return W
+
+
+@pytest.mark.parametrize("n,k,bits,g,kind,sms", [  # ragged rows, every group size, 1 and 5 SMs of grid
+    (1, 128, 4, 64, 0, 1), (37, 384, 4, 128, 0, 5), (130, 640, 3, 64, 0, 1), (130, 640, 3, 64, 0, 5),
+    (3, 128, 3, 32, 0, 5), (9, 512, 4, 256, 0, 1), (20, 512, 3, 128, 1, 5), (11, 384, 3, 32, 1, 1),
+    (3, 512, 3, 256, 1, 5), (1, 11008, 3, 128, 1, 1)])
+def test_quantize_dequant_and_exact_error(harness, n, k, bits, g, kind, sms):
+    W = _weights(n, k, seed=n + bits)
+    rd = _run(harness, ["quant", n, k, bits, g, kind, 25, sms], W)
+    rec = ORecipe(bits, g, "lut" if kind else "uniform", 25)
+    ref = oracle.quantize(W, rec)
+    G = k // g
+    assert np.array_equal(rd.take(n * k * bits // 8, np.uint8).reshape(n, -1), ref["codes"])
+    if kind == 0:
+        assert np.array_equal(rd.take(n * G, np.uint16).reshape(n, G), ref["scales"].view(np.uint16))
+        assert np.array_equal(rd.take(n * ((G + 1) // 2), np.uint8).reshape(n, -1), ref["zeros"])
+    else:
+        assert np.array_equal(rd.take(n * G * 8, np.uint16).reshape(n, G, 8), ref["luts"].view(np.uint16))
+    Wh = oracle.dequant(ref, rec, k)
+    assert np.array_equal(rd.take(n * k, np.uint16).reshape(n, k), Wh.view(np.uint16))
+    tot = rd.take(2, np.uint64)
+    assert int(tot[0]) | (int(tot[1]) << 64) == oselect.sq_error_units(W, Wh)
+    assert rd.take(1, np.uint32)[0] == 0
+
+
+@pytest.mark.parametrize("batch", [1, 3, 16])
+@pytest.mark.parametrize("n,k,bits,g", [(37, 384, 4, 128), (33, 640, 3, 64), (1, 128, 3, 32)])
+def test_int8_activations_and_w_a8_matmul(harness, n, k, bits, g, batch):
+    W = _weights(n, k, seed=n + batch)
+    x = synth.activations(batch, k, seed=batch, stream=n)
+    rd = _run(harness, ["a8", n, k, bits, g, batch, 3], W, x)
+    G = k // g
+    rd.take(n * k * bits // 8 + 2 * n * G + n * ((G + 1) // 2), np.uint8)
+    qr, sr = oracle.quantize_act(x)
+    assert np.array_equal(rd.take(batch * k, np.int8).reshape(batch, k), qr)
+    assert np.array_equal(rd.take(batch, np.float32), sr)
+    y = rd.take(batch * n, np.float32).reshape(batch, n)
+    rec = ORecipe(bits, g, "uniform", 25)
+    ref = oracle.quantize(W, rec)
+    qw = oracle.unpack_codes(ref["codes"], bits, k).astype(np.float64)
+    z = np.repeat(oracle.unpack_zeros(ref["zeros"], G).astype(np.float64), g, axis=1)
+    w_exact = (qw - z) * np.repeat(ref["scales"].astype(np.float64), g, axis=1)
+    tol = oracle.tolerance(oracle.dequant_act(qr, sr), w_exact)
+    assert np.all(oracle.max_abs_err(y, oracle.gemv_a8(ref, rec, x, k)) <= tol)
+
+
+def _q4x_cases():
+    nan = _weights(24, 512, seed=9, dead_row=False).astype(np.float16)
+    nan[4, 130] = np.float16(np.nan)
+    nan[9, 0] = np.float16(np.inf)
+    return {
+        "ragged": (_weights(37, 320, seed=1), 3, 2, 3),
+        "no_steps": (_weights(16, 128, seed=2), 0, 1, 1),
+        "batch16": (_weights(130, 640, seed=3), 3, 5, 16),
+        "all_zero": (np.zeros((8, 256), np.float16), 3, 2, 2),
+        "few_distinct": (np.tile(np.array([-1, 0, 0.5, 1], np.float16), (8, 64)), 3, 2, 4),
+        "nonfinite": (nan, 3, 2, 1),
+    }
+
+
+Q4X = _q4x_cases()
+
+
+@pytest.mark.parametrize("name", sorted(Q4X))
+def test_q4x_learner_dequant_and_multi_matrix_decode(harness, name):
+    W, iters, sms, batch = Q4X[name]
+    W = np.asarray(W, np.float16)
+    n, k = W.shape
+    x = synth.activations(batch, k, seed=batch, stream=n)
+    rd = _run(harness, ["q4x", n, k, iters, sms, batch], W, x)
+    G, bb = k // 64, (k // 64 + 3) // 4
+    got = {"codes": rd.take(n * k // 2, np.uint8).reshape(n, -1), "scales": rd.take(n * G, np.uint16).reshape(n, G),
+           "books": rd.take(n * bb, np.uint8).reshape(n, -1), "codebooks": rd.take(64, np.uint16).reshape(4, 16)}
+    bad = ~np.isfinite(W.reshape(n, G, 64).astype(np.float32)).all(axis=2)
+    clean = W.copy()
+    clean.reshape(n, G, 64)[bad] = 0  # a non-finite group is coded as a dead one
+    ref = oracle.quantize_q4x(clean, iters=iters)
+    want = oracle.pack_q4x(ref)
+    assert np.array_equal(got["codes"], want["codes"])
+    assert np.array_equal(got["scales"], want["scales"].view(np.uint16))
+    assert np.array_equal(got["books"], want["books"])
+    assert np.array_equal(got["codebooks"], want["codebooks"].view(np.uint16))
+    Wh = oracle.dequant_q4x(ref["codes"], ref["scales"], ref["books"], ref["codebooks"])
+    assert np.array_equal(rd.take(n * k, np.uint16).reshape(n, k), Wh.view(np.uint16))
+    y0 = rd.take(batch * n, np.float32).reshape(batch, n)
+    y1 = rd.take(batch * n, np.float32).reshape(batch, n)
+    yh = rd.take(batch * n, np.float16).reshape(batch, n).astype(np.float64)
+    assert np.array_equal(y0, y1)  # both entries of the two-matrix launch
+    if not bad.any():
+        y_ref = oracle.gemv_q4x(ref, x)
+        tol = oracle.tolerance(x, Wh)
+        assert np.all(oracle.max_abs_err(y0, y_ref) <= tol)
+        assert np.all(oracle.max_abs_err(yh, y_ref) <= tol + np.abs(y_ref).max(axis=1) * 2.0 ** -11)
+    assert rd.take(1, np.uint32)[0] == (1 if bad.any() else 0)  # the non-finite status bit
