@@ -1,6 +1,6 @@
 """The kernel sources that use no TMA, mbarrier or tensor-core instructions run
 on host threads, compiled with AddressSanitizer and UBSan (a stand-in for
-compute-sanitizer, which this pool does not offer): every index they form must
+compute-sanitizer): every index they form must
 stay inside buffers of exactly the sizes the C ABI states, and their results
 must equal the oracle's (bit-exact codes, LUTs, dequantized weights, exact
 squared errors and int8 activations; matmuls within the tolerance).  No GPU;
