@@ -307,7 +307,9 @@ qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream);
 
 /* Decode matmul y = x W_hat^T for a Q4X matrix: x device fp16 [batch][k],
  * 16-byte aligned; y device [batch][n] of y_dtype, 4-byte aligned; batch
- * 1..16.  w_hat exactly as above, products and sums in fp32. */
+ * 1..16.  w_hat exactly as above; the products with x and their sums over 16
+ * consecutive weight pairs are formed in fp16 (so they must stay within its
+ * range, |.| < 65504), then summed in fp32. */
 qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream);
 
 /* Several Q4X decode matmuls in one launch: y[i] = x[i] W_hat_i^T, i < count

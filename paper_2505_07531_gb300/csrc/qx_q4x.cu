@@ -656,40 +656,38 @@ constexpr int kGemvWarps = 8;  // warps per block
 
 // w_hat of one 32-weight unit (16 code bytes): half2 pairs (k = 2i, 2i + 1),
 // the codebook entries times s in fp16, which is exactly fp16(fp32(s) fp32(CB)).
-__device__ __forceinline__ void unit_weights(const uint4 &cw, const __half *tb, __half2 s2, float2 (&wf)[16]) {
+__device__ __forceinline__ void unit_weights(const uint4 &cw, const __half *tb, __half2 s2, __half2 (&w)[16]) {
     const uint32_t ws[4] = {cw.x, cw.y, cw.z, cw.w};
 #pragma unroll
     for (int t = 0; t < 4; ++t) {
 #pragma unroll
         for (int i = 0; i < 4; ++i) {
             const uint32_t sel = (ws[t] >> (4 * i)) & 0x000F000Fu;  // codes of k = 8t+2i, 8t+2i+1
-            const __half2 e = __halves2half2(tb[sel & 15u], tb[sel >> 16]);
-            wf[4 * t + i] = __half22float2(__hmul2(e, s2));
+            w[4 * t + i] = __hmul2(__halves2half2(tb[sel & 15u], tb[sel >> 16]), s2);
         }
     }
 }
 
-// acc[b] += the unit's 32 products with x[b][32u .. 32u+31], in fp32.
+// acc[b] += the unit's 32 products with x[b][32u .. 32u+31]: the products and
+// their sums over 16 pairs in fp16 (two chains of eight HFMA2), then fp32.
 template <int NB>
-__device__ __forceinline__ void unit_dot(const float2 (&wf)[16], const __half *x, int64_t k, int u, int batch,
+__device__ __forceinline__ void unit_dot(const __half2 (&w)[16], const __half *x, int64_t k, int u, int batch,
                                          float (&acc)[NB]) {
 #pragma unroll
     for (int b = 0; b < NB; ++b) {
         if (b >= batch) break;
         const uint4 *xr = reinterpret_cast<const uint4 *>(x + (int64_t)b * k + 32 * (int64_t)u);
-        float a = acc[b];
+        __half2 c0 = u2h2(0u), c1 = u2h2(0u);
 #pragma unroll
         for (int v = 0; v < 4; ++v) {
             const uint4 xv = __ldg(xr + v);
-            const uint32_t xs[4] = {xv.x, xv.y, xv.z, xv.w};
-#pragma unroll
-            for (int p = 0; p < 4; ++p) {
-                const float2 xf = __half22float2(u2h2(xs[p]));
-                a = fmaf(wf[4 * v + p].x, xf.x, a);
-                a = fmaf(wf[4 * v + p].y, xf.y, a);
-            }
+            c0 = __hfma2(w[4 * v + 0], u2h2(xv.x), c0);
+            c1 = __hfma2(w[4 * v + 1], u2h2(xv.y), c1);
+            c0 = __hfma2(w[4 * v + 2], u2h2(xv.z), c0);
+            c1 = __hfma2(w[4 * v + 3], u2h2(xv.w), c1);
         }
-        acc[b] = a;
+        const float2 f0 = __half22float2(c0), f1 = __half22float2(c1);
+        acc[b] += (f0.x + f0.y) + (f1.x + f1.y);
     }
 }
 
@@ -730,12 +728,12 @@ __global__ void __launch_bounds__(32 * kGemvWarps) q4x_gemv_kernel(const __grid_
             const uint4 c1 = two ? __ldg(crow + u1) : make_uint4(0u, 0u, 0u, 0u);
             const __half s0 = srow[u0 >> 1], s1 = srow[(two ? u1 : u0) >> 1];
             const uint32_t b0 = book_index(brow, u0 >> 1), b1 = book_index(brow, (two ? u1 : u0) >> 1);
-            float2 wf[16];
-            unit_weights(c0, cbm + kLevels * b0, __halves2half2(s0, s0), wf);
-            unit_dot<NB>(wf, x, m.k, u0, a.batch, acc);
+            __half2 w[16];
+            unit_weights(c0, cbm + kLevels * b0, __halves2half2(s0, s0), w);
+            unit_dot<NB>(w, x, m.k, u0, a.batch, acc);
             if (two) {
-                unit_weights(c1, cbm + kLevels * b1, __halves2half2(s1, s1), wf);
-                unit_dot<NB>(wf, x, m.k, u1, a.batch, acc);
+                unit_weights(c1, cbm + kLevels * b1, __halves2half2(s1, s1), w);
+                unit_dot<NB>(w, x, m.k, u1, a.batch, acc);
             }
         }
 #pragma unroll
