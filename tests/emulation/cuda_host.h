@@ -29,6 +29,8 @@
 #include <memory>
 #include <mutex>
 #include <thread>
+#include <unordered_map>
+#include <cstdio>
 #include <vector>
 
 #define __global__
@@ -37,7 +39,7 @@
 #define __forceinline__ inline
 #define __launch_bounds__(...)
 #define __shared__ static
-#define __align__(x) alignas(x)
+#define __align__(x) __attribute__((aligned(x)))
 #define __grid_constant__
 
 struct dim3 {
@@ -50,20 +52,28 @@ struct Warp {
     std::unique_ptr<std::barrier<>> bar;
     uint64_t buf[32];
 };
+struct MBar {  // an mbarrier: arrivals still expected, transaction bytes, phase
+    uint32_t count = 0, pending = 0, phase = 0;
+    int64_t tx = 0;
+};
 struct Block {
     std::unique_ptr<std::barrier<>> bar;
     std::vector<Warp> warps;
     uint8_t *dyn = nullptr;  // dynamic shared memory, exactly the launch's size
+    size_t dyn_bytes = 0;
+    std::mutex mbar_mu;
+    std::unordered_map<uint32_t, MBar> mbars;  // by shared-memory address
 };
 inline thread_local dim3 t_tid, t_bid;
 inline thread_local Block *t_block = nullptr;
 inline dim3 g_grid, g_blockdim;
 }  // namespace emu
 
-#define threadIdx (emu::t_tid)
-#define blockIdx (emu::t_bid)
-#define gridDim (emu::g_grid)
-#define blockDim (emu::g_blockdim)
+// the built-in indices, as variables (the grid's for the running launch)
+inline thread_local dim3 &threadIdx = emu::t_tid;
+inline thread_local dim3 &blockIdx = emu::t_bid;
+inline dim3 &gridDim = emu::g_grid;
+inline dim3 &blockDim = emu::g_blockdim;
 
 using std::isfinite;
 inline uint8_t *emu_dyn_smem();
@@ -112,6 +122,7 @@ inline unsigned __ballot_sync(unsigned, bool p) {
     return r;
 }
 inline bool __any_sync(unsigned m, bool p) { return __ballot_sync(m, p) != 0; }
+inline bool __all_sync(unsigned m, bool p) { return __ballot_sync(m, p) == 0xffffffffu; }
 
 template <class T, class U>
 inline T atomicAdd(T *p, U v) {
@@ -280,6 +291,7 @@ inline void launch(const Cfg &c, const std::function<void()> &f) {
                 ~Dyn() { if (p) ::operator delete[](p, std::align_val_t(16)); }
             } dyn{c.smem ? new (std::align_val_t(16)) uint8_t[c.smem] : nullptr};
             blk.dyn = dyn.p;
+            blk.dyn_bytes = c.smem;
             blk.bar = std::make_unique<std::barrier<>>(nt);
             const int nw = (nt + 31) / 32;
             blk.warps.resize(nw);
@@ -345,3 +357,183 @@ template <class F>
 inline cudaError_t cudaFuncSetAttribute(F, cudaFuncAttribute, int) { return cudaSuccess; }
 
 inline uint8_t *emu_dyn_smem() { return emu::t_block->dyn; }
+
+// ------------------------------------------------------------------ TMA, mbarrier, launch
+#define __noinline__ __attribute__((noinline))
+
+[[noreturn]] inline void emu_fail(const char *what) {
+    std::fprintf(stderr, "emulation check failed: %s\n", what);
+    std::abort();
+}
+inline void __threadfence_block() { std::atomic_thread_fence(std::memory_order_seq_cst); }
+inline void __threadfence() { std::atomic_thread_fence(std::memory_order_seq_cst); }
+template <class T, class U>
+inline T atomicMax(T *p, U v) {
+    std::atomic_ref<T> r(*p);
+    T o = r.load();
+    while (o < (T)v && !r.compare_exchange_weak(o, (T)v)) {
+    }
+    return o;
+}
+
+// The shared state space is the block's dynamic shared memory: a shared
+// address is an offset into it, checked on every use.
+inline uint32_t __cvta_generic_to_shared(const void *p) {
+    const emu::Block *b = emu::t_block;
+    const ptrdiff_t o = static_cast<const uint8_t *>(p) - b->dyn;
+    if (b->dyn == nullptr || o < 0 || (size_t)o >= b->dyn_bytes) emu_fail("generic address outside shared memory");
+    return (uint32_t)o;
+}
+inline uint8_t *emu_shared(uint32_t a, size_t bytes) {
+    const emu::Block *b = emu::t_block;
+    if ((size_t)a + bytes > b->dyn_bytes) emu_fail("shared-memory access out of range");
+    return b->dyn + a;
+}
+inline uint4 emu_lds128(uint32_t a) {
+    if (a & 15u) emu_fail("misaligned 16-byte shared load");
+    uint4 v;
+    std::memcpy(&v, emu_shared(a, 16), 16);
+    return v;
+}
+
+inline emu::MBar &emu_mbar(uint32_t a) {
+    auto it = emu::t_block->mbars.find(a);
+    if (it == emu::t_block->mbars.end()) emu_fail("mbarrier used before init");
+    return it->second;
+}
+inline void emu_mbar_settle(emu::MBar &m) {
+    if (m.pending == 0 && m.tx == 0) {
+        m.phase ^= 1u;
+        m.pending = m.count;
+    }
+}
+inline void emu_mbar_init(uint32_t a, uint32_t count) {
+    if (a & 7u) emu_fail("misaligned mbarrier");
+    emu_shared(a, 8);
+    std::lock_guard<std::mutex> l(emu::t_block->mbar_mu);
+    emu::MBar &m = emu::t_block->mbars[a];
+    m.count = m.pending = count;
+    m.phase = 0;
+    m.tx = 0;
+}
+inline void emu_mbar_arrive_expect_tx(uint32_t a, uint32_t bytes) {
+    std::lock_guard<std::mutex> l(emu::t_block->mbar_mu);
+    emu::MBar &m = emu_mbar(a);
+    if (m.pending == 0) emu_fail("arrival on a completed mbarrier phase");
+    m.tx += bytes;
+    --m.pending;
+    emu_mbar_settle(m);
+}
+inline void emu_mbar_complete_tx(uint32_t a, uint32_t bytes) {
+    std::lock_guard<std::mutex> l(emu::t_block->mbar_mu);
+    emu::MBar &m = emu_mbar(a);
+    m.tx -= bytes;
+    emu_mbar_settle(m);
+}
+// true once the phase of the given parity has completed
+inline bool emu_mbar_try_wait(uint32_t a, uint32_t parity) {
+    bool done;
+    {
+        std::lock_guard<std::mutex> l(emu::t_block->mbar_mu);
+        done = emu_mbar(a).phase != (parity & 1u);
+    }
+    if (!done) std::this_thread::yield();
+    return done;
+}
+
+// Tensor maps: the parameters cuTensorMapEncodeTiled takes, checked as the
+// driver checks them, kept in the 128-byte descriptor.
+enum { CUDA_SUCCESS = 0, CUDA_ERROR_INVALID_VALUE = 1 };
+enum { CU_TENSOR_MAP_DATA_TYPE_UINT8 = 0, CU_TENSOR_MAP_DATA_TYPE_FLOAT16 = 6 };
+enum { CU_TENSOR_MAP_INTERLEAVE_NONE = 0 };
+enum { CU_TENSOR_MAP_SWIZZLE_NONE = 0, CU_TENSOR_MAP_SWIZZLE_128B = 3 };
+enum { CU_TENSOR_MAP_L2_PROMOTION_L2_256B = 3 };
+enum { CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE = 0 };
+struct EmuTensorMap {
+    const uint8_t *base;
+    uint32_t rank, esize, swizzle128, pad;
+    uint64_t dims[5], strides[5];  // strides[0] = element size; strides[i] in bytes
+    uint32_t box[5];
+};
+static_assert(sizeof(EmuTensorMap) <= sizeof(CUtensorMap), "tensor map fits its descriptor");
+inline CUresult emu_encode_tiled(CUtensorMap *out, CUtensorMapDataType dt, cuuint32_t rank, void *base,
+                                 const cuuint64_t *dims, const cuuint64_t *strides, const cuuint32_t *box,
+                                 const cuuint32_t *estr, CUtensorMapInterleave, CUtensorMapSwizzle sw,
+                                 CUtensorMapL2promotion, CUtensorMapFloatOOBfill) {
+    EmuTensorMap m{};
+    m.esize = dt == CU_TENSOR_MAP_DATA_TYPE_FLOAT16 ? 2 : 1;
+    if (rank < 1 || rank > 5 || ((uintptr_t)base & 15u)) return CUDA_ERROR_INVALID_VALUE;
+    m.base = static_cast<const uint8_t *>(base);
+    m.rank = rank;
+    m.swizzle128 = sw == CU_TENSOR_MAP_SWIZZLE_128B;
+    m.strides[0] = m.esize;
+    for (uint32_t i = 0; i < rank; ++i) {
+        if (dims[i] < 1 || box[i] < 1 || box[i] > 256 || estr[i] != 1) return CUDA_ERROR_INVALID_VALUE;
+        m.dims[i] = dims[i];
+        m.box[i] = box[i];
+        if (i > 0) {
+            if (strides[i - 1] % 16) return CUDA_ERROR_INVALID_VALUE;
+            m.strides[i] = strides[i - 1];
+        }
+    }
+    if ((m.box[0] * m.esize) % 16 || (m.swizzle128 && m.box[0] * m.esize > 128)) return CUDA_ERROR_INVALID_VALUE;
+    std::memset(out, 0, sizeof(CUtensorMap));
+    std::memcpy(out, &m, sizeof(m));
+    return CUDA_SUCCESS;
+}
+
+// A tiled TMA load: the whole box lands at once (out-of-range elements as
+// zeros), with the 128-byte swizzle taken from the shared address bits, then
+// its bytes complete on the mbarrier.
+inline void emu_tma_load(uint32_t dst, const void *map, uint32_t bar, const int *c, int rank) {
+    const EmuTensorMap &m = *static_cast<const EmuTensorMap *>(map);
+    if ((uint32_t)rank != m.rank) emu_fail("TMA rank differs from the tensor map");
+    if (((int64_t)c[0] * m.esize) % 16) emu_fail("TMA innermost coordinate not 16-byte aligned");
+    if (m.swizzle128 && (dst & 1023u)) emu_fail("swizzled TMA destination not 1024-byte aligned");
+    if (!m.swizzle128 && (dst & 127u)) emu_fail("TMA destination not 128-byte aligned");
+    uint64_t total = 1;
+    for (int d = 0; d < rank; ++d) total *= m.box[d];
+    const uint64_t bytes = total * m.esize;
+    emu_shared(dst, bytes);
+    for (uint64_t idx = 0; idx < total; ++idx) {
+        uint64_t rem = idx, src = 0;
+        bool in = true;
+        for (int d = 0; d < rank; ++d) {
+            const int64_t g = (int64_t)c[d] + (int64_t)(rem % m.box[d]);
+            rem /= m.box[d];
+            if (g < 0 || (uint64_t)g >= m.dims[d]) in = false;
+            else src += (uint64_t)g * m.strides[d];
+        }
+        uint32_t a = dst + (uint32_t)(idx * m.esize);
+        if (m.swizzle128) a ^= ((a >> 7) & 7u) << 4;
+        uint8_t *p = emu_shared(a, m.esize);
+        if (in)
+            std::memcpy(p, m.base + src, m.esize);
+        else
+            std::memset(p, 0, m.esize);
+    }
+    emu_mbar_complete_tx(bar, (uint32_t)bytes);
+}
+
+// cudaLaunchKernelEx with its configuration (launch attributes are ignored:
+// kernels run one after another).
+enum cudaLaunchAttributeID { cudaLaunchAttributeProgrammaticStreamSerialization = 1 };
+struct cudaLaunchAttributeValue {
+    int programmaticStreamSerializationAllowed;
+};
+struct cudaLaunchAttribute {
+    cudaLaunchAttributeID id;
+    cudaLaunchAttributeValue val;
+};
+struct cudaLaunchConfig_t {
+    dim3 gridDim, blockDim;
+    size_t dynamicSmemBytes;
+    cudaStream_t stream;
+    cudaLaunchAttribute *attrs;
+    unsigned numAttrs;
+};
+template <class K, class... A>
+inline cudaError_t cudaLaunchKernelEx(const cudaLaunchConfig_t *c, K k, A... args) {
+    emu::launch(emu::Cfg{c->gridDim, c->blockDim, c->dynamicSmemBytes, c->stream}, [&] { k(args...); });
+    return cudaSuccess;
+}

@@ -3,12 +3,19 @@
 //   harness quant n k bits g kind iters sms in out : quantize, dequant, exact error
 //   harness a8    n k bits g batch sms in out      : uniform quantize, int8 activations, W.A8 matmul
 //   harness q4x   n k iters sms batch in out       : Q4X learner, dequant, two-matrix decode
+//   harness gemv  n k bits g kind batch sms in out : quantize, then the TMA-pipelined decode
+//                                                    GEMV on one matrix and on a two-entry launch
 // `in` holds W (fp16 [n][k]) and, for a8 and q4x, x (fp16 [batch][k]).
 #include <cstdio>
 #include <new>
 #include <string>
 
 #include "qx_kernels.cuh"
+
+namespace qx {
+// tensor maps come from the emulated encoder
+EncodeTiledFn encode_fn() { return &emu_encode_tiled; }
+}  // namespace qx
 
 namespace {
 template <class T>
@@ -25,7 +32,8 @@ int main(int argc, char **argv) {
     if (argc < 2) return 2;
     const std::string cmd = argv[1];
     const bool q4x = cmd == "q4x";
-    if ((q4x && argc != 9) || (!q4x && argc != (cmd == "quant" ? 11 : 10))) return 2;
+    const int want = q4x ? 9 : (cmd == "quant" || cmd == "gemv") ? 11 : 10;
+    if (argc != want) return 2;
     const int64_t n = atoll(argv[2]), k = atoll(argv[3]);
     FILE *fi = fopen(argv[argc - 2], "rb"), *fo = fopen(argv[argc - 1], "wb");
     if (fi == nullptr || fo == nullptr) return 2;
@@ -73,8 +81,9 @@ int main(int argc, char **argv) {
         put(fo, yh, 2 * batch * n);
     } else {
         const int bits = atoi(argv[4]), g = atoi(argv[5]);
-        const int kind = cmd == "quant" ? atoi(argv[6]) : 0;
-        const int extra = atoi(argv[cmd == "quant" ? 7 : 6]), sms = atoi(argv[cmd == "quant" ? 8 : 7]);
+        const bool three = cmd == "quant" || cmd == "gemv";  // commands that take a kind
+        const int kind = three ? atoi(argv[6]) : 0;
+        const int extra = atoi(argv[three ? 7 : 6]), sms = atoi(argv[three ? 8 : 7]);
         const int G = (int)(k / g), zb = (G + 1) / 2;
         const size_t cb = n * k * bits / 8, sb = kind == 0 ? 2 * n * G : 0, zbb = kind == 0 ? n * zb : 0,
                      lb = kind == 1 ? 2 * n * G * 8 : 0;
@@ -86,7 +95,44 @@ int main(int argc, char **argv) {
         put(fo, scales, sb);
         put(fo, zeros, zbb);
         put(fo, luts, lb);
-        if (cmd == "quant") {
+        if (cmd == "gemv") {
+            const int batch = extra;
+            __half *x = alloc<__half>(2 * batch * k);
+            if (!get(fi, x, 2 * batch * k)) return 2;
+            float *y0 = alloc<float>(4 * batch * n), *y1 = alloc<float>(4 * batch * n),
+                  *y2 = alloc<float>(4 * batch * n);
+            int l = 0;
+            while ((1 << l) < g) ++l;
+            for (int launch = 0; launch < 2; ++launch) {
+                qx::GemvMulti m{};
+                m.count = launch == 0 ? 1 : 2;
+                m.bits = bits;
+                m.kind = kind;
+                m.batch = batch;
+                m.y_f32 = 1;
+                m.status = status;
+                m.wait_limit_ns = 60000000000ull;  // the emulation is slow; a real stall still ends
+                for (int i = 0; i < m.count; ++i) {
+                    qx::GemvMat &M = m.mat[i];
+                    M.codes = codes;
+                    M.scales = scales;
+                    M.zeros = zeros;
+                    M.luts = luts;
+                    M.x = x;
+                    M.y = launch == 0 ? y0 : (i == 0 ? y1 : y2);
+                    M.n = n;
+                    M.k = k;
+                    M.G = G;
+                    M.zbytes = zb;
+                    M.log2g = l;
+                }
+                if (!qx::plan_gemv(m, sms)) return 3;
+                qx::launch_gemv_multi(m, nullptr, launch == 1);
+            }
+            put(fo, y0, 4 * batch * n);
+            put(fo, y1, 4 * batch * n);
+            put(fo, y2, 4 * batch * n);
+        } else if (cmd == "quant") {
             __half *Wh = alloc<__half>(2 * n * k);
             qx::DequantArgs d{codes, scales, zeros, luts, n, k, bits, g, kind, G, zb, Wh};
             qx::launch_dequant(d, sms, nullptr);

@@ -1,10 +1,12 @@
-"""The kernel sources that use no TMA, mbarrier or tensor-core instructions run
-on host threads, compiled with AddressSanitizer and UBSan (a stand-in for
-compute-sanitizer): every index they form must
-stay inside buffers of exactly the sizes the C ABI states, and their results
-must equal the oracle's (bit-exact codes, LUTs, dequantized weights, exact
-squared errors and int8 activations; matmuls within the tolerance).  No GPU;
-the library never loads this code (tests/emulation/cuda_host.h)."""
+"""The kernel sources that use no tensor-core instructions run on host threads,
+compiled with AddressSanitizer and UBSan (a stand-in for compute-sanitizer):
+the quantizers, dequantizers, the exact-error reduction, the W.A8 pair, the Q4X
+path, and the TMA-pipelined decode GEMV (its mbarriers and tensor copies are
+emulated with the hardware's alignment rules checked).  Every index must stay
+inside buffers of exactly the sizes the C ABI states, and the results must
+equal the oracle's (bit-exact codes, LUTs, dequantized weights, exact squared
+errors and int8 activations; matmuls within the tolerance).  No GPU; the
+library never loads this code (tests/emulation/cuda_host.h)."""
 import os
 import shutil
 import subprocess
@@ -113,6 +115,28 @@ def test_int8_activations_and_w_a8_matmul(harness, n, k, bits, g, batch):
     w_exact = (qw - z) * np.repeat(ref["scales"].astype(np.float64), g, axis=1)
     tol = oracle.tolerance(oracle.dequant_act(qr, sr), w_exact)
     assert np.all(oracle.max_abs_err(y, oracle.gemv_a8(ref, rec, x, k)) <= tol)
+
+
+@pytest.mark.parametrize("n,k,bits,g,kind,batch,sms", [  # 1..4 and 8 rows of x, ragged row blocks
+    (37, 384, 4, 64, 0, 1, 2), (130, 640, 3, 64, 0, 4, 3), (33, 256, 4, 32, 0, 8, 2),
+    (20, 512, 3, 128, 1, 3, 2), (5, 4096, 4, 128, 0, 2, 4), (70, 1152, 3, 128, 0, 1, 3)])
+def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms):
+    """qx_gemv's kernel and host plan (tensor maps, byte-balanced CTA slices):
+    one matrix, and the same matrix twice in one launch (with PDL set)."""
+    W = _weights(n, k, seed=n + g)
+    x = synth.activations(batch, k, seed=batch, stream=n)
+    rd = _run(harness, ["gemv", n, k, bits, g, kind, batch, sms], W, x)
+    G = k // g
+    rd.take(n * k * bits // 8 + (2 * n * G + n * ((G + 1) // 2) if kind == 0 else 2 * n * G * 8), np.uint8)
+    ys = [rd.take(batch * n, np.float32).reshape(batch, n) for _ in range(3)]
+    assert rd.take(1, np.uint32)[0] == 0  # no bounded wait gave up
+    rec = ORecipe(bits, g, "lut" if kind else "uniform", 25)
+    ref = oracle.quantize(W, rec)
+    y_ref = oracle.gemv(ref, rec, x, k)
+    tol = oracle.tolerance(x, oracle.dequant(ref, rec, k))
+    for y in ys:
+        assert np.all(oracle.max_abs_err(y, y_ref) <= tol)
+    assert np.array_equal(ys[0], ys[1]) and np.array_equal(ys[1], ys[2])
 
 
 def _q4x_cases():
