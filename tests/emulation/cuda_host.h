@@ -30,6 +30,7 @@
 #include <mutex>
 #include <thread>
 #include <unordered_map>
+#include <limits>
 #include <cstdio>
 #include <vector>
 
@@ -63,6 +64,8 @@ struct Block {
     size_t dyn_bytes = 0;
     std::mutex mbar_mu;
     std::unordered_map<uint32_t, MBar> mbars;  // by shared-memory address
+    std::vector<float> tmem;                   // tensor memory: 128 lanes x 512 columns
+    uint32_t tmem_cols = 0;
 };
 inline thread_local dim3 t_tid, t_bid;
 inline thread_local Block *t_block = nullptr;
@@ -190,7 +193,7 @@ inline float2 __half22float2(__half2 h) { return float2{__half2float(h.x), __hal
 
 // ------------------------------------------------------------------ runtime
 typedef void *cudaStream_t;
-enum cudaError_t { cudaSuccess = 0 };
+enum cudaError_t { cudaSuccess = 0, cudaErrorInvalidValue = 1, cudaErrorInvalidConfiguration = 9, cudaErrorInvalidDevice = 101, cudaErrorNotSupported = 801 };
 inline cudaError_t cudaMemsetAsync(void *p, int v, size_t n, cudaStream_t) {
     std::memset(p, v, n);
     return cudaSuccess;
@@ -490,7 +493,7 @@ inline void emu_tma_load(uint32_t dst, const void *map, uint32_t bar, const int 
     if ((uint32_t)rank != m.rank) emu_fail("TMA rank differs from the tensor map");
     if (((int64_t)c[0] * m.esize) % 16) emu_fail("TMA innermost coordinate not 16-byte aligned");
     if (m.swizzle128 && (dst & 1023u)) emu_fail("swizzled TMA destination not 1024-byte aligned");
-    if (!m.swizzle128 && (dst & 127u)) emu_fail("TMA destination not 128-byte aligned");
+    if (dst & 15u) emu_fail("TMA destination not 16-byte aligned");
     uint64_t total = 1;
     for (int d = 0; d < rank; ++d) total *= m.box[d];
     const uint64_t bytes = total * m.esize;
@@ -535,5 +538,106 @@ struct cudaLaunchConfig_t {
 template <class K, class... A>
 inline cudaError_t cudaLaunchKernelEx(const cudaLaunchConfig_t *c, K k, A... args) {
     emu::launch(emu::Cfg{c->gridDim, c->blockDim, c->dynamicSmemBytes, c->stream}, [&] { k(args...); });
+    return cudaSuccess;
+}
+
+// ------------------------------------------------------------------ tensor cores
+inline float __uint_as_float(uint32_t u) {
+    float f;
+    std::memcpy(&f, &u, 4);
+    return f;
+}
+inline __half2 __float2half2_rn(float x) { return __half2{__float2half_rn(x), __float2half_rn(x)}; }
+template <class T>
+inline T __ldcg(const T *p) { return *p; }
+inline uint32_t emu_lds32(uint32_t a) {
+    if (a & 3u) emu_fail("misaligned 4-byte shared load");
+    uint32_t v;
+    std::memcpy(&v, emu_shared(a, 4), 4);
+    return v;
+}
+inline void emu_mbar_arrive(uint32_t a) {
+    std::lock_guard<std::mutex> l(emu::t_block->mbar_mu);
+    emu::MBar &m = emu_mbar(a);
+    if (m.pending == 0) emu_fail("arrival on a completed mbarrier phase");
+    --m.pending;
+    emu_mbar_settle(m);
+}
+
+// Allocation is warp-collective: lane 0 acts for the warp.  Columns: a power
+// of two in 32..512; unwritten accumulators read as NaN.
+inline void emu_tmem_alloc(uint32_t dst, uint32_t cols) {
+    if (emu_lane() != 0) return;
+    emu::Block &b = *emu::t_block;
+    if (cols < 32 || cols > 512 || (cols & (cols - 1))) emu_fail("TMEM allocation size");
+    if (b.tmem_cols != 0) emu_fail("second TMEM allocation in a CTA");
+    b.tmem.assign(128 * 512, std::numeric_limits<float>::quiet_NaN());
+    b.tmem_cols = cols;
+    const uint32_t base = 0;  // lane 0, column 0
+    std::memcpy(emu_shared(dst, 4), &base, 4);
+}
+inline void emu_tmem_dealloc(uint32_t taddr, uint32_t cols) {
+    if (emu_lane() != 0) return;
+    emu::Block &b = *emu::t_block;
+    if (taddr != 0 || cols != b.tmem_cols) emu_fail("TMEM deallocation differs from the allocation");
+    b.tmem_cols = 0;
+}
+// 32x32b load: lane l of the warp reads row (lane base + l), n columns.  A warp
+// reaches only the 32 lanes of its quarter (warp id % 4).
+inline void emu_tmem_ld(uint32_t taddr, uint32_t *r, int n) {
+    const emu::Block &b = *emu::t_block;
+    const uint32_t lane0 = taddr >> 16, col = taddr & 0xFFFFu;
+    if (lane0 != 32u * ((threadIdx.x >> 5) & 3u)) emu_fail("TMEM lanes outside the warp's quarter");
+    if (col + (uint32_t)n > b.tmem_cols) emu_fail("TMEM columns outside the allocation");
+    const float *row = b.tmem.data() + (size_t)(lane0 + emu_lane()) * 512 + col;
+    std::memcpy(r, row, 4 * (size_t)n);
+}
+// K-major operand, 128-byte swizzle: row r, element k (fp16) of the tile a
+// shared-memory descriptor names.
+inline double emu_desc_elem(uint64_t desc, int r, int k) {
+    if ((desc >> 61) != 2u || ((desc >> 46) & 3u) != 1u || ((desc >> 49) & 7u) != 0u)
+        emu_fail("shared-memory descriptor: not a 128-byte-swizzle K-major tcgen05 descriptor");
+    const uint32_t start = (uint32_t)(desc & 0x3FFFu) << 4, sbo = (uint32_t)((desc >> 32) & 0x3FFFu) << 4;
+    const uint32_t lin = start + (uint32_t)(r / 8) * sbo + (uint32_t)(r % 8) * 128u + 2u * (uint32_t)k;
+    const uint32_t phys = lin ^ (((lin >> 7) & 7u) << 4);
+    __half h;
+    std::memcpy(&h, emu_shared(phys, 2), 2);
+    return (double)__half2float(h);
+}
+// D[M][N] (+)= A[M][16] B[N][16]^T, fp16 operands, fp32 accumulators.
+inline void emu_mma_f16(uint32_t d, uint64_t adesc, uint64_t bdesc, uint32_t idesc, uint32_t acc) {
+    emu::Block &b = *emu::t_block;
+    if (((idesc >> 4) & 3u) != 1u || ((idesc >> 7) & 7u) != 0u || ((idesc >> 10) & 7u) != 0u ||
+        ((idesc >> 15) & 3u) != 0u)
+        emu_fail("instruction descriptor: expected fp16 K-major operands and fp32 accumulators");
+    const int N = (int)((idesc >> 17) & 63u) << 3, M = (int)((idesc >> 24) & 31u) << 4;
+    if (M != 128 || N < 16 || N > 256 || N % 16) emu_fail("MMA shape for cta_group::1, M = 128");
+    const uint32_t lane0 = d >> 16, col0 = d & 0xFFFFu;
+    if (lane0 != 0 || col0 + (uint32_t)N > b.tmem_cols) emu_fail("MMA accumulator outside the allocation");
+    for (int m = 0; m < M; ++m) {
+        double a[16];
+        for (int k = 0; k < 16; ++k) a[k] = emu_desc_elem(adesc, m, k);
+        float *row = b.tmem.data() + (size_t)m * 512 + col0;
+        for (int n = 0; n < N; ++n) {
+            double sum = 0.0;
+            for (int k = 0; k < 16; ++k) sum += a[k] * emu_desc_elem(bdesc, n, k);
+            row[n] = acc ? row[n] + (float)sum : (float)sum;
+        }
+    }
+}
+
+// runtime lookups the host code makes
+enum cudaDriverEntryPointQueryResult { cudaDriverEntryPointSuccess = 0, cudaDriverEntryPointSymbolNotFound = 1 };
+enum { cudaEnableDefault = 0 };
+inline cudaError_t cudaGetDriverEntryPointByVersion(const char *name, void **p, unsigned, unsigned long long,
+                                                    cudaDriverEntryPointQueryResult *q) {
+    const bool ok = std::strcmp(name, "cuTensorMapEncodeTiled") == 0;
+    *p = ok ? reinterpret_cast<void *>(&emu_encode_tiled) : nullptr;
+    *q = ok ? cudaDriverEntryPointSuccess : cudaDriverEntryPointSymbolNotFound;
+    return cudaSuccess;
+}
+template <class T>
+inline cudaError_t cudaGetSymbolAddress(void **p, T &sym) {
+    *p = static_cast<void *>(&sym);
     return cudaSuccess;
 }

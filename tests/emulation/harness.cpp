@@ -5,17 +5,14 @@
 //   harness q4x   n k iters sms batch in out       : Q4X learner, dequant, two-matrix decode
 //   harness gemv  n k bits g kind batch sms in out : quantize, then the TMA-pipelined decode
 //                                                    GEMV on one matrix and on a two-entry launch
+//   harness gemm  n k bits g kind m sms in out     : quantize, then the tensor-core matmul: one
+//                                                    CTA per tile, split-k, split-k with PDL
 // `in` holds W (fp16 [n][k]) and, for a8 and q4x, x (fp16 [batch][k]).
 #include <cstdio>
 #include <new>
 #include <string>
 
 #include "qx_kernels.cuh"
-
-namespace qx {
-// tensor maps come from the emulated encoder
-EncodeTiledFn encode_fn() { return &emu_encode_tiled; }
-}  // namespace qx
 
 namespace {
 template <class T>
@@ -32,7 +29,7 @@ int main(int argc, char **argv) {
     if (argc < 2) return 2;
     const std::string cmd = argv[1];
     const bool q4x = cmd == "q4x";
-    const int want = q4x ? 9 : (cmd == "quant" || cmd == "gemv") ? 11 : 10;
+    const int want = q4x ? 9 : (cmd == "quant" || cmd == "gemv" || cmd == "gemm") ? 11 : 10;
     if (argc != want) return 2;
     const int64_t n = atoll(argv[2]), k = atoll(argv[3]);
     FILE *fi = fopen(argv[argc - 2], "rb"), *fo = fopen(argv[argc - 1], "wb");
@@ -81,7 +78,7 @@ int main(int argc, char **argv) {
         put(fo, yh, 2 * batch * n);
     } else {
         const int bits = atoi(argv[4]), g = atoi(argv[5]);
-        const bool three = cmd == "quant" || cmd == "gemv";  // commands that take a kind
+        const bool three = cmd == "quant" || cmd == "gemv" || cmd == "gemm";  // commands that take a kind
         const int kind = three ? atoi(argv[6]) : 0;
         const int extra = atoi(argv[three ? 7 : 6]), sms = atoi(argv[three ? 8 : 7]);
         const int G = (int)(k / g), zb = (G + 1) / 2;
@@ -95,7 +92,54 @@ int main(int argc, char **argv) {
         put(fo, scales, sb);
         put(fo, zeros, zbb);
         put(fo, luts, lb);
-        if (cmd == "gemv") {
+        if (cmd == "gemm") {
+            const int64_t m = extra;
+            __half *X = alloc<__half>(2 * m * k);
+            if (!get(fi, X, 2 * m * k)) return 2;
+            int l = 0;
+            while ((1 << l) < g) ++l;
+            for (int run = 0; run < 3; ++run) {
+                const qx::GemmPlan plan = qx::plan_gemm(n, k, m, sms, run > 0);
+                qx::GemmArgs a{};
+                a.codes = codes;
+                a.scales = scales;
+                a.zeros = zeros;
+                a.luts = luts;
+                a.n = n;
+                a.k = k;
+                a.m = m;
+                a.bits = bits;
+                a.kind = kind;
+                a.log2g = l;
+                a.G = G;
+                a.zbytes = zb;
+                a.X = X;
+                __half *Y = alloc<__half>(2 * m * n);
+                a.Y = Y;
+                a.status = status;
+                a.wait_limit_ns = 60000000000ull;
+                a.bn = plan.bn;
+                a.splits = plan.splits;
+                a.pdl = run == 2;
+                static uint8_t *ws = nullptr;  // one workspace, reused by both split-k runs
+                if (plan.splits > 1) {
+                    if (ws == nullptr) {
+                        ws = alloc<uint8_t>(plan.ws_bytes);
+                        std::memset(ws, 0, plan.ws_bytes);
+                    }
+                    a.ws_cnt = reinterpret_cast<uint32_t *>(ws);
+                    a.ws_part = reinterpret_cast<float *>(ws + qx::kSplitCounterBytes);
+                }
+                qx::launch_gemm(a, sms, nullptr);
+                put(fo, Y, 2 * m * n);
+                uint32_t clean = 1;  // the counters are back to zero after every call
+                if (plan.splits > 1)
+                    for (size_t i = 0; i < qx::kSplitCounterBytes; ++i) clean &= ws[i] == 0;
+                put(fo, &clean, 4);
+                const uint32_t shape[2] = {(uint32_t)plan.bn, (uint32_t)plan.splits};
+                put(fo, shape, 8);
+            }
+        } else if (cmd == "gemv") {
             const int batch = extra;
             __half *x = alloc<__half>(2 * batch * k);
             if (!get(fi, x, 2 * batch * k)) return 2;

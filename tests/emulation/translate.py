@@ -1,13 +1,13 @@
-"""Host C++ copies of the library's kernel sources that use no tensor-core
-instructions (tests only).
+"""Host C++ copies of the library's kernel sources (tests only).
 
 Rewrites, in copies written to `out_dir`:
   * the CUDA headers -> cuda_host.h (next to this file);
-  * each inline-PTX statement -> the same operation in C (cuda_host.h), chosen by
-    the instruction it holds; the operand names are those of the sources;
+  * each inline-PTX statement -> the same operation in C (cuda_host.h), chosen
+    by the instruction it holds and filled with its own output and input
+    operands ({o0}, {i0}, ... in order);
   * `extern __shared__ T name[];` -> the launch's dynamic shared memory;
   * `kernel<<<cfg>>>(args);` -> emu::launch(cfg, [&] { kernel(args); }).
-Fails if any inline PTX is left untranslated.
+Fails if an inline-PTX statement holds no known instruction.
 """
 from __future__ import annotations
 
@@ -17,42 +17,70 @@ import re
 CSRC = os.path.join(os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__)))),
                     "paper_2505_07531_gb300", "csrc")
 FILES = ["qx_common.cuh", "qx_kernels.cuh", "qx_quant.cu", "qx_act8.cu", "qx_select.cu", "qx_q4x.cu",
-         "qx_gemv.cu"]
+         "qx_gemv.cu", "qx_gemm.cu"]
 
-# instruction -> C statement, in the operand names the sources use
+# first match wins: longer instruction names before their prefixes
 BY_INSTRUCTION = [
-    ("lop3.b32", "d = (a & b) | c;"),
-    ("prmt.b32", "d = emu_prmt(a, b, sel);"),
-    ("mul.hi.u32", "d = (uint32_t)(((uint64_t)x * (uint64_t)(1u << (32 - n))) >> 32);"),
-    ("%%globaltimer", "t = emu_globaltimer();"),
-    ("cvt.rn.f16.f64", "h = emu_f64_to_f16(x);"),
-    ("mbarrier.init", "emu_mbar_init(b, count);"),
-    ("mbarrier.arrive.expect_tx", "emu_mbar_arrive_expect_tx(b, bytes);"),
-    ("mbarrier.try_wait.parity", "ok = emu_mbar_try_wait(b, parity) ? 1u : 0u;"),
-    ("cp.async.bulk.tensor.2d", "{ const int c_[2] = {x, y}; emu_tma_load(dst, map, bar, c_, 2); }"),
-    ("cp.async.bulk.tensor.3d", "{ const int c_[3] = {x, y, z}; emu_tma_load(dst, map, bar, c_, 3); }"),
-    ("cp.async.bulk.prefetch.L2", "(void)p; (void)bytes;"),
-    ("ld.shared.v4.u32", "v = emu_lds128(a);"),
+    ("lop3.b32", "{o0} = ({i0} & {i1}) | {i2};"),
+    ("prmt.b32", "{o0} = emu_prmt({i0}, {i1}, {i2});"),
+    ("mul.hi.u32", "{o0} = (uint32_t)(((uint64_t)({i0}) * (uint64_t)({i1})) >> 32);"),
+    ("%%globaltimer", "{o0} = emu_globaltimer();"),
+    ("cvt.rn.f16.f64", "{o0} = emu_f64_to_f16({i0});"),
+    ("mbarrier.init", "emu_mbar_init({i0}, {i1});"),
+    ("mbarrier.arrive.expect_tx", "emu_mbar_arrive_expect_tx({i0}, {i1});"),
+    ("mbarrier.arrive.shared", "emu_mbar_arrive({i0});"),
+    ("mbarrier.try_wait.parity", "{o0} = emu_mbar_try_wait({i0}, {i1}) ? 1u : 0u;"),
+    ("cp.async.bulk.tensor.2d", "{{ const int c_[2] = {{{i3}, {i4}}}; emu_tma_load({i0}, {i1}, {i2}, c_, 2); }}"),
+    ("cp.async.bulk.tensor.3d",
+     "{{ const int c_[3] = {{{i3}, {i4}, {i5}}}; emu_tma_load({i0}, {i1}, {i2}, c_, 3); }}"),
+    ("cp.async.bulk.prefetch.L2", ";"),
+    ("ld.shared.v4.u32", "{{ const uint4 t_ = emu_lds128({i0}); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
+    ("ld.shared.u32", "{o0} = emu_lds32({i0});"),
     ("griddepcontrol", ";"),
     ("prefetch.tensormap", ";"),
     ("fence.mbarrier_init", "__threadfence_block();"),
     ("fence.proxy.async", "__threadfence_block();"),
+    ("tcgen05.mma.cta_group::1.kind::f16", "emu_mma_f16({i0}, {i1}, {i2}, {i3}, {i4});"),
+    ("tcgen05.commit", "emu_mbar_arrive({i0});"),
+    ("tcgen05.ld.sync.aligned.32x32b.x32", "emu_tmem_ld({i0}, &{o0}, 32);"),
+    ("tcgen05.ld.sync.aligned.32x32b.x16", "emu_tmem_ld({i0}, &{o0}, 16);"),
+    ("tcgen05.alloc", "emu_tmem_alloc({i0}, {i1});"),
+    ("tcgen05.dealloc", "emu_tmem_dealloc({i0}, {i1});"),
+    ("tcgen05.relinquish_alloc_permit", ";"),
+    ("tcgen05.wait::", ";"),
+    ("tcgen05.fence", "__threadfence_block();"),
 ]
 ASM = re.compile(r"\basm\s*(?:volatile\s*)?\((.*?)\);", re.S)
 LAUNCH = re.compile(r"(\w+(?:<[^<>;]*>)?)<<<(.*?)>>>\((.*?)\);", re.S)
+CONSTRAINT = re.compile(r'"(=?[a-z])"\s*\(')
+
+
+def operands(body: str):
+    """Output and input operand expressions of an asm statement, in order."""
+    outs, ins = [], []
+    for m in CONSTRAINT.finditer(body):
+        depth, j = 1, m.end()
+        while depth:
+            depth += {"(": 1, ")": -1}.get(body[j], 0)
+            j += 1
+        (outs if m.group(1).startswith("=") else ins).append(body[m.end():j - 1].strip())
+    return outs, ins
 
 
 def _asm(m):
-    for key, rep in BY_INSTRUCTION:
-        if key in m.group(1):
-            return rep
-    raise ValueError("untranslated inline PTX: " + m.group(0)[:80])
+    body = m.group(1)
+    for key, tmpl in BY_INSTRUCTION:
+        if key in body:
+            outs, ins = operands(body)
+            return tmpl.format(**{f"o{i}": e for i, e in enumerate(outs)}, **{f"i{i}": e for i, e in enumerate(ins)})
+    raise ValueError("untranslated inline PTX: " + m.group(0)[:100])
 
 
 def translate(src: str) -> str:
     src = src.replace("#include <cuda_fp16.h>", '#include "cuda_host.h"')
     src = src.replace("#include <cuda.h>", '#include "cuda_host.h"').replace("#include <cuda_runtime.h>", "")
-    src = re.sub(r"extern __shared__ (\w+) (\w+)\[\];", r"\1 *\2 = reinterpret_cast<\1 *>(emu_dyn_smem());", src)
+    src = re.sub(r"extern __shared__ (?:__align__\(\d+\) )?(\w+) (\w+)\[\];",
+                 r"\1 *\2 = reinterpret_cast<\1 *>(emu_dyn_smem());", src)
     src = ASM.sub(_asm, src)
     return LAUNCH.sub(lambda m: f"emu::launch(emu::Cfg{{{m.group(2)}}}, [&] {{ {m.group(1)}({m.group(3)}); }});", src)
 

@@ -1,8 +1,8 @@
-"""The kernel sources that use no tensor-core instructions run on host threads,
-compiled with AddressSanitizer and UBSan (a stand-in for compute-sanitizer):
-the quantizers, dequantizers, the exact-error reduction, the W.A8 pair, the Q4X
-path, and the TMA-pipelined decode GEMV (its mbarriers and tensor copies are
-emulated with the hardware's alignment rules checked).  Every index must stay
+"""Every kernel source of the library runs on host threads, compiled with
+AddressSanitizer and UBSan (a stand-in for compute-sanitizer): the quantizers,
+dequantizers, the exact-error reduction, the W.A8 pair, the Q4X path, the
+TMA-pipelined decode GEMV and the tcgen05 matmul (its mbarriers, tensor copies,
+tensor memory and MMAs are emulated with the hardware's rules checked).  Every index must stay
 inside buffers of exactly the sizes the C ABI states, and the results must
 equal the oracle's (bit-exact codes, LUTs, dequantized weights, exact squared
 errors and int8 activations; matmuls within the tolerance).  No GPU; the
@@ -137,6 +137,30 @@ def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms):
     for y in ys:
         assert np.all(oracle.max_abs_err(y, y_ref) <= tol)
     assert np.array_equal(ys[0], ys[1]) and np.array_equal(ys[1], ys[2])
+
+
+@pytest.mark.parametrize("n,k,bits,g,kind,m,sms", [  # 16-, 64- and 256-token tiles, 1..4 k splits
+    (37, 384, 4, 64, 0, 5, 2), (128, 2048, 4, 128, 0, 16, 4), (200, 1024, 3, 64, 0, 40, 4),
+    (64, 1152, 4, 32, 0, 1, 8), (130, 256, 4, 256, 0, 300, 2), (40, 256, 3, 128, 1, 3, 2)])
+def test_tensor_core_matmul(harness, n, k, bits, g, kind, m, sms):
+    """qx_gemm (one CTA per tile), then qx_gemm_splitk twice on one workspace,
+    the second with PDL: each within tolerance (fp16 output), and the split
+    counters back to zero after every call."""
+    W = _weights(n, k, seed=n + m)
+    X = synth.activations(m, k, seed=m, stream=n)
+    rd = _run(harness, ["gemm", n, k, bits, g, kind, m, sms], W, X)
+    G = k // g
+    rd.take(n * k * bits // 8 + (2 * n * G + n * ((G + 1) // 2) if kind == 0 else 2 * n * G * 8), np.uint8)
+    rec = ORecipe(bits, g, "lut" if kind else "uniform", 25)
+    ref = oracle.quantize(W, rec)
+    y_ref = oracle.gemm(ref, rec, X, k)
+    tol = oracle.tolerance(X, oracle.dequant(ref, rec, k)) + np.abs(y_ref).max(axis=1) * 2.0 ** -11
+    for _ in range(3):
+        Y = rd.take(m * n, np.float16).reshape(m, n).astype(np.float64)
+        assert np.all(oracle.max_abs_err(Y, y_ref) <= tol)
+        assert rd.take(1, np.uint32)[0] == 1  # counters rearmed
+        rd.take(2, np.uint32)  # the plan: token tile, splits
+    assert rd.take(1, np.uint32)[0] == 0
 
 
 def _q4x_cases():
