@@ -321,6 +321,21 @@ qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, in
 qx_status qx_q4x_gemv_multi(const qx_q4x *mats, int32_t count, const void *const *x, int32_t batch,
                             void *const *y, int32_t y_dtype, void *stream);
 
+/* Prefill matmul Y = X W_hat^T for a Q4X matrix on the tcgen05 tensor cores,
+ * as qx_gemm: W_hat tiles are dequantized into shared memory (the four
+ * codebooks staged there once per CTA, w_hat exactly as above) and multiplied
+ * in fp16 with fp32 accumulation.  X: device fp16 [m][k], 16-byte aligned;
+ * Y: device fp16 [m][n], 2-byte aligned; m >= 1; k a multiple of 128. */
+qx_status qx_q4x_gemm(const qx_q4x *p, const void *X, int64_t m, void *Y, void *stream);
+
+/* qx_q4x_gemm with the contraction split along k when the tiles alone leave
+ * SMs idle, exactly as qx_gemm_splitk (same plan, workspace rules, PDL flag and
+ * split-order sum).  qx_q4x_gemm_splitk_workspace gives the workspace bytes
+ * on the current device (0: no split). */
+qx_status qx_q4x_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, size_t *bytes);
+qx_status qx_q4x_gemm_splitk(const qx_q4x *p, const void *X, int64_t m, void *Y, void *workspace,
+                             size_t workspace_bytes, int32_t flags, void *stream);
+
 /* Failure-detection self-test.  Launches one CTA on `stream` whose bounded
  * wait (the mbarrier wait of the decode and prefill pipelines) is for a phase
  * that nothing completes.  After limit_us microseconds (1..1000000) it gives

@@ -754,6 +754,89 @@ QX_API qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void
     return qx_q4x_gemv_multi(p, 1, &x, batch, &y, y_dtype, stream);
 }
 
+namespace {
+
+qx_status check_q4x_gemm(const qx_q4x *p, const void *X, int64_t m, const void *Y) {
+    qx_status s = check_q4x(p);
+    if (s != QX_OK) return s;
+    if (p->k % 128 != 0) return QX_ERR_UNSUPPORTED;  // the matmul works in 128-weight superblocks
+    if (p->n > (int64_t)1 << 22 || p->k > (int64_t)1 << 20) return QX_ERR_UNSUPPORTED;
+    if (X == nullptr || Y == nullptr || m < 1) return QX_ERR_INVALID_ARG;
+    if (m > ((int64_t)1 << 31) - 1) return QX_ERR_UNSUPPORTED;
+    if (!aligned(X, 16)) return QX_ERR_ALIGNMENT;
+    if (!aligned(Y, 2)) return QX_ERR_ALIGNMENT;
+    return QX_OK;
+}
+
+// The tensor-core matmul's arguments for Q4X weights: kind 2, the book bytes
+// in `zeros`, the codebooks in `luts`.
+qx::GemmArgs q4x_gemm_args(const qx_q4x *p, const void *X, int64_t m, void *Y, const DeviceInfo *d) {
+    const qx::Q4xMat q = q4x_mat(p);
+    qx::GemmArgs a{};
+    a.codes = q.codes;
+    a.scales = q.scales;
+    a.zeros = q.books;
+    a.luts = q.codebooks;
+    a.n = p->n;
+    a.k = p->k;
+    a.m = m;
+    a.bits = 4;
+    a.kind = 2;
+    a.log2g = 6;
+    a.G = q.G;
+    a.zbytes = q.bbytes;
+    a.X = static_cast<const __half *>(X);
+    a.Y = static_cast<__half *>(Y);
+    a.status = d->status;
+    a.wait_limit_ns = wait_limit_ns();
+    return a;
+}
+
+}  // namespace
+
+QX_API qx_status qx_q4x_gemm(const qx_q4x *p, const void *X, int64_t m, void *Y, void *stream) {
+    qx_status s = check_q4x_gemm(p, X, m, Y);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    qx::GemmArgs a = q4x_gemm_args(p, X, m, Y, d);
+    const qx::GemmPlan plan = qx::plan_gemm(p->n, p->k, m, d->num_sms, false);
+    a.bn = plan.bn;
+    a.splits = 1;
+    return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_q4x_gemm_splitk_workspace(int64_t n, int64_t k, int64_t m, size_t *bytes) {
+    if (bytes == nullptr || n < 1 || k < 1 || m < 1) return QX_ERR_INVALID_ARG;
+    if (k % 128 != 0 || n > (int64_t)1 << 22 || k > (int64_t)1 << 20) return QX_ERR_UNSUPPORTED;
+    DeviceInfo *d = nullptr;
+    const qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    *bytes = qx::plan_gemm(n, k, m, d->num_sms, true).ws_bytes;
+    return QX_OK;
+}
+
+QX_API qx_status qx_q4x_gemm_splitk(const qx_q4x *p, const void *X, int64_t m, void *Y, void *workspace,
+                                    size_t workspace_bytes, int32_t flags, void *stream) {
+    qx_status s = check_q4x_gemm(p, X, m, Y);
+    if (s != QX_OK) return s;
+    if ((flags & ~QX_GEMM_PDL) != 0) return QX_ERR_INVALID_ARG;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    const qx::GemmPlan plan = qx::plan_gemm(p->n, p->k, m, d->num_sms, true);
+    qx::GemmArgs a = q4x_gemm_args(p, X, m, Y, d);
+    a.bn = plan.bn;
+    a.splits = plan.splits;
+    a.pdl = (flags & QX_GEMM_PDL) ? 1 : 0;
+    if (plan.splits > 1) {
+        if (workspace == nullptr || workspace_bytes < plan.ws_bytes) return QX_ERR_INVALID_ARG;
+        if (!aligned(workspace, 256)) return QX_ERR_ALIGNMENT;
+        a.ws_cnt = static_cast<uint32_t *>(workspace);
+        a.ws_part = reinterpret_cast<float *>(static_cast<uint8_t *>(workspace) + qx::kSplitCounterBytes);
+    }
+    return from_cuda(qx::launch_gemm(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+}
+
 QX_API qx_status qx_selftest_wait_timeout(int32_t limit_us, void *stream) {
     if (limit_us < 1 || limit_us > 1000000) return QX_ERR_INVALID_ARG;
     DeviceInfo *d = nullptr;

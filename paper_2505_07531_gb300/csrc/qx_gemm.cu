@@ -300,11 +300,17 @@ struct UnitRaw {
 };
 
 // Uniform metadata of one unit, from global memory (read ahead of use).
+// Q4X (KIND 2): the group's fp16 scale and its 2-bit codebook index (books in
+// `zeros`, four per byte, zbytes per row), held in u.scale and u.zero.
 template <int KIND>
 __device__ __forceinline__ void load_meta(const GemmArgs &a, int64_t row, int64_t k0, UnitRaw &u) {
     if (KIND == 0) {
         const int grp = (int)(k0 >> a.log2g);
         u.zero = zero_nibble(a.zeros + row * a.zbytes, grp);
+        u.scale = a.scales[row * a.G + grp];
+    } else if (KIND == 2) {
+        const int grp = (int)(k0 >> a.log2g);
+        u.zero = (a.zeros[row * a.zbytes + (grp >> 2)] >> (2 * (grp & 3))) & 3u;
         u.scale = a.scales[row * a.G + grp];
     }
 }
@@ -355,6 +361,22 @@ __device__ __forceinline__ void dequant_unit(const UnitRaw &u, __half2 (&v)[16])
     }
 }
 
+// Q4X unit: w_hat = codebook[book][q] * s in fp16 (the exact product rounded
+// once, as the dequant defines), the four codebooks in shared memory at `cb`
+// (128 bytes, one word per bank: any lookup pattern is conflict-free).
+__device__ __forceinline__ void dequant_unit_q4x(const UnitRaw &u, const __half *cb, __half2 (&v)[16]) {
+    const __half2 s2 = __halves2half2(u.scale, u.scale);
+    const __half *tb = cb + 16 * u.zero;
+#pragma unroll
+    for (int t = 0; t < 4; ++t) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+            const uint32_t sel = (u.w[t] >> (4 * i)) & 0x000F000Fu;  // codes of k = 8t+2i, 8t+2i+1
+            v[4 * t + i] = __hmul2(__halves2half2(tb[sel & 15u], tb[sel >> 16]), s2);
+        }
+    }
+}
+
 template <int BITS, int KIND, int BN>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tmap_x, const __grid_constant__ CUtensorMap tmap_c,
@@ -366,6 +388,8 @@ __global__ void __launch_bounds__(THREADS, 1)
     uint8_t *base = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~(uintptr_t)1023);
     SmemLayout<BN> &s = *reinterpret_cast<SmemLayout<BN> *>(base);
     const uint32_t pk_s = smem_u32(base + layout_bytes<BN>());  // packed-code ring
+    // Q4X: the matrix's four codebooks (64 fp16) after the ring
+    __half *q4x_cb = reinterpret_cast<__half *>(base + layout_bytes<BN>() + (size_t)a.pslots * a.pslot_bytes);
     volatile uint32_t *abort_flag = &s.abort_flag;
     uint32_t *abort_w = &s.abort_flag;
     const int warp = threadIdx.x >> 5;
@@ -401,6 +425,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_c) : "memory");
         if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&tmap_l) : "memory");
     }
+    if (KIND == 2 && threadIdx.x >= 64 && threadIdx.x < 128) q4x_cb[threadIdx.x - 64] = a.luts[threadIdx.x - 64];
     if (warp == 1) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
                          smem_u32(&s.tmem_base)),
@@ -498,7 +523,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int u = 2 * h2 + half_id;
                 // with g >= 128 both units use the first unit's table
                 read_codes<BITS, KIND>(base_ps, r, u, (32 * u) >> a.log2g, a.lut_box, h2 == 0 || a.log2g < 7, w[h2]);
-                if (KIND == 0 && row < a.n) load_meta<KIND>(a, row, (int64_t)sbl * 128 + 32 * u, w[h2]);
+                if (KIND != 1 && row < a.n) load_meta<KIND>(a, row, (int64_t)sbl * 128 + 32 * u, w[h2]);
             }
             // every lane has its codes in registers: release the slot
             __syncwarp();
@@ -553,7 +578,10 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                     for (int h2 = 0; h2 < 2; ++h2) {
                         if (valid) {
-                            dequant_unit<BITS, KIND>(cur[h2], v[h2]);
+                            if constexpr (KIND == 2)
+                                dequant_unit_q4x(cur[h2], q4x_cb, v[h2]);
+                            else
+                                dequant_unit<BITS, KIND>(cur[h2], v[h2]);
                         } else {
 #pragma unroll
                             for (int p = 0; p < 16; ++p) v[h2][p] = __float2half2_rn(0.0f);
@@ -844,10 +872,12 @@ cudaError_t launch_gemm(const GemmArgs &args, int num_sms, cudaStream_t st) {
     a.pslot_bytes = (a.bits == 3 ? BM * 48 + BM * a.lut_box : BM * 64 + 0);
     a.pslot_bytes = (a.pslot_bytes + 1023) / 1024 * 1024;
     const int layout = (int)(a.bn == 16 ? layout_bytes<16>() : a.bn == 64 ? layout_bytes<64>() : layout_bytes<256>());
-    const int budget = 227 * 1024 - layout - 1024;
+    const int cb_bytes = a.kind == 2 ? 128 : 0;  // Q4X codebooks after the ring
+    const int budget = 227 * 1024 - layout - 1024 - cb_bytes;
     a.pslots = std::min(kMaxPSlots, budget / a.pslot_bytes);
     if (a.pslots < 2) return cudaErrorInvalidConfiguration;
-    a.smem_bytes = layout + 1024 + a.pslots * a.pslot_bytes;
+    a.smem_bytes = layout + 1024 + a.pslots * a.pslot_bytes + cb_bytes;
+    if (a.bits == 4 && a.kind == 2) return launch_bn<4, 2>(mx, mc, ml, a, units, num_sms, st);
     if (a.bits == 4) return launch_bn<4, 0>(mx, mc, ml, a, units, num_sms, st);
     if (a.kind == 1) return launch_bn<3, 1>(mx, mc, ml, a, units, num_sms, st);
     return launch_bn<3, 0>(mx, mc, ml, a, units, num_sms, st);

@@ -106,6 +106,9 @@ def _lib():
         lib.qx_q4x_dequant.argtypes = [P(_Q4x), VP, VP]
         lib.qx_q4x_gemv.argtypes = [P(_Q4x), VP, I32, VP, I32, VP]
         lib.qx_q4x_gemv_multi.argtypes = [P(_Q4x), I32, P(VP), I32, P(VP), I32, VP]
+        lib.qx_q4x_gemm.argtypes = [P(_Q4x), VP, I64, VP, VP]
+        lib.qx_q4x_gemm_splitk_workspace.argtypes = [I64, I64, I64, P(ctypes.c_size_t)]
+        lib.qx_q4x_gemm_splitk.argtypes = [P(_Q4x), VP, I64, VP, VP, ctypes.c_size_t, I32, VP]
         lib.qx_selftest_wait_timeout.argtypes = [I32, VP]
         lib.qx_get_device_status.argtypes = [VP]
         lib.qx_status_string.argtypes = [ctypes.c_int]
@@ -116,7 +119,8 @@ def _lib():
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
-                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_selftest_wait_timeout",
+                   "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_q4x_gemm", "qx_q4x_gemm_splitk_workspace",
+                   "qx_q4x_gemm_splitk", "qx_selftest_wait_timeout",
                    "qx_get_device_status", "qx_version"):
             getattr(lib, fn).restype = ctypes.c_int
         _LIB = lib
@@ -527,6 +531,35 @@ def selftest_wait_timeout(limit_us: int, device=None) -> None:
     bounded wait that runs out; device_status() then returns 5 (QX_ERR_TIMEOUT)."""
     dev = device if device is not None else torch.device("cuda", torch.cuda.current_device())
     _check(_lib().qx_selftest_wait_timeout(int(limit_us), _stream(dev)), "qx_selftest_wait_timeout")
+
+
+def q4x_gemm(P: Q4xMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+    """Prefill Y = X W_hat^T for a Q4X matrix on the tensor cores (qx_q4x_gemm); fp16 [m][n]."""
+    _dev_tensor(X, "X")
+    m = X.shape[0]
+    Y = out if out is not None else torch.empty((m, P.n), dtype=torch.float16, device=X.device)
+    _dev_tensor(Y, "out")
+    pc = P.c()
+    _check(_lib().qx_q4x_gemm(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _stream(X.device)), "qx_q4x_gemm")
+    return Y
+
+
+def q4x_gemm_splitk(P: Q4xMatrix, X: torch.Tensor, out: torch.Tensor | None = None,
+                    workspace: torch.Tensor | None = None, pdl: bool = False) -> torch.Tensor:
+    """qx_q4x_gemm with k split across CTAs when the tiles leave SMs idle
+    (qx_q4x_gemm_splitk); the workspace is kept per device and stream as for
+    gemm_splitk.  Returns fp16 [m][n]."""
+    _dev_tensor(X, "X")
+    m = X.shape[0]
+    Y = out if out is not None else torch.empty((m, P.n), dtype=torch.float16, device=X.device)
+    _dev_tensor(Y, "out")
+    need = ctypes.c_size_t(0)
+    _check(_lib().qx_q4x_gemm_splitk_workspace(P.n, P.k, m, ctypes.byref(need)), "qx_q4x_gemm_splitk_workspace")
+    ws = workspace if workspace is not None else splitk_workspace(X.device, int(need.value))
+    pc = P.c()
+    _check(_lib().qx_q4x_gemm_splitk(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _ptr(ws), ws.numel(),
+                                     GEMM_PDL if pdl else 0, _stream(X.device)), "qx_q4x_gemm_splitk")
+    return Y
 
 
 # ------------------------------------------------------------ save / load

@@ -7,12 +7,51 @@
 //                                                    GEMV on one matrix and on a two-entry launch
 //   harness gemm  n k bits g kind m sms in out     : quantize, then the tensor-core matmul: one
 //                                                    CTA per tile, split-k, split-k with PDL
+//   harness q4xgemm n k iters m sms in out         : Q4X learner, then the same three matmuls
+//                                                    on the Q4X weights
 // `in` holds W (fp16 [n][k]) and, for a8 and q4x, x (fp16 [batch][k]).
 #include <cstdio>
 #include <new>
 #include <string>
 
 #include "qx_kernels.cuh"
+
+namespace {
+template <class T>
+T *alloc(size_t bytes);
+void put(FILE *f, const void *p, size_t b);
+
+// qx_gemm, then qx_gemm_splitk twice on one workspace (the second with PDL):
+// Y, whether the split counters are back to zero, and the plan, per run.
+void three_matmuls(qx::GemmArgs base, int sms, FILE *fo) {
+    uint8_t *ws = nullptr;
+    for (int run = 0; run < 3; ++run) {
+        const qx::GemmPlan plan = qx::plan_gemm(base.n, base.k, base.m, sms, run > 0);
+        qx::GemmArgs a = base;
+        __half *Y = alloc<__half>(2 * base.m * base.n);
+        a.Y = Y;
+        a.bn = plan.bn;
+        a.splits = plan.splits;
+        a.pdl = run == 2;
+        if (plan.splits > 1) {
+            if (ws == nullptr) {
+                ws = alloc<uint8_t>(plan.ws_bytes);
+                std::memset(ws, 0, plan.ws_bytes);
+            }
+            a.ws_cnt = reinterpret_cast<uint32_t *>(ws);
+            a.ws_part = reinterpret_cast<float *>(ws + qx::kSplitCounterBytes);
+        }
+        qx::launch_gemm(a, sms, nullptr);
+        put(fo, Y, 2 * base.m * base.n);
+        uint32_t clean = 1;
+        if (plan.splits > 1)
+            for (size_t i = 0; i < qx::kSplitCounterBytes; ++i) clean &= ws[i] == 0;
+        put(fo, &clean, 4);
+        const uint32_t shape[2] = {(uint32_t)plan.bn, (uint32_t)plan.splits};
+        put(fo, shape, 8);
+    }
+}
+}  // namespace
 
 namespace {
 template <class T>
@@ -28,6 +67,48 @@ bool get(FILE *f, void *p, size_t b) { return fread(p, 1, b, f) == b; }
 int main(int argc, char **argv) {
     if (argc < 2) return 2;
     const std::string cmd = argv[1];
+    if (cmd == "q4xgemm") {  // n k iters m sms in out
+        if (argc != 9) return 2;
+        const int64_t n = atoll(argv[2]), k = atoll(argv[3]), m = atoll(argv[5]);
+        const int iters = atoi(argv[4]), sms = atoi(argv[6]);
+        FILE *fi = fopen(argv[7], "rb"), *fo = fopen(argv[8], "wb");
+        if (fi == nullptr || fo == nullptr) return 2;
+        const int G = (int)(k / 64), bb = (G + 3) / 4;
+        __half *W = alloc<__half>(2 * n * k), *X = alloc<__half>(2 * m * k);
+        if (!get(fi, W, 2 * n * k) || !get(fi, X, 2 * m * k)) return 2;
+        uint32_t *status = alloc<uint32_t>(4);
+        *status = 0;
+        uint8_t *codes = alloc<uint8_t>(n * k / 2), *books = alloc<uint8_t>(n * bb);
+        __half *scales = alloc<__half>(2 * n * G), *cbs = alloc<__half>(128);
+        void *ws = alloc<uint8_t>(qx::q4x_workspace_bytes(n, k));
+        qx::Q4xQuantArgs q{W, n, k, G, bb, iters, codes, scales, books, cbs, ws, status};
+        qx::launch_q4x_quantize(q, sms, nullptr);
+        put(fo, codes, n * k / 2);
+        put(fo, scales, 2 * n * G);
+        put(fo, books, n * bb);
+        put(fo, cbs, 128);
+        qx::GemmArgs a{};
+        a.codes = codes;
+        a.scales = scales;
+        a.zeros = books;     // Q4X: the 2-bit book indices
+        a.luts = cbs;        // Q4X: the four codebooks
+        a.n = n;
+        a.k = k;
+        a.m = m;
+        a.bits = 4;
+        a.kind = 2;
+        a.log2g = 6;
+        a.G = G;
+        a.zbytes = bb;
+        a.X = X;
+        a.status = status;
+        a.wait_limit_ns = 60000000000ull;
+        three_matmuls(a, sms, fo);
+        put(fo, status, 4);
+        fclose(fo);
+        fclose(fi);
+        return 0;
+    }
     const bool q4x = cmd == "q4x";
     const int want = q4x ? 9 : (cmd == "quant" || cmd == "gemv" || cmd == "gemm") ? 11 : 10;
     if (argc != want) return 2;
@@ -98,47 +179,23 @@ int main(int argc, char **argv) {
             if (!get(fi, X, 2 * m * k)) return 2;
             int l = 0;
             while ((1 << l) < g) ++l;
-            for (int run = 0; run < 3; ++run) {
-                const qx::GemmPlan plan = qx::plan_gemm(n, k, m, sms, run > 0);
-                qx::GemmArgs a{};
-                a.codes = codes;
-                a.scales = scales;
-                a.zeros = zeros;
-                a.luts = luts;
-                a.n = n;
-                a.k = k;
-                a.m = m;
-                a.bits = bits;
-                a.kind = kind;
-                a.log2g = l;
-                a.G = G;
-                a.zbytes = zb;
-                a.X = X;
-                __half *Y = alloc<__half>(2 * m * n);
-                a.Y = Y;
-                a.status = status;
-                a.wait_limit_ns = 60000000000ull;
-                a.bn = plan.bn;
-                a.splits = plan.splits;
-                a.pdl = run == 2;
-                static uint8_t *ws = nullptr;  // one workspace, reused by both split-k runs
-                if (plan.splits > 1) {
-                    if (ws == nullptr) {
-                        ws = alloc<uint8_t>(plan.ws_bytes);
-                        std::memset(ws, 0, plan.ws_bytes);
-                    }
-                    a.ws_cnt = reinterpret_cast<uint32_t *>(ws);
-                    a.ws_part = reinterpret_cast<float *>(ws + qx::kSplitCounterBytes);
-                }
-                qx::launch_gemm(a, sms, nullptr);
-                put(fo, Y, 2 * m * n);
-                uint32_t clean = 1;  // the counters are back to zero after every call
-                if (plan.splits > 1)
-                    for (size_t i = 0; i < qx::kSplitCounterBytes; ++i) clean &= ws[i] == 0;
-                put(fo, &clean, 4);
-                const uint32_t shape[2] = {(uint32_t)plan.bn, (uint32_t)plan.splits};
-                put(fo, shape, 8);
-            }
+            qx::GemmArgs a{};
+            a.codes = codes;
+            a.scales = scales;
+            a.zeros = zeros;
+            a.luts = luts;
+            a.n = n;
+            a.k = k;
+            a.m = m;
+            a.bits = bits;
+            a.kind = kind;
+            a.log2g = l;
+            a.G = G;
+            a.zbytes = zb;
+            a.X = X;
+            a.status = status;
+            a.wait_limit_ns = 60000000000ull;
+            three_matmuls(a, sms, fo);
         } else if (cmd == "gemv") {
             const int batch = extra;
             __half *x = alloc<__half>(2 * batch * k);

@@ -229,3 +229,22 @@ def test_cuda_errors_are_reported_with_their_name():
         status, name = line.split(" ", 1)
         assert status == "4" and name.startswith("cuda") and name != "cudaSuccess", line
     assert lines[2] == "1 1"  # limit outside 1 us .. 1 s
+
+
+def test_q4x_gemm_rejects_bad_arguments_before_launching(qx):
+    lib = qx._lib()
+    A = ctypes.c_void_p
+    good = qx._Q4x(64, 512, A(0x10000), A(0x20000), A(0x30000), A(0x40000))
+    assert lib.qx_q4x_gemm(None, A(0x1000), 4, A(0x2000), None) == 1
+    assert lib.qx_q4x_gemm(ctypes.byref(good), None, 4, A(0x2000), None) == 1
+    assert lib.qx_q4x_gemm(ctypes.byref(good), A(0x1000), 0, A(0x2000), None) == 1
+    assert lib.qx_q4x_gemm(ctypes.byref(good), A(0x1008), 4, A(0x2000), None) == 3
+    assert lib.qx_q4x_gemm(ctypes.byref(good), A(0x1000), 4, A(0x2001), None) == 3
+    k64 = qx._Q4x(64, 320, A(0x10000), A(0x20000), A(0x30000), A(0x40000))  # k not a multiple of 128
+    assert lib.qx_q4x_gemm(ctypes.byref(k64), A(0x1000), 4, A(0x2000), None) == 2
+    assert lib.qx_q4x_gemm_splitk(ctypes.byref(good), A(0x1000), 4, A(0x2000), None, 0, 2, None) == 1  # flag
+    assert lib.qx_q4x_gemm_splitk(ctypes.byref(k64), A(0x1000), 4, A(0x2000), None, 0, 0, None) == 2
+    nbytes = ctypes.c_size_t(0)
+    assert lib.qx_q4x_gemm_splitk_workspace(64, 320, 4, ctypes.byref(nbytes)) == 2
+    assert lib.qx_q4x_gemm_splitk_workspace(64, 512, 0, ctypes.byref(nbytes)) == 1
+    assert lib.qx_q4x_gemm_splitk_workspace(64, 512, 4, None) == 1

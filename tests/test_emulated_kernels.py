@@ -33,12 +33,22 @@ def harness(tmp_path_factory):
     sys.path.insert(0, HERE)
     import translate
 
-    cpps = translate.write_all(str(out))
+    import concurrent.futures as cf
+
+    cpps = translate.write_all(str(out)) + [os.path.join(HERE, "harness.cpp")]
+    flags = ["-std=c++20", "-O1", "-g", "-fsanitize=address,undefined", "-fno-sanitize-recover=undefined",
+             "-ffp-contract=off", "-Wno-unknown-pragmas", "-pthread", "-I", str(out), "-I", HERE]
+
+    def compile_one(src):
+        obj = str(out / (os.path.basename(src)[:-4] + ".o"))
+        r = subprocess.run([gxx, *flags, "-c", src, "-o", obj], capture_output=True, text=True)
+        assert r.returncode == 0, r.stderr[-3000:]
+        return obj
+
+    with cf.ThreadPoolExecutor(max_workers=len(cpps)) as ex:
+        objs = list(ex.map(compile_one, cpps))
     exe = str(out / "harness")
-    cmd = [gxx, "-std=c++20", "-O1", "-g", "-fsanitize=address,undefined", "-fno-sanitize-recover=undefined",
-           "-ffp-contract=off", "-Wno-unknown-pragmas", "-pthread", "-I", str(out), "-I", HERE, *cpps,
-           os.path.join(HERE, "harness.cpp"), "-o", exe]
-    r = subprocess.run(cmd, capture_output=True, text=True)
+    r = subprocess.run([gxx, *flags, *objs, "-o", exe], capture_output=True, text=True)
     assert r.returncode == 0, r.stderr[-3000:]
     return exe, out
 
@@ -160,6 +170,30 @@ def test_tensor_core_matmul(harness, n, k, bits, g, kind, m, sms):
         assert np.all(oracle.max_abs_err(Y, y_ref) <= tol)
         assert rd.take(1, np.uint32)[0] == 1  # counters rearmed
         rd.take(2, np.uint32)  # the plan: token tile, splits
+    assert rd.take(1, np.uint32)[0] == 0
+
+
+@pytest.mark.parametrize("n,k,iters,m,sms", [  # Q4X weights: 16-, 64- and 256-token tiles, 1..4 splits
+    (37, 384, 3, 5, 2), (128, 2048, 2, 16, 4), (200, 1024, 2, 40, 4), (64, 1152, 2, 300, 2)])
+def test_q4x_tensor_core_matmul(harness, n, k, iters, m, sms):
+    W = _weights(n, k, seed=n + m).astype(np.float16)
+    X = synth.activations(m, k, seed=m, stream=n)
+    rd = _run(harness, ["q4xgemm", n, k, iters, m, sms], np.concatenate([W.ravel(), X.astype(np.float16).ravel()]))
+    ref = oracle.quantize_q4x(W, iters=iters)
+    want = oracle.pack_q4x(ref)
+    G, bb = k // 64, (k // 64 + 3) // 4
+    assert np.array_equal(rd.take(n * k // 2, np.uint8).reshape(n, -1), want["codes"])
+    assert np.array_equal(rd.take(n * G, np.uint16).reshape(n, G), want["scales"].view(np.uint16))
+    assert np.array_equal(rd.take(n * bb, np.uint8).reshape(n, -1), want["books"])
+    assert np.array_equal(rd.take(64, np.uint16).reshape(4, 16), want["codebooks"].view(np.uint16))
+    y_ref = oracle.gemv_q4x(ref, X)
+    Wh = oracle.dequant_q4x(ref["codes"], ref["scales"], ref["books"], ref["codebooks"])
+    tol = oracle.tolerance(X, Wh) + np.abs(y_ref).max(axis=1) * 2.0 ** -11
+    for _ in range(3):
+        Y = rd.take(m * n, np.float16).reshape(m, n).astype(np.float64)
+        assert np.all(oracle.max_abs_err(Y, y_ref) <= tol)
+        assert rd.take(1, np.uint32)[0] == 1
+        rd.take(2, np.uint32)
     assert rd.take(1, np.uint32)[0] == 0
 
 

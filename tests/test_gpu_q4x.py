@@ -84,6 +84,38 @@ def test_gemv_within_tolerance(qx, learned, c, batch):
     assert np.all(oracle.max_abs_err(y, oracle.gemv_q4x(ref, x)) <= oracle.tolerance(x, Wh))
 
 
+@pytest.mark.parametrize("m", [1, 5, 17, 200])
+@pytest.mark.parametrize("c", CASES, ids=_ids)
+def test_tensor_core_matmul_within_tolerance(qx, learned, c, m):
+    """Prefill on the tensor cores (qx_q4x_gemm and the split-k form) against
+    the oracle; k must be a multiple of 128, else the call is refused."""
+    _, P, ref = learned[c]
+    X = torch.from_numpy(synth.activations(m, c[1], seed=m, stream=c[0] + 2)).cuda()
+    if c[1] % 128:
+        with pytest.raises(qx.QxError):
+            qx.q4x_gemm(P, X)
+        return
+    Xn = X.cpu().numpy()
+    y_ref = oracle.gemv_q4x(ref, Xn)
+    Wh = oracle.dequant_q4x(ref["codes"], ref["scales"], ref["books"], ref["codebooks"])
+    tol = oracle.tolerance(Xn, Wh) + np.abs(y_ref).max(axis=1) * 2.0 ** -11  # fp16 output
+    Y = qx.q4x_gemm(P, X).cpu().numpy().astype(np.float64)
+    Ys = qx.q4x_gemm_splitk(P, X).cpu().numpy().astype(np.float64)
+    assert qx.device_status() == 0
+    assert np.all(oracle.max_abs_err(Y, y_ref) <= tol)
+    assert np.all(oracle.max_abs_err(Ys, y_ref) <= tol)
+
+
+def test_split_k_repeats_and_pdl_are_bit_identical(qx, learned):
+    _, P, _ = learned[(96, 4096, 1)]
+    X = torch.from_numpy(synth.activations(16, 4096, seed=3, stream=3)).cuda()
+    a = qx.q4x_gemm_splitk(P, X)
+    b = qx.q4x_gemm_splitk(P, X)
+    c = qx.q4x_gemm_splitk(P, X, pdl=True)
+    assert qx.device_status() == 0
+    assert torch.equal(a, b) and torch.equal(b, c)
+
+
 def test_gemv_fp16_output(qx, learned):
     c = CASES[5]
     _, P, ref = learned[c]
@@ -191,3 +223,8 @@ def test_full_size_llama_projection(qx):
         x = synth.activations(batch, k, seed=batch, stream=11)
         y = qx.q4x_gemv(P, torch.from_numpy(x).cuda(), out_dtype=torch.float32).cpu().numpy()
         assert np.all(oracle.max_abs_err(y, oracle.gemv_q4x(ref, x)) <= oracle.tolerance(x, Wh))
+    # a 512-token prefill on the tensor cores
+    X = synth.activations(512, k, seed=5, stream=11)
+    Y = qx.q4x_gemm(P, torch.from_numpy(X).cuda()).cpu().numpy().astype(np.float64)
+    y_ref = oracle.gemv_q4x(ref, X)
+    assert np.all(oracle.max_abs_err(Y, y_ref) <= oracle.tolerance(X, Wh) + np.abs(y_ref).max(axis=1) * 2.0 ** -11)
