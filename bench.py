@@ -448,7 +448,7 @@ def run_ours(args):
         extra["config5"] = run_config5(qx, torch, dev, stream)
         torch.cuda.empty_cache()
         try:  # last: its result or its error is reported, the sections above stand
-            extra["q4x"] = run_q4x(qx, torch, dev, stream, l2, hbm)
+            extra["q4x"] = run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst)
         except Exception as e:  # noqa: BLE001
             extra["q4x"] = {"error": f"{type(e).__name__}: {e}"[:300]}
 
@@ -643,13 +643,14 @@ def run_config3(qx, torch, dev, stream, l2):
     return out
 
 
-def run_q4x(qx, torch, dev, stream, l2, hbm):
+def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
     """Q4X shared codebooks (groups of 64 with an fp16 scale and a 2-bit book
     index, 4-bit codes, four 16-level codebooks learned per matrix): the
     learner's device time per Llama-7B layer matrix, and the decode matmul over
     the layer at batch 1 and 4 (q,k,v | o | gate,up | down: four
     qx_q4x_gemv_multi launches per layer copy in one CUDA graph, weights
-    rotated over copies larger than 4x L2)."""
+    rotated over copies larger than 4x L2), and the tensor-core prefill
+    (qx_q4x_gemm) at M = 2048 against the two MLP shapes."""
     import synth
 
     def learn(name, n, k, sigma, sid):
@@ -702,6 +703,29 @@ def run_q4x(qx, torch, dev, stream, l2, hbm):
             "path": "4 qx_q4x_gemv_multi launches (persistent warps over the rows, codebooks in shared memory)"}
     if qx.device_status(stream) != 0:
         raise RuntimeError("q4x decode reported a device error")
+    # prefill on the tensor cores (qx_q4x_gemm): M = 2048 tokens against the two
+    # MLP shapes, as the per-group prefill benchmark
+    del layers
+    pre = {}
+    for nm in ("gate_proj", "down_proj"):
+        P = base[nm]
+        X = synth.activations_torch(GEMM_M, P.k, seed=3, stream=80, device=dev)
+        Y = torch.empty((GEMM_M, P.n), dtype=torch.float16, device=dev)
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                qx.q4x_gemm(P, X, out=Y)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            e0.record(stream)
+            for _ in range(10):
+                qx.q4x_gemm(P, X, out=Y)
+            e1.record(stream)
+        torch.cuda.synchronize(dev)
+        us = e0.elapsed_time(e1) * 1e3 / 10
+        tflops = 2.0 * GEMM_M * P.n * P.k / (us * 1e-6) / 1e12
+        pre[f"{P.n}x{P.k}"] = {"us": us, "TFLOPs": tflops, "frac_of_measured_bf16": tflops / tf_burst}
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("q4x prefill reported a device error")
+    out[f"prefill_m{GEMM_M}"] = pre
     return out
 
 
