@@ -20,3 +20,10 @@ def cuda_dev():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     return torch.device("cuda:0")
+
+
+@pytest.fixture(scope="session")
+def emulation_dir(tmp_path_factory):
+    """One build directory for the host builds of the kernel sources (the
+    sanitizer tests share its objects)."""
+    return tmp_path_factory.mktemp("emulated")

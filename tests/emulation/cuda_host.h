@@ -641,3 +641,25 @@ inline cudaError_t cudaGetSymbolAddress(void **p, T &sym) {
     *p = static_cast<void *>(&sym);
     return cudaSuccess;
 }
+
+// ------------------------------------------------------------------ the C ABI's runtime calls
+// One emulated device; its SM count comes from QX_EMU_SMS (default 4).
+enum cudaDeviceAttr { cudaDevAttrMultiProcessorCount = 16 };
+enum cudaMemcpyKind { cudaMemcpyHostToHost = 0, cudaMemcpyHostToDevice = 1, cudaMemcpyDeviceToHost = 2,
+                      cudaMemcpyDeviceToDevice = 3, cudaMemcpyDefault = 4 };
+inline cudaError_t cudaDeviceGetAttribute(int *v, cudaDeviceAttr attr, int) {
+    if (attr != cudaDevAttrMultiProcessorCount) return cudaErrorInvalidValue;
+    const char *e = std::getenv("QX_EMU_SMS");
+    *v = e != nullptr ? std::atoi(e) : 4;
+    return *v > 0 ? cudaSuccess : cudaErrorInvalidValue;
+}
+inline cudaError_t cudaMemcpy(void *d, const void *s, size_t n, cudaMemcpyKind) {
+    std::memcpy(d, s, n);
+    return cudaSuccess;
+}
+inline cudaError_t cudaMemcpyAsync(void *d, const void *s, size_t n, cudaMemcpyKind, cudaStream_t) {
+    std::memcpy(d, s, n);
+    return cudaSuccess;
+}
+inline cudaError_t cudaStreamSynchronize(cudaStream_t) { return cudaSuccess; }
+inline const char *cudaGetErrorName(cudaError_t e) { return e == cudaSuccess ? "cudaSuccess" : "cudaErrorEmulated"; }

@@ -17,7 +17,7 @@ import re
 CSRC = os.path.join(os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__)))),
                     "paper_2505_07531_gb300", "csrc")
 FILES = ["qx_common.cuh", "qx_kernels.cuh", "qx_quant.cu", "qx_act8.cu", "qx_select.cu", "qx_q4x.cu",
-         "qx_gemv.cu", "qx_gemm.cu"]
+         "qx_gemv.cu", "qx_gemm.cu", "qx_api.cu"]
 
 # first match wins: longer instruction names before their prefixes
 BY_INSTRUCTION = [
@@ -98,3 +98,43 @@ def write_all(out_dir: str) -> list:
         if name.endswith(".cpp"):
             cpps.append(os.path.join(out_dir, name))
     return cpps
+
+
+INCLUDE = os.path.join(os.path.dirname(CSRC), "..", "include")
+FLAGS = ["-std=c++20", "-O1", "-g", "-fPIC", "-fsanitize=address,undefined", "-fno-sanitize-recover=undefined",
+         "-ffp-contract=off", "-Wno-unknown-pragmas", "-Wno-narrowing", "-Wno-psabi", "-pthread"]
+
+
+def build(gxx: str, out_dir: str, target: str) -> str:
+    """Translate, compile in parallel and link with the sanitizers.  target
+    "harness": the exact-size buffer executable (harness.cpp); "library": a
+    shared library exporting the C ABI (load it with the sanitizer runtimes
+    preloaded).  Returns the path built."""
+    import concurrent.futures as cf
+    import subprocess
+
+    here = os.path.dirname(os.path.abspath(__file__))
+    srcs = [os.path.join(out_dir, f[:-3] + ".cpp") for f in FILES if f.endswith(".cu")]
+    if not all(os.path.exists(f) for f in srcs):
+        srcs = write_all(out_dir)
+    if target == "harness":
+        srcs.append(os.path.join(here, "harness.cpp"))
+    inc = ["-I", out_dir, "-I", here, "-I", os.path.normpath(INCLUDE)]
+
+    def one(src):
+        obj = os.path.join(out_dir, os.path.basename(src).rsplit(".", 1)[0] + ".o")
+        if os.path.exists(obj) and os.path.getmtime(obj) >= os.path.getmtime(src):
+            return obj  # both targets share the objects of one build directory
+        r = subprocess.run([gxx, *FLAGS, *inc, "-c", src, "-o", obj], capture_output=True, text=True)
+        if r.returncode != 0:
+            raise RuntimeError(r.stderr[-3000:])
+        return obj
+
+    with cf.ThreadPoolExecutor(max_workers=len(srcs)) as ex:
+        objs = list(ex.map(one, srcs))
+    out = os.path.join(out_dir, "harness" if target == "harness" else "libqx_emulated.so")
+    link = [gxx, *FLAGS, *objs, "-o", out] + (["-shared"] if target == "library" else [])
+    r = subprocess.run(link, capture_output=True, text=True)
+    if r.returncode != 0:
+        raise RuntimeError(r.stderr[-3000:])
+    return out
