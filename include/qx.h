@@ -153,6 +153,23 @@ enum {
 qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const *x, int32_t batch,
                         void *const *y, int32_t y_dtype, int32_t flags, void *stream);
 
+/* One group of a qx_gemv_chain call: the arguments of one qx_gemv_multi. */
+typedef struct qx_gemv_group {
+    const qx_packed *mats;   /* count matrices sharing bits and kind */
+    int32_t count;           /* 1..8 */
+    const void *const *x;    /* count device pointers, as in qx_gemv_multi */
+    void *const *y;          /* count device pointers */
+} qx_gemv_group;
+
+/* A decode step in one call: qx_gemv_multi(groups[i]...) for i = 0..ngroups-1
+ * (ngroups 1..64) in order on `stream`, all with the same batch, y_dtype and
+ * flags (e.g. the q,k,v | o | gate,up | down groups of a decoder layer, with
+ * QX_GEMV_PDL).  The results equal the separate calls bit for bit; the host
+ * cost of the step is one call.  All groups are validated before the first
+ * launch; a failing group returns its status and nothing is launched. */
+qx_status qx_gemv_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                        int32_t flags, void *stream);
+
 /* Prefill matmul Y = X W_hat^T (Table 2 "Prefill") on the tcgen05 tensor cores:
  * W_hat tiles are dequantized into shared memory and multiplied in fp16 with
  * fp32 accumulation in tensor memory, 256 tokens per tile (16 when m <= 16).

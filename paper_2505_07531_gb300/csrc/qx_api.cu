@@ -342,8 +342,10 @@ QX_API qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void 
     return run_gemv(p, 1, &x, batch, &y, y_dtype, 0, static_cast<cudaStream_t>(stream), d);
 }
 
-QX_API qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const *x, int32_t batch,
-                               void *const *y, int32_t y_dtype, int32_t flags, void *stream) {
+namespace {
+
+qx_status check_gemv_multi(const qx_packed *mats, int32_t count, const void *const *x, int32_t batch,
+                           void *const *y, int32_t y_dtype, int32_t flags) {
     if (mats == nullptr || x == nullptr || y == nullptr || count < 1) return QX_ERR_INVALID_ARG;
     if (count > qx::kMaxGemvMats) return QX_ERR_UNSUPPORTED;
     if ((flags & ~QX_GEMV_PDL) != 0) return QX_ERR_INVALID_ARG;
@@ -353,10 +355,36 @@ QX_API qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void 
         if (mats[i].recipe.bits != mats[0].recipe.bits || mats[i].recipe.kind != mats[0].recipe.kind)
             return QX_ERR_INVALID_ARG;
     }
-    DeviceInfo *d = nullptr;
-    qx_status s = device_info(&d);
+    return QX_OK;
+}
+
+}  // namespace
+
+QX_API qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void *const *x, int32_t batch,
+                               void *const *y, int32_t y_dtype, int32_t flags, void *stream) {
+    qx_status s = check_gemv_multi(mats, count, x, batch, y, y_dtype, flags);
     if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
     return run_gemv(mats, count, x, batch, y, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
+}
+
+QX_API qx_status qx_gemv_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                               int32_t flags, void *stream) {
+    if (groups == nullptr || ngroups < 1 || ngroups > 64) return QX_ERR_INVALID_ARG;
+    qx_status s;
+    for (int i = 0; i < ngroups; ++i) {
+        const qx_gemv_group &g = groups[i];
+        if ((s = check_gemv_multi(g.mats, g.count, g.x, batch, g.y, y_dtype, flags)) != QX_OK) return s;
+    }
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    for (int i = 0; i < ngroups; ++i) {
+        const qx_gemv_group &g = groups[i];
+        s = run_gemv(g.mats, g.count, g.x, batch, g.y, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
+        if (s != QX_OK) return s;
+    }
+    return QX_OK;
 }
 
 namespace {

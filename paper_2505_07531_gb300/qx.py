@@ -59,6 +59,11 @@ class _Packed(ctypes.Structure):
                 ("zeros", ctypes.c_void_p), ("luts", ctypes.c_void_p)]
 
 
+class _GemvGroup(ctypes.Structure):
+    _fields_ = [("mats", ctypes.POINTER(_Packed)), ("count", ctypes.c_int32),
+                ("x", ctypes.POINTER(ctypes.c_void_p)), ("y", ctypes.POINTER(ctypes.c_void_p))]
+
+
 class _Q4x(ctypes.Structure):
     _fields_ = [("n", ctypes.c_int64), ("k", ctypes.c_int64), ("codes", ctypes.c_void_p),
                 ("scales", ctypes.c_void_p), ("books", ctypes.c_void_p), ("codebooks", ctypes.c_void_p)]
@@ -100,6 +105,7 @@ def _lib():
         lib.qx_select_recipe.argtypes = [VP, I64, I64, P(_Recipe), I32, ctypes.c_double, VP, ctypes.c_size_t,
                                          P(I32), P(ctypes.c_uint64), P(ctypes.c_double), VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
+        lib.qx_gemv_chain.argtypes = [P(_GemvGroup), I32, I32, I32, I32, VP]
         lib.qx_q4x_size.argtypes = [I64, I64, P(_Q4xSizes)]
         lib.qx_q4x_workspace.argtypes = [I64, I64, P(ctypes.c_size_t)]
         lib.qx_q4x_quantize.argtypes = [VP, I32, P(_Q4x), VP, ctypes.c_size_t, VP]
@@ -116,7 +122,7 @@ def _lib():
         lib.qx_version.argtypes = []
         lib.qx_last_error_string.argtypes = []
         lib.qx_last_error_string.restype = ctypes.c_char_p
-        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemm",
+        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemv_chain", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
                    "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_q4x_gemm", "qx_q4x_gemm_splitk_workspace",
@@ -286,6 +292,49 @@ def gemv_multi(mats, xs, outs=None, out_dtype=torch.float16, pdl: bool = False):
     _check(_lib().qx_gemv_multi(arr, len(mats), xp, b, yp, code, GEMV_PDL if pdl else 0, _stream(xs[0].get_device())),
            "qx_gemv_multi")
     return ys
+
+
+class GemvChain:
+    """A decode step as one qx_gemv_chain call.  `groups` lists (matrices, xs,
+    outs) triples, each the arguments of one gemv_multi (same batch and output
+    dtype throughout); the ctypes arguments are built here once, so calling
+    the object costs one library call.  Build a new chain if any of the
+    tensors is replaced."""
+
+    def __init__(self, groups, pdl: bool = True):
+        self._keep, built = [], []
+        batch, dt, dev = None, None, None
+        for mats, xs, outs in groups:
+            mats, xs, outs = list(mats), list(xs), list(outs)
+            if not (len(mats) == len(xs) == len(outs)) or not 1 <= len(mats) <= 8:
+                raise ValueError("each group: 1..8 matrices, one x and one output per matrix")
+            for P, x, y in zip(mats, xs, outs):
+                x2 = x.view(-1, P.k)
+                _dev_tensor(x2, "x")
+                b = x2.shape[0]
+                batch = b if batch is None else batch
+                dt = y.dtype if dt is None else dt
+                dev = x.device if dev is None else dev
+                if b != batch or y.dtype != dt or tuple(y.shape) != (b, P.n):
+                    raise ValueError("every group must share the batch and the output dtype")
+                _dev_tensor(y, "out", dt)
+            cnt = len(mats)
+            pa = (_Packed * cnt)(*[P.c() for P in mats])
+            xa = (ctypes.c_void_p * cnt)(*[x.data_ptr() for x in xs])
+            ya = (ctypes.c_void_p * cnt)(*[y.data_ptr() for y in outs])
+            self._keep += [pa, xa, ya, mats, xs, outs]
+            built.append(_GemvGroup(ctypes.cast(pa, ctypes.POINTER(_Packed)), cnt,
+                                    ctypes.cast(xa, ctypes.POINTER(ctypes.c_void_p)),
+                                    ctypes.cast(ya, ctypes.POINTER(ctypes.c_void_p))))
+        if not built:
+            raise ValueError("no groups")
+        self._groups = (_GemvGroup * len(built))(*built)
+        self._args = (self._groups, len(built), batch, F32 if dt == torch.float32 else F16,
+                      GEMV_PDL if pdl else 0)
+        self._dev = dev
+
+    def __call__(self):
+        _check(_lib().qx_gemv_chain(*self._args, _stream(self._dev)), "qx_gemv_chain")
 
 
 def gemm(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:

@@ -114,6 +114,32 @@ def check_per_group(n, k, bits, g, kind):
                        (ctypes.c_void_p * 3)(*[P(v) for v in ys]), 1, 1, None), "qx_gemv_multi")
     for v in ys:
         within(v.reshape(2, n), oracle.gemv(ref, orec, x, k), oracle.tolerance(x, Wh))
+    # a decode step as one call: groups (S, S) and (S), each equal to its qx_gemv_multi
+    VPA = ctypes.POINTER(ctypes.c_void_p)
+
+    def group(mlist, xs, ys_):
+        c = len(mlist)
+        pa, xa, ya = (qx._Packed * c)(*mlist), (ctypes.c_void_p * c)(*xs), (ctypes.c_void_p * c)(*ys_)
+        _keep.extend([pa, xa, ya])
+        return qx._GemvGroup(ctypes.cast(pa, ctypes.POINTER(qx._Packed)), c, ctypes.cast(xa, VPA),
+                             ctypes.cast(ya, VPA))
+
+    yc = [buf(8 * n, np.float32, fill=np.nan) for _ in range(3)]
+    ok(L.qx_gemv_chain((qx._GemvGroup * 2)(group([S, S], [P(xd)] * 2, [P(yc[0]), P(yc[1])]),
+                                           group([S], [P(xd)], [P(yc[2])])), 2, 2, 1, 1, None), "qx_gemv_chain")
+    sep = [buf(8 * n, np.float32) for _ in range(3)]
+    ok(L.qx_gemv_multi((qx._Packed * 2)(S, S), 2, (ctypes.c_void_p * 2)(P(xd), P(xd)), 2,
+                       (ctypes.c_void_p * 2)(P(sep[0]), P(sep[1])), 1, 1, None), "multi (S, S)")
+    ok(L.qx_gemv_multi((qx._Packed * 1)(S), 1, (ctypes.c_void_p * 1)(P(xd)), 2, (ctypes.c_void_p * 1)(P(sep[2])),
+                       1, 1, None), "multi (S)")
+    for a_, b_ in zip(yc, sep):
+        assert np.array_equal(a_, b_), "chain equals the separate calls"
+    untouched = buf(8 * n, np.float32, fill=np.nan)
+    bad_y = buf(8 * n + 4, np.uint8)[2:]  # misaligned output of the second group
+    assert L.qx_gemv_chain((qx._GemvGroup * 2)(group([S], [P(xd)], [P(untouched)]),
+                                               group([S], [P(xd)], [ctypes.c_void_p(bad_y.ctypes.data)])),
+                           2, 2, 1, 1, None) == 3, "misaligned y"
+    assert np.isnan(untouched).all(), "nothing launched when a later group is invalid"
     # prefill: one CTA per tile, split-k (twice on one workspace, the second with PDL), no-alloc
     for m in (3, 17, 200):
         X = synth.activations(m, k, seed=m, stream=n)
