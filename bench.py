@@ -422,20 +422,23 @@ def run_ours(args):
     # back (one copy), then a stream synchronisation, per step
     hx = x_flat.cpu().pin_memory()
     hy = torch.empty(y_flat.shape, dtype=y_flat.dtype).pin_memory()
-    # a step is one qx_gemv_chain call (its arguments bound once per weight
-    # copy); a chain that cannot be built or run falls back to the four calls
-    e2e_step, e2e_path = step, "4 qx_gemv_multi calls per step"
+    # a step is one qx_decode_step call (copy in, the four launches, copy out,
+    # synchronize; arguments bound once per weight copy); if it cannot be built
+    # or run, the step is the torch copies around the four qx_gemv_multi calls
+    e2e_call, e2e_path = None, "torch copies + 4 qx_gemv_multi calls + synchronize per step"
     try:
-        chains = [qx.GemvChain([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
-                                for names, x in CHAIN]) for c in range(copies)]
+        dsteps = [qx.DecodeStep([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
+                                 for names, x in CHAIN], h2d=[(x_flat, hx)], d2h=[(hy, y_flat)])
+                  for c in range(copies)]
         with torch.cuda.stream(stream):
-            for ch in chains:
-                ch()
+            for ds in dsteps:
+                ds()
         if qx.device_status(stream) != 0:
-            raise RuntimeError("device status after the chain")
-        e2e_step, e2e_path = (lambda c: chains[c]()), "1 qx_gemv_chain call per step (4 PDL launches)"
+            raise RuntimeError("device status after the decode step")
+        e2e_call = lambda c: dsteps[c]()  # noqa: E731
+        e2e_path = "1 qx_decode_step call per step: copy in, 4 PDL launches, copy out, synchronize"
     except Exception as e:  # noqa: BLE001
-        e2e_path += f" (chain unavailable: {type(e).__name__}: {e})"[:200]
+        e2e_path += f" (decode step unavailable: {type(e).__name__}: {e})"[:200]
     e2e_steps = max(3, min(args.steps, 2000))
     if dist is not None:
         dist.barrier()
@@ -444,8 +447,11 @@ def run_ours(args):
     with torch.cuda.stream(stream):
         for i in range(e2e_steps):
             c = i % copies
+            if e2e_call is not None:
+                e2e_call(c)
+                continue
             x_flat.copy_(hx, non_blocking=True)
-            e2e_step(c)
+            step(c)
             hy.copy_(y_flat, non_blocking=True)
             stream.synchronize()
     e2e_ms = _max_over_ranks(dist, (time.perf_counter() - t0) * 1e3 / e2e_steps, dev)

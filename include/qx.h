@@ -170,6 +170,24 @@ typedef struct qx_gemv_group {
 qx_status qx_gemv_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
                         int32_t flags, void *stream);
 
+/* A copy of a decode step: `bytes` from src to dst (host to device for the
+ * inputs, device to host for the outputs). */
+typedef struct qx_copy {
+    void *dst;
+    const void *src;
+    size_t bytes;
+} qx_copy;
+
+/* A whole decode step in one call, in order on `stream`: the nin copies `in`
+ * (host to device; pinned host memory keeps them asynchronous), the groups as
+ * in qx_gemv_chain, the nout copies `out` (device to host), then, when sync is
+ * non-zero, a synchronization of the stream (the outputs are then in host
+ * memory).  nin, nout 0..16.  Every group is validated before the first copy;
+ * a failing argument returns its status and nothing is issued. */
+qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
+                         int32_t batch, int32_t y_dtype, int32_t flags, const qx_copy *out, int32_t nout,
+                         int32_t sync, void *stream);
+
 /* Prefill matmul Y = X W_hat^T (Table 2 "Prefill") on the tcgen05 tensor cores:
  * W_hat tiles are dequantized into shared memory and multiplied in fp16 with
  * fp32 accumulation in tensor memory, 256 tokens per tile (16 when m <= 16).

@@ -369,22 +369,65 @@ QX_API qx_status qx_gemv_multi(const qx_packed *mats, int32_t count, const void 
     return run_gemv(mats, count, x, batch, y, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
 }
 
-QX_API qx_status qx_gemv_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
-                               int32_t flags, void *stream) {
+namespace {
+
+qx_status check_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype, int32_t flags) {
     if (groups == nullptr || ngroups < 1 || ngroups > 64) return QX_ERR_INVALID_ARG;
-    qx_status s;
     for (int i = 0; i < ngroups; ++i) {
         const qx_gemv_group &g = groups[i];
-        if ((s = check_gemv_multi(g.mats, g.count, g.x, batch, g.y, y_dtype, flags)) != QX_OK) return s;
-    }
-    DeviceInfo *d = nullptr;
-    if ((s = device_info(&d)) != QX_OK) return s;
-    for (int i = 0; i < ngroups; ++i) {
-        const qx_gemv_group &g = groups[i];
-        s = run_gemv(g.mats, g.count, g.x, batch, g.y, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
+        const qx_status s = check_gemv_multi(g.mats, g.count, g.x, batch, g.y, y_dtype, flags);
         if (s != QX_OK) return s;
     }
     return QX_OK;
+}
+
+qx_status run_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype, int32_t flags,
+                    cudaStream_t st, DeviceInfo *d) {
+    for (int i = 0; i < ngroups; ++i) {
+        const qx_gemv_group &g = groups[i];
+        const qx_status s = run_gemv(g.mats, g.count, g.x, batch, g.y, y_dtype, flags, st, d);
+        if (s != QX_OK) return s;
+    }
+    return QX_OK;
+}
+
+qx_status check_copies(const qx_copy *c, int32_t n) {
+    if (n < 0 || n > 16 || (n > 0 && c == nullptr)) return QX_ERR_INVALID_ARG;
+    for (int i = 0; i < n; ++i)
+        if (c[i].dst == nullptr || c[i].src == nullptr) return QX_ERR_INVALID_ARG;
+    return QX_OK;
+}
+
+}  // namespace
+
+QX_API qx_status qx_gemv_chain(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                               int32_t flags, void *stream) {
+    qx_status s = check_chain(groups, ngroups, batch, y_dtype, flags);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    return run_chain(groups, ngroups, batch, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
+}
+
+QX_API qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
+                                int32_t batch, int32_t y_dtype, int32_t flags, const qx_copy *out, int32_t nout,
+                                int32_t sync, void *stream) {
+    qx_status s = check_copies(in, nin);
+    if (s == QX_OK) s = check_copies(out, nout);
+    if (s == QX_OK) s = check_chain(groups, ngroups, batch, y_dtype, flags);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    for (int i = 0; i < nin; ++i)
+        if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
+            return s;
+    if ((s = run_chain(groups, ngroups, batch, y_dtype, flags, st, d)) != QX_OK) return s;
+    for (int i = 0; i < nout; ++i)
+        if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
+            QX_OK)
+            return s;
+    return sync ? from_cuda(cudaStreamSynchronize(st)) : QX_OK;
 }
 
 namespace {

@@ -64,6 +64,10 @@ class _GemvGroup(ctypes.Structure):
                 ("x", ctypes.POINTER(ctypes.c_void_p)), ("y", ctypes.POINTER(ctypes.c_void_p))]
 
 
+class _Copy(ctypes.Structure):
+    _fields_ = [("dst", ctypes.c_void_p), ("src", ctypes.c_void_p), ("bytes", ctypes.c_size_t)]
+
+
 class _Q4x(ctypes.Structure):
     _fields_ = [("n", ctypes.c_int64), ("k", ctypes.c_int64), ("codes", ctypes.c_void_p),
                 ("scales", ctypes.c_void_p), ("books", ctypes.c_void_p), ("codebooks", ctypes.c_void_p)]
@@ -106,6 +110,7 @@ def _lib():
                                          P(I32), P(ctypes.c_uint64), P(ctypes.c_double), VP]
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_gemv_chain.argtypes = [P(_GemvGroup), I32, I32, I32, I32, VP]
+        lib.qx_decode_step.argtypes = [P(_Copy), I32, P(_GemvGroup), I32, I32, I32, I32, P(_Copy), I32, I32, VP]
         lib.qx_q4x_size.argtypes = [I64, I64, P(_Q4xSizes)]
         lib.qx_q4x_workspace.argtypes = [I64, I64, P(ctypes.c_size_t)]
         lib.qx_q4x_quantize.argtypes = [VP, I32, P(_Q4x), VP, ctypes.c_size_t, VP]
@@ -122,7 +127,7 @@ def _lib():
         lib.qx_version.argtypes = []
         lib.qx_last_error_string.argtypes = []
         lib.qx_last_error_string.restype = ctypes.c_char_p
-        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemv_chain", "qx_gemm",
+        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemv_chain", "qx_decode_step", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
                    "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_q4x_gemm", "qx_q4x_gemm_splitk_workspace",
@@ -335,6 +340,39 @@ class GemvChain:
 
     def __call__(self):
         _check(_lib().qx_gemv_chain(*self._args, _stream(self._dev)), "qx_gemv_chain")
+
+
+class DecodeStep(GemvChain):
+    """A whole decode step as one qx_decode_step call: the host-to-device
+    copies `h2d` [(device tensor, host tensor)], the groups of a GemvChain, the
+    device-to-host copies `d2h` [(host tensor, device tensor)], then (sync) a
+    synchronization of the stream.  Host tensors should be pinned.  Arguments
+    are bound once; build a new step if a tensor is replaced."""
+
+    def __init__(self, groups, h2d=(), d2h=(), pdl: bool = True, sync: bool = True):
+        super().__init__(groups, pdl)
+
+        def copies(pairs, to_device):
+            arr = []
+            for dst, src in pairs:
+                if dst.is_cuda != to_device or src.is_cuda == to_device:
+                    raise ValueError("h2d pairs are (device, host), d2h pairs (host, device)")
+                if not (dst.is_contiguous() and src.is_contiguous()):
+                    raise ValueError("copies need contiguous tensors")
+                nb = src.numel() * src.element_size()
+                if dst.numel() * dst.element_size() != nb:
+                    raise ValueError("a copy's two tensors differ in size")
+                arr.append(_Copy(dst.data_ptr(), src.data_ptr(), nb))
+                self._keep += [dst, src]
+            return ((_Copy * len(arr))(*arr) if arr else None), len(arr)
+
+        self._in, nin = copies(list(h2d), True)
+        self._out, nout = copies(list(d2h), False)
+        groups_arr, ng, batch, ydt, flags = self._args
+        self._step = (self._in, nin, groups_arr, ng, batch, ydt, flags, self._out, nout, 1 if sync else 0)
+
+    def __call__(self):
+        _check(_lib().qx_decode_step(*self._step, _stream(self._dev)), "qx_decode_step")
 
 
 def gemm(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:

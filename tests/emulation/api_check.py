@@ -140,6 +140,19 @@ def check_per_group(n, k, bits, g, kind):
                                                group([S], [P(xd)], [ctypes.c_void_p(bad_y.ctypes.data)])),
                            2, 2, 1, 1, None) == 3, "misaligned y"
     assert np.isnan(untouched).all(), "nothing launched when a later group is invalid"
+    # the whole step in one call: host x in, the groups, host y out, synchronize
+    hx = put(x)
+    dx = buf(x.nbytes, np.float16)
+    dys = [buf(8 * n, np.float32) for _ in range(3)]
+    hys = [buf(8 * n, np.float32, fill=np.nan) for _ in range(3)]
+    cin = (qx._Copy * 1)(qx._Copy(dx.ctypes.data, hx.ctypes.data, x.nbytes))
+    cout = (qx._Copy * 3)(*[qx._Copy(h.ctypes.data, d.ctypes.data, h.nbytes) for h, d in zip(hys, dys)])
+    steps = (qx._GemvGroup * 2)(group([S, S], [P(dx)] * 2, [P(dys[0]), P(dys[1])]), group([S], [P(dx)], [P(dys[2])]))
+    ok(L.qx_decode_step(cin, 1, steps, 2, 2, 1, 1, cout, 3, 1, None), "qx_decode_step")
+    for a_, b_ in zip(hys, sep):
+        assert np.array_equal(a_, b_), "decode step equals the separate calls"
+    assert L.qx_decode_step(cin, 17, steps, 2, 2, 1, 1, cout, 3, 1, None) == 1, "too many copies"
+    assert L.qx_decode_step(None, 1, steps, 2, 2, 1, 1, cout, 3, 1, None) == 1, "missing copy list"
     # prefill: one CTA per tile, split-k (twice on one workspace, the second with PDL), no-alloc
     for m in (3, 17, 200):
         X = synth.activations(m, k, seed=m, stream=n)

@@ -265,3 +265,22 @@ def test_gemv_chain_rejects_bad_arguments_before_launching(qx):
     assert lib.qx_gemv_chain((qx._GemvGroup * 1)(g), 1, 1, 0, 2, None) == 1    # unknown flag
     bad = qx._GemvGroup(ctypes.cast(mats, ctypes.POINTER(qx._Packed)), 0, ctypes.cast(xs, VPA), ctypes.cast(ys, VPA))
     assert lib.qx_gemv_chain((qx._GemvGroup * 2)(g, bad), 2, 1, 0, 0, None) == 1  # count 0 in the second group
+
+
+def test_decode_step_rejects_bad_arguments_before_launching(qx):
+    lib = qx._lib()
+    A = ctypes.c_void_p
+    P3 = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), A(0x1000), A(0x2000), A(0x3000), None)
+    mats = (qx._Packed * 1)(P3)
+    xs, ys = (A * 1)(A(0x4000)), (A * 1)(A(0x5000))
+    VPA = ctypes.POINTER(ctypes.c_void_p)
+    g = (qx._GemvGroup * 1)(qx._GemvGroup(ctypes.cast(mats, ctypes.POINTER(qx._Packed)), 1, ctypes.cast(xs, VPA),
+                                          ctypes.cast(ys, VPA)))
+    c = (qx._Copy * 1)(qx._Copy(0x4000, 0x9000, 256))
+    nul = (qx._Copy * 1)(qx._Copy(0x4000, None, 256))
+    assert lib.qx_decode_step(c, 17, g, 1, 1, 0, 0, c, 1, 1, None) == 1
+    assert lib.qx_decode_step(c, 1, g, 1, 1, 0, 0, c, -1, 1, None) == 1
+    assert lib.qx_decode_step(None, 1, g, 1, 1, 0, 0, None, 0, 1, None) == 1
+    assert lib.qx_decode_step(nul, 1, g, 1, 1, 0, 0, None, 0, 1, None) == 1
+    assert lib.qx_decode_step(c, 1, None, 1, 1, 0, 0, None, 0, 1, None) == 1
+    assert lib.qx_decode_step(c, 1, g, 1, 17, 0, 0, None, 0, 1, None) == 2

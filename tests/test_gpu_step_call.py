@@ -34,3 +34,21 @@ def test_chain_equals_the_separate_calls(qx, batch):
         for nm, y in zip(names, sep):
             assert torch.equal(ys[nm], y), nm
     assert qx.device_status() == 0
+
+
+def test_decode_step_copies_in_and_out(qx):
+    """qx_decode_step: pinned host x in, the groups, host y out, synchronized:
+    the host outputs equal the device results of the separate calls."""
+    rec = qx.Recipe(4, 128, qx.UNIFORM)
+    mats = [qx.quantize(torch.from_numpy(synth.student_t_weights(n, 512, 0.02, seed=n, stream=1)).cuda(), rec)
+            for n in (256, 384)]
+    hx = torch.from_numpy(synth.activations(2, 512, seed=3, stream=3)).pin_memory()
+    dx = torch.empty(hx.shape, dtype=hx.dtype, device="cuda")
+    dys = [torch.empty((2, P.n), dtype=torch.float16, device="cuda") for P in mats]
+    hys = [torch.full((2, P.n), float("nan"), dtype=torch.float16).pin_memory() for P in mats]
+    step = qx.DecodeStep([(mats, [dx, dx], dys)], h2d=[(dx, hx)], d2h=list(zip(hys, dys)))
+    step()
+    ref = qx.gemv_multi(mats, [hx.cuda(), hx.cuda()])
+    for h, r in zip(hys, ref):
+        assert torch.equal(h, r.cpu())
+    assert qx.device_status() == 0
