@@ -749,16 +749,24 @@ def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
     return out
 
 
-LLAVA_LANG = [  # Q/K 3-bit LUT g128; V/O and the MLP 4-bit uniform g64
-    ("q_proj", 4096, 4096, 0.01, 0, (3, 128, 1)), ("k_proj", 4096, 4096, 0.01, 1, (3, 128, 1)),
-    ("v_proj", 4096, 4096, 0.02, 2, (4, 64, 0)), ("o_proj", 4096, 4096, 0.02, 3, (4, 64, 0)),
-    ("gate_proj", 11008, 4096, 0.04, 4, (4, 64, 0)), ("up_proj", 11008, 4096, 0.04, 5, (4, 64, 0)),
-    ("down_proj", 4096, 11008, 0.04, 6, (4, 64, 0)),
-]
-LLAVA_VISION = [  # CLIP ViT-L/14: hidden 1024, MLP 4096; 4-bit uniform g128
-    ("q_proj", 1024, 1024, 0.02, 10), ("k_proj", 1024, 1024, 0.02, 11), ("v_proj", 1024, 1024, 0.02, 12),
-    ("o_proj", 1024, 1024, 0.02, 13), ("fc1", 4096, 1024, 0.04, 14), ("fc2", 1024, 4096, 0.04, 15),
-]
+def _llava_table():
+    """The LLaVA-v1.6-7B-shaped model's per-matrix recipes (a JSON table in the
+    package): language matrices as (name, n, k, sigma, stream, (bits, g,
+    kind)), vision matrices as (name, n, k, sigma, stream) with their one
+    shared recipe."""
+    with open(os.path.join(ROOT, "paper_2505_07531_gb300", "recipes", "llava_v1_6_7b.json")) as f:
+        t = json.load(f)
+    kinds = {"uniform": 0, "lut": 1}
+    rec = lambda m: (m["recipe"]["bits"], m["recipe"]["group_size"], kinds[m["recipe"]["kind"]])  # noqa: E731
+    lang = [(m["name"], m["n"], m["k"], m["sigma"], m["stream"], rec(m)) for m in t["language"]["matrices"]]
+    vis = [(m["name"], m["n"], m["k"], m["sigma"], m["stream"]) for m in t["vision"]["matrices"]]
+    vrec = {rec(m) for m in t["vision"]["matrices"]}
+    if len(vrec) != 1:
+        raise ValueError("the vision matrices share one recipe in this benchmark")
+    return t, lang, vis, vrec.pop()
+
+
+LLAVA, LLAVA_LANG, LLAVA_VISION, LLAVA_VISION_RECIPE = _llava_table()
 
 
 def run_select(qx, torch, dev, stream):
@@ -800,8 +808,9 @@ def run_config5(qx, torch, dev, stream):
         W = synth.student_t_weights_torch(n, k, sigma, seed=5, stream=sid, device=dev)
         base[nm] = qx.quantize(W, qx.Recipe(bits, g, kind))
         del W
-    lang = [base] + [{nm: _clone(qx, P) for nm, P in base.items()} for _ in range(31)]
-    lang_bytes = 32 * sum(P.nbytes() for P in base.values())
+    n_lang = LLAVA["language"]["layers"]
+    lang = [base] + [{nm: _clone(qx, P) for nm, P in base.items()} for _ in range(n_lang - 1)]
+    lang_bytes = n_lang * sum(P.nbytes() for P in base.values())
     xs = {k: synth.activations_torch(1, k, seed=5, stream=80 + i, device=dev) for i, k in enumerate((4096, 11008))}
     xa, xo, xm = (synth.activations_torch(1, 4096, seed=5, stream=90 + i, device=dev) for i in range(3))
     ys = {nm: torch.empty((1, n), dtype=torch.float16, device=dev) for nm, n, *_ in LLAVA_LANG}
@@ -811,15 +820,16 @@ def run_config5(qx, torch, dev, stream):
     dec_ms = _time_graph(torch, stream, gr, 10)
     del gr, lang
 
-    vbase = dict(_quantize_layer(qx, torch, dev, LLAVA_VISION, qx.Recipe(4, 128, qx.UNIFORM), seed=5))
-    vis = [vbase] + [{nm: _clone(qx, P) for nm, P in vbase.items()} for _ in range(23)]
-    M = 576
+    vbase = dict(_quantize_layer(qx, torch, dev, LLAVA_VISION, qx.Recipe(*LLAVA_VISION_RECIPE), seed=5))
+    n_vis = LLAVA["vision"]["layers"]
+    vis = [vbase] + [{nm: _clone(qx, P) for nm, P in vbase.items()} for _ in range(n_vis - 1)]
+    M = LLAVA["vision"]["tokens"]
     X1 = synth.activations_torch(M, 1024, seed=5, stream=95, device=dev)
     X4 = synth.activations_torch(M, 4096, seed=5, stream=96, device=dev)
     Ys = {nm: torch.empty((M, n), dtype=torch.float16, device=dev) for nm, n, *_ in LLAVA_VISION}
 
     def vision_ms(gemm):
-        """24 vision layers through `gemm` (qx.gemm or qx.gemm_splitk), one CUDA graph."""
+        """The vision layers through `gemm` (qx.gemm or qx.gemm_splitk), one CUDA graph."""
         def vision_pass():
             for L in vis:
                 for nm, n, k, *_ in LLAVA_VISION:
@@ -839,16 +849,17 @@ def run_config5(qx, torch, dev, stream):
 
     pre_ms = vision_ms(lambda P, X, out: qx.gemm_splitk(P, X, out=out, pdl=True))
     pre_ms_tile = vision_ms(qx.gemm)
-    flops = 24 * sum(2.0 * M * n * k for _, n, k, *_ in LLAVA_VISION)
+    flops = n_vis * sum(2.0 * M * n * k for _, n, k, *_ in LLAVA_VISION)
     del vis
     return {"workload": "llava16_7b_mixed_recipe",
             "recipe": {"language": "q,k L3g128; v,o,gate,up,down U4g64", "vision": "all U4g128"},
             "decode_token_us": dec_ms * 1e3, "decode_GBps": lang_bytes / (dec_ms * 1e-3) / 1e9,
-            "decode_launches": 32 * len(chain), "language_weight_bytes": lang_bytes,
+            "decode_launches": n_lang * len(chain), "language_weight_bytes": lang_bytes,
             "vision_prefill_us": pre_ms * 1e3, "vision_prefill_TFLOPs": flops / (pre_ms * 1e-3) / 1e12,
             "vision_prefill_path": "qx_gemm_splitk with PDL (64- or 256-token tiles, k split where the tiles leave SMs idle)",
             "vision_prefill_us_one_cta_per_tile": pre_ms_tile * 1e3,
-            "vision_tokens": M, "vision_gemm_launches": 24 * len(LLAVA_VISION)}
+            "vision_tokens": M, "vision_gemm_launches": n_vis * len(LLAVA_VISION),
+            "recipe_table": "paper_2505_07531_gb300/recipes/llava_v1_6_7b.json"}
 
 
 def main():

@@ -649,6 +649,26 @@ def q4x_gemm_splitk(P: Q4xMatrix, X: torch.Tensor, out: torch.Tensor | None = No
     return Y
 
 
+def recipe_table(path: str) -> dict:
+    """A per-matrix recipe table (JSON, as recipes/llava_v1_6_7b.json): for
+    each sub-model, its layer count and a list of (name, n, k, Recipe); the
+    recipe is chosen per matrix (Sections 2.1, 2.3)."""
+    import json
+
+    kinds = {"uniform": UNIFORM, "lut": LUT}
+    with open(path) as f:
+        t = json.load(f)
+    out = {}
+    for sub, body in t.items():
+        if not isinstance(body, dict) or "matrices" not in body:
+            continue
+        mats = [(m["name"], int(m["n"]), int(m["k"]),
+                 Recipe(int(m["recipe"]["bits"]), int(m["recipe"]["group_size"]), kinds[m["recipe"]["kind"]]))
+                for m in body["matrices"]]
+        out[sub] = {"layers": int(body["layers"]), "matrices": mats}
+    return out
+
+
 # ------------------------------------------------------------ save / load
 # A packed matrix on disk: an 80-byte little-endian header, then its four
 # buffers in header order.
