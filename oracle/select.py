@@ -15,12 +15,19 @@ activations and is not part of this step.  Reading:
   eligible: bpw_r <= max_bpw (every candidate when max_bpw is None)
   chosen:   the eligible r with the smallest E_r, ties to the smaller bpw_r,
             then to the earlier candidate; None when none is eligible.
+
+A candidate of kind "q4x" (bits 4, group size 64) is the shared-codebook
+format of Section 3.2 (oracle/q4x.py, lloyd_iters as its step limit); its
+bytes include the matrix's four codebooks.
 """
 from __future__ import annotations
 
 import numpy as np
 
 from .pack import Recipe, dequant, packed_sizes, quantize
+from .q4x import dequant_q4x, q4x_sizes, quantize_q4x
+
+Q4X = "q4x"
 
 
 def sq_error_units(W: np.ndarray, W_hat: np.ndarray) -> int:
@@ -31,9 +38,26 @@ def sq_error_units(W: np.ndarray, W_hat: np.ndarray) -> int:
     return int((d * d).sum())
 
 
+def _check_q4x(r: Recipe):
+    if r.bits != 4 or r.group_size != 64:
+        raise ValueError("a q4x candidate has 4 bits and groups of 64")
+
+
 def bits_per_weight(n: int, k: int, r: Recipe) -> float:
     """8 * packed bytes / weights, as the float64 division of two integers."""
+    if r.kind == Q4X:
+        _check_q4x(r)
+        return 8.0 * sum(q4x_sizes(n, k).values()) / (n * k)
     return 8.0 * sum(packed_sizes(n, k, r).values()) / (n * k)
+
+
+def dequantized(W: np.ndarray, r: Recipe) -> np.ndarray:
+    """W_hat of candidate r."""
+    if r.kind == Q4X:
+        _check_q4x(r)
+        q = quantize_q4x(W, iters=r.lloyd_iters)
+        return dequant_q4x(q["codes"], q["scales"], q["books"], q["codebooks"])
+    return dequant(quantize(W, r), r, np.asarray(W).shape[1])
 
 
 def select_recipe(W: np.ndarray, recipes: list, max_bpw: float | None = None):
@@ -48,7 +72,7 @@ def select_recipe(W: np.ndarray, recipes: list, max_bpw: float | None = None):
         if max_bpw is not None and bpw > max_bpw:
             errs.append(None)
             continue
-        e = sq_error_units(W, dequant(quantize(W, r), r, k))
+        e = sq_error_units(W, dequantized(W, r))
         errs.append(e)
         if best is None or (e, bpw) < (errs[best], bpws[best]):
             best = i

@@ -3,6 +3,7 @@ non-uniform per matrix by the Frobenius error; bit-widths per layer)."""
 from fractions import Fraction
 
 import numpy as np
+import pytest
 
 from oracle import select
 from oracle.pack import Recipe
@@ -51,3 +52,31 @@ def test_budget_excludes_recipes_and_can_exclude_all():
     best, errs_b, _ = select.select_recipe(W, [U3, U4, L3], max_bpw=4.0)
     assert best == 0 and errs_b[1] is None and errs_b[2] is None
     assert select.select_recipe(W, [U4, L3], max_bpw=3.0)[0] is None
+
+
+def test_q4x_candidate_bits_per_weight_and_lossless_choice():
+    """Groups made of 16 shared levels (times a per-group power of two, with
+    the group maximum present) are coded without error by Q4X, which must then
+    win against every per-group recipe; its bits per weight are the paper's
+    4 + 18/64 plus the 128-byte codebooks."""
+    from fractions import Fraction
+
+    from oracle.select import Q4X
+
+    n, k = 16, 256
+    levels = np.array([-1, -0.75, -0.5, -0.375, -0.25, -0.125, -0.0625, 0,
+                       0.0625, 0.125, 0.25, 0.375, 0.5, 0.625, 0.75, 1.0])
+    rng = np.random.default_rng(4)
+    W = np.empty((n, k))
+    for r in range(n):
+        for g in range(k // 64):
+            v = levels[rng.integers(0, 16, 64)]
+            v[0] = 1.0  # the group maximum, so that s is the power of two below
+            W[r, 64 * g:64 * g + 64] = v * 2.0 ** -int(rng.integers(3, 8))
+    W = W.astype(np.float16)
+    cands = [Recipe(4, 64, "uniform"), Recipe(3, 128, "lut"), Recipe(4, 64, Q4X)]
+    chosen, errs, bpws = select.select_recipe(W, cands)
+    assert errs[2] == 0 and all(e > 0 for e in errs[:2]) and chosen == 2
+    assert Fraction(bpws[2]).limit_denominator(1 << 20) == Fraction(8 * (n * k // 2 + 2 * n * 4 + n * 1 + 128), n * k)
+    with pytest.raises(ValueError):
+        select.bits_per_weight(n, k, Recipe(3, 64, Q4X))
