@@ -72,7 +72,9 @@ typedef enum qx_status {
 
 typedef enum qx_kind {
     QX_UNIFORM = 0, /* per-group fp16 scale + 4-bit zero-point, RTN (Section 3.2)   */
-    QX_LUT = 1      /* per-group 2^bits-entry fp16 codebook, Lloyd-Max (Section 2.2) */
+    QX_LUT = 1,     /* per-group 2^bits-entry fp16 codebook, Lloyd-Max (Section 2.2) */
+    QX_Q4X = 2      /* shared codebooks (Section 3.2): a qx_select_recipe candidate
+                       only; every qx_packed entry point rejects it (INVALID_ARG) */
 } qx_kind;
 
 typedef enum qx_dtype { QX_F16 = 0, QX_F32 = 1 } qx_dtype;
@@ -276,6 +278,10 @@ qx_status qx_gemv_a8(const qx_packed *p, const void *q, const void *scales, int3
  * candidate over the budget.  *chosen = the eligible candidate with the
  * smallest E_i, ties to the smaller bpw, then to the earlier index; -1 when
  * none is eligible.
+ * A candidate of kind QX_Q4X (bits 4, group_size 64, lloyd_iters 0..1000 as
+ * the learner's step limit, else UNSUPPORTED / INVALID_ARG) is quantized by
+ * qx_q4x_quantize and dequantized by qx_q4x_dequant; its bytes are the four
+ * Q4X buffers of qx_q4x_size, codebooks included.
  * W: device fp16 [n][k], 16-byte aligned, as for qx_quantize.  candidates,
  * chosen, sq_error (2 count words), bpw (count): host memory.  workspace:
  * device memory, 256-byte aligned, of at least qx_select_workspace() bytes.

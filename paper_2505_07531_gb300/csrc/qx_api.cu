@@ -591,27 +591,51 @@ QX_API qx_status qx_gemv_a8(const qx_packed *p, const void *q, const void *scale
 namespace {
 
 // Workspace of qx_select_recipe: the largest candidate's packed buffers, the
-// dequantized matrix, the error partials and one 16-byte result per candidate.
+// dequantized matrix, the error partials, one 16-byte result per candidate
+// and, when a Q4X candidate is present, the Q4X learner's workspace.
 struct SelectLayout {
-    size_t packed, what, partials, results, total;
+    size_t packed, what, partials, results, q4x, total;
 };
 
 size_t round256(size_t x) { return (x + 255) / 256 * 256; }
 
+// Byte sizes of one candidate's four buffers: {codes, scales, zeros, luts}
+// for the per-group kinds, {codes, scales, books, codebooks} for Q4X.
+qx_status candidate_sizes(int64_t n, int64_t k, const qx_recipe *r, uint64_t out[4]) {
+    if (r == nullptr) return QX_ERR_INVALID_ARG;
+    if (r->kind == QX_Q4X) {
+        if (r->lloyd_iters < 0 || r->lloyd_iters > 1000) return QX_ERR_INVALID_ARG;
+        if (r->bits != 4 || r->group_size != qx::kQ4xGroup) return QX_ERR_UNSUPPORTED;
+        qx_q4x_sizes sz{};
+        const qx_status s = qx_q4x_size(n, k, &sz);
+        if (s != QX_OK) return s;
+        out[0] = sz.codes, out[1] = sz.scales, out[2] = sz.books, out[3] = sz.codebooks;
+        return QX_OK;
+    }
+    qx_sizes sz{};
+    const qx_status s = qx_packed_size(n, k, r, &sz);
+    if (s != QX_OK) return s;
+    out[0] = sz.codes, out[1] = sz.scales, out[2] = sz.zeros, out[3] = sz.luts;
+    return QX_OK;
+}
+
 qx_status select_layout(int64_t n, int64_t k, const qx_recipe *cands, int32_t count, int num_sms, SelectLayout *L) {
     if (cands == nullptr || count < 1 || count > 16) return QX_ERR_INVALID_ARG;
     size_t packed = 0;
+    bool q4x = false;
     for (int i = 0; i < count; ++i) {
-        qx_sizes sz{};
-        qx_status s = qx_packed_size(n, k, &cands[i], &sz);
+        uint64_t sz[4] = {};
+        qx_status s = candidate_sizes(n, k, &cands[i], sz);
         if (s != QX_OK) return s;
-        packed = std::max(packed, round256(sz.codes) + round256(sz.scales) + round256(sz.zeros) + round256(sz.luts));
+        packed = std::max(packed, round256(sz[0]) + round256(sz[1]) + round256(sz[2]) + round256(sz[3]));
+        q4x = q4x || cands[i].kind == QX_Q4X;
     }
     L->packed = packed;
     L->what = round256((size_t)n * k * 2);
     L->partials = round256((size_t)qx::sq_error_blocks(num_sms) * 16);
     L->results = round256((size_t)count * 16);
-    L->total = L->packed + L->what + L->partials + L->results;
+    L->q4x = q4x ? round256(qx::q4x_workspace_bytes(n, k)) : 0;
+    L->total = L->packed + L->what + L->partials + L->results + L->q4x;
     return QX_OK;
 }
 
@@ -648,28 +672,37 @@ QX_API qx_status qx_select_recipe(const void *W, int64_t n, int64_t k, const qx_
     void *what = ws + L.packed;
     auto *partials = reinterpret_cast<unsigned long long *>(ws + L.packed + L.what);
     auto *results = reinterpret_cast<unsigned long long *>(ws + L.packed + L.what + L.partials);
+    uint8_t *q4x_ws = ws + L.packed + L.what + L.partials + L.results;
     bool eligible[16] = {};
     for (int i = 0; i < count; ++i) {
-        qx_sizes sz{};
-        qx_packed_size(n, k, &candidates[i], &sz);
-        bpw[i] = 8.0 * (double)(sz.codes + sz.scales + sz.zeros + sz.luts) / ((double)n * (double)k);
+        uint64_t sz[4] = {};
+        candidate_sizes(n, k, &candidates[i], sz);
+        bpw[i] = 8.0 * (double)(sz[0] + sz[1] + sz[2] + sz[3]) / ((double)n * (double)k);
         eligible[i] = !(max_bpw > 0.0) || bpw[i] <= max_bpw;
         if (!eligible[i]) continue;
         // quantize into the workspace, dequantize, take the exact error
-        qx_packed p{};
-        p.n = n;
-        p.k = k;
-        p.recipe = candidates[i];
+        void *buf[4] = {};
         uint8_t *at = ws;
-        p.codes = at;
-        at += round256(sz.codes);
-        p.scales = sz.scales ? at : nullptr;
-        at += round256(sz.scales);
-        p.zeros = sz.zeros ? at : nullptr;
-        at += round256(sz.zeros);
-        p.luts = sz.luts ? at : nullptr;
-        if ((s = qx_quantize(W, n, k, &candidates[i], &p, stream)) != QX_OK) return s;
-        if ((s = qx_dequant(&p, what, stream)) != QX_OK) return s;
+        for (int j = 0; j < 4; ++j) {
+            buf[j] = sz[j] ? at : nullptr;
+            at += round256(sz[j]);
+        }
+        if (candidates[i].kind == QX_Q4X) {
+            const qx_q4x p{n, k, buf[0], buf[1], buf[2], buf[3]};
+            if ((s = qx_q4x_quantize(W, candidates[i].lloyd_iters, &p, q4x_ws, L.q4x, stream)) != QX_OK) return s;
+            if ((s = qx_q4x_dequant(&p, what, stream)) != QX_OK) return s;
+        } else {
+            qx_packed p{};
+            p.n = n;
+            p.k = k;
+            p.recipe = candidates[i];
+            p.codes = buf[0];
+            p.scales = buf[1];
+            p.zeros = buf[2];
+            p.luts = buf[3];
+            if ((s = qx_quantize(W, n, k, &candidates[i], &p, stream)) != QX_OK) return s;
+            if ((s = qx_dequant(&p, what, stream)) != QX_OK) return s;
+        }
         if ((s = from_cuda(qx::launch_sq_error(static_cast<const __half *>(W), static_cast<const __half *>(what),
                                                n * k, partials, results + 2 * i, d->num_sms, st))) != QX_OK)
             return s;

@@ -15,7 +15,7 @@ import torch
 
 _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "libqx.so")
 
-UNIFORM, LUT = 0, 1
+UNIFORM, LUT, Q4X = 0, 1, 2
 F16, F32 = 0, 1
 GEMV_PDL = 1
 GEMM_PDL = 1
@@ -145,7 +145,8 @@ def _check(code: int, where: str):
 
 @dataclass(frozen=True)
 class Recipe:
-    """Per-matrix recipe: bit-width, group size along k, uniform (0) or LUT (1)."""
+    """Per-matrix recipe: bit-width, group size along k, uniform (0) or LUT (1);
+    Q4X (2, bits 4, group 64) only as a select_recipe candidate."""
 
     bits: int
     group_size: int

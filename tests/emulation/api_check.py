@@ -194,19 +194,30 @@ def check_per_group(n, k, bits, g, kind):
 
 def check_select(n, k):
     W = synth.student_t_weights(n, k, 0.02, seed=5, stream=6, outlier_frac=0.001)
-    cands = [qx.Recipe(3, 64, 0), qx.Recipe(3, 128, 1), qx.Recipe(4, 64, 0), qx.Recipe(4, 128, 0)]
-    arr = (qx._Recipe * 4)(*[c.c() for c in cands])
-    nb = ctypes.c_size_t(0)
-    ok(L.qx_select_workspace(n, k, arr, 4, ctypes.byref(nb)), "qx_select_workspace")
-    ws = buf(nb.value)
-    chosen, err, bpw = ctypes.c_int32(-1), (ctypes.c_uint64 * 8)(), (ctypes.c_double * 4)()
-    ok(L.qx_select_recipe(P(put(W)), n, k, arr, 4, 0.0, P(ws), ws.nbytes, ctypes.byref(chosen), err, bpw, None),
-       "qx_select_recipe")
-    orecs = [ORecipe(c.bits, c.group_size, "lut" if c.kind else "uniform", 25) for c in cands]
-    want = oselect.select_recipe(W, orecs)
-    got_e = [err[2 * i] | (err[2 * i + 1] << 64) for i in range(4)]
-    assert chosen.value == want[0], f"chosen {chosen.value} vs {want[0]}"
-    assert got_e == [int(e) for e in want[1]], "exact errors"
+    cands = [qx.Recipe(3, 64, qx.UNIFORM), qx.Recipe(3, 128, qx.LUT), qx.Recipe(4, 64, qx.UNIFORM),
+             qx.Recipe(4, 128, qx.UNIFORM), qx.Recipe(4, 64, qx.Q4X, 4)]
+    c = len(cands)
+    arr = (qx._Recipe * c)(*[r.c() for r in cands])
+    names = {qx.UNIFORM: "uniform", qx.LUT: "lut", qx.Q4X: oselect.Q4X}
+    orecs = [ORecipe(r.bits, r.group_size, names[r.kind], r.lloyd_iters) for r in cands]
+    Wd = put(W)
+    for budget in (0.0, 4.3):
+        nb = ctypes.c_size_t(0)
+        ok(L.qx_select_workspace(n, k, arr, c, ctypes.byref(nb)), "qx_select_workspace")
+        ws = buf(nb.value)
+        chosen, err, bpw = ctypes.c_int32(-1), (ctypes.c_uint64 * (2 * c))(), (ctypes.c_double * c)()
+        ok(L.qx_select_recipe(P(Wd), n, k, arr, c, budget, P(ws), ws.nbytes, ctypes.byref(chosen), err, bpw, None),
+           "qx_select_recipe")
+        want = oselect.select_recipe(W, orecs, max_bpw=budget or None)
+        got_e = [None if err[2 * i] == err[2 * i + 1] == 2 ** 64 - 1 else err[2 * i] | (err[2 * i + 1] << 64)
+                 for i in range(c)]
+        assert chosen.value == (-1 if want[0] is None else want[0]), f"chosen {chosen.value} vs {want[0]}"
+        assert got_e == [None if e is None else int(e) for e in want[1]], "exact errors"
+        assert list(bpw) == list(want[2]), "bits per weight"
+    # a Q4X candidate outside bits 4 / group 64 is not built
+    bad = (qx._Recipe * 1)(qx._Recipe(4, 128, qx.Q4X, 4))
+    assert L.qx_select_workspace(n, k, bad, 1, ctypes.byref(nb)) == 2
+    assert status() == 0
 
 
 def check_q4x(n, k, iters):

@@ -119,6 +119,14 @@ def test_entry_points_reject_bad_arguments_before_launching(qx):
     assert lib.qx_select_workspace(64, 200, cands, 2, ctypes.byref(nbytes)) == 2
     bad = (qx._Recipe * 1)(qx._Recipe(4, 64, 1, 0))  # 4-bit LUT is not built
     assert lib.qx_select_workspace(64, 256, bad, 1, ctypes.byref(nbytes)) == 2
+    # Q4X: a selection candidate only, with bits 4, groups of 64, 0..1000 steps
+    q4 = qx._Recipe(4, 64, qx.Q4X, 0)
+    assert lib.qx_packed_size(64, 256, ctypes.byref(q4), ctypes.byref(qx._Sizes())) == 1
+    for r, code in [((3, 64, qx.Q4X, 0), 2), ((4, 128, qx.Q4X, 0), 2), ((4, 64, qx.Q4X, 1001), 1),
+                    ((4, 64, qx.Q4X, -1), 1), ((4, 64, 3, 0), 1)]:
+        one = (qx._Recipe * 1)(qx._Recipe(*r))
+        assert lib.qx_select_workspace(64, 256, one, 1, ctypes.byref(nbytes)) == code, r
+    assert lib.qx_select_workspace(64, 224, (qx._Recipe * 1)(q4), 1, ctypes.byref(nbytes)) == 2  # k % 64
     ch, err, bpw = ctypes.c_int32(0), (ctypes.c_uint64 * 4)(), (ctypes.c_double * 2)()
     assert lib.qx_select_recipe(None, 64, 256, cands, 2, 0.0, None, 0, ctypes.byref(ch), err, bpw, None) == 1
     assert lib.qx_select_recipe(ctypes.c_void_p(0x4008), 64, 256, cands, 2, 0.0, None, 0, ctypes.byref(ch), err, bpw,

@@ -207,6 +207,41 @@ def test_nonfinite_group_is_flagged_and_coded_as_dead(qx):
     _assert_same(P, oracle.quantize_q4x(clean))
 
 
+@pytest.mark.parametrize("shape", [(96, 512), (37, 320)])
+def test_select_recipe_with_q4x_candidate(qx, shape):
+    """Recipe selection with a Q4X candidate beside per-group ones: the same
+    choice, exact errors and bits per weight as the oracle, with budgets that
+    keep or exclude Q4X (its 128 codebook bytes count)."""
+    from oracle import select as oselect
+    from oracle.pack import Recipe as ORecipe
+    n, k = shape
+    W = _weights(n, k, seed=700 + n)
+    spec = [(3, 64, qx.UNIFORM, "uniform", 25), (4, 64, qx.Q4X, oselect.Q4X, 6), (3, 128, qx.LUT, "lut", 25),
+            (4, 128, qx.UNIFORM, "uniform", 25)]
+    cands = [qx.Recipe(b, g, kd, it) for b, g, kd, _, it in spec]
+    orecs = [ORecipe(b, g, name, it) for b, g, _, name, it in spec]
+    Wd = torch.from_numpy(W).cuda()
+    for max_bpw in (None, 4.35, 4.2):
+        got = qx.select_recipe(Wd, cands, max_bpw)
+        want = oselect.select_recipe(W, orecs, max_bpw)
+        assert got[0] == want[0] and got[1] == want[1] and got[2] == want[2], max_bpw
+    assert qx.device_status() == 0
+
+
+def test_select_recipe_q4x_lossless(qx):
+    """Groups drawn from 16 shared levels with their maximum present: Q4X codes
+    them without error and is chosen over the per-group recipes."""
+    rng = np.random.default_rng(9)
+    levels = np.array([-1, -0.75, -0.5, -0.375, -0.25, -0.125, -0.0625, 0,
+                       0.0625, 0.125, 0.25, 0.375, 0.5, 0.625, 0.75, 1.0])
+    W = levels[rng.integers(0, 16, (32, 512))]
+    W[:, ::64] = 1.0
+    W = (W * 2.0 ** -rng.integers(3, 8, (32, 8)).repeat(64, axis=1)).astype(np.float16)
+    best, errs, _ = qx.select_recipe(torch.from_numpy(W).cuda(),
+                                     [qx.Recipe(4, 64, qx.UNIFORM), qx.Recipe(4, 64, qx.Q4X)])
+    assert best == 1 and errs[1] == 0 and errs[0] > 0
+
+
 @pytest.mark.slow
 def test_full_size_llama_projection(qx):
     """4096 x 4096 (a Llama-7B attention projection), the default 25 steps:
