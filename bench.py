@@ -457,20 +457,24 @@ def run_ours(args):
     e2e_ms = _max_over_ranks(dist, (time.perf_counter() - t0) * 1e3 / e2e_steps, dev)
     e2e_value = _job_rate(step_bytes, ws, e2e_ms) / 1e9
 
-    gemm = run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
+    def section(fn, *a):
+        # a section that fails reports its error in its own key; the headline
+        # figures above and the other sections stand
+        try:
+            return fn(*a)
+        except Exception as e:  # noqa: BLE001
+            return {"error": f"{type(e).__name__}: {e}"[:300]}
+        finally:
+            torch.cuda.empty_cache()
+
+    gemm = section(run_gemm_part, qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
     del layers, graphs
     extra = {}
     if not args.skip_configs:
-        torch.cuda.empty_cache()
-        extra["config3"] = run_config3(qx, torch, dev, stream, l2)
-        extra["recipe_select"] = run_select(qx, torch, dev, stream)
-        torch.cuda.empty_cache()
-        extra["config5"] = run_config5(qx, torch, dev, stream)
-        torch.cuda.empty_cache()
-        try:  # last: its result or its error is reported, the sections above stand
-            extra["q4x"] = run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst)
-        except Exception as e:  # noqa: BLE001
-            extra["q4x"] = {"error": f"{type(e).__name__}: {e}"[:300]}
+        extra["config3"] = section(run_config3, qx, torch, dev, stream, l2)
+        extra["recipe_select"] = section(run_select, qx, torch, dev, stream)
+        extra["config5"] = section(run_config5, qx, torch, dev, stream)
+        extra["q4x"] = section(run_q4x, qx, torch, dev, stream, l2, hbm, tf_burst)
 
     if rank == 0:
         cpu = run_cpu_baseline() if not args.skip_cpu_baseline else None
@@ -786,11 +790,23 @@ def run_select(qx, torch, dev, stream):
         e1.record(stream)
     torch.cuda.synchronize()
     names = ["U3g64", "L3g128", "U4g64", "U4g128"]
-    return {"matrix": [4096, 4096], "candidates": names, "ms": e0.elapsed_time(e1),
-            "chosen": names[best] if best is not None else None,
-            "rel_frobenius_error": {nm: math.sqrt(e / float(1 << 48)) / float(W.float().norm())
-                                    for nm, e in zip(names, errs)},
-            "bpw": dict(zip(names, bpws))}
+    norm = float(W.float().norm())
+    out = {"matrix": [4096, 4096], "candidates": names, "ms": e0.elapsed_time(e1),
+           "chosen": names[best] if best is not None else None,
+           "rel_frobenius_error": {nm: math.sqrt(e / float(1 << 48)) / norm for nm, e in zip(names, errs)},
+           "bpw": dict(zip(names, bpws))}
+    # the same four and a Q4X candidate (shared codebooks, 25 learner steps)
+    cands5 = cands + [qx.Recipe(4, 64, qx.Q4X, 25)]
+    with torch.cuda.stream(stream):
+        qx.select_recipe(W, cands5)  # warm-up
+        e0.record(stream)
+        best5, errs5, bpws5 = qx.select_recipe(W, cands5)
+        e1.record(stream)
+    torch.cuda.synchronize()
+    names5 = names + ["Q4Xg64"]
+    out["with_q4x"] = {"ms": e0.elapsed_time(e1), "chosen": names5[best5] if best5 is not None else None,
+                       "rel_frobenius_error": math.sqrt(errs5[4] / float(1 << 48)) / norm, "bpw": bpws5[4]}
+    return out
 
 
 def run_config5(qx, torch, dev, stream):
