@@ -836,19 +836,32 @@ def run_config5(qx, torch, dev, stream):
     dec_ms = _time_graph(torch, stream, gr, 10)
     del gr, lang
 
-    vbase = dict(_quantize_layer(qx, torch, dev, LLAVA_VISION, qx.Recipe(*LLAVA_VISION_RECIPE), seed=5))
+    vrec = qx.Recipe(*LLAVA_VISION_RECIPE)
+    vbase = dict(_quantize_layer(qx, torch, dev, LLAVA_VISION, vrec, seed=5))
+    # q, k and v read the same activations and share the recipe: stacked along
+    # n they are one 3n x k matrix (a fused QKV projection).  Every group lies
+    # within one row, so its codes are those of the three matrices, row for row.
+    qkv = [m for m in LLAVA_VISION if m[0] in ("q_proj", "k_proj", "v_proj")]
+    Wqkv = torch.cat([synth.student_t_weights_torch(n, k, sig, seed=5, stream=sid, device=dev)
+                      for _, n, k, sig, sid in qkv])
+    vbase["qkv_proj"] = qx.quantize(Wqkv, vrec)
+    del Wqkv
     n_vis = LLAVA["vision"]["layers"]
     vis = [vbase] + [{nm: _clone(qx, P) for nm, P in vbase.items()} for _ in range(n_vis - 1)]
     M = LLAVA["vision"]["tokens"]
     X1 = synth.activations_torch(M, 1024, seed=5, stream=95, device=dev)
     X4 = synth.activations_torch(M, 4096, seed=5, stream=96, device=dev)
-    Ys = {nm: torch.empty((M, n), dtype=torch.float16, device=dev) for nm, n, *_ in LLAVA_VISION}
+    separate = [(nm, n, k) for nm, n, k, *_ in LLAVA_VISION]
+    fused = [("qkv_proj", sum(m[1] for m in qkv), qkv[0][2])] + [m for m in separate if m[0] not in
+                                                                  ("q_proj", "k_proj", "v_proj")]
+    Ys = {nm: torch.empty((M, n), dtype=torch.float16, device=dev) for nm, n, _ in separate + fused}
 
-    def vision_ms(gemm):
-        """The vision layers through `gemm` (qx.gemm or qx.gemm_splitk), one CUDA graph."""
+    def vision_ms(gemm, mats):
+        """The vision layers' matrices `mats` through `gemm` (qx.gemm or
+        qx.gemm_splitk), one CUDA graph."""
         def vision_pass():
             for L in vis:
-                for nm, n, k, *_ in LLAVA_VISION:
+                for nm, n, k in mats:
                     gemm(L[nm], X4 if k == 4096 else X1, out=Ys[nm])
 
         with torch.cuda.stream(stream):
@@ -863,8 +876,10 @@ def run_config5(qx, torch, dev, stream):
         del gv
         return ms
 
-    pre_ms = vision_ms(lambda P, X, out: qx.gemm_splitk(P, X, out=out, pdl=True))
-    pre_ms_tile = vision_ms(qx.gemm)
+    splitk = lambda P, X, out: qx.gemm_splitk(P, X, out=out, pdl=True)  # noqa: E731
+    pre_ms = vision_ms(splitk, fused)
+    pre_ms_sep = vision_ms(splitk, separate)
+    pre_ms_tile = vision_ms(qx.gemm, separate)
     flops = n_vis * sum(2.0 * M * n * k for _, n, k, *_ in LLAVA_VISION)
     del vis
     return {"workload": "llava16_7b_mixed_recipe",
@@ -872,9 +887,12 @@ def run_config5(qx, torch, dev, stream):
             "decode_token_us": dec_ms * 1e3, "decode_GBps": lang_bytes / (dec_ms * 1e-3) / 1e9,
             "decode_launches": n_lang * len(chain), "language_weight_bytes": lang_bytes,
             "vision_prefill_us": pre_ms * 1e3, "vision_prefill_TFLOPs": flops / (pre_ms * 1e-3) / 1e12,
-            "vision_prefill_path": "qx_gemm_splitk with PDL (64- or 256-token tiles, k split where the tiles leave SMs idle)",
+            "vision_prefill_path": "qx_gemm_splitk with PDL (64- or 256-token tiles, k split where the tiles "
+                                   "leave SMs idle); q, k, v stacked as one 3072x1024 matrix",
+            "vision_prefill_us_separate_qkv": pre_ms_sep * 1e3,
             "vision_prefill_us_one_cta_per_tile": pre_ms_tile * 1e3,
-            "vision_tokens": M, "vision_gemm_launches": n_vis * len(LLAVA_VISION),
+            "vision_tokens": M, "vision_gemm_launches": n_vis * len(fused),
+            "vision_gemm_launches_separate_qkv": n_vis * len(separate),
             "recipe_table": "paper_2505_07531_gb300/recipes/llava_v1_6_7b.json"}
 
 

@@ -102,3 +102,21 @@ def test_shape_checks():
         oracle.pack_codes(np.zeros((1, 64), np.uint8), 4)
     with pytest.raises(ValueError):
         oracle.pack_codes(np.full((1, 128), 8, np.uint8), 3)
+
+
+@pytest.mark.parametrize("bits,g,kind", [(3, 64, "uniform"), (4, 128, "uniform"), (3, 128, "lut")])
+def test_rows_are_quantized_independently(bits, g, kind):
+    """Every group lies within one row (Section 2.1: groups of consecutive
+    weights along a row), so matrices stacked along n pack to their packed
+    buffers stacked row for row: a fused projection is the same model."""
+    import synth
+
+    r = Recipe(bits, g, kind, 6)
+    A = synth.student_t_weights(40, 256, 0.02, seed=1, stream=2).astype(np.float16)
+    B = synth.student_t_weights(24, 256, 0.05, seed=1, stream=3).astype(np.float16)
+    pa, pb, pab = oracle.quantize(A, r), oracle.quantize(B, r), oracle.quantize(np.vstack([A, B]), r)
+    for key in ("codes", "scales", "zeros", "luts"):
+        if pab[key] is None:
+            assert pa[key] is None
+            continue
+        assert np.array_equal(pab[key].view(np.uint8), np.vstack([pa[key], pb[key]]).view(np.uint8)), key
