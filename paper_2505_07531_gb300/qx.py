@@ -229,8 +229,13 @@ class PackedMatrix:
         return out
 
 
+def _on_device(t: torch.Tensor) -> bool:
+    """Whether the library may take t's memory as device memory."""
+    return t.is_cuda
+
+
 def _dev_tensor(t: torch.Tensor, name: str, dtype=torch.float16):
-    if not t.is_cuda:
+    if not _on_device(t):
         raise ValueError(f"{name} must be a CUDA tensor")
     if t.dtype != dtype:
         raise ValueError(f"{name} must be {dtype}")
@@ -356,7 +361,7 @@ class DecodeStep(GemvChain):
         def copies(pairs, to_device):
             arr = []
             for dst, src in pairs:
-                if dst.is_cuda != to_device or src.is_cuda == to_device:
+                if _on_device(dst) != to_device or _on_device(src) == to_device:
                     raise ValueError("h2d pairs are (device, host), d2h pairs (host, device)")
                 if not (dst.is_contiguous() and src.is_contiguous()):
                     raise ValueError("copies need contiguous tensors")
@@ -432,7 +437,7 @@ def gemm_splitk(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = Non
     _dev_tensor(Y, "out")
     need = gemm_splitk_workspace_bytes(P.n, P.k, m, P.recipe)
     ws = workspace if workspace is not None else splitk_workspace(X.device, need)
-    if not ws.is_cuda or ws.dtype != torch.uint8:
+    if not _on_device(ws) or ws.dtype != torch.uint8:
         raise ValueError("workspace must be a CUDA uint8 tensor")
     pc = P.c()
     _check(_lib().qx_gemm_splitk(ctypes.byref(pc), _ptr(X), m, _ptr(Y), _ptr(ws), ws.numel(),
@@ -467,7 +472,7 @@ def quantize_act(x: torch.Tensor):
 def gemv_a8(P: PackedMatrix, q: torch.Tensor, scales: torch.Tensor, out: torch.Tensor | None = None,
             out_dtype=torch.float16) -> torch.Tensor:
     """W.A8 decode y = s_b x (q_w - z) q x s_g (qx_gemv_a8) for uniform weights; returns [batch][n]."""
-    if not q.is_cuda or q.dtype != torch.int8 or not q.is_contiguous():
+    if not _on_device(q) or q.dtype != torch.int8 or not q.is_contiguous():
         raise ValueError("q must be a contiguous CUDA int8 tensor")
     _dev_tensor(scales, "scales", torch.float32)
     b = q.shape[0]

@@ -1,8 +1,9 @@
 """Every C-ABI entry point, built for the host from the kernel and API sources
 with AddressSanitizer and UBSan, called through ctypes the way a user calls
 it, on buffers of exactly the sizes include/qx.h states; results against the
-oracle (tests/emulation/api_check.py).  No GPU; the library never loads this
-build."""
+oracle (tests/emulation/api_check.py); and the Python binding driven against
+that build (tests/emulation/binding_check.py).  No GPU; the library never
+loads this build."""
 import os
 import shutil
 import subprocess
@@ -13,7 +14,7 @@ import pytest
 HERE = os.path.join(os.path.dirname(os.path.abspath(__file__)), "emulation")
 
 
-def test_every_entry_point_under_the_sanitizers(emulation_dir):
+def _run_under_sanitizers(emulation_dir, script, marker):
     gxx = shutil.which("g++")
     if gxx is None:
         pytest.skip("g++ is not available")
@@ -24,6 +25,17 @@ def test_every_entry_point_under_the_sanitizers(emulation_dir):
     runtimes = [subprocess.run([gxx, f"-print-file-name={n}"], capture_output=True, text=True).stdout.strip()
                 for n in ("libasan.so", "libubsan.so")]
     env = dict(os.environ, LD_PRELOAD=" ".join(runtimes), ASAN_OPTIONS="detect_leaks=0", QX_EMU_SMS="3")
-    r = subprocess.run([sys.executable, os.path.join(HERE, "api_check.py"), lib], capture_output=True, text=True,
+    r = subprocess.run([sys.executable, os.path.join(HERE, script), lib], capture_output=True, text=True,
                        env=env, timeout=1800)
-    assert r.returncode == 0 and "api ok" in r.stdout, (r.stdout[-2000:] + r.stderr[-4000:])
+    assert r.returncode == 0 and marker in r.stdout, (r.stdout[-2000:] + r.stderr[-4000:])
+
+
+def test_every_entry_point_under_the_sanitizers(emulation_dir):
+    _run_under_sanitizers(emulation_dir, "api_check.py", "api ok")
+
+
+def test_python_binding_under_the_sanitizers(emulation_dir):
+    """The wrappers of paper_2505_07531_gb300/qx.py (Q4X calls, recipe selection
+    with a Q4X candidate, GemvChain, DecodeStep) with host tensors standing in
+    for device tensors (tests/emulation/binding_check.py)."""
+    _run_under_sanitizers(emulation_dir, "binding_check.py", "binding ok")
