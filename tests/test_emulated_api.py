@@ -24,7 +24,10 @@ def _run_under_sanitizers(emulation_dir, script, marker):
     lib = translate.build(gxx, str(emulation_dir), "library")
     runtimes = [subprocess.run([gxx, f"-print-file-name={n}"], capture_output=True, text=True).stdout.strip()
                 for n in ("libasan.so", "libubsan.so")]
-    env = dict(os.environ, LD_PRELOAD=" ".join(runtimes), ASAN_OPTIONS="detect_leaks=0", QX_EMU_SMS="3")
+    # the emulation runs kernels thousands of times slower than a GPU: its bounded
+    # waits get minutes, not the default two seconds
+    env = dict(os.environ, LD_PRELOAD=" ".join(runtimes), ASAN_OPTIONS="detect_leaks=0", QX_EMU_SMS="3",
+               QX_WAIT_LIMIT_MS="300000")
     r = subprocess.run([sys.executable, os.path.join(HERE, script), lib], capture_output=True, text=True,
                        env=env, timeout=1800)
     assert r.returncode == 0 and marker in r.stdout, (r.stdout[-2000:] + r.stderr[-4000:])
