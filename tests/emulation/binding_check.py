@@ -162,10 +162,30 @@ def check_chain_and_step():
     assert qx.device_status() == 0
 
 
+def check_stacked():
+    """q, k, v stacked along n: the same packed rows and, per 128-row tile, the
+    same prefill outputs bit for bit."""
+    r = qx.Recipe(4, 128, qx.UNIFORM)
+    k, m = 256, 20
+    Ws = [synth.student_t_weights(n, k, 0.02, seed=7, stream=i).astype(np.float16)
+          for i, n in enumerate((256, 128, 128))]
+    parts = [qx.quantize(dev(W), r) for W in Ws]
+    S = qx.quantize(dev(np.vstack(Ws)), r)
+    for key in ("codes", "scales", "zeros"):
+        assert torch.equal(getattr(S, key).view(torch.uint8),
+                           torch.cat([getattr(P, key).view(torch.uint8) for P in parts])), key
+    X = dev(synth.activations(m, k, seed=3, stream=m))
+    Y = qx.gemm(S, X)
+    Yp = torch.cat([qx.gemm(P, X) for P in parts], dim=1)
+    assert torch.equal(Y.view(torch.int16), Yp.view(torch.int16))
+    assert qx.device_status() == 0
+
+
 def main():
     check_q4x(37, 384, 2)
     check_select()
     check_chain_and_step()
+    check_stacked()
     print("binding ok")
 
 
