@@ -56,4 +56,4 @@ from .q4x import (  # noqa: F401
     gemv_q4x,
 )
 from .select import select_recipe, sq_error_units, bits_per_weight  # noqa: F401
-from .act8 import quantize_act, gemv_a8, dequant_act  # noqa: F401
+from .act8 import quantize_act, gemv_a8, dequant_act, dequant_act_f16, gemm_a8  # noqa: F401

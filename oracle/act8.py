@@ -13,7 +13,13 @@ Readings:
   Matmul, uniform weights (codes q_w, zero-points z, fp16 scales s_g):
       y[b][n] = s_b * sum_g s_g * sum_{k in g} (q_w[n][k] - z[n][g]) * q[b][k]
       The inner sums are exact integers; the oracle takes the rest in float64.
-  Non-uniform (LUT) weights have no integer form: W.A8 is uniform only.
+  Non-uniform (LUT) weights have no integer form: W.A8 decode is uniform only.
+  Prefill (any weight format): the tensor cores take fp16 operands, so the
+  int8 activations enter as
+      x_hat[b][k] = fp16(fp32(s_b * q[b][k]))      one fp32 product, then RN
+  and Y = x_hat W_hat^T is the fp16 matmul of the prefill, in float64 here.
+  For uniform weights it differs from the decode form above only by the
+  rounding of x_hat (at most 2^-11 of each |s_b q|).
 """
 from __future__ import annotations
 
@@ -59,3 +65,16 @@ def gemv_a8(p: dict, r, x: np.ndarray, k: int) -> np.ndarray:
 def dequant_act(q: np.ndarray, s: np.ndarray) -> np.ndarray:
     """x_hat = s q (float64), the activations the W.A8 decode multiplies."""
     return q.astype(F64) * s.astype(F64)[:, None]
+
+
+def dequant_act_f16(q: np.ndarray, s: np.ndarray) -> np.ndarray:
+    """x_hat = fp16(fp32(s_b q)) [b][k], the prefill's fp16 activations."""
+    prod = np.asarray(q, dtype=np.int8).astype(F32) * np.asarray(s, dtype=F32)[:, None]  # one fp32 RN product
+    return prod.astype(np.float16)
+
+
+def gemm_a8(W_hat: np.ndarray, x: np.ndarray) -> np.ndarray:
+    """float64 Y [b][n] of the W.A8 prefill for fp16 activations x [b][k] and
+    dequantized fp16 weights W_hat [n][k]."""
+    q, s = quantize_act(x)
+    return dequant_act_f16(q, s).astype(F64) @ np.asarray(W_hat, dtype=np.float16).astype(F64).T

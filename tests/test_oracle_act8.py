@@ -75,3 +75,49 @@ def test_lut_weights_have_no_integer_path():
     r = Recipe(3, 64, "lut")
     with pytest.raises(ValueError):
         act8.gemv_a8(oracle.quantize(W, r), r, synth.activations(1, 128, seed=1, stream=1), 128)
+
+
+# ---------------------------------------------------------------- W.A8 prefill
+def test_prefill_activations_closed_form():
+    """x = j 2^-7: s = 2^-7, q = j and x_hat = x exactly, so the prefill is the
+    plain product with x."""
+    j = np.arange(-127, 129)[:256].reshape(2, 128)
+    j[j > 127] = 0
+    x = (j * 2.0 ** -7).astype(np.float16)
+    q, s = act8.quantize_act(x)
+    xh = act8.dequant_act_f16(q, s)
+    assert np.array_equal(xh.view(np.uint16), x.view(np.uint16))
+    W = synth.student_t_weights(24, 128, 0.02, seed=2, stream=3).astype(np.float16)
+    assert np.array_equal(act8.gemm_a8(W, x), x.astype(np.float64) @ W.astype(np.float64).T)
+
+
+def test_prefill_largest_activation_round_trips():
+    """s_b = fp32(m / 127) is within 2^-24 of m / 127, so fp16(fp32(127 s_b))
+    lands back on the fp16 value m: the largest |x| of every token is kept
+    exactly (including fp16 subnormals)."""
+    x = synth.activations(64, 256, seed=4, stream=5)
+    x[3] *= np.float16(2.0 ** -20)  # a token in the subnormal range
+    q, s = act8.quantize_act(x)
+    xh = act8.dequant_act_f16(q, s)
+    for b in range(x.shape[0]):
+        i = int(np.argmax(np.abs(x[b].astype(np.float64))))
+        assert abs(int(q[b, i])) == 127 and xh[b, i] == x[b, i], b
+
+
+def test_prefill_matches_the_integer_decode_form_within_one_rounding():
+    """For uniform weights the prefill and the decode (exact integer group
+    sums) differ only by x_hat's rounding: |diff| <= 2^-11 sum_k |s_b q_k w_hat_k|."""
+    k = 256
+    r = Recipe(4, 64, "uniform")
+    W = synth.student_t_weights(40, k, 0.02, seed=6, stream=7).astype(np.float16)
+    x = synth.activations(5, k, seed=8, stream=9)
+    x[2] = 0  # a dead token: zero output
+    p = oracle.quantize(W, r)
+    Wh = oracle.dequant(p, r, k)
+    y_pre, y_dec = act8.gemm_a8(Wh, x), act8.gemv_a8(p, r, x, k)
+    q, s = act8.quantize_act(x)
+    bound = 2.0 ** -11 * (np.abs(act8.dequant_act(q, s)) @ np.abs(Wh.astype(np.float64)).T)
+    assert np.all(np.abs(y_pre - y_dec) <= bound * (1 + 1e-9) + 1e-300)
+    assert not y_pre[2].any()
+    # a dropped scale or a transposed operand is far outside that bound
+    assert np.abs(y_pre - y_dec).max() < 1e-2 * np.abs(y_dec).max()
