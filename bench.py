@@ -542,7 +542,11 @@ def run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src):
     per = {mats[j][0]: 1e3 * sum(evs[r][j][0].elapsed_time(evs[r][j][1]) for r in range(reps)) / reps
            for j in range(len(mats))}
     tflops = flops / (ms * 1e-3) / 1e12
-    return {"value": tflops, "unit": "TFLOP/s", "ms_per_step": ms, "per_matrix_us": per,
+    try:
+        a8 = _a8_prefill(qx, torch, dev, stream, mats, Xs, Ys, flops)
+    except Exception as e:  # noqa: BLE001
+        a8 = {"error": f"{type(e).__name__}: {e}"[:300]}
+    return {"value": tflops, "unit": "TFLOP/s", "ms_per_step": ms, "per_matrix_us": per, "a8_prefill": a8,
             "config": {"workload": "prefill_M2048_L3g128", "m": GEMM_M,
                        "matrices": {nm: [P.n, P.k] for nm, P in mats}, "mma": "tcgen05 kind::f16, fp32 accumulate",
                        "l2": "weights 22.5 MB and X 16-22 MB are L2-resident (compute-bound kernel)"},
@@ -550,6 +554,39 @@ def run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src):
                          "frac": tflops / tf_burst,
                          "peak_source": f"{peak_src} bf16_tflops (burst) x 1.0 nominal fp16/bf16 ratio",
                          "kernel": "gemm_kernel<3,LUT>", "traffic": _traffic("qx_gemm.cu", "gemm_L3g128_m2048")}}
+
+
+def _a8_prefill(qx, torch, dev, stream, mats, Xs, Ys, flops):
+    """The same prefill with 8-bit per-token activations (Tables 1-2, W.A8):
+    qx_quantize_act, qx_dequant_act (x_hat = fp16(s_b q)) and qx_gemm per
+    matrix, all three timed."""
+    bufs = [(torch.empty(X.shape, dtype=torch.int8, device=dev), torch.empty((X.shape[0],), dtype=torch.float32,
+                                                                              device=dev), torch.empty_like(X))
+            for X in Xs]
+    lib = qx._lib()
+
+    def step():
+        for (nm, P), X, Y, (q, s, xh) in zip(mats, Xs, Ys, bufs):
+            m, k = X.shape
+            qx._check(lib.qx_quantize_act(qx._ptr(X), m, k, qx._ptr(q), qx._ptr(s), qx._stream(dev)),
+                      "qx_quantize_act")
+            qx.dequant_act(q, s, out=xh)
+            qx.gemm(P, xh, out=Y)
+
+    with torch.cuda.stream(stream):
+        for _ in range(3):
+            step()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(stream)
+        for _ in range(10):
+            step()
+        e1.record(stream)
+    torch.cuda.synchronize(dev)
+    if qx.device_status(stream) != 0:
+        raise RuntimeError("W.A8 prefill reported a device error")
+    ms = e0.elapsed_time(e1) / 10
+    return {"ms_per_step": ms, "TFLOPs": flops / (ms * 1e-3) / 1e12,
+            "path": "qx_quantize_act + qx_dequant_act + qx_gemm per matrix (fp16 tensor cores on x_hat)"}
 
 
 def _chain_graph(qx, torch, stream, layers, chain, outs, pdl=True):

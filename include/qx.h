@@ -257,8 +257,19 @@ qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64_t m, v
  * (row of x): s_b = fp32(max_k |x[b][k]| / 127) and q[b][k] = clamp(rint(x / s_b),
  * -127, 127) in IEEE fp32 (q = 0 when s_b = 0); bit-exact with the CPU oracle.
  * x: device fp16 [batch][k], finite; q: device int8 [batch][k], 16-byte
- * aligned; scales: device fp32 [batch].  batch 1..16, k a multiple of 16. */
+ * aligned; scales: device fp32 [batch].  batch 1..2^24 (decode batches and
+ * prefill token counts alike), k a multiple of 16 up to 2^20. */
 qx_status qx_quantize_act(const void *x, int32_t batch, int64_t k, void *q, void *scales, void *stream);
+
+/* W.A8 prefill activations: the tensor cores take fp16 operands, so the int8
+ * codes of qx_quantize_act enter the matmul as x_hat[b][k] = fp16(fp32(s_b *
+ * q[b][k])), one IEEE fp32 product then a round to nearest even; bit-exact
+ * with the CPU oracle.  Y = x_hat W_hat^T is then qx_gemm (or qx_gemm_splitk,
+ * qx_q4x_gemm) on x_hat: the W.A8 prefill, for any weight format.
+ * q: device int8 [m][k], 16-byte aligned; scales: device fp32 [m]; x_hat:
+ * device fp16 [m][k], 16-byte aligned.  m 1..2^24, k a multiple of 16 up to
+ * 2^20.  Asynchronous on `stream`. */
+qx_status qx_dequant_act(const void *q, const void *scales, int64_t m, int64_t k, void *x_hat, void *stream);
 
 /* W.A8 decode matmul for uniform weights: y[b][n] = s_b * sum_g s_g *
  * sum_{k in g} (q_w - z) q[b][k], the group sums exact integers (dp4a), the

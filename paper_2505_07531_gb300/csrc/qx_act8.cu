@@ -44,6 +44,38 @@ __global__ void __launch_bounds__(kActThreads) quantize_act_kernel(const __half 
     if (threadIdx.x == 0) scales[blockIdx.x] = s;
 }
 
+// W.A8 prefill: the tensor cores take fp16 operands, so the int8 activations
+// enter the matmul as x_hat = fp16(fp32(s_b q)), one IEEE fp32 product then a
+// round to nearest even.  One thread per 16 codes: a 16-byte load, two
+// 16-byte stores.
+constexpr int kDqThreads = 256;
+
+__global__ void __launch_bounds__(kDqThreads) dequant_act_kernel(const int8_t *q, const float *scales, int64_t m,
+                                                                 int64_t k, __half *xh) {
+    const int64_t vpr = k / 16, total = m * vpr;
+    for (int64_t i = (int64_t)blockIdx.x * kDqThreads + threadIdx.x; i < total;
+         i += (int64_t)gridDim.x * kDqThreads) {
+        const float s = scales[i / vpr];
+        const uint4 v = reinterpret_cast<const uint4 *>(q)[i];
+        const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+        uint32_t o[8];
+#pragma unroll
+        for (int t = 0; t < 4; ++t) {
+#pragma unroll
+            for (int e = 0; e < 2; ++e) {
+                const int c0 = (int)(int8_t)((w[t] >> (16 * e)) & 0xffu);
+                const int c1 = (int)(int8_t)((w[t] >> (16 * e + 8)) & 0xffu);
+                const uint32_t h0 = __half_as_ushort(__float2half_rn(__fmul_rn(s, (float)c0)));
+                const uint32_t h1 = __half_as_ushort(__float2half_rn(__fmul_rn(s, (float)c1)));
+                o[2 * t + e] = h0 | (h1 << 16);
+            }
+        }
+        uint4 *dst = reinterpret_cast<uint4 *>(xh) + 2 * i;
+        dst[0] = make_uint4(o[0], o[1], o[2], o[3]);
+        dst[1] = make_uint4(o[4], o[5], o[6], o[7]);
+    }
+}
+
 __device__ __forceinline__ uint32_t prmt_b(uint32_t a, uint32_t b, uint32_t sel) {
     uint32_t d;
     asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
@@ -164,6 +196,14 @@ cudaError_t launch_a8_bits(const GemvA8Args &a, cudaStream_t st) {
 
 cudaError_t launch_quantize_act(const __half *x, int batch, int64_t k, int8_t *q, float *scales, cudaStream_t st) {
     quantize_act_kernel<<<batch, kActThreads, 0, st>>>(x, k, q, scales);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_dequant_act(const int8_t *q, const float *scales, int64_t m, int64_t k, __half *xh, int num_sms,
+                              cudaStream_t st) {
+    const int64_t need = (m * (k / 16) + kDqThreads - 1) / kDqThreads;
+    const unsigned grid = (unsigned)std::max<int64_t>(1, std::min<int64_t>(need, (int64_t)num_sms * 8));
+    dequant_act_kernel<<<grid, kDqThreads, 0, st>>>(q, scales, m, k, xh);
     return cudaGetLastError();
 }
 

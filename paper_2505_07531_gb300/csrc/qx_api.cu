@@ -71,6 +71,9 @@ uint64_t wait_limit_ns() {
 
 bool aligned(const void *p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
+// rows (tokens) of one qx_quantize_act / qx_dequant_act call
+constexpr int64_t kMaxActRows = (int64_t)1 << 24;
+
 int ilog2(int v) {
     int r = 0;
     while ((1 << r) < v) ++r;
@@ -550,14 +553,27 @@ QX_API qx_status qx_gemm_splitk_noalloc(const qx_packed *p, const void *X, int64
 
 QX_API qx_status qx_quantize_act(const void *x, int32_t batch, int64_t k, void *q, void *scales, void *stream) {
     if (x == nullptr || q == nullptr || scales == nullptr) return QX_ERR_INVALID_ARG;
-    if (batch < 1 || batch > 16 || k < 1) return QX_ERR_INVALID_ARG;
-    if (k % 16 != 0 || k > ((int64_t)1 << 20)) return QX_ERR_UNSUPPORTED;
+    if (batch < 1 || k < 1) return QX_ERR_INVALID_ARG;
+    if (batch > kMaxActRows || k % 16 != 0 || k > ((int64_t)1 << 20)) return QX_ERR_UNSUPPORTED;
     if (!aligned(x, 2) || !aligned(q, 16) || !aligned(scales, 4)) return QX_ERR_ALIGNMENT;
     DeviceInfo *d = nullptr;
     qx_status s = device_info(&d);
     if (s != QX_OK) return s;
     return from_cuda(qx::launch_quantize_act(static_cast<const __half *>(x), batch, k, static_cast<int8_t *>(q),
                                              static_cast<float *>(scales), static_cast<cudaStream_t>(stream)));
+}
+
+QX_API qx_status qx_dequant_act(const void *q, const void *scales, int64_t m, int64_t k, void *x_hat, void *stream) {
+    if (q == nullptr || scales == nullptr || x_hat == nullptr) return QX_ERR_INVALID_ARG;
+    if (m < 1 || k < 1) return QX_ERR_INVALID_ARG;
+    if (m > kMaxActRows || k % 16 != 0 || k > ((int64_t)1 << 20)) return QX_ERR_UNSUPPORTED;
+    if (!aligned(q, 16) || !aligned(scales, 4) || !aligned(x_hat, 16)) return QX_ERR_ALIGNMENT;
+    DeviceInfo *d = nullptr;
+    const qx_status s = device_info(&d);
+    if (s != QX_OK) return s;
+    return from_cuda(qx::launch_dequant_act(static_cast<const int8_t *>(q), static_cast<const float *>(scales), m, k,
+                                            static_cast<__half *>(x_hat), d->num_sms,
+                                            static_cast<cudaStream_t>(stream)));
 }
 
 QX_API qx_status qx_gemv_a8(const qx_packed *p, const void *q, const void *scales, int32_t batch, void *y,

@@ -130,6 +130,8 @@ struct GemvA8Args {
     int y_f32;
 };
 cudaError_t launch_quantize_act(const __half *x, int batch, int64_t k, int8_t *q, float *scales, cudaStream_t st);
+cudaError_t launch_dequant_act(const int8_t *q, const float *scales, int64_t m, int64_t k, __half *xh, int num_sms,
+                              cudaStream_t st);
 cudaError_t launch_gemv_a8(const GemvA8Args &a, cudaStream_t st);
 
 // Exact sum of (W - W_hat)^2 2^48 over `count` fp16 elements (a multiple of 8,

@@ -105,6 +105,7 @@ def _lib():
         lib.qx_gemm_splitk_noalloc.argtypes = [P(_Packed), VP, I64, VP, VP]
         lib.qx_quantize_act.argtypes = [VP, I32, I64, VP, VP, VP]
         lib.qx_gemv_a8.argtypes = [P(_Packed), VP, VP, I32, VP, I32, VP]
+        lib.qx_dequant_act.argtypes = [VP, VP, I64, I64, VP, VP]
         lib.qx_select_workspace.argtypes = [I64, I64, P(_Recipe), I32, P(ctypes.c_size_t)]
         lib.qx_select_recipe.argtypes = [VP, I64, I64, P(_Recipe), I32, ctypes.c_double, VP, ctypes.c_size_t,
                                          P(I32), P(ctypes.c_uint64), P(ctypes.c_double), VP]
@@ -129,7 +130,7 @@ def _lib():
         lib.qx_last_error_string.restype = ctypes.c_char_p
         for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemv_chain", "qx_decode_step", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
-                   "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_gemv_a8",
+                   "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_dequant_act", "qx_gemv_a8",
                    "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_q4x_gemm", "qx_q4x_gemm_splitk_workspace",
                    "qx_q4x_gemm_splitk", "qx_selftest_wait_timeout",
                    "qx_get_device_status", "qx_version"):
@@ -467,6 +468,30 @@ def quantize_act(x: torch.Tensor):
     s = torch.empty((b,), dtype=torch.float32, device=x.device)
     _check(_lib().qx_quantize_act(_ptr(x2), b, k, _ptr(q), _ptr(s), _stream(x.device)), "qx_quantize_act")
     return q, s
+
+
+def dequant_act(q: torch.Tensor, scales: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:
+    """fp16 x_hat = fp16(fp32(s_b q)) [m][k] of int8 activations (qx_dequant_act)."""
+    if not _on_device(q) or q.dtype != torch.int8 or not q.is_contiguous():
+        raise ValueError("q must be a contiguous CUDA int8 tensor")
+    _dev_tensor(scales, "scales", torch.float32)
+    m, k = q.shape
+    xh = out if out is not None else torch.empty((m, k), dtype=torch.float16, device=q.device)
+    _dev_tensor(xh, "out")
+    _check(_lib().qx_dequant_act(_ptr(q), _ptr(scales), m, k, _ptr(xh), _stream(q.device)), "qx_dequant_act")
+    return xh
+
+
+def gemm_a8(P, x: torch.Tensor, out: torch.Tensor | None = None, splitk: bool = False) -> torch.Tensor:
+    """W.A8 prefill Y = x_hat W_hat^T: per-token int8 activations
+    (qx_quantize_act), their fp16 form (qx_dequant_act), then the tensor-core
+    matmul (qx_gemm, qx_gemm_splitk with ``splitk``, or qx_q4x_gemm for a
+    Q4xMatrix).  Returns fp16 [m][n]."""
+    q, s = quantize_act(x)
+    xh = dequant_act(q, s)
+    if isinstance(P, Q4xMatrix):
+        return q4x_gemm_splitk(P, xh, out=out) if splitk else q4x_gemm(P, xh, out=out)
+    return gemm_splitk(P, xh, out=out) if splitk else gemm(P, xh, out=out)
 
 
 def gemv_a8(P: PackedMatrix, q: torch.Tensor, scales: torch.Tensor, out: torch.Tensor | None = None,

@@ -181,7 +181,38 @@ def check_stacked():
     assert qx.device_status() == 0
 
 
+def check_a8_prefill():
+    """W.A8 prefill: int8 codes and scales for more tokens than a decode batch,
+    x_hat bit-exact, and the matmul on x_hat within tolerance, for per-group
+    and Q4X weights."""
+    k, m = 256, 37
+    x = synth.activations(m, k, seed=11, stream=12)
+    x[4] = 0  # a dead token
+    q, s = qx.quantize_act(dev(x))
+    qr, sr = oracle.quantize_act(x)
+    assert np.array_equal(q.numpy(), qr) and np.array_equal(s.numpy().view(np.uint32), sr.view(np.uint32))
+    xh = qx.dequant_act(q, s)
+    xr = oracle.dequant_act_f16(qr, sr)
+    assert np.array_equal(bits(xh), xr.view(np.uint16))
+    W = synth.student_t_weights(72, k, 0.02, seed=13, stream=14).astype(np.float16)
+    for rec, orec in [((4, 128, qx.UNIFORM), ORecipe(4, 128, "uniform")), ((3, 128, qx.LUT, 3), ORecipe(3, 128, "lut", 3))]:
+        P = qx.quantize(dev(W), qx.Recipe(*rec))
+        Wh = oracle.dequant(oracle.quantize(W, orec), orec, k)
+        y_ref = oracle.gemm_a8(Wh, x)
+        tol = oracle.tolerance(xr, Wh) + np.abs(y_ref).max(axis=1) * 2.0 ** -11
+        Y = qx.gemm_a8(P, dev(x)).numpy().astype(np.float64)
+        assert np.all(oracle.max_abs_err(Y, y_ref) <= tol), rec
+    P4 = qx.q4x_quantize(dev(W), 2)
+    ref = oracle.quantize_q4x(W, iters=2)
+    Wh = oracle.dequant_q4x(ref["codes"], ref["scales"], ref["books"], ref["codebooks"])
+    y_ref = oracle.gemm_a8(Wh, x)
+    Y = qx.gemm_a8(P4, dev(x)).numpy().astype(np.float64)
+    assert np.all(oracle.max_abs_err(Y, y_ref) <= oracle.tolerance(xr, Wh) + np.abs(y_ref).max(axis=1) * 2.0 ** -11)
+    assert qx.device_status() == 0
+
+
 def main():
+    check_a8_prefill()
     check_q4x(37, 384, 2)
     check_select()
     check_chain_and_step()

@@ -101,8 +101,19 @@ def test_entry_points_reject_bad_arguments_before_launching(qx):
     assert lib.qx_gemm_splitk_workspace(4096, 4096, 1, None, ctypes.byref(nbytes)) == 1
     # W.A8: activation and matmul argument checks
     assert lib.qx_quantize_act(None, 1, 128, None, None, None) == 1
-    assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 17, 128, ctypes.c_void_p(0x5000), ctypes.c_void_p(0x6000),
+    assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 0, 128, ctypes.c_void_p(0x5000), ctypes.c_void_p(0x6000),
                                None) == 1
+    assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), (1 << 24) + 1, 128, ctypes.c_void_p(0x5000),
+                               ctypes.c_void_p(0x6000), None) == 2  # up to 2^24 tokens
+    # W.A8 prefill activations: pointers, sizes, alignment
+    A, S, X = ctypes.c_void_p(0x4000), ctypes.c_void_p(0x5000), ctypes.c_void_p(0x6000)
+    assert lib.qx_dequant_act(None, S, 4, 128, X, None) == 1
+    assert lib.qx_dequant_act(A, S, 0, 128, X, None) == 1
+    assert lib.qx_dequant_act(A, S, 4, 120, X, None) == 2
+    assert lib.qx_dequant_act(A, S, (1 << 24) + 1, 128, X, None) == 2
+    assert lib.qx_dequant_act(ctypes.c_void_p(0x4008), S, 4, 128, X, None) == 3
+    assert lib.qx_dequant_act(A, ctypes.c_void_p(0x5002), 4, 128, X, None) == 3
+    assert lib.qx_dequant_act(A, S, 4, 128, ctypes.c_void_p(0x6008), None) == 3
     assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 1, 120, ctypes.c_void_p(0x5000), ctypes.c_void_p(0x6000),
                                None) == 2
     assert lib.qx_quantize_act(ctypes.c_void_p(0x4000), 1, 128, ctypes.c_void_p(0x5008), ctypes.c_void_p(0x6000),
