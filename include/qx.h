@@ -268,7 +268,9 @@ qx_status qx_quantize_act(const void *x, int32_t batch, int64_t k, void *q, void
  * qx_q4x_gemm) on x_hat: the W.A8 prefill, for any weight format.
  * q: device int8 [m][k], 16-byte aligned; scales: device fp32 [m]; x_hat:
  * device fp16 [m][k], 16-byte aligned.  m 1..2^24, k a multiple of 16 up to
- * 2^20.  Asynchronous on `stream`. */
+ * 2^20.  Asynchronous on `stream`.  Errors (nothing launched): INVALID_ARG
+ * (NULL, m < 1, k < 1), UNSUPPORTED (k not a multiple of 16, k > 2^20,
+ * m > 2^24), ALIGNMENT (q or x_hat not 16-byte, scales not 4-byte aligned). */
 qx_status qx_dequant_act(const void *q, const void *scales, int64_t m, int64_t k, void *x_hat, void *stream);
 
 /* W.A8 decode matmul for uniform weights: y[b][n] = s_b * sum_g s_g *
