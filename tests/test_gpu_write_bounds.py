@@ -86,6 +86,16 @@ def test_per_group_entry_points_stay_in_bounds(qx, n, k, bits, gs, kind):
         qx.gemv_a8(P, q.t.view(batch, k), s.t, out=y.t.view(batch, n))
         assert torch.equal(y.t.view(batch, n), qx.gemv_a8(ref, q2, s2, out_dtype=torch.float32))
         bands += [q, s, y]
+        # W.A8 prefill: more tokens than a decode batch, then x_hat
+        m = 20
+        X = torch.from_numpy(synth.activations(m, k, seed=8, stream=n)).cuda()
+        q, s, xh = Guarded(m * k, torch.int8), Guarded(4 * m, torch.float32), Guarded(2 * m * k, torch.float16)
+        qx._check(qx._lib().qx_quantize_act(qx._ptr(X), m, k, qx._ptr(q.t), qx._ptr(s.t),
+                                            qx._stream(X.device)), "qx_quantize_act")
+        qx.dequant_act(q.t.view(m, k), s.t, out=xh.t.view(m, k))
+        q2, s2 = qx.quantize_act(X)
+        assert torch.equal(xh.t.view(m, k), qx.dequant_act(q2, s2))
+        bands += [q, s, xh]
     assert qx.device_status() == 0
     assert all(b.intact() for b in bands)
 
