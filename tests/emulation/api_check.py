@@ -189,6 +189,15 @@ def check_per_group(n, k, bits, g, kind):
         w_exact = (qw - z) * np.repeat(ref["scales"].astype(np.float64), g, axis=1)
         within(y.reshape(batch, n), oracle.gemv_a8(ref, orec, x, k), oracle.tolerance(oracle.dequant_act(qr, sr),
                                                                                       w_exact))
+    # W.A8 prefill activations for more tokens than a decode batch, any weight format
+    m = 19
+    x = synth.activations(m, k, seed=12, stream=n)
+    q, s, xh = buf(m * k, np.int8), buf(4 * m, np.float32), buf(2 * m * k, np.float16)
+    ok(L.qx_quantize_act(P(put(x)), m, k, P(q), P(s), None), "qx_quantize_act (prefill)")
+    ok(L.qx_dequant_act(P(q), P(s), m, k, P(xh), None), "qx_dequant_act")
+    qr, sr = oracle.quantize_act(x)
+    assert np.array_equal(q.reshape(m, k), qr) and np.array_equal(s, sr), "prefill int8 activations"
+    assert np.array_equal(xh.view(np.uint16), oracle.dequant_act_f16(qr, sr).view(np.uint16).ravel()), "x_hat"
     assert status() == 0
 
 
