@@ -457,16 +457,7 @@ def run_ours(args):
     e2e_ms = _max_over_ranks(dist, (time.perf_counter() - t0) * 1e3 / e2e_steps, dev)
     e2e_value = _job_rate(step_bytes, ws, e2e_ms) / 1e9
 
-    def section(fn, *a):
-        # a section that fails reports its error in its own key; the headline
-        # figures above and the other sections stand
-        try:
-            return fn(*a)
-        except Exception as e:  # noqa: BLE001
-            return {"error": f"{type(e).__name__}: {e}"[:300]}
-        finally:
-            torch.cuda.empty_cache()
-
+    section = lambda fn, *a: _section(torch, fn, *a)  # noqa: E731
     gemm = section(run_gemm_part, qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
     del layers, graphs
     extra = {}
@@ -510,6 +501,18 @@ def run_ours(args):
         print(json.dumps(line))
     if dist is not None:
         dist.destroy_process_group()
+
+
+def _section(torch, fn, *a):
+    """fn(*a), or {"error": ...} if it raises: a section that fails reports its
+    error in its own key, and the headline figures and the other sections
+    stand.  The caching allocator's free blocks are released either way."""
+    try:
+        return fn(*a)
+    except Exception as e:  # noqa: BLE001
+        return {"error": f"{type(e).__name__}: {e}"[:300]}
+    finally:
+        torch.cuda.empty_cache()
 
 
 def run_gemm_part(qx, torch, dev, stream, tf_burst, peak_src):

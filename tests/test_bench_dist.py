@@ -53,6 +53,32 @@ def test_single_process_needs_no_process_group(monkeypatch):
     assert bench._job_rate(2e9, 1, 1.0) == pytest.approx(2e12)
 
 
+def test_a_failing_section_reports_its_error_and_the_run_goes_on():
+    """bench.py's sections after the headline (GEMM, configs, Q4X) each return
+    their figures or an {"error": ...} of their own; the allocator's cache is
+    released after each either way."""
+    sys.path.insert(0, ROOT)
+    import bench
+
+    released = []
+
+    class _Cuda:
+        @staticmethod
+        def empty_cache():
+            released.append(1)
+
+    class _Torch:
+        cuda = _Cuda
+
+    def boom(n):
+        raise RuntimeError("device error " * n)
+
+    assert bench._section(_Torch, lambda a, b: {"v": a + b}, 2, 3) == {"v": 5}
+    out = bench._section(_Torch, boom, 100)
+    assert out["error"].startswith("RuntimeError: device error") and len(out["error"]) == 300
+    assert released == [1, 1]
+
+
 def test_reference_arm_under_torchrun_prints_once_from_rank_0():
     """`bench.py --impl reference` launched as the driver launches N = 2: rank 0
     alone runs the oracle and prints one JSON line; rank 1 exits 0 without work."""
