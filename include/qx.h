@@ -127,11 +127,10 @@ qx_status qx_dequant(const qx_packed *p, void *W_out, void *stream);
 /* Decode matmul y = x W_hat^T (Section 2.4: memory-bound decoding; Table 2
  * "Decode").  x: device fp16 [batch][k], row-major, 16-byte aligned;
  * y: device [batch][n] of y_dtype (QX_F16 or QX_F32), 4-byte aligned.
- * batch in 1..16; k <= 32768.  fp16 products summed in fp32 per 32 weights
- * and across groups; the products and their sums over 16 consecutive weight
- * pairs are formed in fp16, so they must stay within its range (|.| < 65504),
- * which LLM weights and activations satisfy by orders of magnitude.  Batches above four stream the weights once per eight
- * rows of x (once per four where eight rows of x do not fit on chip). */
+ * batch in 1..16; k <= 32768.  The weights are dequantized in registers
+ * (w_hat exactly as qx_dequant) and multiplied on the tensor cores with x:
+ * the fp16 products are exact and summed in fp32.  One launch streams the
+ * weights once for the whole batch. */
 qx_status qx_gemv(const qx_packed *p, const void *x, int32_t batch, void *y,
                   int32_t y_dtype, void *stream);
 
@@ -189,6 +188,33 @@ typedef struct qx_copy {
 qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
                          int32_t batch, int32_t y_dtype, int32_t flags, const qx_copy *out, int32_t nout,
                          int32_t sync, void *stream);
+
+/* Bytes of workspace qx_gemv_fused and qx_decode_step_fused need (host only;
+ * a small constant). */
+qx_status qx_gemv_fused_workspace(size_t *bytes);
+
+/* The groups of qx_gemv_chain (Section 2.4: decoding is memory-bound, so the
+ * weight stream should not stop between the projections of a layer) in ONE
+ * persistent launch: one CTA per SM streams the weights of every group without
+ * a break, and group i + 1 reads its x only once every CTA has finished group
+ * i (its y written), so x of a later group may be the y of an earlier one.
+ * The results equal qx_gemv_chain's bit for bit.  ngroups 1..64; the groups
+ * run as one launch when there are at most 4 of them with at most 16 matrices
+ * in all, sharing bits and kind (else as qx_gemv_chain runs them).
+ * workspace: caller-owned device memory, 256-byte aligned, of at least
+ * qx_gemv_fused_workspace() bytes, all zero before the first call: every
+ * completed call leaves it zero (zero it again after QX_ERR_TIMEOUT).  Calls
+ * that may run at the same time need separate workspaces.  flags: 0 or
+ * QX_GEMV_PDL.  Errors: those of qx_gemv_chain; INVALID_ARG (workspace NULL
+ * or too small), ALIGNMENT (workspace). */
+qx_status qx_gemv_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                        int32_t flags, void *workspace, size_t workspace_bytes, void *stream);
+
+/* qx_decode_step with the groups run by qx_gemv_fused (same workspace rules). */
+qx_status qx_decode_step_fused(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
+                               int32_t batch, int32_t y_dtype, int32_t flags, void *workspace,
+                               size_t workspace_bytes, const qx_copy *out, int32_t nout, int32_t sync,
+                               void *stream);
 
 /* Prefill matmul Y = X W_hat^T (Table 2 "Prefill") on the tcgen05 tensor cores:
  * W_hat tiles are dequantized into shared memory and multiplied in fp16 with

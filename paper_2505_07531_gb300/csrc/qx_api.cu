@@ -227,8 +227,11 @@ std::mutex g_plan_mu;
 
 bool same_inputs(const qx::GemvMulti &p, const qx::GemvMulti &a) {
     if (p.count != a.count || p.bits != a.bits || p.kind != a.kind || p.batch != a.batch || p.y_f32 != a.y_f32 ||
-        p.status != a.status || p.wait_limit_ns != a.wait_limit_ns)
+        p.status != a.status || p.wait_limit_ns != a.wait_limit_ns || p.nphase != a.nphase ||
+        p.phase_ctr != a.phase_ctr)
         return false;
+    for (int i = 0; i <= a.nphase; ++i)
+        if (p.phase_first[i] != a.phase_first[i]) return false;
     for (int i = 0; i < a.count; ++i) {
         const qx::GemvMat &u = p.mat[i], &v = a.mat[i];
         if (u.codes != v.codes || u.scales != v.scales || u.zeros != v.zeros || u.luts != v.luts || u.x != v.x ||
@@ -261,35 +264,39 @@ bool plan_cached(qx::GemvMulti &a, const DeviceInfo *d) {
     return true;
 }
 
-// One decode launch over `count` matrices for activation rows b0 .. b0+nb-1
-// (nb <= 4, or 8).  When the group's activations do not fit one CTA's shared
-// memory, the group is split per matrix, then the rows are halved.
+// One decode launch over `count` matrices for activation rows b0 .. b0+nb-1.
+// Should a plan not fit (a tensor map the driver refuses, or shared memory),
+// the group is split per matrix, then the rows are halved.
+// The per-matrix launch fields of packed matrix p with activation rows b0..
+void fill_mat(qx::GemvMat &M, const qx_packed &p, const void *x, void *y, int b0, int esz) {
+    M.codes = static_cast<const uint8_t *>(p.codes);
+    M.scales = static_cast<const __half *>(p.scales);
+    M.zeros = static_cast<const uint8_t *>(p.zeros);
+    M.luts = static_cast<const __half *>(p.luts);
+    M.x = static_cast<const __half *>(x) + (int64_t)b0 * p.k;
+    M.y = static_cast<uint8_t *>(y) + (int64_t)b0 * p.n * esz;
+    M.n = p.n;
+    M.k = p.k;
+    M.G = (int)(p.k / p.recipe.group_size);
+    M.zbytes = (M.G + 1) / 2;
+    M.log2g = ilog2(p.recipe.group_size);
+}
+
 qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int b0, int nb, void *const *y,
                      int y_dtype, int flags, cudaStream_t st, DeviceInfo *d) {
     const int esz = y_dtype == QX_F32 ? 4 : 2;
     qx::GemvMulti a{};
     a.count = count;
+    a.nphase = 1;
+    a.phase_first[0] = 0;
+    a.phase_first[1] = count;
     a.bits = mats[0].recipe.bits;
     a.kind = mats[0].recipe.kind;
     a.batch = nb;
     a.y_f32 = y_dtype == QX_F32;
     a.status = d->status;
     a.wait_limit_ns = wait_limit_ns();
-    for (int i = 0; i < count; ++i) {
-        const qx_packed &p = mats[i];
-        qx::GemvMat &M = a.mat[i];
-        M.codes = static_cast<const uint8_t *>(p.codes);
-        M.scales = static_cast<const __half *>(p.scales);
-        M.zeros = static_cast<const uint8_t *>(p.zeros);
-        M.luts = static_cast<const __half *>(p.luts);
-        M.x = static_cast<const __half *>(x[i]) + (int64_t)b0 * p.k;
-        M.y = static_cast<uint8_t *>(y[i]) + (int64_t)b0 * p.n * esz;
-        M.n = p.n;
-        M.k = p.k;
-        M.G = (int)(p.k / p.recipe.group_size);
-        M.zbytes = (M.G + 1) / 2;
-        M.log2g = ilog2(p.recipe.group_size);
-    }
+    for (int i = 0; i < count; ++i) fill_mat(a.mat[i], mats[i], x[i], y[i], b0, esz);
     if (plan_cached(a, d))
         return from_cuda(qx::launch_gemv_multi(a, st, (flags & QX_GEMV_PDL) != 0));
     if (count > 1) {
@@ -307,18 +314,11 @@ qx_status gemv_chunk(const qx_packed *mats, int count, const void *const *x, int
     return QX_ERR_UNSUPPORTED;
 }
 
-// Kernels exist for 1..4 and 8 rows of x: a batch is processed eight rows at
-// a time while at least eight remain, then four at a time; each chunk
-// streams the weights once.
+// One launch covers the whole batch (1..16 rows of x): the kernel reads x from
+// global memory, so the weights are streamed once whatever the batch.
 qx_status run_gemv(const qx_packed *mats, int count, const void *const *x, int batch, void *const *y,
                    int y_dtype, int flags, cudaStream_t st, DeviceInfo *d) {
-    for (int b0 = 0; b0 < batch;) {
-        const int nb = batch - b0 >= 8 ? 8 : std::min(4, batch - b0);
-        qx_status s = gemv_chunk(mats, count, x, b0, nb, y, y_dtype, flags, st, d);
-        if (s != QX_OK) return s;
-        b0 += nb;
-    }
-    return QX_OK;
+    return gemv_chunk(mats, count, x, 0, batch, y, y_dtype, flags, st, d);
 }
 
 qx_status check_gemv_args(const qx_packed *p, const void *x, int32_t batch, const void *y, int32_t y_dtype) {
@@ -426,6 +426,107 @@ QX_API qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_gr
         if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
             return s;
     if ((s = run_chain(groups, ngroups, batch, y_dtype, flags, st, d)) != QX_OK) return s;
+    for (int i = 0; i < nout; ++i)
+        if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
+            QX_OK)
+            return s;
+    return sync ? from_cuda(cudaStreamSynchronize(st)) : QX_OK;
+}
+
+namespace {
+
+constexpr size_t kFusedWorkspaceBytes = 256;  // one phase counter per group, padded
+
+// The groups of a decode step in one persistent launch (qx::GemvMulti with one
+// phase per group).  *launched is false, with nothing launched, when they
+// cannot share one: more groups or matrices than a launch holds, different
+// bits or kinds, or a plan that does not fit.
+qx_status run_fused(const qx_gemv_group *groups, int ngroups, int batch, int y_dtype, int flags, void *ws,
+                    cudaStream_t st, DeviceInfo *d, bool *launched) {
+    *launched = false;
+    if (ngroups > qx::kMaxGemvPhases) return QX_OK;
+    const int esz = y_dtype == QX_F32 ? 4 : 2;
+    qx::GemvMulti a{};
+    a.bits = groups[0].mats[0].recipe.bits;
+    a.kind = groups[0].mats[0].recipe.kind;
+    a.batch = batch;
+    a.y_f32 = y_dtype == QX_F32;
+    a.status = d->status;
+    a.wait_limit_ns = wait_limit_ns();
+    a.nphase = ngroups;
+    a.phase_ctr = static_cast<uint32_t *>(ws);
+    int count = 0;
+    for (int gi = 0; gi < ngroups; ++gi) {
+        const qx_gemv_group &g = groups[gi];
+        a.phase_first[gi] = count;
+        for (int i = 0; i < g.count; ++i) {
+            if (count == qx::kMaxGemvTotal) return QX_OK;
+            if (g.mats[i].recipe.bits != a.bits || g.mats[i].recipe.kind != a.kind) return QX_OK;
+            fill_mat(a.mat[count++], g.mats[i], g.x[i], g.y[i], 0, esz);
+        }
+    }
+    a.count = count;
+    a.phase_first[ngroups] = count;
+    if (!plan_cached(a, d)) return QX_OK;
+    const cudaError_t e = qx::launch_gemv_multi(a, st, (flags & QX_GEMV_PDL) != 0);
+    if (e == cudaErrorCooperativeLaunchTooLarge) {  // not all CTAs resident at once: run them apart
+        cudaGetLastError();
+        return QX_OK;
+    }
+    *launched = true;
+    return from_cuda(e);
+}
+
+qx_status check_fused_ws(const void *ws, size_t bytes) {
+    if (ws == nullptr || bytes < kFusedWorkspaceBytes) return QX_ERR_INVALID_ARG;
+    if (!aligned(ws, 256)) return QX_ERR_ALIGNMENT;
+    return QX_OK;
+}
+
+qx_status run_chain_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                          int32_t flags, void *ws, cudaStream_t st, DeviceInfo *d) {
+    if (ngroups > 1) {
+        bool launched = false;
+        const qx_status s = run_fused(groups, ngroups, batch, y_dtype, flags, ws, st, d, &launched);
+        if (s != QX_OK || launched) return s;
+    }
+    return run_chain(groups, ngroups, batch, y_dtype, flags, st, d);
+}
+
+}  // namespace
+
+QX_API qx_status qx_gemv_fused_workspace(size_t *bytes) {
+    if (bytes == nullptr) return QX_ERR_INVALID_ARG;
+    *bytes = kFusedWorkspaceBytes;
+    return QX_OK;
+}
+
+QX_API qx_status qx_gemv_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                               int32_t flags, void *workspace, size_t workspace_bytes, void *stream) {
+    qx_status s = check_chain(groups, ngroups, batch, y_dtype, flags);
+    if (s == QX_OK) s = check_fused_ws(workspace, workspace_bytes);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    return run_chain_fused(groups, ngroups, batch, y_dtype, flags, workspace, static_cast<cudaStream_t>(stream), d);
+}
+
+QX_API qx_status qx_decode_step_fused(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
+                                      int32_t batch, int32_t y_dtype, int32_t flags, void *workspace,
+                                      size_t workspace_bytes, const qx_copy *out, int32_t nout, int32_t sync,
+                                      void *stream) {
+    qx_status s = check_copies(in, nin);
+    if (s == QX_OK) s = check_copies(out, nout);
+    if (s == QX_OK) s = check_chain(groups, ngroups, batch, y_dtype, flags);
+    if (s == QX_OK) s = check_fused_ws(workspace, workspace_bytes);
+    if (s != QX_OK) return s;
+    DeviceInfo *d = nullptr;
+    if ((s = device_info(&d)) != QX_OK) return s;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    for (int i = 0; i < nin; ++i)
+        if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
+            return s;
+    if ((s = run_chain_fused(groups, ngroups, batch, y_dtype, flags, workspace, st, d)) != QX_OK) return s;
     for (int i = 0; i < nout; ++i)
         if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
             QX_OK)

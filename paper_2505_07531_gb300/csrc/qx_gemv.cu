@@ -1,62 +1,59 @@
-// Decode matmul y[b][n] = sum_k w_hat[n][k] x[b][k] on CUDA cores, fed by TMA.
+// Decode matmul y[b][n] = sum_k w_hat[n][k] x[b][k] for 1..16 rows of x, the
+// weights dequantized in registers.
 //
 // Decoding reads every weight once per token, so it is bound by HBM bandwidth
 // and by the cost of unpacking the codes (paper Section 2.4).  On GB300 the
 // unpack of a 3-bit code through an 8-entry table costs about one byte-permute
-// per weight, which at HBM speed keeps the integer pipe nearly busy: the
-// kernel is built to spend as few issue slots as possible on anything else.
+// per weight on the integer pipe; everything else a weight needs is kept off
+// that pipe and off the issue slots:
 //
-//   * Work unit: a 32-row block of one matrix.  Lane r of every warp owns row
-//     r of the block, so a row's dot product never needs a warp shuffle and
-//     the activations x are the same for all lanes (a broadcast load).
-//   * The rows are streamed in slices of 1024 weights: one stage of the
-//     shared-memory ring holds the codes (and LUTs) of 32 rows x 1024 k,
-//     fetched with 2-D/3-D TMA tensor copies in the 128-byte swizzled layout,
-//     which makes the per-lane 16-byte reads of 32 different rows free of bank
-//     conflicts.
-//   * Sixteen warps in four groups of four: group g decodes the stages q with
-//     q % 4 == g, and each of its warps one 256-weight part of each of them
-//     (two 3-bit superblocks), so four stages are in decode at once.
-//   * No producer warp (a seventeenth warp puts five warps on one SM
-//     sub-partition, which caps every thread at 96 registers): the first
-//     stages are issued from the kernel parameters by one lane each before the
-//     programmatic-dependent-launch wait (weights do not depend on the
-//     previous kernel); the rest of the ring is requested as those land, and
-//     afterwards the last warp of a group to release a stage refills it.
-//   * Partial sums of a row block stay in registers across its slices; at the
+//   * Lane (g, t) = (lane / 4, lane % 4) of a warp takes the 32-weight unit t
+//     of a 128-weight superblock for rows g and g + 8 of a 16-row tile.  Ten
+//     code words per lane arrive by two ldmatrix instructions from the
+//     128-byte swizzled TMA stage (free of bank conflicts), and the lane
+//     decodes them in their natural order.
+//   * Products: one or two rows of x on the CUDA cores (fp16 products summed
+//     over 8 weight pairs per chain, then fp32); three or more on the tensor
+//     cores, mma.sync m16n8k16 with the dequantized weights as A (16 rows x
+//     16 k) and x as B (16 k x 8 rows of x), fp32 accumulation.  The order of
+//     the contraction inside an MMA is free as long as A and B agree, so a
+//     lane loads x for the same 32 k it decodes.  One MMA serves up to 8 rows
+//     of x (two up to 16): a small batch costs the weight traffic of one.
+//   * A stage of the shared-memory ring holds the codes (and LUTs) of 32 rows
+//     x 1024 k.  Sixteen warps in two groups: group g takes the stages q with
+//     q % 2 == g, and warp w of a group decodes superblock w of each of its
+//     stages for both 16-row tiles (its x fragments serve both).
+//   * A producer warp issues the copies, each once the eight warps of the
+//     slot's group have released its previous fill (an mbarrier every lane
+//     arrives at); waits suspend in hardware rather than spin.
+//   * Partial sums of a row block stay in registers across its stages; at the
 //     end of the block each warp stores its partials and the last contributor
 //     adds them in a fixed order (deterministic) and writes y.
-//   * Uniform scales and zero-points are read by each lane from global memory
-//     one stage ahead, after the block's first copy has pulled its metadata
-//     into L2 with a bulk prefetch.
-// One CTA of 512 threads per SM.  Under programmatic dependent launch the
-// next decode kernel's CTA takes an SM as soon as this kernel's CTA there has
-// exited and issues its weight copies before it waits.  Every wait is
-// bounded in time and reports QX_ERR_TIMEOUT through the device status.
+//   * x is read from global memory (L1/L2): no per-launch staging.
+//   * One launch may run several groups of matrices one after another
+//     (qx_gemv_fused): the producer streams the weights of every group without
+//     a break, and the consumers of group p + 1 read x only once every CTA has
+//     counted group p done in a device-side counter.
+// Every wait is bounded in time and reports QX_ERR_TIMEOUT through the device
+// status.
 #include "qx_kernels.cuh"
 
 namespace qx {
 
 namespace {
 
-constexpr int kGroups = 4;       // warp groups; group g takes the stages q with q % kGroups == g
-constexpr int kGroupWarps = 4;   // warps per group, one 256-weight part of a stage each
-constexpr int kWarps = kGroups * kGroupWarps;
-constexpr int kThreads = 32 * kWarps;
-constexpr int kRows = 32;           // rows per block (one per lane)
-constexpr int kSliceK = 1024;       // weights per row per stage
-constexpr int kPartK = kSliceK / kGroupWarps;  // weights per warp per stage
-constexpr int kBox = kRows * 128;   // one 32-row x 128-byte TMA box
-constexpr int kMaxRing = 8;
-// Stages issued at start (GemvMulti::initial): one per warp group for a
-// standalone launch -- requesting the whole ring at once makes every stage
-// land late, as the memory system serves them interleaved; the rest of the
-// ring is issued as the first stages land.  A launch that follows another
-// kernel under programmatic dependent launch requests the whole ring, whose
-// latency then hides behind the previous kernel.
-constexpr int kMaxRbSlots = 16;
-constexpr int kHeader = 1024;       // barriers, counters, per-matrix CTA plan
+constexpr int kWarps = 8;        // warps per group: warp w decodes superblock w of a stage
+constexpr int kGroups = 2;       // group g takes the stages q with q % kGroups == g
+constexpr int kProducer = kWarps * kGroups;  // the warp after the consumers issues the copies
+constexpr int kThreads = 32 * (kWarps * kGroups + 1);
+constexpr int kRows = 32;        // rows per block: two 16-row MMA tiles
+constexpr int kSliceK = 1024;    // weights per row per stage: eight 128-weight superblocks
+constexpr int kBox = kRows * 128;  // one 32-row x 128-byte TMA box
+constexpr int kMaxRing = 12;
+constexpr int kMaxRbSlots = 8;
+constexpr int kHeader = 2048;    // barriers, counters, per-matrix and per-phase CTA plan
 constexpr int kSmemBudget = 220 * 1024;
+constexpr int kCoreBatch = 2;    // batches up to this take the CUDA-core products
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -68,6 +65,10 @@ __device__ __forceinline__ void mbar_init(uint32_t b, uint32_t count) {
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint32_t b, uint32_t bytes) {
     asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(b), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t b) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(b) : "memory");
 }
 
 __device__ __forceinline__ bool mbar_try_wait(uint32_t b, uint32_t parity) {
@@ -82,6 +83,21 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t b, uint32_t parity) {
     return ok != 0;
 }
 
+// try_wait that lets the hardware suspend the warp until the phase completes
+// (for at most about `hint_ns`): a waiting warp takes no issue slots from the
+// warps that share its scheduler.
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint32_t b, uint32_t parity, uint32_t hint_ns) {
+    uint32_t ok;
+    asm volatile(
+        "{\n\t.reg .pred p;\n\t"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+        "selp.u32 %0, 1, 0, p;\n\t}"
+        : "=r"(ok)
+        : "r"(b), "r"(parity), "r"(hint_ns)
+        : "memory");
+    return ok != 0;
+}
+
 // Bounded wait: false after `limit_ns`, or once another warp has raised the
 // abort flag (when `abort_flag` is not null).
 __device__ __noinline__ bool mbar_wait(uint32_t b, uint32_t parity, uint64_t limit_ns,
@@ -89,19 +105,21 @@ __device__ __noinline__ bool mbar_wait(uint32_t b, uint32_t parity, uint64_t lim
     if (mbar_try_wait(b, parity)) return true;
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
-        if (mbar_try_wait(b, parity)) return true;
+        if (mbar_try_wait_sleep(b, parity, 1000u)) return true;
         if (abort_flag != nullptr && *abort_flag) return false;
         if (globaltimer_ns() - t0 > limit_ns) return false;
     }
 }
 
-// Bounded wait for a shared-memory word to reach `want`.
+// Bounded wait for a shared-memory word to reach `want` (backing off between
+// reads, so that the waiting warp leaves the scheduler to the others).
 __device__ __noinline__ bool wait_equal(uint32_t *p, uint32_t want, uint64_t limit_ns,
                                         volatile uint32_t *abort_flag) {
     volatile uint32_t *v = p;
     if (*v == want) return true;
     const uint64_t t0 = globaltimer_ns();
     for (;;) {
+        __nanosleep(64);
         if (*v == want) {
             __threadfence_block();
             return true;
@@ -109,6 +127,18 @@ __device__ __noinline__ bool wait_equal(uint32_t *p, uint32_t want, uint64_t lim
         if (*abort_flag) return false;
         if (globaltimer_ns() - t0 > limit_ns) return false;
     }
+}
+
+// Shared-memory counter increment with acquire-release ordering at CTA scope:
+// the caller's earlier shared stores are visible to whoever sees the new count,
+// and the caller sees the stores of those that counted before it.
+__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t *p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], %2;"
+                 : "=r"(old)
+                 : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))), "r"(v)
+                 : "memory");
+    return old;
 }
 
 __device__ __forceinline__ void tma_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
@@ -140,30 +170,43 @@ __device__ __forceinline__ uint4 lds128(uint32_t a) {
     return v;
 }
 
-__device__ __forceinline__ float dot16(const __half2 (&w)[16], const __half2 (&x)[16]) {
-    __half2 a0 = __hmul2(w[0], x[0]);
-    __half2 a1 = __hmul2(w[1], x[1]);
-#pragma unroll
-    for (int i = 2; i < 16; i += 2) {
-        a0 = __hfma2(w[i], x[i], a0);
-        a1 = __hfma2(w[i + 1], x[i + 1], a1);
-    }
-    const float2 f0 = __half22float2(a0);
-    const float2 f1 = __half22float2(a1);
-    return (f0.x + f0.y) + (f1.x + f1.y);
+// ldmatrix (8x8 b16 matrices): lanes 8i..8i+7 give the row addresses of matrix
+// i; lane (g, t) receives bytes 4t..4t+3 of row g of each matrix.
+__device__ __forceinline__ void ldsm_x4(uint32_t a, uint32_t &d0, uint32_t &d1, uint32_t &d2, uint32_t &d3) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(d0), "=r"(d1), "=r"(d2), "=r"(d3)
+                 : "r"(a));
 }
 
-// 32 activations x[k .. k+31] from shared memory (the same address in every
-// lane: a broadcast).
-__device__ __forceinline__ void load_x32(uint32_t p, __half2 (&x)[16]) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        const uint4 t = lds128(p + 16u * i);
-        x[4 * i + 0] = u2h2(t.x);
-        x[4 * i + 1] = u2h2(t.y);
-        x[4 * i + 2] = u2h2(t.z);
-        x[4 * i + 3] = u2h2(t.w);
-    }
+__device__ __forceinline__ void ldsm_x2(uint32_t a, uint32_t &d0, uint32_t &d1) {
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(d0), "=r"(d1) : "r"(a));
+}
+
+// D += A B, m16n8k16, fp16 operands, fp32 accumulators.  Lane (g, t) holds
+// a0 = A[g][2t..2t+1], a1 = A[g+8][2t..2t+1], a2 = A[g][2t+8..2t+9],
+// a3 = A[g+8][2t+8..2t+9]; b0 = B[2t..2t+1][g], b1 = B[2t+8..2t+9][g];
+// d = D[g][2t], D[g][2t+1], D[g+8][2t], D[g+8][2t+1].
+__device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                         uint32_t b0, uint32_t b1) {
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+        "{%0, %1, %2, %3};"
+        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// 16 bytes of x: through the read-only path, or (fused launches, whose x may
+// be written by an earlier phase of the same launch) from L2.
+__device__ __forceinline__ uint4 ldg_x(const __half *p, bool l2) {
+    uint4 v;
+    if (l2)
+        asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                     : "l"(p));
+    else
+        asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
+                     : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
+                     : "l"(p));
+    return v;
 }
 
 // Offset of 16-byte chunk `c` of 128-byte box row `r` inside a 1024-byte-aligned
@@ -179,7 +222,6 @@ struct MatS {
     const __half *x;
     void *y;
     int n, K, G, zbytes, log2g, nks, nlb;
-    int xoff;   // shared-memory offset (halves) of this matrix's x
     int q0;     // first CTA-local stage of this matrix
     int rbq0;   // first CTA-local row block of this matrix
     int rb0;    // first matrix-local row block of this CTA
@@ -187,32 +229,19 @@ struct MatS {
 };
 
 struct Header {
-    uint64_t full[kMaxRing];
-    uint32_t rel[kMaxRing];        // warps done with the stage's current fill
+    uint64_t full[kMaxRing];       // a stage's copies have landed
+    uint64_t empty[kMaxRing];      // the eight warps of its group are done with it
     uint32_t cnt[kMaxRbSlots];     // warps that stored their partials of a block
     uint32_t gen[kMaxRbSlots];     // blocks finished in each partial-sum slot
     uint32_t abort_flag;
-    uint32_t issued;               // stages issued so far
-    int nstages;
-    MatS mats[kMaxGemvMats];
-    int q_end[kMaxGemvMats];       // q0 of the next matrix (nstages for the last)
+    int ph_q0[kMaxGemvPhases + 1];  // first CTA-local stage of each phase (multiples of kGroups)
+    int ph_nst[kMaxGemvPhases];     // stages of each phase in this CTA (before the padding)
+    MatS mats[kMaxGemvTotal];
 };
 static_assert(sizeof(Header) <= kHeader, "header does not fit");
 
-// Stage q of this CTA: matrix, matrix-local row block, slice.
-__device__ __forceinline__ void stage_coords(const Header &h, int count, int q, int &m, int &rb, int &ks) {
-    m = 0;
-    while (m + 1 < count && q >= h.q_end[m]) ++m;
-    const int local = q - h.mats[m].q0;
-    const int nks = h.mats[m].nks;
-    const int rbl = local / nks;
-    rb = h.mats[m].rb0 + rbl;
-    ks = local - rbl * nks;
-}
-
-// Issue the TMA copies of stage q into its ring slot (one thread).
 // Geometry a stage copy needs, from the shared-memory table or straight from
-// the kernel parameters (the first copy is issued before the table exists).
+// the kernel parameters (the first copies are issued before the table exists).
 struct Geom {
     int K, log2g, nlb, G, n, zbytes;
     const __half *scales;
@@ -228,7 +257,7 @@ __device__ __forceinline__ Geom geom_of(const GemvMat &M) {
 }
 
 // Issue the TMA copies of one stage (matrix m, matrix-local row block rb,
-// slice ks) into ring slot `slot` (one thread).
+// slice ks) into the ring slot at `base` with full barrier `bar` (one thread).
 template <int BITS, int KIND>
 __device__ void issue_geom(const GemvMulti &a, const Geom &M, int m, uint32_t bar, uint32_t base, int rb, int ks) {
     const int row0 = rb * kRows;
@@ -259,7 +288,7 @@ __device__ void issue_geom(const GemvMulti &a, const Geom &M, int m, uint32_t ba
     if (KIND == 1) {
         const CUtensorMap *tl = &a.tm_luts[m];
         const int gps = kSliceK >> M.log2g;
-        const uint32_t lbase = base + 3 * kBox;
+        const uint32_t lbase = base + (BITS == 3 ? 3 : 4) * kBox;
         for (int b = 0; b < nlb; ++b) tma_2d(lbase + b * kBox, tl, bar, (ks * gps + 8 * b) * 16, row0);
     } else if (ks == 0) {
         // pull this block's scales and zero-points into L2; the lanes read
@@ -279,193 +308,215 @@ __device__ __forceinline__ void issue_at(const GemvMulti &a, Header &h, uint32_t
                            ring_s + (uint32_t)(slot * a.stage_bytes), rb, ks);
 }
 
-// Issue stage q (set-up path: coordinates from the stage number).
-template <int BITS, int KIND>
-__device__ void issue_stage(const GemvMulti &a, Header &h, uint32_t ring_s, int q) {
-    int m, rb, ks;
-    stage_coords(h, a.count, q, m, rb, ks);
-    issue_at<BITS, KIND>(a, h, ring_s, m, rb, ks, q % a.ring);
-}
-
-// Scales and zero-points of one lane's 256-weight part: up to eight fp16
-// scales and eight 4-bit zero-points (group order, lowest first).
+// Uniform scales and zero-points of a lane's four rows (tile rows g, g + 8 of
+// both 16-row tiles) for its 32-weight unit of a stage: scales as half2
+// pairs (rows g, g + 8) per tile, zero-points in nibbles 0..3.
 struct Meta {
-    uint32_t s0, s1, s2, s3;  // scales 0-1, 2-3, 4-5, 6-7
+    uint32_t s[2];
     uint32_t z;
 };
 
-__device__ __forceinline__ Meta load_meta(const MatS &M, int row, int k0) {
-    Meta t{0u, 0u, 0u, 0u, 0u};
-    if (row >= M.n || k0 >= M.K) return t;
-    const int g0 = k0 >> M.log2g;
-    // groups in the part, within the row (a part may run past k: then only
-    // its first half is valid)
-    const int ng = min(M.log2g >= 8 ? 1 : kPartK >> M.log2g, M.G - g0);
-    const unsigned short *sp = reinterpret_cast<const unsigned short *>(M.scales) + (int64_t)row * M.G + g0;
-    const uint8_t *zp = M.zeros + (int64_t)row * M.zbytes;
-    uint32_t s[4] = {0u, 0u, 0u, 0u};
+__device__ __forceinline__ Meta load_meta(const MatS &M, int row0, int k0) {
+    Meta t{{0u, 0u}, 0u};
+    if (k0 >= M.K) return t;
+    const int grp = k0 >> M.log2g;
+    const unsigned short *sp = reinterpret_cast<const unsigned short *>(M.scales);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
-        if (j < ng) {
-            s[j >> 1] |= (uint32_t)sp[j] << ((j & 1) * 16);
-            t.z |= (((uint32_t)zp[(g0 + j) >> 1] >> (((g0 + j) & 1) * 4)) & 15u) << (4 * j);
+    for (int i = 0; i < 4; ++i) {
+        const int row = row0 + 8 * i;  // g, g + 8, 16 + g, 24 + g
+        if (row < M.n) {
+            t.s[i >> 1] |= (uint32_t)__ldg(sp + (int64_t)row * M.G + grp) << ((i & 1) * 16);
+            const uint32_t zb = __ldg(M.zeros + (int64_t)row * M.zbytes + (grp >> 1));
+            t.z |= ((zb >> ((grp & 1) * 4)) & 15u) << (4 * i);
         }
     }
-    t.s0 = s[0];
-    t.s1 = s[1];
-    t.s2 = s[2];
-    t.s3 = s[3];
     return t;
 }
 
-__device__ __forceinline__ float meta_scale(const Meta &t, int gl) {
-    uint32_t w = t.s0;
-    if (gl >= 2) w = t.s1;
-    if (gl >= 4) w = t.s2;
-    if (gl >= 6) w = t.s3;
-    return __half2float(__ushort_as_half((unsigned short)(w >> ((gl & 1) * 16))));
-}
-
-__device__ __forceinline__ uint32_t meta_zero(const Meta &t, int gl) { return (t.z >> (4 * gl)) & 15u; }
-
-// Row blocks of matrix m in this CTA's range [lo, hi) of the launch's list.
+// Row blocks of matrix m in this CTA's range [lo, hi) of its phase's list.
 __device__ __forceinline__ int cta_nrb(const GemvMulti &a, int m, int lo, int hi) {
     const int f = max(lo, a.mat[m].rb_off), e = min(hi, a.mat[m].rb_off + a.mat[m].nrb);
     return e > f ? e - f : 0;
 }
 
-// Matrix m is the first matrix of this CTA with its activations: it owns
-// their shared-memory copy (matrices of a launch may share one x).
-__device__ __forceinline__ bool x_owner_p(const GemvMulti &a, int m, int lo, int hi) {
-    if (cta_nrb(a, m, lo, hi) == 0) return false;
-    for (int j = 0; j < m; ++j)
-        if (cta_nrb(a, j, lo, hi) > 0 && a.mat[j].x == a.mat[m].x && a.mat[j].k == a.mat[m].k) return false;
-    return true;
+__device__ __forceinline__ int phase_of(const GemvMulti &a, int m) {
+    int p = 0;
+    while (p + 1 < a.nphase && m >= a.phase_first[p + 1]) ++p;
+    return p;
 }
 
-// Offset (halves) of matrix m's activations in the shared-memory copy.
-template <int NB>
-__device__ __forceinline__ int x_offset(const GemvMulti &a, int m, int lo, int hi) {
-    int off = 0;
-    for (int j = 0; j < m; ++j) {
-        if (!x_owner_p(a, j, lo, hi)) continue;
-        if (a.mat[j].x == a.mat[m].x && a.mat[j].k == a.mat[m].k) return off;
-        off += NB * (int)a.mat[j].k;
-    }
-    return off;
+// This CTA's stages of phase p (its row blocks times their slices).
+__device__ __forceinline__ int phase_stages(const GemvMulti &a, int p) {
+    const int lo = a.cta_rb[p][blockIdx.x], hi = a.cta_rb[p][blockIdx.x + 1];
+    int q = 0;
+    for (int m = a.phase_first[p]; m < a.phase_first[p + 1]; ++m) q += cta_nrb(a, m, lo, hi) * a.mat[m].nks;
+    return q;
 }
 
-// Cursor over one warp's stages: matrix, CTA-local row block of that matrix,
-// slice, and the CTA-local stage number.
-struct Cursor {
-    int m, rbl, ks, q;
-};
+__device__ __forceinline__ int round_groups(int q) { return (q + kGroups - 1) / kGroups * kGroups; }
 
-__device__ __forceinline__ void advance_by(const Header &h, int count, Cursor &c, int d) {
-    c.q += d;
-    c.ks += d;
-    while (c.m < count && c.ks >= h.mats[c.m].nks) {
-        c.ks -= h.mats[c.m].nks;
-        if (++c.rbl == h.mats[c.m].nrb) {
-            c.rbl = 0;
-            ++c.m;
-            while (c.m < count && h.mats[c.m].nrb == 0) ++c.m;
+// Grid-scope counter of a fused launch: a release increment (everything the
+// CTA wrote before it, ordered by the consumers' barrier, is visible to whoever
+// acquires the new count) and an acquire read.
+__device__ __forceinline__ uint32_t atom_add_release_gpu(uint32_t *p, uint32_t v) {
+    uint32_t old;
+    asm volatile("atom.add.release.gpu.global.u32 %0, [%1], %2;" : "=r"(old) : "l"(p), "r"(v) : "memory");
+    return old;
+}
+
+__device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
+    uint32_t v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+
+// Named barrier of the consumer warps (the producer warp does not take part).
+__device__ __forceinline__ void consumers_sync() {
+    asm volatile("bar.sync 1, %0;" ::"n"(32 * kWarps * kGroups) : "memory");
+}
+
+// Products of one 16-row tile's decoded weights with x.  NT = 1, 2: the
+// tensor cores (mma.sync m16n8k16, 8 rows of x per n-tile).  NT = -1, -2: CUDA
+// cores for one or two rows of x, where an MMA would waste most of its 8
+// columns: fp16 products summed in fp16 over 8 weight pairs per chain, then in
+// fp32 (the same products the MMA forms; `scaled` false means w holds q - z and
+// the group's scale is applied to the fp32 sum).
+template <int NT>
+struct Dot {
+    static constexpr bool kCores = NT < 0;
+    static constexpr int NX = kCores ? -NT : NT;  // rows of x (CUDA cores) or n-tiles held
+    __half2 h[NX][4];                             // CUDA cores: fp16 chains, rows g and g + 8
+    __device__ __forceinline__ void start() {
+        if (kCores) {
+#pragma unroll
+            for (int b = 0; b < NX; ++b)
+#pragma unroll
+                for (int i = 0; i < 4; ++i) h[b][i] = u2h2(0u);
         }
     }
-}
-
-// Wait for a full-barrier phase: a try in line, the bounded loop out of line.
-__device__ __forceinline__ bool wait_full(uint32_t bar, uint32_t par, uint64_t limit_ns,
-                                          volatile uint32_t *abort_flag) {
-    bool ok = mbar_try_wait(bar, par);
-    if (!__all_sync(0xffffffffu, ok)) ok = __all_sync(0xffffffffu, mbar_wait(bar, par, limit_ns, abort_flag));
-    return ok;
-}
-
-// One 3-bit superblock (128 k = four 32-weight units) of one row: codes words
-// A/B/C, tables built TPS times (once per group), products with NB rows of x.
-template <int KIND, int NB, int TPS>
-__device__ __forceinline__ void superblock3(const uint4 &A, const uint4 &B, const uint4 &C, uint32_t lut_s,
-                                            int lg0, int r, const Meta &meta, int gl0, uint32_t xk, int K,
-                                            bool half_only, float (&acc)[NB]) {
-    const uint32_t Aw[4] = {A.x, A.y, A.z, A.w};
-    const uint32_t Bw[4] = {B.x, B.y, B.z, B.w};
-    const uint32_t Cw[4] = {C.x, C.y, C.z, C.w};
-    (void)half_only;
-    Table8 tab{};
-    float s = 1.0f;
+    // weights (row g: p01 p23, row g + 8: r01 r23) of codes m = 4j .. 4j + 3
+    __device__ __forceinline__ void step(int j, __half2 p01, __half2 p23, __half2 r01, __half2 r23,
+                                         const uint32_t (&xw)[NX][16], int nb, float (&acc)[NX][4]) {
+        if (kCores) {
 #pragma unroll
-    for (int i = 0; i < 4; ++i) {
-        // up to four rows of x are held at once (batch 8 takes them one by one)
-        constexpr int XB = NB <= 4 ? NB : 1;
-        __half2 xv[XB][16];
+            for (int b = 0; b < NX; ++b) {
+                h[b][0] = __hfma2(p01, u2h2(xw[b][2 * j]), h[b][0]);
+                h[b][1] = __hfma2(p23, u2h2(xw[b][2 * j + 1]), h[b][1]);
+                h[b][2] = __hfma2(r01, u2h2(xw[b][2 * j]), h[b][2]);
+                h[b][3] = __hfma2(r23, u2h2(xw[b][2 * j + 1]), h[b][3]);
+            }
+        } else {
 #pragma unroll
-        for (int b = 0; b < XB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
-        if (i % (4 / TPS) == 0) {
-            const int t = i / (4 / TPS);
-            if (KIND == 1) {
-                const int lg = lg0 + t;
-                const uint4 l = lds128(lut_s + (uint32_t)((lg >> 3) * kBox) + swz(r, lg & 7));
-                tab = make_table8(l.x, l.y, l.z, l.w);
-            } else {
-                tab = table8_offsets(meta_zero(meta, gl0 + t));
-                s = meta_scale(meta, gl0 + t);
+            for (int nt = 0; nt < NX; ++nt)
+                mma16816(acc[nt], h22u(p01), h22u(r01), h22u(p23), h22u(r23), xw[nt][2 * j], xw[nt][2 * j + 1]);
+        }
+    }
+    // CUDA cores: the fp16 chains into the fp32 sums (times the scales s0, s1 of
+    // rows g, g + 8 when the weights were q - z)
+    __device__ __forceinline__ void finish(int nb, float s0, float s1, float (&acc)[NX][4]) {
+        if (kCores) {
+#pragma unroll
+            for (int b = 0; b < NX; ++b) {
+                const float2 f0 = __half22float2(h[b][0]), f1 = __half22float2(h[b][1]);
+                const float2 f2 = __half22float2(h[b][2]), f3 = __half22float2(h[b][3]);
+                acc[b][0] += s0 * ((f0.x + f0.y) + (f1.x + f1.y));
+                acc[b][1] += s1 * ((f2.x + f2.y) + (f3.x + f3.y));
             }
         }
-        __half2 w[16];
-        lookup_triple(tab, Aw[i], Bw[i], Cw[i], w);
+    }
+};
+
+// One 16-row tile, 3-bit codes: the lane's code words of rows g (A0 B0 C0) and
+// g + 8 (A1 B1 C1) for its 32-weight unit, their 8-entry tables (a group's LUT,
+// or the uniform offsets j - z with scales s0, s1), products with x.
+template <int KIND, int NT>
+__device__ __forceinline__ void tile3(const Table8 &t0, const Table8 &t1, uint32_t A0, uint32_t B0, uint32_t C0,
+                                      uint32_t A1, uint32_t B1, uint32_t C1, __half2 s0, __half2 s1,
+                                      const uint32_t (&xw)[Dot<NT>::NX][16], int nb,
+                                      float (&acc)[Dot<NT>::NX][4]) {
+    const uint32_t msk = 0x77777777u;
+    uint32_t e0[4], e1[4];  // selectors of codes m = 8q + nibble
+    e0[0] = A0 & msk;
+    e0[1] = B0 & msk;
+    e0[2] = C0 & msk;
+    e0[3] = (shr_fma(A0, 3) & 0x11111111u) | (shr_fma(B0, 2) & 0x22222222u) | (shr_fma(C0, 1) & 0x44444444u);
+    e1[0] = A1 & msk;
+    e1[1] = B1 & msk;
+    e1[2] = C1 & msk;
+    e1[3] = (shr_fma(A1, 3) & 0x11111111u) | (shr_fma(B1, 2) & 0x22222222u) | (shr_fma(C1, 1) & 0x44444444u);
+    Dot<NT> d;
+    d.start();
 #pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            const __half2(&xb)[16] = xv[XB == NB ? b : 0];
-            if (XB != NB && b > 0) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[0]);
-            if (KIND == 1)
-                acc[b] += dot16(w, xb);
-            else
-                acc[b] += s * dot16(w, xb);
+    for (int q = 0; q < 4; ++q) {
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {  // codes m = 8q + 4hh .. +3: step j = 2q + hh
+            const uint32_t s0w = hh ? shr_fma(e0[q], 16) : e0[q];
+            const uint32_t s1w = hh ? shr_fma(e1[q], 16) : e1[q];
+            __half2 p01, p23, r01, r23;
+            lookup4(t0, s0w, p01, p23);
+            lookup4(t1, s1w, r01, r23);
+            if (KIND == 0 && !Dot<NT>::kCores) {  // tensor cores: the dequantized weights themselves
+                p01 = __hmul2(p01, s0);
+                p23 = __hmul2(p23, s0);
+                r01 = __hmul2(r01, s1);
+                r23 = __hmul2(r23, s1);
+            }
+            d.step(2 * q + hh, p01, p23, r01, r23, xw, nb, acc);
         }
     }
+    if (KIND == 0)
+        d.finish(nb, __low2float(s0), __low2float(s1), acc);
+    else
+        d.finish(nb, 1.0f, 1.0f, acc);
 }
 
-// Eight 4-bit units (256 k) of one row, UPG units per group.
-template <int NB, int UPG>
-__device__ __forceinline__ void part4(uint32_t cb, int r, const Meta &meta, uint32_t xk, int K, bool half_only,
-                                      float (&acc)[NB]) {
-    float s = 1.0f;
-    __half2 zl{}, zh{};
+// One 16-row tile, 4-bit uniform codes: the lane's 16 code bytes of rows g
+// (c0) and g + 8 (c1), zero-point constants and scales, products with x.
+template <int NT>
+__device__ __forceinline__ void tile4(const uint4 &c0, const uint4 &c1, uint32_t z0, uint32_t z1, __half2 s0,
+                                      __half2 s1, const uint32_t (&xw)[Dot<NT>::NX][16], int nb,
+                                      float (&acc)[Dot<NT>::NX][4]) {
+    const uint32_t w0[4] = {c0.x, c0.y, c0.z, c0.w};
+    const uint32_t w1[4] = {c1.x, c1.y, c1.z, c1.w};
+    const __half2 zl0 = zlo_of(z0), zh0 = zhi_of(z0), zl1 = zlo_of(z1), zh1 = zhi_of(z1);
+    Dot<NT> d;
+    d.start();
 #pragma unroll
-    for (int i = 0; i < 8; ++i) {
-        if (i == 4 && half_only) break;  // k is a multiple of 128, not of 256
-        constexpr int XB = NB <= 4 ? NB : 1;
-        __half2 xv[XB][16];
+    for (int wd = 0; wd < 4; ++wd) {  // codes m = 8 wd .. 8 wd + 7: steps 2 wd, 2 wd + 1
+        __half2 o0[4], o1[4];
+        unpack4_qz(w0[wd], zl0, zh0, o0);
+        unpack4_qz(w1[wd], zl1, zh1, o1);
+        if (!Dot<NT>::kCores) {
 #pragma unroll
-        for (int b = 0; b < XB; ++b) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[b]);
-        if (i % UPG == 0) {
-            const int gl = i / UPG;
-            const uint32_t z = meta_zero(meta, gl);
-            zl = zlo_of(z);
-            zh = zhi_of(z);
-            s = meta_scale(meta, gl);
-        }
-        const uint4 cw = lds128(cb + swz(r, i));
-        const uint32_t wd[4] = {cw.x, cw.y, cw.z, cw.w};
-        __half2 w[16];
-#pragma unroll
-        for (int t = 0; t < 4; ++t) {
-            __half2 o[4];
-            unpack4_qz(wd[t], zl, zh, o);
-#pragma unroll
-            for (int u = 0; u < 4; ++u) w[4 * t + u] = o[u];
+            for (int i = 0; i < 4; ++i) {
+                o0[i] = __hmul2(o0[i], s0);
+                o1[i] = __hmul2(o1[i], s1);
+            }
         }
 #pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            const __half2(&xb)[16] = xv[XB == NB ? b : 0];
-            if (XB != NB && b > 0) load_x32(xk + 2u * (uint32_t)(b * K + 32 * i), xv[0]);
-            acc[b] += s * dot16(w, xb);
-        }
+        for (int hh = 0; hh < 2; ++hh)
+            d.step(2 * wd + hh, o0[2 * hh], o0[2 * hh + 1], o1[2 * hh], o1[2 * hh + 1], xw, nb, acc);
     }
+    d.finish(nb, __low2float(s0), __low2float(s1), acc);
 }
 
-template <int BITS, int KIND, int NB>
+// Row stride (floats) of a block's partial sums in shared memory.  CUDA-core
+// path (one or two rows of x, scalar reads): odd, so that the finisher's
+// lane-strided reads hit 32 different banks.  Tensor-core path (16-byte
+// reads): 4 times an odd number, so that 8 lanes' 16-byte reads cover all 32
+// banks.
+__host__ __device__ __forceinline__ int partial_stride(int nb, bool cores) {
+    if (cores) return nb | 1;
+    const int r = (nb + 3) & ~3;
+    return (r / 4) % 2 ? r : r + 4;
+}
+
+__device__ __forceinline__ __half2 half2_of(uint32_t pair, int hi) {
+    const unsigned short v = (unsigned short)(hi ? pair >> 16 : pair);
+    return __halves2half2(__ushort_as_half(v), __ushort_as_half(v));
+}
+
+template <int BITS, int KIND, int NT>
 __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant__ GemvMulti a) {
     extern __shared__ uint8_t smem_raw[];
     // 1024-byte alignment for the swizzled TMA boxes
@@ -474,25 +525,38 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     uint8_t *base = smem_raw + (base_s - raw_s);
     Header &h = *reinterpret_cast<Header *>(base);
     float *red = reinterpret_cast<float *>(base + kHeader);
-    __half *xs = reinterpret_cast<__half *>(base + kHeader + a.red_bytes);
-    const uint32_t xs_s = base_s + (uint32_t)(kHeader + a.red_bytes);
-    const uint32_t ring_s = base_s + (uint32_t)(kHeader + a.red_bytes + a.x_smem_bytes);
+    const uint32_t ring_s = base_s + (uint32_t)(kHeader + a.red_bytes);
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
-    const int count = a.count, ring = a.ring;
+    const int count = a.count, ring = a.ring, nb = a.batch;
+    constexpr int NX = Dot<NT>::NX;
 
     // let the next kernel in the stream start streaming its own weights; it
     // still waits for this grid's completion before it reads activations
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 
-    // ---- set-up from the kernel parameters, spread over threads, with a
-    // single barrier before the main loop: the first copies start at once and
-    // the activations are staged while the tables are built
-    const int lo = a.cta_rb[blockIdx.x], hi = a.cta_rb[blockIdx.x + 1];
-    if (warp == 0) {
-        if (lane < count) {  // matrix `lane`: this CTA's row blocks, stage numbering, x offset
+    // ---- set-up from the kernel parameters, with a single barrier before
+    // the main loops
+    const bool fused = a.nphase > 1;
+    if (warp == kProducer) {
+        if (lane == 0) {
+            for (int i = 0; i < ring; ++i) {
+                mbar_init(smem_u32(&h.full[i]), 1);
+                mbar_init(smem_u32(&h.empty[i]), 32 * kWarps);
+            }
+            h.abort_flag = 0;
+            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        }
+        if (lane < count) {
+            asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_codes[lane]) : "memory");
+            if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_luts[lane]) : "memory");
+        }
+    } else if (warp == 0) {
+        if (lane < count) {  // matrix `lane`: this CTA's row blocks and stage numbering
             const int t = lane;
+            const int p = phase_of(a, t);
+            const int lo = a.cta_rb[p][blockIdx.x], hi = a.cta_rb[p][blockIdx.x + 1];
             const GemvMat &G = a.mat[t];
             MatS &S = h.mats[t];
             const int f = max(lo, G.rb_off);
@@ -509,262 +573,382 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             S.nlb = G.nlb;
             S.rb0 = f - G.rb_off;
             S.nrb = cta_nrb(a, t, lo, hi);
+            // stages and blocks before this matrix: earlier phases (their stage
+            // counts padded to a multiple of kGroups), then this phase's earlier matrices
             int q = 0, rbq = 0;
-            for (int m = 0; m < t; ++m) {
+            for (int pp = 0; pp < p; ++pp) {
+                q += round_groups(phase_stages(a, pp));
+                const int l2 = a.cta_rb[pp][blockIdx.x], h2 = a.cta_rb[pp][blockIdx.x + 1];
+                for (int m = a.phase_first[pp]; m < a.phase_first[pp + 1]; ++m) rbq += cta_nrb(a, m, l2, h2);
+            }
+            for (int m = a.phase_first[p]; m < t; ++m) {
                 const int nr = cta_nrb(a, m, lo, hi);
                 q += nr * a.mat[m].nks;
                 rbq += nr;
             }
             S.q0 = q;
             S.rbq0 = rbq;
-            h.q_end[t] = q + S.nrb * G.nks;
-            S.xoff = x_offset<NB>(a, t, lo, hi);
+        }
+    } else if (warp == 1) {
+        if (lane < kMaxRbSlots) {
+            h.cnt[lane] = 0;
+            h.gen[lane] = 0;
         }
         if (lane == 0) {
             int q = 0;
-            for (int m = 0; m < count; ++m) q += cta_nrb(a, m, lo, hi) * a.mat[m].nks;
-            h.nstages = q;
-        }
-    } else if (warp == 1) {
-        if (lane < count) {
-            asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_codes[lane]) : "memory");
-            if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_luts[lane]) : "memory");
-        }
-    } else if (warp == 2) {
-        if (lane == 0) {
-            for (int i = 0; i < ring; ++i) mbar_init(smem_u32(&h.full[i]), 1);
-            h.abort_flag = 0;
-            asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-        }
-        __syncwarp();
-        // the CTA's first stages straight from the parameters, one per lane, so
-        // that their data is on the way while the rest of the set-up runs
-        int q = 0;
-        for (int m = 0; m < count; ++m) {
-            const GemvMat &G = a.mat[m];
-            const int nq = cta_nrb(a, m, lo, hi) * G.nks;
-            if (lane < a.initial && lane >= q && lane < q + nq) {
-                const int j = lane - q, rbl = j / G.nks, ks = j - rbl * G.nks;
-                const int rb0 = max(lo, G.rb_off) - G.rb_off;
-                issue_geom<BITS, KIND>(a, geom_of(G), m, smem_u32(&h.full[lane]),
-                                       ring_s + (uint32_t)(lane * a.stage_bytes), rb0 + rbl, ks);
+            for (int p = 0; p < a.nphase; ++p) {
+                h.ph_q0[p] = q;
+                h.ph_nst[p] = phase_stages(a, p);
+                q += round_groups(h.ph_nst[p]);
             }
-            q += nq;
+            h.ph_q0[a.nphase] = q;
         }
-        if (lane == 0) h.issued = (uint32_t)min(a.initial, q);
-    } else if (threadIdx.x >= 96 && threadIdx.x < 96 + kMaxRing) {
-        h.rel[threadIdx.x - 96] = 0;
-    } else if (threadIdx.x >= 128 && threadIdx.x < 128 + kMaxRbSlots) {
-        h.cnt[threadIdx.x - 128] = 0;
-        h.gen[threadIdx.x - 128] = 0;
-    }
-    // activations -> shared memory (every lane of a warp then reads the same
-    // address: a broadcast), after the previous kernel in the stream is done
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    for (int m = 0; m < count; ++m) {
-        if (!x_owner_p(a, m, lo, hi)) continue;
-        const int vecs = NB * (int)a.mat[m].k / 8;
-        const uint4 *src = reinterpret_cast<const uint4 *>(a.mat[m].x);
-        uint4 *dst = reinterpret_cast<uint4 *>(xs + x_offset<NB>(a, m, lo, hi));
-        for (int i = threadIdx.x; i < vecs; i += kThreads) dst[i] = src[i];
     }
     __syncthreads();
 
-    const int nst = h.nstages;
-    const int r = lane;
-    const int grp = warp / kGroupWarps;   // stages q with q % kGroups == grp
-    const int part = warp % kGroupWarps;  // 256-weight part of each of those stages
+    if (warp == kProducer) {
+        // ---- producer: every stage in order, each once its slot's previous
+        // fill has been released by the eight warps of its group; a phase's
+        // stages are padded to a multiple of kGroups with empty stages (a full
+        // barrier phase with no bytes), so that every phase starts on group 0
+        // as a launch of its own does
+        if (lane == 0) {
+            bool okp = true;
+            int q = 0;
+            for (int p = 0; p < a.nphase && okp; ++p) {
+                const int qend = h.ph_q0[p + 1];
+                int m = a.phase_first[p], rbl = 0, ks = 0;
+                while (m < a.phase_first[p + 1] && h.mats[m].nrb == 0) ++m;
+                for (; q < qend; ++q) {
+                    const int slot = q % ring;
+                    if (q >= ring) {
+                        okp = mbar_wait(smem_u32(&h.empty[slot]), (uint32_t)((q / ring) - 1) & 1u, a.wait_limit_ns,
+                                        &h.abort_flag);
+                        if (!okp) break;
+                    }
+                    if (m >= a.phase_first[p + 1]) {  // padding
+                        mbar_arrive_expect_tx(smem_u32(&h.full[slot]), 0);
+                        continue;
+                    }
+                    issue_at<BITS, KIND>(a, h, ring_s, m, h.mats[m].rb0 + rbl, ks, slot);
+                    if (++ks == h.mats[m].nks) {
+                        ks = 0;
+                        if (++rbl == h.mats[m].nrb) {
+                            rbl = 0;
+                            ++m;
+                            while (m < a.phase_first[p + 1] && h.mats[m].nrb == 0) ++m;
+                        }
+                    }
+                }
+            }
+            if (!okp) {
+                h.abort_flag = 1u;
+                atomicOr(a.status, kStatusTimeout);
+            }
+            // every issued copy lands before the CTA's shared memory is released
+            for (int qq = max(0, q - ring); qq < q; ++qq)
+                mbar_wait(smem_u32(&h.full[qq % ring]), (uint32_t)(qq / ring) & 1u, a.wait_limit_ns, nullptr);
+        }
+        return;
+    }
+
+    // ---- consumers: x is read, and y written, only after the previous kernel
+    // in the stream has finished
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int grp = warp / kWarps;   // stages q with q % kGroups == grp
+    const int sb = warp % kWarps;    // superblock of each of those stages
+    const int g = lane >> 2, t = lane & 3;
+    const int nbs = partial_stride(nb, Dot<NT>::kCores);  // row stride (floats) of the partial sums
+    const int kunit = 128 * sb + 32 * t;  // the lane's 32-weight unit within a slice
     bool ok = true;
 
-    // this warp's first stage, and the one after it
-    Cursor c{0, 0, 0, 0};
-    while (c.m < count && h.mats[c.m].nrb == 0) ++c.m;
-    advance_by(h, count, c, grp);
-    Cursor cn = c;
-    advance_by(h, count, cn, kGroups);
-    // the stage that refills this warp's current slot, q + ring: ring is a
-    // multiple of kGroups, so it is one of this warp's own later stages
-    Cursor cr = c;
-    advance_by(h, count, cr, ring);
-    // uniform metadata of this warp's stages, loaded one stage ahead
-    Meta cur{}, nxt{};
-    if (KIND == 0 && c.m < count)
-        cur = load_meta(h.mats[c.m], (h.mats[c.m].rb0 + c.rbl) * kRows + r, c.ks * kSliceK + part * kPartK);
-
-    // per-lane offsets of this warp's 3-bit code chunks in a stage (planes 0-2
-    // of row r are box rows 3r..3r+2; superblocks 2 part and 2 part + 1)
-    uint32_t co[2][3];
+    // per-lane shared-memory offsets of the code words of both tiles
+    uint32_t co[2][2];
 #pragma unroll
-    for (int hb = 0; hb < 2; ++hb)
-#pragma unroll
-        for (int p = 0; p < 3; ++p) co[hb][p] = swz(3 * r + p, part * 2 + hb);
-
-    float acc[NB];
-#pragma unroll
-    for (int b = 0; b < NB; ++b) acc[b] = 0.0f;
-    int slot = grp, fm = -1, frbl = 0;
-    uint32_t par = 0;
-
-    // partials of row block (m, rbl) -> shared memory; the last contributor
-    // sums them in a fixed order and writes y
-    auto flush = [&](int m, int rbl) -> bool {
-        const MatS &M = h.mats[m];
-        const int rbi = M.rbq0 + rbl;
-        const int rs = rbi % a.rb_slots;
-        const uint32_t use = (uint32_t)(rbi / a.rb_slots);
-        // the warp groups run independently: the slot's previous block must
-        // have been summed before this warp overwrites its partials
-        bool okf = true;
-        if (lane == 0 && *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) != use)
-            okf = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
-        if (!__shfl_sync(0xffffffffu, okf, 0)) return false;
-        float *rp = red + (size_t)rs * (kWarps * NB * 32);
-#pragma unroll
-        for (int b = 0; b < NB; ++b) rp[(warp * NB + b) * 32 + r] = acc[b];
-        __syncwarp();
-        const int ng = min(M.nks, kGroups);  // groups that worked on this block
-        uint32_t fin = 0;
-        if (lane == 0) {
-            __threadfence_block();
-            fin = atomicAdd(&h.cnt[rs], 1u) + 1u == (uint32_t)(ng * kGroupWarps);
-            __threadfence_block();
-        }
-        fin = __shfl_sync(0xffffffffu, fin, 0);
-        if (fin) {
-            const int q0 = M.q0 + rbl * M.nks;  // the block's first stage
-            const int row = (M.rb0 + rbl) * kRows + r;
-            float v[NB];
-#pragma unroll
-            for (int b = 0; b < NB; ++b) {
-                v[b] = 0.0f;
-                for (int j = 0; j < ng; ++j) {
-                    const int g = (q0 + j) % kGroups;
-#pragma unroll
-                    for (int p = 0; p < kGroupWarps; ++p) v[b] += rp[((g * kGroupWarps + p) * NB + b) * 32 + r];
-                }
-            }
-            // free the slot first: the fence must not wait for the y stores
-            __syncwarp();
-            if (lane == 0) {
-                h.cnt[rs] = 0;
-                __threadfence_block();
-                *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
-            }
-            if (row < M.n) {
-#pragma unroll
-                for (int b = 0; b < NB; ++b) {
-                    if (a.y_f32)
-                        reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v[b];
-                    else
-                        reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v[b]);
-                }
-            }
-        }
-        return true;
-    };
-
-    while (c.m < count) {
-        const MatS &M = h.mats[c.m];
-        if (fm >= 0 && (fm != c.m || frbl != c.rbl)) {  // left the previous row block
-            ok = flush(fm, frbl);
-            if (!ok) break;
-#pragma unroll
-            for (int b = 0; b < NB; ++b) acc[b] = 0.0f;
-        }
-        fm = c.m;
-        frbl = c.rbl;
-        if (KIND == 0 && cn.m < count) {
-            const MatS &N = h.mats[cn.m];
-            nxt = load_meta(N, (N.rb0 + cn.rbl) * kRows + r, cn.ks * kSliceK + part * kPartK);
-        }
-        ok = wait_full(smem_u32(&h.full[slot]), par, a.wait_limit_ns, &h.abort_flag);
-        if (!ok) break;
-        const int q = c.q;
-        if (part == 0 && lane == 0 && q + a.initial < min(ring, nst)) {
-            // ramp-up: a stage has landed, request one more of the ring
-            issue_stage<BITS, KIND>(a, h, ring_s, q + a.initial);
-            atomicMax(&h.issued, (uint32_t)(q + a.initial + 1));
-        }
-        const int K = M.K;
-        const int k0 = c.ks * kSliceK + part * kPartK;
-        if (k0 < K) {
-            const uint32_t sb = ring_s + (uint32_t)(slot * a.stage_bytes);
-            const uint32_t xk = xs_s + 2u * (uint32_t)(M.xoff + k0);
-            const bool half_only = k0 + 128 >= K;  // k is a multiple of 128, not of 256
-            const int log2g = M.log2g;
-            if (BITS == 3) {
-                const uint32_t lut_s = sb + 3 * kBox;
-#pragma unroll
-                for (int hb = 0; hb < 2; ++hb) {
-                    if (hb == 1 && half_only) break;
-                    const uint4 A = lds128(sb + co[hb][0]);
-                    const uint4 B = lds128(sb + co[hb][1]);
-                    const uint4 C = lds128(sb + co[hb][2]);
-                    const int kk = part * kPartK + 128 * hb;  // within the slice
-                    const int gl0 = (128 * hb) >> log2g;       // first group of the superblock in the part
-                    const int lg0 = kk >> log2g;               // ... in the slice (LUT boxes)
-                    if (log2g >= 7)
-                        superblock3<KIND, NB, 1>(A, B, C, lut_s, lg0, r, cur, gl0, xk + 256u * hb, K, half_only, acc);
-                    else if (log2g == 6)
-                        superblock3<KIND, NB, 2>(A, B, C, lut_s, lg0, r, cur, gl0, xk + 256u * hb, K, half_only, acc);
-                    else
-                        superblock3<KIND, NB, 4>(A, B, C, lut_s, lg0, r, cur, gl0, xk + 256u * hb, K, half_only, acc);
-                }
-            } else {
-                // 4-bit: box `part` holds this part's 256 k, 16 bytes per 32 k
-                const uint32_t cb = sb + (uint32_t)(part * kBox);
-                if (log2g >= 8)
-                    part4<NB, 8>(cb, r, cur, xk, K, half_only, acc);
-                else if (log2g == 7)
-                    part4<NB, 4>(cb, r, cur, xk, K, half_only, acc);
-                else if (log2g == 6)
-                    part4<NB, 2>(cb, r, cur, xk, K, half_only, acc);
-                else
-                    part4<NB, 1>(cb, r, cur, xk, K, half_only, acc);
-            }
-        }
-        // release the stage; the last warp of the group refills it
-        __syncwarp();
-        if (lane == 0) {
-            __threadfence_block();
-            const uint32_t old = atomicAdd(&h.rel[slot], 1u);
-            if (old == kGroupWarps - 1) {
-                h.rel[slot] = 0;
-                __threadfence_block();
-                asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
-                if (cr.m < count && !*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) {
-                    issue_at<BITS, KIND>(a, h, ring_s, cr.m, h.mats[cr.m].rb0 + cr.rbl, cr.ks, slot);
-                    atomicMax(&h.issued, (uint32_t)(q + ring + 1));
-                }
-            }
-        }
-        if (KIND == 0) cur = nxt;
-        c = cn;
-        advance_by(h, count, cn, kGroups);
-        advance_by(h, count, cr, kGroups);
-        slot += kGroups;
-        if (slot >= ring) {
-            slot -= ring;
-            par ^= 1u;
+    for (int rt = 0; rt < 2; ++rt) {
+        if (BITS == 3) {
+            // ldmatrix.x4: planes 0, 1 of rows g and g + 8; ldmatrix.x2: plane 2
+            const int mat = lane >> 3, rr = lane & 7;
+            const int row4 = 16 * rt + 8 * (mat & 1) + rr, rho4 = 3 * row4 + (mat >> 1);
+            const int row2 = 16 * rt + 8 * ((lane >> 3) & 1) + rr, rho2 = 3 * row2 + 2;
+            co[rt][0] = swz(rho4, sb);
+            co[rt][1] = swz(rho2, sb);
+        } else {
+            const int r0 = 16 * rt + g;
+            const int chunk = 4 * (sb & 1) + t;
+            co[rt][0] = (uint32_t)((sb >> 1) * kBox) + swz(r0, chunk);
+            co[rt][1] = (uint32_t)((sb >> 1) * kBox) + swz(r0 + 8, chunk);
         }
     }
-    if (ok && fm >= 0) ok = flush(fm, frbl);
+
+    int slot = grp;
+    uint32_t par = 0;
+    float *rp_base = red;
+    for (int p = 0; p < a.nphase; ++p) {
+        if (fused && p > 0) {
+            // phase p reads its x only once every CTA has finished phase p - 1
+            if (threadIdx.x == 0 && ok && ld_acquire_gpu(a.phase_ctr + (p - 1)) < gridDim.x) {
+                const uint64_t t0 = globaltimer_ns();
+                while (ld_acquire_gpu(a.phase_ctr + (p - 1)) < gridDim.x) {
+                    if (*reinterpret_cast<volatile uint32_t *>(&h.abort_flag) ||
+                        globaltimer_ns() - t0 > a.wait_limit_ns) {
+                        h.abort_flag = 1u;
+                        atomicOr(a.status, kStatusTimeout);
+                        break;
+                    }
+                }
+            }
+            consumers_sync();
+            if (*reinterpret_cast<volatile uint32_t *>(&h.abort_flag)) ok = false;
+        }
+        for (int m = a.phase_first[p]; m < a.phase_first[p + 1] && ok; ++m) {
+            const MatS &M = h.mats[m];
+            const int nrb = M.nrb;
+            if (nrb == 0) continue;
+            const int K = M.K, nks = M.nks, n = M.n, log2g = M.log2g;
+            const int q0 = M.q0, rb0 = M.rb0, rbq0 = M.rbq0;
+            const __half *xm = M.x;
+            // the lane's LUT chunk in a stage (LUT kind): its group within the slice
+            uint32_t lo_off[2][2] = {{0u, 0u}, {0u, 0u}};
+            if (KIND == 1) {
+                const int lg = kunit >> log2g;
+    #pragma unroll
+                for (int rt = 0; rt < 2; ++rt) {
+                    lo_off[rt][0] = (uint32_t)(3 * kBox + (lg >> 3) * kBox) + swz(16 * rt + g, lg & 7);
+                    lo_off[rt][1] = (uint32_t)(3 * kBox + (lg >> 3) * kBox) + swz(16 * rt + g + 8, lg & 7);
+                }
+            }
+            // x fragments of the lane's 32 k of slice ks: rows g (and g + 8) of x
+            auto load_x = [&](int ks, uint32_t (&xv)[NX][16]) {
+                const int k0 = ks * kSliceK + kunit;
+                const bool in = ks * kSliceK + 128 * sb < K;
+    #pragma unroll
+                for (int nt = 0; nt < NX; ++nt) {
+                    const int b = Dot<NT>::kCores ? nt : g + 8 * nt;  // CUDA cores: every lane takes every row of x
+                    if (in && b < nb) {
+                        const __half *xp = xm + (int64_t)b * K + k0;
+    #pragma unroll
+                        for (int i = 0; i < 4; ++i) {
+                            const uint4 v = ldg_x(xp + 8 * i, fused);
+                            xv[nt][4 * i + 0] = v.x;
+                            xv[nt][4 * i + 1] = v.y;
+                            xv[nt][4 * i + 2] = v.z;
+                            xv[nt][4 * i + 3] = v.w;
+                        }
+                    } else {
+    #pragma unroll
+                        for (int i = 0; i < 16; ++i) xv[nt][i] = 0u;
+                    }
+                }
+            };
+            for (int rbl = 0; rbl < nrb && ok; ++rbl) {
+                const int qb = q0 + rbl * nks;  // the block's first stage
+                const int ks0 = (grp - qb % kGroups + kGroups) % kGroups;
+                if (ks0 >= nks) continue;  // this group has no stage of the block
+                const int row0 = (rb0 + rbl) * kRows + g;  // the lane's first row (of g, g + 8, g + 16, g + 24)
+                float acc[2][NX][4];
+    #pragma unroll
+                for (int rt = 0; rt < 2; ++rt)
+    #pragma unroll
+                    for (int nt = 0; nt < NX; ++nt)
+    #pragma unroll
+                        for (int i = 0; i < 4; ++i) acc[rt][nt][i] = 0.0f;
+                Meta cur{};
+                if (KIND == 0) cur = load_meta(M, row0, ks0 * kSliceK + kunit);
+                for (int ks = ks0; ks < nks; ks += kGroups) {
+                    Meta nxt{};
+                    if (KIND == 0 && ks + kGroups < nks) nxt = load_meta(M, row0, (ks + kGroups) * kSliceK + kunit);
+                    const bool live = ks * kSliceK + 128 * sb < K;  // K is a multiple of 128
+                    uint32_t xw[NX][16];
+                    load_x(ks, xw);
+                    const uint32_t fb = smem_u32(&h.full[slot]);
+                    if (!mbar_try_wait(fb, par) && !mbar_wait(fb, par, a.wait_limit_ns, &h.abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    if (live) {
+                        const uint32_t sbase = ring_s + (uint32_t)(slot * a.stage_bytes);
+    #pragma unroll
+                        for (int rt = 0; rt < 2; ++rt) {
+                            if (BITS == 3) {
+                                uint32_t A0, A1, B0, B1, C0, C1;
+                                ldsm_x4(sbase + co[rt][0], A0, A1, B0, B1);
+                                ldsm_x2(sbase + co[rt][1], C0, C1);
+                                Table8 t0, t1;
+                                __half2 s0 = u2h2(0u), s1 = s0;
+                                if (KIND == 1) {
+                                    const uint4 l0 = lds128(sbase + lo_off[rt][0]);
+                                    const uint4 l1 = lds128(sbase + lo_off[rt][1]);
+                                    t0 = make_table8(l0.x, l0.y, l0.z, l0.w);
+                                    t1 = make_table8(l1.x, l1.y, l1.z, l1.w);
+                                } else {
+                                    t0 = table8_offsets((cur.z >> (8 * rt)) & 15u);
+                                    t1 = table8_offsets((cur.z >> (8 * rt + 4)) & 15u);
+                                    s0 = half2_of(cur.s[rt], 0);
+                                    s1 = half2_of(cur.s[rt], 1);
+                                }
+                                tile3<KIND, NT>(t0, t1, A0, B0, C0, A1, B1, C1, s0, s1, xw, nb, acc[rt]);
+                            } else {
+                                const uint4 c0 = lds128(sbase + co[rt][0]);
+                                const uint4 c1 = lds128(sbase + co[rt][1]);
+                                tile4<NT>(c0, c1, (cur.z >> (8 * rt)) & 15u, (cur.z >> (8 * rt + 4)) & 15u,
+                                          half2_of(cur.s[rt], 0), half2_of(cur.s[rt], 1), xw, nb, acc[rt]);
+                            }
+                        }
+                    }
+                    // release the slot (every lane arrives: no warp-level sync needed)
+                    mbar_arrive(smem_u32(&h.empty[slot]));
+                    if (KIND == 0) cur = nxt;
+                    slot += kGroups;
+                    if (slot >= ring) {
+                        slot -= ring;
+                        par ^= 1u;
+                    }
+                }
+                if (!ok) break;
+                // ---- partials of this block -> shared memory; the last contributor
+                // sums them in a fixed order and writes y
+                const int rbi = rbq0 + rbl;
+                const int rs = rbi % a.rb_slots;
+                const uint32_t use = (uint32_t)(rbi / a.rb_slots);
+                // the warp groups run independently: the slot's previous block must
+                // have been summed before this warp overwrites its partials
+                bool okf = true;
+                if (lane == 0 && *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) != use)
+                    okf = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
+                if (!__shfl_sync(0xffffffffu, okf, 0)) {
+                    ok = false;
+                    break;
+                }
+                // slot layout: [group][superblock warp][32 rows][nbs]
+                float *rp = rp_base + (size_t)rs * (kGroups * kWarps * kRows * nbs);
+                float *mine = rp + (size_t)(grp * kWarps + sb) * (kRows * nbs);
+                if (Dot<NT>::kCores) {
+                    // CUDA cores: sum the four lanes of a row (units t = 0..3), then lane t
+                    // stores row of x t
+    #pragma unroll
+                    for (int rt = 0; rt < 2; ++rt)
+    #pragma unroll
+                        for (int b = 0; b < NX; ++b)
+    #pragma unroll
+                            for (int r = 0; r < 2; ++r) {
+                                float v = acc[rt][b][r];
+                                v += __shfl_xor_sync(0xffffffffu, v, 1);
+                                v += __shfl_xor_sync(0xffffffffu, v, 2);
+                                if (t == b && b < nb) mine[(16 * rt + g + 8 * r) * nbs + b] = v;
+                            }
+                } else {
+    #pragma unroll
+                    for (int rt = 0; rt < 2; ++rt)
+    #pragma unroll
+                        for (int nt = 0; nt < NX; ++nt) {
+                            const int col = 8 * nt + 2 * t;
+                            const int r0 = 16 * rt + g;
+                            if (col < nb) {
+                                mine[r0 * nbs + col] = acc[rt][nt][0];
+                                mine[(r0 + 8) * nbs + col] = acc[rt][nt][2];
+                            }
+                            if (col + 1 < nb) {
+                                mine[r0 * nbs + col + 1] = acc[rt][nt][1];
+                                mine[(r0 + 8) * nbs + col + 1] = acc[rt][nt][3];
+                            }
+                        }
+                }
+                __syncwarp();
+                const int ng = min(nks, kGroups);  // groups that worked on this block
+                uint32_t fin = 0;
+                if (lane == 0) fin = atom_add_acq_rel(&h.cnt[rs], 1u) + 1u == (uint32_t)(ng * kWarps);
+                fin = __shfl_sync(0xffffffffu, fin, 0);
+                if (fin) {
+                    __syncwarp();  // lane 0's acquire orders the whole warp's reads below
+                    const int row = (rb0 + rbl) * kRows + lane;
+                    // the block's partials in a fixed order: group by the block's
+                    // stage order, then superblock warp
+                    constexpr int VMAX = Dot<NT>::kCores ? 2 : 8 * NX;
+                    float v[VMAX];
+    #pragma unroll
+                    for (int b = 0; b < VMAX; ++b) v[b] = 0.0f;
+                    for (int j = 0; j < ng; ++j) {
+                        const float *src = rp + (size_t)((qb + j) % kGroups * kWarps) * (kRows * nbs) + lane * nbs;
+    #pragma unroll
+                        for (int w = 0; w < kWarps; ++w) {
+                            const float *sw = src + (size_t)w * (kRows * nbs);
+                            if (Dot<NT>::kCores) {
+    #pragma unroll
+                                for (int b = 0; b < VMAX; ++b)
+                                    if (b < nb) v[b] += sw[b];
+                            } else {
+    #pragma unroll
+                                for (int c4 = 0; c4 < VMAX / 4; ++c4) {
+                                    if (4 * c4 < nb) {
+                                        const float4 f = *reinterpret_cast<const float4 *>(sw + 4 * c4);
+                                        v[4 * c4] += f.x;
+                                        v[4 * c4 + 1] += f.y;
+                                        v[4 * c4 + 2] += f.z;
+                                        v[4 * c4 + 3] += f.w;
+                                    }
+                                }
+                            }
+                        }
+                    }
+                    // free the slot first: the fence must not wait for the y stores
+                    __syncwarp();
+                    if (lane == 0) {
+                        h.cnt[rs] = 0;
+                        __threadfence_block();
+                        *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
+                    }
+                    if (row < n) {
+    #pragma unroll
+                        for (int b = 0; b < VMAX; ++b) {
+                            if (b >= nb) break;
+                            if (a.y_f32)
+                                reinterpret_cast<float *>(M.y)[(int64_t)b * n + row] = v[b];
+                            else
+                                reinterpret_cast<__half *>(M.y)[(int64_t)b * n + row] = __float2half_rn(v[b]);
+                        }
+                    }
+                }
+            }
+        }
+        // the padding stages of this phase that belong to this group
+        for (int q = h.ph_q0[p] + h.ph_nst[p]; q < h.ph_q0[p + 1] && ok; ++q) {
+            if (q % kGroups != grp) continue;
+            const uint32_t fb = smem_u32(&h.full[slot]);
+            if (!mbar_try_wait(fb, par) && !mbar_wait(fb, par, a.wait_limit_ns, &h.abort_flag)) {
+                ok = false;
+                break;
+            }
+            mbar_arrive(smem_u32(&h.empty[slot]));
+            slot += kGroups;
+            if (slot >= ring) {
+                slot -= ring;
+                par ^= 1u;
+            }
+        }
+        if (fused) {
+            // every consumer warp of this CTA is done with phase p (partials
+            // summed, y written): count the CTA in
+            consumers_sync();
+            if (threadIdx.x == 0) {
+                const uint32_t old = atom_add_release_gpu(a.phase_ctr + p, 1u);
+                if (p == a.nphase - 1 && old == gridDim.x - 1) {
+                    // the last CTA of the launch: every other CTA has passed
+                    // every wait, so the counters go back to zero for the next launch
+                    for (int i = 0; i < a.nphase; ++i) a.phase_ctr[i] = 0u;
+                }
+            }
+        }
+    }
     if (!ok && lane == 0) {
         h.abort_flag = 1u;
         atomicOr(a.status, kStatusTimeout);
     }
-    if (lane == 0 && (!ok || *reinterpret_cast<volatile uint32_t *>(&h.abort_flag))) {
-        // a warp that gives up lets the copies still in flight land before
-        // it exits, so the CTA's shared memory outlives them
-        const int iss = (int)*reinterpret_cast<volatile uint32_t *>(&h.issued);
-        for (int qq = max(0, iss - ring); qq < iss; ++qq)
-            mbar_wait(smem_u32(&h.full[qq % ring]), (uint32_t)(qq / ring) & 1u, a.wait_limit_ns, nullptr);
-    }
 }
 
-template <int BITS, int KIND, int NB>
+template <int BITS, int KIND, int NT>
 cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
-    auto kern = gemv_kernel<BITS, KIND, NB>;
+    auto kern = gemv_kernel<BITS, KIND, NT>;
     static std::atomic<uint64_t> attrs_ready{0};
     cudaError_t e = ensure_kernel_attrs(reinterpret_cast<const void *>(kern), attrs_ready, true);
     if (e != cudaSuccess) return e;
@@ -773,11 +957,21 @@ cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
     cfg.blockDim = dim3(kThreads);
     cfg.dynamicSmemBytes = (size_t)a.smem_bytes;
     cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchAttribute attr[2];
+    int na = 0;
+    if (pdl) {
+        attr[na].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[na].val.programmaticStreamSerializationAllowed = 1;
+        ++na;
+    }
+    if (a.nphase > 1) {
+        // the phases wait on one another across CTAs: every CTA must be resident
+        attr[na].id = cudaLaunchAttributeCooperative;
+        attr[na].val.cooperative = 1;
+        ++na;
+    }
     cfg.attrs = attr;
-    cfg.numAttrs = pdl ? 1 : 0;
+    cfg.numAttrs = (unsigned)na;
     return cudaLaunchKernelEx(&cfg, kern, a);
 }
 
@@ -793,22 +987,21 @@ bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims
 
 }  // namespace
 
-// Host-side plan: tensor maps, byte-balanced CTA row-block ranges and the
+// Host-side plan: tensor maps, byte-balanced CTA row-block ranges (per phase,
+// exactly as a launch of that phase alone would have them) and the
 // shared-memory budget.  Returns false if the matrices cannot share one launch.
 bool plan_gemv(GemvMulti &a, int num_sms) {
-    const int bmax = a.batch;  // kernels are built for batch 1..4 exactly
+    if (a.nphase < 1 || a.nphase > kMaxGemvPhases || a.count < 1 || a.count > kMaxGemvTotal) return false;
+    if (a.phase_first[0] != 0 || a.phase_first[a.nphase] != a.count) return false;
     int nks_min = 1 << 30, nlb_max = 1;
-    int64_t total = 0, rbs = 0;
     for (int m = 0; m < a.count; ++m) {
         GemvMat &M = a.mat[m];
         M.nks = (int)((M.k + kSliceK - 1) / kSliceK);
         M.nlb = a.kind == 1 ? std::max(1, 128 >> M.log2g) : 0;
         M.nrb = (int)((M.n + kRows - 1) / kRows);
-        M.rb_off = (int)rbs;
-        rbs += M.nrb;
         nks_min = std::min(nks_min, M.nks);
         nlb_max = std::max(nlb_max, M.nlb);
-        if (M.n > (int64_t)1 << 30 || rbs > (int64_t)1 << 30) return false;
+        if (M.n > (int64_t)1 << 30) return false;
         const uint8_t *codes = M.codes;
         if (a.bits == 3) {
             // bytes within a plane, plane, row: box = [32 rows][3 planes][128 bytes]
@@ -829,61 +1022,59 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
             if (!encode(&a.tm_luts[m], M.luts, 2, dims, strides, box)) return false;
         }
     }
-    // bytes per row block (balancing only)
-    int64_t rb_bytes[kMaxGemvMats];
-    for (int m = 0; m < a.count; ++m) {
-        const GemvMat &M = a.mat[m];
-        const int64_t row = M.k * a.bits / 8 + (a.kind == 1 ? (int64_t)M.G * 16 : (int64_t)M.G * 2 + M.zbytes);
-        rb_bytes[m] = row * kRows;
-        total += rb_bytes[m] * M.nrb;
-    }
-    a.total_bytes = total;
-    a.grid = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), rbs);
-    // CTA c owns the row blocks whose first byte lies in [c T / grid, (c+1) T / grid)
-    for (int c = 0; c <= a.grid; ++c) {
-        const int64_t b = (int64_t)((__int128)c * total / a.grid);
-        int64_t acc = 0, r = rbs;
-        for (int m = 0; m < a.count; ++m) {
-            const GemvMat &M = a.mat[m];
-            const int64_t mb = rb_bytes[m] * M.nrb;
-            if (b < acc + mb) {
-                r = M.rb_off + std::min<int64_t>((b - acc + rb_bytes[m] - 1) / rb_bytes[m], M.nrb);
-                break;
-            }
-            acc += mb;
+    a.total_bytes = 0;
+    a.grid = 1;
+    int grids[kMaxGemvPhases];
+    for (int p = 0; p < a.nphase; ++p) {
+        const int m0 = a.phase_first[p], m1 = a.phase_first[p + 1];
+        if (m1 <= m0) return false;
+        int64_t rbs = 0, total = 0;
+        int64_t rb_bytes[kMaxGemvTotal];  // bytes per row block (balancing only)
+        for (int m = m0; m < m1; ++m) {
+            GemvMat &M = a.mat[m];
+            M.rb_off = (int)rbs;
+            rbs += M.nrb;
+            const int64_t row = M.k * a.bits / 8 + (a.kind == 1 ? (int64_t)M.G * 16 : (int64_t)M.G * 2 + M.zbytes);
+            rb_bytes[m] = row * kRows;
+            total += rb_bytes[m] * M.nrb;
         }
-        a.cta_rb[c] = (int32_t)r;
-    }
-    // activations of the matrices a CTA touches (one copy per distinct x)
-    int64_t xmax = 0;
-    for (int c = 0; c < a.grid; ++c) {
-        int64_t xb = 0;
-        for (int m = 0; m < a.count; ++m) {
-            const GemvMat &M = a.mat[m];
-            if (std::max<int64_t>(a.cta_rb[c], M.rb_off) >= std::min<int64_t>(a.cta_rb[c + 1], M.rb_off + M.nrb))
-                continue;
-            bool dup = false;
-            for (int j = 0; j < m && !dup; ++j) {
-                const GemvMat &P = a.mat[j];
-                const bool touched =
-                    std::max<int64_t>(a.cta_rb[c], P.rb_off) < std::min<int64_t>(a.cta_rb[c + 1], P.rb_off + P.nrb);
-                dup = touched && P.x == M.x && P.k == M.k;
+        if (rbs > (int64_t)1 << 30) return false;
+        a.total_bytes += total;
+        const int grid = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), rbs);
+        grids[p] = grid;
+        a.grid = std::max(a.grid, grid);
+        // CTA c owns the row blocks whose first byte lies in [c T / grid, (c+1) T / grid)
+        for (int c = 0; c <= grid; ++c) {
+            const int64_t b = (int64_t)((__int128)c * total / grid);
+            int64_t acc = 0, r = rbs;
+            for (int m = m0; m < m1; ++m) {
+                const GemvMat &M = a.mat[m];
+                const int64_t mb = rb_bytes[m] * M.nrb;
+                if (b < acc + mb) {
+                    r = M.rb_off + std::min<int64_t>((b - acc + rb_bytes[m] - 1) / rb_bytes[m], M.nrb);
+                    break;
+                }
+                acc += mb;
             }
-            if (!dup) xb += (int64_t)a.batch * M.k * 2;
+            a.cta_rb[p][c] = (int32_t)r;
         }
-        xmax = std::max(xmax, xb);
     }
-    a.x_smem_bytes = (int)((xmax + 1023) / 1024 * 1024);  // the ring after it stays 1024-aligned
+    // CTAs beyond a phase's own grid have no row block of that phase
+    for (int p = 0; p < a.nphase; ++p)
+        for (int c = grids[p] + 1; c <= a.grid; ++c) a.cta_rb[p][c] = a.cta_rb[p][grids[p]];
     a.stage_bytes = (a.bits == 3 ? 3 * kBox : 4 * kBox) + (a.kind == 1 ? nlb_max * kBox : 0);
     // The ring is a multiple of the number of warp groups, so that every
     // slot is only ever used by one group: a warp then never waits on a
     // barrier phase more than one ahead of the slot's current one.
+    const int nbs = partial_stride(a.batch, a.batch <= kCoreBatch);
+    const int slot_bytes = kGroups * kWarps * kRows * nbs * 4;
     for (int ring = kMaxRing; ring >= kGroups; ring -= kGroups) {
         // partial-sum slots: any count is safe (a warp waits for the slot's
         // previous block); enough of them keep the warp groups from waiting
-        const int slots = bmax > 4 ? 1 : std::min(kMaxRbSlots, (ring + nks_min - 1) / nks_min + 2);
-        const int red = (slots * kWarps * bmax * 32 * 4 + 1023) / 1024 * 1024;
-        const int smem = 1024 + kHeader + red + a.x_smem_bytes + ring * a.stage_bytes;
+        int slots = std::min(kMaxRbSlots, (ring + nks_min - 1) / nks_min + 2);
+        while (slots > 2 && slots * slot_bytes > 48 * 1024) --slots;
+        const int red = (slots * slot_bytes + 1023) / 1024 * 1024;
+        const int smem = 1024 + kHeader + red + ring * a.stage_bytes;
         if (smem <= kSmemBudget || ring == kGroups) {
             a.ring = ring;
             a.rb_slots = slots;
@@ -895,18 +1086,14 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
     return a.ring >= kGroups && a.smem_bytes <= 227 * 1024;
 }
 
-template <int BITS, int KIND>
-cudaError_t launch_nb(const GemvMulti &a, cudaStream_t st, bool pdl) {
-    switch (a.batch) {
-        case 1: return launch_one<BITS, KIND, 1>(a, st, pdl);
-        case 2: return launch_one<BITS, KIND, 2>(a, st, pdl);
-        case 3: return launch_one<BITS, KIND, 3>(a, st, pdl);
-        case 4: return launch_one<BITS, KIND, 4>(a, st, pdl);
-        default: return launch_one<BITS, KIND, 8>(a, st, pdl);
-    }
-}
-
 namespace {
+
+template <int BITS, int KIND>
+cudaError_t launch_nt(const GemvMulti &a, cudaStream_t st, bool pdl) {
+    if (a.batch == 1) return launch_one<BITS, KIND, -1>(a, st, pdl);
+    if (a.batch <= kCoreBatch) return launch_one<BITS, KIND, -2>(a, st, pdl);
+    return a.batch <= 8 ? launch_one<BITS, KIND, 1>(a, st, pdl) : launch_one<BITS, KIND, 2>(a, st, pdl);
+}
 
 // Failure-detection self-test: one thread waits, with the bounded mbarrier
 // wait of the decode and prefill rings, for a phase that nothing completes
@@ -931,10 +1118,9 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t *status, cudaStream
 }
 
 cudaError_t launch_gemv_multi(GemvMulti &a, cudaStream_t st, bool pdl) {
-    a.initial = pdl ? a.ring : kGroups;
-    if (a.bits == 4) return launch_nb<4, 0>(a, st, pdl);
-    if (a.kind == 1) return launch_nb<3, 1>(a, st, pdl);
-    return launch_nb<3, 0>(a, st, pdl);
+    if (a.bits == 4) return launch_nt<4, 0>(a, st, pdl);
+    if (a.kind == 1) return launch_nt<3, 1>(a, st, pdl);
+    return launch_nt<3, 0>(a, st, pdl);
 }
 
 }  // namespace qx

@@ -35,8 +35,10 @@ struct DequantArgs {
     __half *W;
 };
 
-constexpr int kMaxGemvMats = 8;
-constexpr int kMaxGemvCtas = 512;
+constexpr int kMaxGemvMats = 8;     // matrices of one group (one phase)
+constexpr int kMaxGemvPhases = 4;   // groups of one fused launch (qx_gemv_fused)
+constexpr int kMaxGemvTotal = 16;   // matrices of one launch over all its phases
+constexpr int kMaxGemvCtas = 256;
 
 // One matrix of a (multi-matrix) decode launch.  The fields after log2g are
 // filled by plan_gemv().
@@ -52,22 +54,28 @@ struct GemvMat {
     int nks;         // 1024-weight slices per row
     int nlb;         // LUT boxes (32 rows x 8 groups) per slice
     int nrb;         // 32-row blocks
-    int rb_off;      // first row-block of this matrix in the launch's list
+    int rb_off;      // first row-block of this matrix in its phase's list
 };
 
+// A decode launch: one phase (qx_gemv_multi), or several phases run one after
+// another by one persistent grid (qx_gemv_fused), each phase's x read only
+// after every CTA has finished the phase before it.
 struct GemvMulti {
     // scalars first: the kernel's set-up reads them before anything else
-    int count, bits, kind, batch, y_f32;
-    int grid, ring, initial, rb_slots, stage_bytes, red_bytes, x_smem_bytes, smem_bytes;
+    int count, bits, kind, batch, y_f32;   // count: matrices over all phases
+    int nphase;
+    int phase_first[kMaxGemvPhases + 1];   // first matrix of each phase; [nphase] = count
+    int grid, ring, rb_slots, stage_bytes, red_bytes, smem_bytes;
     int64_t total_bytes;
     uint32_t *status;
+    uint32_t *phase_ctr;                   // nphase counters (nphase > 1): zero between launches
     uint64_t wait_limit_ns;
-    GemvMat mat[kMaxGemvMats];
-    // first row-block of every CTA (byte-balanced, computed on the host);
-    // cta_rb[grid] = total row-blocks
-    int32_t cta_rb[kMaxGemvCtas + 1];
-    CUtensorMap tm_codes[kMaxGemvMats];  // packed codes, 32-row x 128-byte boxes
-    CUtensorMap tm_luts[kMaxGemvMats];   // LUTs, 32-row x 128-byte boxes (LUT kind)
+    GemvMat mat[kMaxGemvTotal];
+    // per phase, the first row-block of every CTA in the phase's list
+    // (byte-balanced, computed on the host); cta_rb[p][grid] = the phase's row-blocks
+    int32_t cta_rb[kMaxGemvPhases][kMaxGemvCtas + 1];
+    CUtensorMap tm_codes[kMaxGemvTotal];  // packed codes, 32-row x 128-byte boxes
+    CUtensorMap tm_luts[kMaxGemvTotal];   // LUTs, 32-row x 128-byte boxes (LUT kind)
 };
 
 struct GemmArgs {

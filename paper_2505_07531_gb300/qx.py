@@ -112,6 +112,10 @@ def _lib():
         lib.qx_gemv_multi.argtypes = [P(_Packed), I32, P(VP), I32, P(VP), I32, I32, VP]
         lib.qx_gemv_chain.argtypes = [P(_GemvGroup), I32, I32, I32, I32, VP]
         lib.qx_decode_step.argtypes = [P(_Copy), I32, P(_GemvGroup), I32, I32, I32, I32, P(_Copy), I32, I32, VP]
+        lib.qx_gemv_fused_workspace.argtypes = [P(ctypes.c_size_t)]
+        lib.qx_gemv_fused.argtypes = [P(_GemvGroup), I32, I32, I32, I32, VP, ctypes.c_size_t, VP]
+        lib.qx_decode_step_fused.argtypes = [P(_Copy), I32, P(_GemvGroup), I32, I32, I32, I32, VP, ctypes.c_size_t,
+                                             P(_Copy), I32, I32, VP]
         lib.qx_q4x_size.argtypes = [I64, I64, P(_Q4xSizes)]
         lib.qx_q4x_workspace.argtypes = [I64, I64, P(ctypes.c_size_t)]
         lib.qx_q4x_quantize.argtypes = [VP, I32, P(_Q4x), VP, ctypes.c_size_t, VP]
@@ -128,7 +132,8 @@ def _lib():
         lib.qx_version.argtypes = []
         lib.qx_last_error_string.argtypes = []
         lib.qx_last_error_string.restype = ctypes.c_char_p
-        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemv_chain", "qx_decode_step", "qx_gemm",
+        for fn in ("qx_packed_size", "qx_quantize", "qx_dequant", "qx_gemv", "qx_gemv_multi", "qx_gemv_chain", "qx_decode_step", "qx_gemv_fused_workspace", "qx_gemv_fused",
+                   "qx_decode_step_fused", "qx_gemm",
                    "qx_gemm_splitk_workspace", "qx_gemm_splitk", "qx_gemm_splitk_noalloc", "qx_gemm_splitk_plan",
                    "qx_select_workspace", "qx_select_recipe", "qx_quantize_act", "qx_dequant_act", "qx_gemv_a8",
                    "qx_q4x_size", "qx_q4x_workspace", "qx_q4x_quantize", "qx_q4x_dequant", "qx_q4x_gemv", "qx_q4x_gemv_multi", "qx_q4x_gemm", "qx_q4x_gemm_splitk_workspace",
@@ -311,9 +316,11 @@ class GemvChain:
     outs) triples, each the arguments of one gemv_multi (same batch and output
     dtype throughout); the ctypes arguments are built here once, so calling
     the object costs one library call.  Build a new chain if any of the
-    tensors is replaced."""
+    tensors is replaced.  With `fused`, the groups run as ONE persistent launch
+    (qx_gemv_fused; same results), on a workspace the object owns: do not call
+    one fused object on two streams at the same time."""
 
-    def __init__(self, groups, pdl: bool = True):
+    def __init__(self, groups, pdl: bool = True, fused: bool = False):
         self._keep, built = [], []
         batch, dt, dev = None, None, None
         for mats, xs, outs in groups:
@@ -344,20 +351,31 @@ class GemvChain:
         self._args = (self._groups, len(built), batch, F32 if dt == torch.float32 else F16,
                       GEMV_PDL if pdl else 0)
         self._dev = dev
+        self._ws = None
+        if fused:
+            nbytes = ctypes.c_size_t(0)
+            _check(_lib().qx_gemv_fused_workspace(ctypes.byref(nbytes)), "qx_gemv_fused_workspace")
+            self._ws = torch.zeros(int(nbytes.value) + 256, dtype=torch.uint8, device=dev)
+            off = (-self._ws.data_ptr()) % 256
+            self._ws_args = (ctypes.c_void_p(self._ws.data_ptr() + off), int(nbytes.value))
 
     def __call__(self):
-        _check(_lib().qx_gemv_chain(*self._args, _stream(self._dev)), "qx_gemv_chain")
+        if self._ws is not None:
+            _check(_lib().qx_gemv_fused(*self._args, *self._ws_args, _stream(self._dev)), "qx_gemv_fused")
+        else:
+            _check(_lib().qx_gemv_chain(*self._args, _stream(self._dev)), "qx_gemv_chain")
 
 
 class DecodeStep(GemvChain):
-    """A whole decode step as one qx_decode_step call: the host-to-device
+    """A whole decode step as one qx_decode_step call (qx_decode_step_fused
+    with `fused`): the host-to-device
     copies `h2d` [(device tensor, host tensor)], the groups of a GemvChain, the
     device-to-host copies `d2h` [(host tensor, device tensor)], then (sync) a
     synchronization of the stream.  Host tensors should be pinned.  Arguments
     are bound once; build a new step if a tensor is replaced."""
 
-    def __init__(self, groups, h2d=(), d2h=(), pdl: bool = True, sync: bool = True):
-        super().__init__(groups, pdl)
+    def __init__(self, groups, h2d=(), d2h=(), pdl: bool = True, sync: bool = True, fused: bool = False):
+        super().__init__(groups, pdl, fused)
 
         def copies(pairs, to_device):
             arr = []
@@ -379,7 +397,12 @@ class DecodeStep(GemvChain):
         self._step = (self._in, nin, groups_arr, ng, batch, ydt, flags, self._out, nout, 1 if sync else 0)
 
     def __call__(self):
-        _check(_lib().qx_decode_step(*self._step, _stream(self._dev)), "qx_decode_step")
+        if self._ws is not None:
+            st = self._step
+            _check(_lib().qx_decode_step_fused(*st[:7], *self._ws_args, *st[7:], _stream(self._dev)),
+                   "qx_decode_step_fused")
+        else:
+            _check(_lib().qx_decode_step(*self._step, _stream(self._dev)), "qx_decode_step")
 
 
 def gemm(P: PackedMatrix, X: torch.Tensor, out: torch.Tensor | None = None) -> torch.Tensor:

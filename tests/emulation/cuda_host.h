@@ -52,6 +52,7 @@ namespace emu {
 struct Warp {
     std::unique_ptr<std::barrier<>> bar;
     uint64_t buf[32];
+    uint32_t mbuf[32][10];  // per-lane operands of a warp-wide matrix instruction
 };
 struct MBar {  // an mbarrier: arrivals still expected, transaction bytes, phase
     uint32_t count = 0, pending = 0, phase = 0;
@@ -66,6 +67,8 @@ struct Block {
     std::unordered_map<uint32_t, MBar> mbars;  // by shared-memory address
     std::vector<float> tmem;                   // tensor memory: 128 lanes x 512 columns
     uint32_t tmem_cols = 0;
+    std::mutex nbar_mu;
+    std::unique_ptr<std::barrier<>> nbar;      // named barrier 1 (the first use sets its count)
 };
 inline thread_local dim3 t_tid, t_bid;
 inline thread_local Block *t_block = nullptr;
@@ -160,6 +163,9 @@ struct alignas(4) __half2 {
 struct float2 {
     float x, y;
 };
+struct alignas(16) float4 {
+    float x, y, z, w;
+};
 struct alignas(16) uint4 {
     unsigned x, y, z, w;
 };
@@ -190,10 +196,11 @@ inline __half2 __hmul2(__half2 a, __half2 b) {
                    __float2half_rn(__half2float(a.y) * __half2float(b.y))};
 }
 inline float2 __half22float2(__half2 h) { return float2{__half2float(h.x), __half2float(h.y)}; }
+inline float __low2float(__half2 h) { return __half2float(h.x); }
 
 // ------------------------------------------------------------------ runtime
 typedef void *cudaStream_t;
-enum cudaError_t { cudaSuccess = 0, cudaErrorInvalidValue = 1, cudaErrorInvalidConfiguration = 9, cudaErrorInvalidDevice = 101, cudaErrorNotSupported = 801 };
+enum cudaError_t { cudaSuccess = 0, cudaErrorInvalidValue = 1, cudaErrorInvalidConfiguration = 9, cudaErrorInvalidDevice = 101, cudaErrorCooperativeLaunchTooLarge = 720, cudaErrorNotSupported = 801 };
 inline cudaError_t cudaMemsetAsync(void *p, int v, size_t n, cudaStream_t) {
     std::memset(p, v, n);
     return cudaSuccess;
@@ -399,6 +406,81 @@ inline uint4 emu_lds128(uint32_t a) {
     return v;
 }
 
+// ldmatrix .m8n8 .b16 (nmat = 1, 2 or 4 matrices): lanes 8i..8i+7 give the
+// 16-byte row addresses of matrix i; lane l receives bytes 4(l%4)..4(l%4)+3
+// of row l/4 of every matrix.
+inline void emu_ldsm(uint32_t a, int nmat, uint32_t *d0, uint32_t *d1, uint32_t *d2, uint32_t *d3) {
+    emu::Warp &w = emu_warp();
+    const unsigned l = emu_lane();
+    w.buf[l] = a;
+    w.bar->arrive_and_wait();
+    uint32_t *d[4] = {d0, d1, d2, d3};
+    for (int i = 0; i < nmat; ++i) {
+        const uint32_t row = (uint32_t)w.buf[8 * i + l / 4];
+        if (row & 15u) emu_fail("misaligned ldmatrix row address");
+        std::memcpy(d[i], emu_shared(row + 4 * (l % 4), 4), 4);
+    }
+    w.bar->arrive_and_wait();
+}
+
+// mma.sync m16n8k16 row.col f32.f16.f16.f32, D = A B + C, with lane (g, t)
+// holding a0 = A[g][2t..2t+1], a1 = A[g+8][2t..], a2 = A[g][2t+8..],
+// a3 = A[g+8][2t+8..], b0 = B[2t..2t+1][g], b1 = B[2t+8..2t+9][g] and
+// D[g][2t], D[g][2t+1], D[g+8][2t], D[g+8][2t+1].  The fp16 products are exact;
+// the sum is formed in double and rounded once to fp32 (the hardware's adder
+// order is not specified, so results are checked within tolerance).
+inline float emu_h2f(uint32_t bits16) {
+    __half h;
+    const uint16_t b = (uint16_t)bits16;
+    std::memcpy(&h, &b, 2);
+    return __half2float(h);
+}
+inline void emu_mma16816(float &d0, float &d1, float &d2, float &d3, uint32_t a0, uint32_t a1, uint32_t a2,
+                         uint32_t a3, uint32_t b0, uint32_t b1) {
+    emu::Warp &w = emu_warp();
+    const unsigned l = emu_lane();
+    uint32_t *m = w.mbuf[l];
+    const float c[4] = {d0, d1, d2, d3};
+    m[0] = a0; m[1] = a1; m[2] = a2; m[3] = a3; m[4] = b0; m[5] = b1;
+    std::memcpy(&m[6], c, 16);
+    w.bar->arrive_and_wait();
+    auto A = [&](int row, int k) {  // A[row][k]
+        const uint32_t r = w.mbuf[4 * (row % 8) + (k % 8) / 2][(row >= 8 ? 1 : 0) + (k >= 8 ? 2 : 0)];
+        return emu_h2f(k % 2 ? r >> 16 : r);
+    };
+    auto B = [&](int k, int col) {  // B[k][col]
+        const uint32_t r = w.mbuf[4 * col + (k % 8) / 2][4 + (k >= 8 ? 1 : 0)];
+        return emu_h2f(k % 2 ? r >> 16 : r);
+    };
+    const int g = (int)l / 4, t = (int)l % 4;
+    float out[4];
+    for (int i = 0; i < 4; ++i) {
+        const int row = g + 8 * (i / 2), col = 2 * t + (i % 2);
+        double s = c[i];
+        for (int k = 0; k < 16; ++k) s += (double)A(row, k) * (double)B(k, col);
+        out[i] = (float)s;
+    }
+    w.bar->arrive_and_wait();
+    d0 = out[0]; d1 = out[1]; d2 = out[2]; d3 = out[3];
+}
+
+// atom.add on a shared-memory word (by its shared address)
+inline uint32_t emu_atom_add_shared(uint32_t a, uint32_t v) {
+    if (a & 3u) emu_fail("misaligned shared atomic");
+    return std::atomic_ref<uint32_t>(*reinterpret_cast<uint32_t *>(emu_shared(a, 4))).fetch_add(v);
+}
+inline void __nanosleep(unsigned) { std::this_thread::yield(); }
+
+// bar.sync 1, n: a barrier of n threads of the block
+inline void emu_named_bar(unsigned n) {
+    emu::Block *b = emu::t_block;
+    {
+        std::lock_guard<std::mutex> l(b->nbar_mu);
+        if (!b->nbar) b->nbar = std::make_unique<std::barrier<>>((std::ptrdiff_t)n);
+    }
+    b->nbar->arrive_and_wait();
+}
+
 inline emu::MBar &emu_mbar(uint32_t a) {
     auto it = emu::t_block->mbars.find(a);
     if (it == emu::t_block->mbars.end()) emu_fail("mbarrier used before init");
@@ -520,9 +602,10 @@ inline void emu_tma_load(uint32_t dst, const void *map, uint32_t bar, const int 
 
 // cudaLaunchKernelEx with its configuration (launch attributes are ignored:
 // kernels run one after another).
-enum cudaLaunchAttributeID { cudaLaunchAttributeProgrammaticStreamSerialization = 1 };
+enum cudaLaunchAttributeID { cudaLaunchAttributeProgrammaticStreamSerialization = 1, cudaLaunchAttributeCooperative = 2 };
 struct cudaLaunchAttributeValue {
     int programmaticStreamSerializationAllowed;
+    int cooperative;
 };
 struct cudaLaunchAttribute {
     cudaLaunchAttributeID id;

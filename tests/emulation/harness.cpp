@@ -207,6 +207,9 @@ int main(int argc, char **argv) {
             for (int launch = 0; launch < 2; ++launch) {
                 qx::GemvMulti m{};
                 m.count = launch == 0 ? 1 : 2;
+                m.nphase = 1;
+                m.phase_first[0] = 0;
+                m.phase_first[1] = m.count;
                 m.bits = bits;
                 m.kind = kind;
                 m.batch = batch;

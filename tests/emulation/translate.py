@@ -29,11 +29,23 @@ BY_INSTRUCTION = [
     ("mbarrier.init", "emu_mbar_init({i0}, {i1});"),
     ("mbarrier.arrive.expect_tx", "emu_mbar_arrive_expect_tx({i0}, {i1});"),
     ("mbarrier.arrive.shared", "emu_mbar_arrive({i0});"),
+    ("atom.acq_rel.cta.shared::cta.add.u32", "{o0} = emu_atom_add_shared({i0}, {i1});"),
     ("mbarrier.try_wait.parity", "{o0} = emu_mbar_try_wait({i0}, {i1}) ? 1u : 0u;"),
     ("cp.async.bulk.tensor.2d", "{{ const int c_[2] = {{{i3}, {i4}}}; emu_tma_load({i0}, {i1}, {i2}, c_, 2); }}"),
     ("cp.async.bulk.tensor.3d",
      "{{ const int c_[3] = {{{i3}, {i4}, {i5}}}; emu_tma_load({i0}, {i1}, {i2}, c_, 3); }}"),
     ("cp.async.bulk.prefetch.L2", ";"),
+    ("ldmatrix.sync.aligned.m8n8.x4", "emu_ldsm({i0}, 4, &{o0}, &{o1}, &{o2}, &{o3});"),
+    ("ldmatrix.sync.aligned.m8n8.x2", "emu_ldsm({i0}, 2, &{o0}, &{o1}, nullptr, nullptr);"),
+    ("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32",
+     "emu_mma16816({o0}, {o1}, {o2}, {o3}, {i0}, {i1}, {i2}, {i3}, {i4}, {i5});"),
+    ("ld.global.cg.v4.u32",
+     "{{ uint4 t_; std::memcpy(&t_, (const void *)({i0}), 16); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
+    ("bar.sync 1", "emu_named_bar({i0});"),
+    ("atom.add.release.gpu.global.u32", "{o0} = std::atomic_ref<uint32_t>(*({i0})).fetch_add({i1});"),
+    ("ld.acquire.gpu.global.u32", "{o0} = std::atomic_ref<uint32_t>(*const_cast<uint32_t *>({i0})).load();"),
+    ("ld.global.nc.v4.u32",
+     "{{ uint4 t_; std::memcpy(&t_, (const void *)({i0}), 16); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
     ("ld.shared.v4.u32", "{{ const uint4 t_ = emu_lds128({i0}); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
     ("ld.shared.u32", "{o0} = emu_lds32({i0});"),
     ("griddepcontrol", ";"),
@@ -52,7 +64,7 @@ BY_INSTRUCTION = [
 ]
 ASM = re.compile(r"\basm\s*(?:volatile\s*)?\((.*?)\);", re.S)
 LAUNCH = re.compile(r"(\w+(?:<[^<>;]*>)?)<<<(.*?)>>>\((.*?)\);", re.S)
-CONSTRAINT = re.compile(r'"(=?[a-z])"\s*\(')
+CONSTRAINT = re.compile(r'"([=+]?[a-z])"\s*\(')
 
 
 def operands(body: str):
@@ -63,7 +75,7 @@ def operands(body: str):
         while depth:
             depth += {"(": 1, ")": -1}.get(body[j], 0)
             j += 1
-        (outs if m.group(1).startswith("=") else ins).append(body[m.end():j - 1].strip())
+        (outs if m.group(1)[0] in "=+" else ins).append(body[m.end():j - 1].strip())
     return outs, ins
 
 

@@ -111,9 +111,10 @@ def test_int8_activations_and_w_a8_matmul(harness, n, k, bits, g, batch):
     assert np.all(oracle.max_abs_err(y, oracle.gemv_a8(ref, rec, x, k)) <= tol)
 
 
-@pytest.mark.parametrize("n,k,bits,g,kind,batch,sms", [  # 1..4 and 8 rows of x, ragged row blocks
+@pytest.mark.parametrize("n,k,bits,g,kind,batch,sms", [  # 1..16 rows of x, ragged row blocks
     (37, 384, 4, 64, 0, 1, 2), (130, 640, 3, 64, 0, 4, 3), (33, 256, 4, 32, 0, 8, 2),
-    (20, 512, 3, 128, 1, 3, 2), (5, 4096, 4, 128, 0, 2, 4), (70, 1152, 3, 128, 0, 1, 3)])
+    (20, 512, 3, 128, 1, 3, 2), (5, 4096, 4, 128, 0, 2, 4), (70, 1152, 3, 128, 0, 1, 3),
+    (40, 512, 3, 128, 1, 16, 2), (33, 384, 4, 64, 0, 11, 2), (24, 768, 3, 32, 1, 5, 2)])
 def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms):
     """qx_gemv's kernel and host plan (tensor maps, byte-balanced CTA slices):
     one matrix, and the same matrix twice in one launch (with PDL set)."""

@@ -207,7 +207,7 @@ def test_nonfinite_group_is_flagged_and_coded_as_dead(qx):
     _assert_same(P, oracle.quantize_q4x(clean))
 
 
-@pytest.mark.parametrize("shape", [(96, 512), (37, 320)])
+@pytest.mark.parametrize("shape", [(96, 512), (37, 384)])
 def test_select_recipe_with_q4x_candidate(qx, shape):
     """Recipe selection with a Q4X candidate beside per-group ones: the same
     choice, exact errors and bits per weight as the oracle, with budgets that

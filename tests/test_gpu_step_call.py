@@ -36,9 +36,11 @@ def test_chain_equals_the_separate_calls(qx, batch):
     assert qx.device_status() == 0
 
 
-def test_decode_step_copies_in_and_out(qx):
-    """qx_decode_step: pinned host x in, the groups, host y out, synchronized:
-    the host outputs equal the device results of the separate calls."""
+@pytest.mark.parametrize("fused", [False, True])
+def test_decode_step_copies_in_and_out(qx, fused):
+    """qx_decode_step (qx_decode_step_fused): pinned host x in, the groups, host
+    y out, synchronized: the host outputs equal the device results of the
+    separate calls."""
     rec = qx.Recipe(4, 128, qx.UNIFORM)
     mats = [qx.quantize(torch.from_numpy(synth.student_t_weights(n, 512, 0.02, seed=n, stream=1)).cuda(), rec)
             for n in (256, 384)]
@@ -46,9 +48,44 @@ def test_decode_step_copies_in_and_out(qx):
     dx = torch.empty(hx.shape, dtype=hx.dtype, device="cuda")
     dys = [torch.empty((2, P.n), dtype=torch.float16, device="cuda") for P in mats]
     hys = [torch.full((2, P.n), float("nan"), dtype=torch.float16).pin_memory() for P in mats]
-    step = qx.DecodeStep([(mats, [dx, dx], dys)], h2d=[(dx, hx)], d2h=list(zip(hys, dys)))
+    step = qx.DecodeStep([(mats, [dx, dx], dys)], h2d=[(dx, hx)], d2h=list(zip(hys, dys)), fused=fused)
     step()
     ref = qx.gemv_multi(mats, [hx.cuda(), hx.cuda()])
     for h, r in zip(hys, ref):
         assert torch.equal(h, r.cpu())
     assert qx.device_status() == 0
+
+
+@pytest.mark.parametrize("bits,g,kind", [(3, 128, 1), (4, 64, 0)])
+@pytest.mark.parametrize("batch", [1, 2, 5, 16])
+def test_fused_launch_equals_the_chain(qx, bits, g, kind, batch):
+    """qx_gemv_fused: the groups of a chain in one persistent launch, bit for
+    bit the chain's results.  With fp16 outputs the third group reads the first
+    group's output as its x, which the launch may read only once every CTA has
+    finished the first group (the outputs start as NaN, so an early read
+    shows).  Three calls in a row share one workspace: each launch leaves its
+    phase counters zero for the next."""
+    rec = qx.Recipe(bits, g, kind)
+    shapes = {"q": (256, 512), "k": (96, 512), "up": (1000, 512), "o": (512, 256), "down": (384, 1024)}
+    mats = {nm: qx.quantize(torch.from_numpy(synth.student_t_weights(n, k, 0.02, seed=i, stream=n)).cuda(), rec)
+            for i, (nm, (n, k)) in enumerate(shapes.items())}
+    xa = torch.from_numpy(synth.activations(batch, 512, seed=1, stream=1)).cuda()
+    xd = torch.from_numpy(synth.activations(batch, 1024, seed=2, stream=2)).cuda()
+    for dt in (torch.float16, torch.float32):
+        ys = {nm: torch.empty((batch, P.n), dtype=dt, device="cuda") for nm, P in mats.items()}
+        handoff = dt == torch.float16
+        xo = ys["q"] if handoff else torch.from_numpy(synth.activations(batch, 256, seed=3, stream=3)).cuda()
+        groups = [(["q", "k"], [xa, xa]), (["up"], [xa]), (["o"], [xo]), (["down"], [xd])]
+        fused = qx.GemvChain([([mats[nm] for nm in names], xs, [ys[nm] for nm in names]) for names, xs in groups],
+                             fused=True)
+        for rep in range(3):
+            for y in ys.values():
+                y.fill_(float("nan"))
+            fused()
+            ref = {}
+            for names, xs in groups:
+                xs_ref = [ref["q"] if handoff and x is ys["q"] else x for x in xs]
+                ref.update(zip(names, qx.gemv_multi([mats[nm] for nm in names], xs_ref, out_dtype=dt, pdl=True)))
+            for nm in mats:
+                assert torch.equal(ys[nm], ref[nm]), (nm, rep)
+        assert qx.device_status() == 0

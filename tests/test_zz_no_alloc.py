@@ -4,7 +4,6 @@ static scratch in place of a caller workspace.  Same results as the oracle
 memory allocated by the calls, and a refusal when the plan needs more scratch
 than the library holds.  Collected last (its name), so that the rest of the
 suite runs first."""
-import ctypes
 
 import numpy as np
 import pytest
@@ -16,16 +15,27 @@ from oracle.pack import Recipe as ORecipe
 
 
 def test_noalloc_rejects_bad_arguments_before_launching():
-    import paper_2505_07531_gb300.qx as qx
+    """Host validation refuses a null struct, m = 0 and a misaligned X before
+    any launch.  The calls run in a child process that sees no CUDA device, so
+    that the placeholder addresses below can never reach a kernel: were the
+    validation ever to let one through, the call would fail in the CUDA
+    runtime (QX_ERR_CUDA = 4), not launch."""
+    import os
+    import subprocess
+    import sys
 
-    lib = qx._lib()
-    assert lib.qx_gemm_splitk_noalloc(None, None, 1, None, None) == 1
-    P = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), ctypes.c_void_p(0x1000), ctypes.c_void_p(0x2000),
-                   ctypes.c_void_p(0x3000), None)
-    assert lib.qx_gemm_splitk_noalloc(ctypes.byref(P), ctypes.c_void_p(0x4000), 0, ctypes.c_void_p(0x5000),
-                                      None) == 1
-    assert lib.qx_gemm_splitk_noalloc(ctypes.byref(P), ctypes.c_void_p(0x4008), 1, ctypes.c_void_p(0x5000),
-                                      None) == 3
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    code = (
+        "import ctypes, paper_2505_07531_gb300.qx as qx\n"
+        "lib = qx._lib(); A = ctypes.c_void_p\n"
+        "P = qx._Packed(64, 128, qx._Recipe(4, 64, 0, 0), A(0x1000), A(0x2000), A(0x3000), None)\n"
+        "print(lib.qx_gemm_splitk_noalloc(None, None, 1, None, None),\n"
+        "      lib.qx_gemm_splitk_noalloc(ctypes.byref(P), A(0x4000), 0, A(0x5000), None),\n"
+        "      lib.qx_gemm_splitk_noalloc(ctypes.byref(P), A(0x4008), 1, A(0x5000), None))\n")
+    env = dict(os.environ, CUDA_VISIBLE_DEVICES="")
+    r = subprocess.run([sys.executable, "-c", code], capture_output=True, text=True, cwd=root, env=env, timeout=300)
+    assert r.returncode == 0, r.stderr[-2000:]
+    assert r.stdout.split() == ["1", "1", "3"]  # QX_ERR_INVALID_ARG twice, then QX_ERR_ALIGNMENT
 
 
 @pytest.fixture(scope="module")
