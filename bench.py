@@ -180,8 +180,53 @@ def _oracle_pass(rec, mats):
         oracle.gemv(p, rec, x, k)
 
 
+_POOL_SAMPLE = None
+
+
+def _pool_init(sample):
+    global _POOL_SAMPLE
+    _POOL_SAMPLE = sample
+
+
+def _pool_passes(passes: int) -> float:
+    rec, mats = _POOL_SAMPLE
+    t0 = time.perf_counter()
+    for _ in range(passes):
+        _oracle_pass(rec, mats)
+    return time.perf_counter() - t0
+
+
+class _OraclePool:
+    """The oracle on every host core: one single-threaded process per core,
+    each making whole passes over its own copy of the sample (started with
+    spawn, in a process that has not touched the GPU)."""
+
+    def __init__(self, rec, mats, workers: int):
+        import multiprocessing as mp
+
+        self.workers = workers
+        self.pool = mp.get_context("spawn").Pool(workers, initializer=_pool_init, initargs=((rec, mats),))
+        self.pool.map(_pool_passes, [1] * workers)  # start-up and first touch
+
+    def run(self, passes: int) -> float:
+        """Wall seconds for `passes` passes on every worker."""
+        t0 = time.perf_counter()
+        self.pool.map(_pool_passes, [passes] * self.workers)
+        return time.perf_counter() - t0
+
+    def close(self):
+        self.pool.close()
+        self.pool.join()
+
+
+def _single_thread_env():
+    return dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+                CUDA_VISIBLE_DEVICES="")
+
+
 def cpu_baseline_child(seconds: float):
-    """Run in a single-threaded subprocess: oracle GB/s on a bounded sample."""
+    """Run in a subprocess with single-threaded numpy: oracle GB/s on a bounded
+    sample, on one core and on every core."""
     rec, mats = _oracle_sample(64)
     nbytes = sum(m[3] for m in mats)
     _oracle_pass(rec, mats)
@@ -193,34 +238,62 @@ def cpu_baseline_child(seconds: float):
         if time.perf_counter() - t0 >= seconds:
             break
     dt = time.perf_counter() - t0
-    print(json.dumps({"value": nbytes * reps / dt / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
-                      "sample": f"{reps} passes over the first 64 rows of each of the 7 layer matrices "
-                                f"({nbytes / 1e6:.2f} MB packed per pass), numpy float64, 1 thread, {dt:.1f} s"}))
+    one = nbytes * reps / dt / 1e9
+    workers = os.cpu_count() or 1
+    pool = _OraclePool(rec, mats, workers)
+    chunk = max(1, int(seconds / (dt / reps)) // 16)  # bounded in time whatever the cores' speed
+    passes, dtp = 0, 0.0
+    while dtp < seconds:
+        dtp += pool.run(chunk)
+        passes += chunk
+    pool.close()
+    allc = nbytes * passes * workers / dtp / 1e9
+    print(json.dumps({"value": allc, "unit": "GB/s", "cores": workers, "kind": "oracle",
+                      "value_1_core": one,
+                      "sample": f"the first 64 rows of each of the 7 layer matrices ({nbytes / 1e6:.2f} MB packed "
+                                f"per pass), numpy float64: {workers} single-threaded processes x {passes} passes "
+                                f"each in {dtp:.1f} s; on 1 core {reps} passes in {dt:.1f} s"}))
 
 
 def run_cpu_baseline(seconds: float = 12.0):
-    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
-               CUDA_VISIBLE_DEVICES="")
     r = subprocess.run([sys.executable, os.path.abspath(__file__), "--cpu-baseline-child", str(seconds)],
-                       capture_output=True, text=True, env=env, timeout=600)
+                       capture_output=True, text=True, env=_single_thread_env(), timeout=900)
     try:
         return json.loads(r.stdout.strip().splitlines()[-1])
     except Exception:
-        return {"value": None, "unit": "GB/s", "cores": 1, "kind": "oracle", "sample": "failed: " + r.stderr[-200:]}
+        return {"value": None, "unit": "GB/s", "cores": None, "kind": "oracle", "sample": "failed: " + r.stderr[-200:]}
 
 
 def run_reference(args):
-    """The oracle as the reference arm: same metric and config, bounded samples per step.
+    """The oracle as the reference arm: same metric and config, on every host
+    core, bounded samples per step.
 
     The oracle quantizes a fixed sample (the first 64 rows of each of the seven
     matrices) once; a step is a whole number of dequantize + float64 matvec passes
-    over that sample, sized so that warm-up plus timed steps take about
-    QX_REF_BUDGET_S seconds of wall time.
+    over that sample on each of os.cpu_count() single-threaded processes, sized so
+    that warm-up plus timed steps take about QX_REF_BUDGET_S seconds of wall time.
     """
     dist, rank, ws, _ = _dist()
     if rank != 0:
         return
+    if os.environ.get("QX_REF_CHILD") != "1":
+        # numpy single-threaded in every process: the processes are the cores
+        env = dict(_single_thread_env(), QX_REF_CHILD="1")
+        env.pop("RANK", None)
+        env.pop("WORLD_SIZE", None)
+        r = subprocess.run([sys.executable, os.path.abspath(__file__), "--impl", "reference", "--gpus", str(ws),
+                            "--steps", str(args.steps), "--warmup", str(args.warmup)], capture_output=True, text=True,
+                           env=env, timeout=1800)
+        out = [ln for ln in r.stdout.splitlines() if ln.startswith("{")]
+        if r.returncode != 0 or not out:
+            print(json.dumps({"impl": "reference", "unavailable": "oracle arm failed: " + r.stderr[-200:]}))
+            return
+        line = json.loads(out[-1])
+        line["n_gpus"] = ws
+        print(json.dumps(line))
+        return
     steps, warmup = args.steps, args.warmup
+    workers = os.cpu_count() or 1
     per_step = REF_BUDGET_S / max(1, steps + warmup)
     rows = 64
     rec, mats = _oracle_sample(rows)
@@ -238,28 +311,23 @@ def run_reference(args):
         _oracle_pass(rec, mats)
         t_pass = max(time.perf_counter() - t0, 1e-6)
     passes = max(1, int(per_step / t_pass))
-
-    def one_step():
-        for _ in range(passes):
-            _oracle_pass(rec, mats)
-
+    pool = _OraclePool(rec, mats, workers)
     for _ in range(warmup):
-        one_step()
-    t0 = time.perf_counter()
+        pool.run(passes)
+    dt = 0.0
     for _ in range(steps):
-        one_step()
-    dt = time.perf_counter() - t0
-    v = nbytes * passes * steps / dt / 1e9
-    cores = 1 if os.environ.get("OPENBLAS_NUM_THREADS") == "1" else (os.cpu_count() or 1)
-    sample = (f"{passes} pass(es) per step over the first {rows} rows of each of the 7 layer matrices "
-              f"({nbytes / 1e6:.2f} MB packed per pass), numpy float64")
+        dt += pool.run(passes)
+    pool.close()
+    v = nbytes * passes * workers * steps / dt / 1e9
+    sample = (f"{workers} single-threaded processes, each {passes} pass(es) per step over the first {rows} rows of "
+              f"each of the 7 layer matrices ({nbytes / 1e6:.2f} MB packed per pass), numpy float64")
     line = {
         "impl": "reference", "metric": METRIC, "value": v, "unit": "GB/s", "n_gpus": ws, "steps": steps,
         "warmup": warmup, "ms_per_step": dt / steps * 1e3, "higher_is_better": True, "scaling": "weak",
         "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": {"workload": "llama7b_layer_decode_L3g128_b1", "sample_rows_per_matrix": rows,
-                   "passes_per_step": passes},
-        "cpu_baseline": {"value": v, "unit": "GB/s", "cores": cores, "kind": "oracle", "sample": sample},
+                   "passes_per_step_per_process": passes},
+        "cpu_baseline": {"value": v, "unit": "GB/s", "cores": workers, "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line))
@@ -282,6 +350,29 @@ def _quantize_layer(qx, torch, dev, mats, recipe, seed=0):
 def _clone(qx, P):
     c = lambda t: None if t is None else t.clone()
     return qx.PackedMatrix(P.n, P.k, P.recipe, c(P.codes), c(P.scales), c(P.zeros), c(P.luts))
+
+
+def _summary(line, hbm, tf_burst):
+    """The headline figures in a few keys (the end of the line)."""
+    def get(d, *path):
+        for p in path:
+            if not isinstance(d, dict) or p not in d:
+                return None
+            d = d[p]
+        return d
+
+    out = {"decode_L3g128_b1_GBps": line["value"], "frac_of_measured_hbm": line["value"] / hbm,
+           "e2e_GBps": get(line, "e2e", "value"),
+           "prefill_TFLOPs": get(line, "gemm", "value"), "prefill_frac_of_bf16_burst": get(line, "gemm", "roofline", "frac")}
+    for rec in ("U4g128", "U3g64"):
+        for b in (1, 4, 16):
+            v = get(line, "config3", f"llama7b_layer_decode_{rec}_b{b}", "GBps")
+            if v is not None:
+                out[f"decode_{rec}_b{b}_GBps"] = v
+    v = get(line, "q4x", "llama7b_layer_decode_Q4X_b1", "GBps")
+    if v is not None:
+        out["decode_Q4X_b1_GBps"] = v
+    return out
 
 
 def run_ours(args):
@@ -344,6 +435,12 @@ def run_ours(args):
         with torch.cuda.graph(g, stream=stream):
             step(c)
         graphs.append(g)
+    # one graph of a step on every copy in turn: programmatic dependent launch
+    # links consecutive steps inside it (it does not cross graph boundaries)
+    g_all = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g_all, stream=stream):
+        for c in range(copies):
+            step(c)
     torch.cuda.synchronize(dev)
 
     uuid = getattr(props, "uuid", None)
@@ -366,8 +463,10 @@ def run_ours(args):
     ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     with torch.cuda.stream(stream):
         ev0.record(stream)
-        for i in range(args.steps):
-            graphs[i % copies].replay()
+        for _ in range(args.steps // copies):  # exactly K steps: whole rounds, then single steps
+            g_all.replay()
+        for i in range(args.steps % copies):
+            graphs[i].replay()
         ev1.record(stream)
     torch.cuda.synchronize(dev)
     clocks = sampler.stop()
@@ -417,6 +516,25 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     one_launch_ms = e0.elapsed_time(e1) / reps
 
+    # the same chain as ONE persistent launch (qx_gemv_fused): the four groups
+    # hand off through device-side counters instead of kernel boundaries
+    fused_us = None
+    try:
+        fsteps = [qx.GemvChain([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
+                                for names, x in CHAIN], fused=True) for c in range(copies)]
+        with torch.cuda.stream(stream):
+            for fs in fsteps:
+                fs()
+        torch.cuda.synchronize(dev)
+        gf = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(gf, stream=stream):
+            for fs in fsteps:
+                fs()
+        fused_us = _time_graph(torch, stream, gf, 20) / copies * 1e3
+        del gf, fsteps
+    except Exception as e:  # noqa: BLE001
+        fused_us = f"unavailable: {type(e).__name__}: {e}"[:160]
+
     # end to end through the public API with host buffers: the step's activations
     # in from pinned host memory (one copy), the four decode calls, the outputs
     # back (one copy), then a stream synchronisation, per step
@@ -459,10 +577,10 @@ def run_ours(args):
 
     section = lambda fn, *a: _section(torch, fn, *a)  # noqa: E731
     gemm = section(run_gemm_part, qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
-    del layers, graphs
+    del layers, graphs, g_all
     extra = {}
     if not args.skip_configs:
-        extra["config3"] = section(run_config3, qx, torch, dev, stream, l2)
+        extra["config3"] = section(run_config3, qx, torch, dev, stream, l2, hbm)
         extra["recipe_select"] = section(run_select, qx, torch, dev, stream)
         extra["config5"] = section(run_config5, qx, torch, dev, stream)
         extra["q4x"] = section(run_q4x, qx, torch, dev, stream, l2, hbm, tf_burst)
@@ -478,26 +596,31 @@ def run_ours(args):
                        "matrices": {nm: [n, k] for nm, n, k, _, _ in LAYER},
                        "recipe": "3-bit LUT (8 fp16 levels, Lloyd-Max) group 128",
                        "batch": 1, "bytes_per_step": step_bytes,
-                       "step": "qkv | o | gate+up | down: 4 qx_gemv_multi launches (PDL) in one CUDA graph",
+                       "step": "qkv | o | gate+up | down: 4 qx_gemv_multi launches (PDL); CUDA graphs of one "
+                               "step on every weight copy in turn",
                        "l2": f"{copies} rotating weight copies ({copies * layer_bytes / 1e6:.0f} MB) > "
                              f"4x L2 ({l2 / 1e6:.0f} MB)"},
+            # the long sections first: the record keeps the end of the line
+            **extra,
             "per_launch_us": per_launch_us,
             "one_launch_7_matrices": {"us": one_launch_ms * 1e3,
                                       "GBps": step_bytes / (one_launch_ms * 1e-3) / 1e9},
-            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
-                         "frac": achieved / hbm, "peak_source": f"{peak_src} hbm_gbs",
-                         "kernel": "gemv_kernel<3,LUT,1>", "launches_per_step": len(CHAIN),
-                         "launch_us": launch_us, "bytes_per_launch": step_bytes / len(CHAIN),
-                         "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
-            "gemm": gemm,
-            **extra,
+            "fused_one_launch_4_groups": ({"us": fused_us, "GBps": step_bytes / (fused_us * 1e-6) / 1e9}
+                                          if isinstance(fused_us, float) else fused_us),
             "cpu_baseline": cpu,
             "clocks": clocks,
             "e2e": {"value": e2e_value, "unit": "GB/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": hx.numel() * hx.element_size(),
                     "d2h_bytes_per_step": hy.numel() * hy.element_size(), "path": e2e_path},
             "gpu_launches": args.steps * len(CHAIN),
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                         "frac": achieved / hbm, "peak_source": f"{peak_src} hbm_gbs",
+                         "kernel": "gemv_kernel<3,LUT,-1>", "launches_per_step": len(CHAIN),
+                         "launch_us": launch_us, "bytes_per_launch": step_bytes / len(CHAIN),
+                         "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
+            "gemm": gemm,
         }
+        line["summary"] = _summary(line, hbm, tf_burst)
         print(json.dumps(line))
     if dist is not None:
         dist.destroy_process_group()
@@ -637,10 +760,11 @@ def _time_graph(torch, stream, g, reps):
     return e0.elapsed_time(e1) / reps  # ms per replay
 
 
-def run_config3(qx, torch, dev, stream, l2):
+def run_config3(qx, torch, dev, stream, l2, hbm):
     """Llama-7B layer, 4-bit uniform g128 and 3-bit uniform g64, batch 1 / 4 / 16:
-    the CUDA-core decode chain (qx_gemv_multi, PDL) and, for batch 4 and 16,
-    the tensor-core path (qx_gemm_splitk, one launch per matrix)."""
+    the decode chain (qx_gemv_multi, PDL; products on the CUDA cores at batch
+    1, on mma.sync at 4 and 16) and, for batch 4 and 16, the tcgen05 split-k
+    matmul (qx_gemm_splitk, one launch per matrix) beside it."""
     import synth
 
     out = {}
@@ -660,9 +784,11 @@ def run_config3(qx, torch, dev, stream, l2):
             ms = _time_graph(torch, stream, gr, 20) / copies
             del gr
             io = sum(x.numel() * 2 for x in xs) + sum(y.numel() * 2 for y in ys.values())
+            gbps = (layer_bytes + io) / (ms * 1e-3) / 1e9
             out[f"llama7b_layer_decode_U{bits}g{g}_b{batch}"] = {
-                "us_per_layer": ms * 1e3, "GBps": (layer_bytes + io) / (ms * 1e-3) / 1e9,
-                "weight_bytes": layer_bytes, "path": "qx_gemv_multi chain (CUDA cores)"}
+                "us_per_layer": ms * 1e3, "GBps": gbps, "frac_of_measured_hbm": gbps / hbm,
+                "weight_bytes": layer_bytes,
+                "path": "4 qx_gemv_multi launches (PDL): " + ("CUDA-core" if batch <= 2 else "mma.sync") + " products"}
             if batch in (1, 4):
                 # W.A8: the four distinct activations quantized per token to int8,
                 # then seven integer-dot matmuls (qx_quantize_act + qx_gemv_a8)
@@ -720,6 +846,7 @@ def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
     def learn(name, n, k, sigma, sid):
         W = synth.student_t_weights_torch(n, k, sigma, seed=0, stream=sid, device=dev)
         with torch.cuda.stream(stream):
+            stream.wait_stream(torch.cuda.default_stream(dev))  # W is drawn on the default stream
             e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
             e0.record(stream)
             P = qx.q4x_quantize(W)
@@ -731,8 +858,9 @@ def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
     base, learn_ms = {}, {}
     for spec in LAYER:
         base[spec[0]], learn_ms[spec[0]] = learn(*spec)
-    if qx.device_status(stream) != 0:
-        raise RuntimeError("q4x_quantize reported a device error")
+    st_code = qx.device_status(stream)
+    if st_code != 0:
+        raise RuntimeError(f"q4x_quantize reported device status {st_code}")
     layer_bytes = sum(P.nbytes() for P in base.values())
     copies = max(2, math.ceil(4 * l2 / layer_bytes))
     dup = lambda P: qx.Q4xMatrix(P.n, P.k, P.codes.clone(), P.scales.clone(), P.books.clone(), P.codebooks.clone())
@@ -823,6 +951,7 @@ def run_select(qx, torch, dev, stream):
     cands = [qx.Recipe(3, 64, qx.UNIFORM), qx.Recipe(3, 128, qx.LUT), qx.Recipe(4, 64, qx.UNIFORM),
              qx.Recipe(4, 128, qx.UNIFORM)]
     with torch.cuda.stream(stream):
+        stream.wait_stream(torch.cuda.default_stream(dev))  # W is drawn on the default stream
         qx.select_recipe(W, cands)  # warm-up
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         e0.record(stream)
@@ -843,6 +972,9 @@ def run_select(qx, torch, dev, stream):
         best5, errs5, bpws5 = qx.select_recipe(W, cands5)
         e1.record(stream)
     torch.cuda.synchronize()
+    st_code = qx.device_status(stream)
+    if st_code != 0:
+        raise RuntimeError(f"recipe selection reported device status {st_code}")
     names5 = names + ["Q4Xg64"]
     out["with_q4x"] = {"ms": e0.elapsed_time(e1), "chosen": names5[best5] if best5 is not None else None,
                        "rel_frobenius_error": math.sqrt(errs5[4] / float(1 << 48)) / norm, "bpw": bpws5[4]}

@@ -105,7 +105,11 @@ typedef struct qx_packed {
     void *luts;
 } qx_packed;
 
-/* Host only: byte sizes of the packed buffers of an n x k matrix.
+/* Host only: byte sizes of the packed buffers of an n x k matrix, from the
+ * packed layout above (the paper gives none: Section 2.4 names the packing
+ * kernels and the data-mover bus widths that shape it; this library's reading
+ * of them is the layout in the header comment).  The bits per weight of
+ * Tables 1-2 are 8 x (these sizes summed) / (n k).
  * Errors: INVALID_ARG (NULL, n < 1, k < 1), UNSUPPORTED (recipe not built or
  * k not a multiple of 128 and of g). */
 qx_status qx_packed_size(int64_t n, int64_t k, const qx_recipe *recipe, qx_sizes *out);
@@ -423,12 +427,14 @@ qx_status qx_q4x_gemm_splitk(const qx_q4x *p, const void *X, int64_t m, void *Y,
  * the context usable; qx_get_device_status() then returns QX_ERR_TIMEOUT. */
 qx_status qx_selftest_wait_timeout(int32_t limit_us, void *stream);
 
-/* Synchronize `stream`, then return and clear the current device's status word
- * (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns QX_ERR_CUDA if the
- * synchronization itself fails. */
+/* Library infrastructure, no passage of the paper (which describes no error
+ * handling): synchronize `stream`, then return and clear the current device's
+ * status word (QX_OK, QX_ERR_NONFINITE or QX_ERR_TIMEOUT).  Returns
+ * QX_ERR_CUDA if the synchronization itself fails. */
 qx_status qx_get_device_status(void *stream);
 
-/* Static, NUL-terminated description of a status code. */
+/* Library infrastructure, no passage of the paper: a static, NUL-terminated
+ * description of a status code. */
 const char *qx_status_string(qx_status s);
 
 /* Name of the last CUDA error an entry point of this thread turned into

@@ -353,6 +353,18 @@ __device__ __forceinline__ int phase_stages(const GemvMulti &a, int p) {
     return q;
 }
 
+// Pull the activations of phase p into L2 (lane i: matrix i of the phase).
+// L2 is the point of coherence, so this is safe even when an earlier phase of
+// the launch still writes them.
+__device__ __forceinline__ void prefetch_x(const GemvMulti &a, int p, int lane) {
+    if (p >= a.nphase) return;
+    const int m = a.phase_first[p] + lane;
+    if (m >= a.phase_first[p + 1]) return;
+    const GemvMat &M = a.mat[m];
+    const uint32_t bytes = (uint32_t)(a.batch * M.k * 2) & ~15u;
+    if (bytes) prefetch_l2_bulk(M.x, bytes);
+}
+
 __device__ __forceinline__ int round_groups(int q) { return (q + kGroups - 1) / kGroups * kGroups; }
 
 // Grid-scope counter of a fused launch: a release increment (everything the
@@ -552,6 +564,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_codes[lane]) : "memory");
             if (KIND == 1) asm volatile("prefetch.tensormap [%0];" ::"l"(&a.tm_luts[lane]) : "memory");
         }
+        prefetch_x(a, 0, lane);
     } else if (warp == 0) {
         if (lane < count) {  // matrix `lane`: this CTA's row blocks and stage numbering
             const int t = lane;
@@ -612,10 +625,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         // stages are padded to a multiple of kGroups with empty stages (a full
         // barrier phase with no bytes), so that every phase starts on group 0
         // as a launch of its own does
-        if (lane == 0) {
-            bool okp = true;
-            int q = 0;
-            for (int p = 0; p < a.nphase && okp; ++p) {
+        bool okp = true;
+        int q = 0;
+        for (int p = 0; p < a.nphase && okp; ++p) {
+            prefetch_x(a, p + 1, lane);  // the next phase's activations, while this one streams
+            if (lane == 0) {
                 const int qend = h.ph_q0[p + 1];
                 int m = a.phase_first[p], rbl = 0, ks = 0;
                 while (m < a.phase_first[p + 1] && h.mats[m].nrb == 0) ++m;
@@ -641,6 +655,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     }
                 }
             }
+            okp = __shfl_sync(0xffffffffu, okp, 0);
+            q = __shfl_sync(0xffffffffu, q, 0);
+        }
+        if (lane == 0) {
             if (!okp) {
                 h.abort_flag = 1u;
                 atomicOr(a.status, kStatusTimeout);

@@ -608,3 +608,32 @@ def test_degenerate_groups_bit_exact(qx, bits, g, kind):
     y = qx.gemv(P, torch.from_numpy(x).cuda(), out_dtype=torch.float32).cpu().numpy()
     keep = [r for r in range(n) if r != 5]
     _check_matmul(y[:, keep], oracle.gemv(ref, rec, x, k)[:, keep], x, Wh[keep])
+
+
+# ---------------------------------------------------------------- heavy-tailed activations
+def _massive_activations(batch, k, seed):
+    """N(0, 1) activations with eight 'massive' channels of |x| 100..1000 (the
+    outlier channels of LLM residual streams), the same channels in every row."""
+    rng = np.random.default_rng(seed)
+    x = rng.standard_normal((batch, k))
+    ch = rng.choice(k, size=8, replace=False)
+    x[:, ch] = rng.choice([-1.0, 1.0], size=(batch, 8)) * rng.uniform(100.0, 1000.0, size=(batch, 8))
+    return x.astype(np.float16)
+
+
+@pytest.mark.parametrize("batch", [1, 2, 4, 16])
+@pytest.mark.parametrize("n,k,bits,g,kind", [(512, 4096, 3, 128, 1), (384, 11008, 4, 64, 0)])
+def test_gemv_heavy_tailed_activations(qx, n, k, bits, g, kind, batch):
+    """Batches of 1 and 2 form fp16 products and their sums over 8 weight pairs
+    on the CUDA cores before the fp32 sum; larger batches accumulate in fp32 on
+    the tensor cores.  With massive activation channels (and the weights' 10
+    sigma outliers) both stay within the tolerance."""
+    W = synth.student_t_weights(n, k, 0.04, seed=n, stream=k, outlier_frac=0.001)
+    rec = _orecipe(bits, g, kind)
+    ref = oracle.quantize(W, rec)
+    Wh = oracle.dequant(ref, rec, k)
+    P = qx.quantize(torch.from_numpy(W).cuda(), qx.Recipe(bits, g, kind))
+    x = _massive_activations(batch, k, seed=batch)
+    y = qx.gemv(P, torch.from_numpy(x).cuda(), out_dtype=torch.float32).cpu().numpy()
+    assert qx.device_status() == 0
+    _check_matmul(y, oracle.gemv(ref, rec, x, k), x, Wh)
