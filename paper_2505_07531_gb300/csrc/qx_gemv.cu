@@ -240,8 +240,7 @@ struct Header {
 };
 static_assert(sizeof(Header) <= kHeader, "header does not fit");
 
-// Geometry a stage copy needs, from the shared-memory table or straight from
-// the kernel parameters (the first copies are issued before the table exists).
+// Geometry a stage copy needs, from the shared-memory table.
 struct Geom {
     int K, log2g, nlb, G, n, zbytes;
     const __half *scales;
@@ -252,9 +251,6 @@ __device__ __forceinline__ Geom geom_of(const MatS &M) {
     return Geom{M.K, M.log2g, M.nlb, M.G, M.n, M.zbytes, M.scales, M.zeros};
 }
 
-__device__ __forceinline__ Geom geom_of(const GemvMat &M) {
-    return Geom{(int)M.k, M.log2g, M.nlb, M.G, (int)M.n, M.zbytes, M.scales, M.zeros};
-}
 
 // Issue the TMA copies of one stage (matrix m, matrix-local row block rb,
 // slice ks) into the ring slot at `base` with full barrier `bar` (one thread).
@@ -701,6 +697,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
 
     int slot = grp;
     uint32_t par = 0;
+    int blk_slot = 0;       // partial-sum slot of the CTA's next row block (blocks in CTA order)
+    uint32_t blk_use = 0;   // uses of that slot before it
     float *rp_base = red;
     for (int p = 0; p < a.nphase; ++p) {
         if (fused && p > 0) {
@@ -724,28 +722,35 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             const int nrb = M.nrb;
             if (nrb == 0) continue;
             const int K = M.K, nks = M.nks, n = M.n, log2g = M.log2g;
-            const int q0 = M.q0, rb0 = M.rb0, rbq0 = M.rbq0;
+            const int q0 = M.q0, rb0 = M.rb0;
             const __half *xm = M.x;
             // the lane's LUT chunk in a stage (LUT kind): its group within the slice
             uint32_t lo_off[2][2] = {{0u, 0u}, {0u, 0u}};
             if (KIND == 1) {
                 const int lg = kunit >> log2g;
-    #pragma unroll
+#pragma unroll
                 for (int rt = 0; rt < 2; ++rt) {
                     lo_off[rt][0] = (uint32_t)(3 * kBox + (lg >> 3) * kBox) + swz(16 * rt + g, lg & 7);
                     lo_off[rt][1] = (uint32_t)(3 * kBox + (lg >> 3) * kBox) + swz(16 * rt + g + 8, lg & 7);
                 }
             }
             // x fragments of the lane's 32 k of slice ks: rows g (and g + 8) of x
+            // the lane's rows of x at its unit of slice 0 (CUDA cores: every lane
+            // takes every row of x; tensor cores: row g of each n-tile)
+            const __half *xl[NX];
+#pragma unroll
+            for (int nt = 0; nt < NX; ++nt) {
+                const int b = Dot<NT>::kCores ? nt : g + 8 * nt;
+                xl[nt] = xm + (int64_t)min(b, nb - 1) * K + kunit;
+            }
             auto load_x = [&](int ks, uint32_t (&xv)[NX][16]) {
-                const int k0 = ks * kSliceK + kunit;
                 const bool in = ks * kSliceK + 128 * sb < K;
-    #pragma unroll
+#pragma unroll
                 for (int nt = 0; nt < NX; ++nt) {
-                    const int b = Dot<NT>::kCores ? nt : g + 8 * nt;  // CUDA cores: every lane takes every row of x
+                    const int b = Dot<NT>::kCores ? nt : g + 8 * nt;
                     if (in && b < nb) {
-                        const __half *xp = xm + (int64_t)b * K + k0;
-    #pragma unroll
+                        const __half *xp = xl[nt] + ks * kSliceK;
+#pragma unroll
                         for (int i = 0; i < 4; ++i) {
                             const uint4 v = ldg_x(xp + 8 * i, fused);
                             xv[nt][4 * i + 0] = v.x;
@@ -754,22 +759,29 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                             xv[nt][4 * i + 3] = v.w;
                         }
                     } else {
-    #pragma unroll
+#pragma unroll
                         for (int i = 0; i < 16; ++i) xv[nt][i] = 0u;
                     }
                 }
             };
             for (int rbl = 0; rbl < nrb && ok; ++rbl) {
+                // the block's partial-sum slot, and how often the slot was used before
+                const int rs = blk_slot;
+                const uint32_t use = blk_use;
+                if (++blk_slot == a.rb_slots) {
+                    blk_slot = 0;
+                    ++blk_use;
+                }
                 const int qb = q0 + rbl * nks;  // the block's first stage
                 const int ks0 = (grp - qb % kGroups + kGroups) % kGroups;
                 if (ks0 >= nks) continue;  // this group has no stage of the block
                 const int row0 = (rb0 + rbl) * kRows + g;  // the lane's first row (of g, g + 8, g + 16, g + 24)
                 float acc[2][NX][4];
-    #pragma unroll
+#pragma unroll
                 for (int rt = 0; rt < 2; ++rt)
-    #pragma unroll
+#pragma unroll
                     for (int nt = 0; nt < NX; ++nt)
-    #pragma unroll
+#pragma unroll
                         for (int i = 0; i < 4; ++i) acc[rt][nt][i] = 0.0f;
                 Meta cur{};
                 if (KIND == 0) cur = load_meta(M, row0, ks0 * kSliceK + kunit);
@@ -786,7 +798,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     }
                     if (live) {
                         const uint32_t sbase = ring_s + (uint32_t)(slot * a.stage_bytes);
-    #pragma unroll
+#pragma unroll
                         for (int rt = 0; rt < 2; ++rt) {
                             if (BITS == 3) {
                                 uint32_t A0, A1, B0, B1, C0, C1;
@@ -826,9 +838,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 if (!ok) break;
                 // ---- partials of this block -> shared memory; the last contributor
                 // sums them in a fixed order and writes y
-                const int rbi = rbq0 + rbl;
-                const int rs = rbi % a.rb_slots;
-                const uint32_t use = (uint32_t)(rbi / a.rb_slots);
                 // the warp groups run independently: the slot's previous block must
                 // have been summed before this warp overwrites its partials
                 bool okf = true;
@@ -844,11 +853,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 if (Dot<NT>::kCores) {
                     // CUDA cores: sum the four lanes of a row (units t = 0..3), then lane t
                     // stores row of x t
-    #pragma unroll
+#pragma unroll
                     for (int rt = 0; rt < 2; ++rt)
-    #pragma unroll
+#pragma unroll
                         for (int b = 0; b < NX; ++b)
-    #pragma unroll
+#pragma unroll
                             for (int r = 0; r < 2; ++r) {
                                 float v = acc[rt][b][r];
                                 v += __shfl_xor_sync(0xffffffffu, v, 1);
@@ -856,9 +865,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                                 if (t == b && b < nb) mine[(16 * rt + g + 8 * r) * nbs + b] = v;
                             }
                 } else {
-    #pragma unroll
+#pragma unroll
                     for (int rt = 0; rt < 2; ++rt)
-    #pragma unroll
+#pragma unroll
                         for (int nt = 0; nt < NX; ++nt) {
                             const int col = 8 * nt + 2 * t;
                             const int r0 = 16 * rt + g;
@@ -884,19 +893,19 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     // stage order, then superblock warp
                     constexpr int VMAX = Dot<NT>::kCores ? 2 : 8 * NX;
                     float v[VMAX];
-    #pragma unroll
+#pragma unroll
                     for (int b = 0; b < VMAX; ++b) v[b] = 0.0f;
                     for (int j = 0; j < ng; ++j) {
                         const float *src = rp + (size_t)((qb + j) % kGroups * kWarps) * (kRows * nbs) + lane * nbs;
-    #pragma unroll
+#pragma unroll
                         for (int w = 0; w < kWarps; ++w) {
                             const float *sw = src + (size_t)w * (kRows * nbs);
                             if (Dot<NT>::kCores) {
-    #pragma unroll
+#pragma unroll
                                 for (int b = 0; b < VMAX; ++b)
                                     if (b < nb) v[b] += sw[b];
                             } else {
-    #pragma unroll
+#pragma unroll
                                 for (int c4 = 0; c4 < VMAX / 4; ++c4) {
                                     if (4 * c4 < nb) {
                                         const float4 f = *reinterpret_cast<const float4 *>(sw + 4 * c4);
@@ -917,7 +926,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                         *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
                     }
                     if (row < n) {
-    #pragma unroll
+#pragma unroll
                         for (int b = 0; b < VMAX; ++b) {
                             if (b >= nb) break;
                             if (a.y_f32)
