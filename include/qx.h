@@ -188,7 +188,13 @@ typedef struct qx_copy {
  * in qx_gemv_chain, the nout copies `out` (device to host), then, when sync is
  * non-zero, a synchronization of the stream (the outputs are then in host
  * memory).  nin, nout 0..16.  Every group is validated before the first copy;
- * a failing argument returns its status and nothing is issued. */
+ * a failing argument returns its status and nothing is issued.
+ * When every host buffer is pinned and `stream` is not being captured, the
+ * first call with a given set of arguments captures the copies and launches
+ * as a CUDA graph (on a stream of the library's own) and every later call
+ * with the same arguments replays it: one launch per step.  The library keeps
+ * up to 16 such graphs, and the device memory they hold, until the process
+ * ends.  Otherwise the copies and launches are issued one by one. */
 qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
                          int32_t batch, int32_t y_dtype, int32_t flags, const qx_copy *out, int32_t nout,
                          int32_t sync, void *stream);

@@ -5,6 +5,7 @@
 #include <cstdlib>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include "qx.h"
 #include "qx_kernels.cuh"
@@ -412,6 +413,146 @@ QX_API qx_status qx_gemv_chain(const qx_gemv_group *groups, int32_t ngroups, int
     return run_chain(groups, ngroups, batch, y_dtype, flags, static_cast<cudaStream_t>(stream), d);
 }
 
+namespace {
+
+qx_status run_chain_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
+                          int32_t flags, void *ws, cudaStream_t st, DeviceInfo *d);
+
+// The copies and launches of one decode step, issued on `st` (ws non-null: the
+// groups as one fused launch).
+qx_status issue_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups, int32_t batch,
+                     int32_t y_dtype, int32_t flags, void *ws, const qx_copy *out, int32_t nout, cudaStream_t st,
+                     DeviceInfo *d) {
+    qx_status s = QX_OK;
+    for (int i = 0; i < nin; ++i)
+        if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
+            return s;
+    s = ws != nullptr ? run_chain_fused(groups, ngroups, batch, y_dtype, flags, ws, st, d)
+                      : run_chain(groups, ngroups, batch, y_dtype, flags, st, d);
+    if (s != QX_OK) return s;
+    for (int i = 0; i < nout; ++i)
+        if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
+            QX_OK)
+            return s;
+    return QX_OK;
+}
+
+// A model repeats the same decode step (same buffers, same shapes) every
+// token.  Its copies and launches are captured once as a CUDA graph and the
+// graph is replayed: one launch instead of a launch per group and a copy per
+// buffer, with the groups' programmatic dependencies kept as graph edges.
+// The graphs are kept by everything the step depends on, like the plans.
+struct StepGraph {
+    bool used = false;
+    int dev = -1;
+    std::vector<uint8_t> key;
+    cudaGraphExec_t exec = nullptr;
+};
+constexpr int kStepGraphs = 16;
+StepGraph g_steps[kStepGraphs];
+int g_step_next = 0;
+std::mutex g_step_mu;
+cudaStream_t g_capture[kMaxDevices] = {};
+
+void key_put(std::vector<uint8_t> &k, const void *p, size_t n) {
+    const uint8_t *b = static_cast<const uint8_t *>(p);
+    k.insert(k.end(), b, b + n);
+}
+
+std::vector<uint8_t> step_key(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
+                              int32_t batch, int32_t y_dtype, int32_t flags, const void *ws, const qx_copy *out,
+                              int32_t nout) {
+    std::vector<uint8_t> k;
+    const int32_t sc[6] = {nin, ngroups, batch, y_dtype, flags, nout};
+    key_put(k, sc, sizeof(sc));
+    key_put(k, &ws, sizeof(ws));
+    for (int i = 0; i < nin; ++i) key_put(k, &in[i], sizeof(qx_copy));
+    for (int i = 0; i < nout; ++i) key_put(k, &out[i], sizeof(qx_copy));
+    for (int gi = 0; gi < ngroups; ++gi) {
+        const qx_gemv_group &g = groups[gi];
+        key_put(k, &g.count, sizeof(g.count));
+        for (int i = 0; i < g.count; ++i) {
+            key_put(k, &g.mats[i], sizeof(qx_packed));
+            key_put(k, &g.x[i], sizeof(void *));
+            key_put(k, &g.y[i], sizeof(void *));
+        }
+    }
+    return k;
+}
+
+// Host memory the graph's copy nodes may take: pinned (page-locked) memory.
+bool copyable(const qx_copy *c, int32_t n, bool host_src) {
+    for (int i = 0; i < n; ++i) {
+        cudaPointerAttributes at;
+        if (cudaPointerGetAttributes(&at, host_src ? c[i].src : c[i].dst) != cudaSuccess) {
+            cudaGetLastError();
+            return false;
+        }
+        if (at.type != cudaMemoryTypeHost) return false;
+    }
+    return true;
+}
+
+qx_status run_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups, int32_t batch,
+                   int32_t y_dtype, int32_t flags, void *ws, const qx_copy *out, int32_t nout, int32_t sync,
+                   cudaStream_t st, DeviceInfo *d) {
+    int dev = -1;
+    qx_status s = from_cuda(cudaGetDevice(&dev));
+    if (s != QX_OK) return s;
+    cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+    bool direct = cudaStreamIsCapturing(st, &cs) != cudaSuccess || cs != cudaStreamCaptureStatusNone ||
+                  dev < 0 || dev >= kMaxDevices;
+    cudaGetLastError();
+    cudaGraphExec_t exec = nullptr;
+    if (!direct) {
+        const std::vector<uint8_t> key = step_key(in, nin, groups, ngroups, batch, y_dtype, flags, ws, out, nout);
+        std::lock_guard<std::mutex> lock(g_step_mu);
+        for (int i = 0; i < kStepGraphs && exec == nullptr; ++i)
+            if (g_steps[i].used && g_steps[i].dev == dev && g_steps[i].key == key) exec = g_steps[i].exec;
+        if (exec == nullptr && copyable(in, nin, true) && copyable(out, nout, false)) {
+            // capture on a stream of the library's own, then keep the instantiated graph
+            if (g_capture[dev] == nullptr &&
+                cudaStreamCreateWithFlags(&g_capture[dev], cudaStreamNonBlocking) != cudaSuccess) {
+                cudaGetLastError();
+                g_capture[dev] = nullptr;
+            }
+            cudaGraph_t graph = nullptr;
+            if (g_capture[dev] != nullptr &&
+                cudaStreamBeginCapture(g_capture[dev], cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
+                const qx_status si =
+                    issue_step(in, nin, groups, ngroups, batch, y_dtype, flags, ws, out, nout, g_capture[dev], d);
+                const cudaError_t ee = cudaStreamEndCapture(g_capture[dev], &graph);
+                if (si == QX_OK && ee == cudaSuccess && graph != nullptr &&
+                    cudaGraphInstantiate(&exec, graph, 0) != cudaSuccess)
+                    exec = nullptr;
+                if (graph != nullptr) cudaGraphDestroy(graph);
+                if (si != QX_OK || ee != cudaSuccess) exec = nullptr;
+            }
+            cudaGetLastError();
+            if (exec != nullptr) {
+                StepGraph &e = g_steps[g_step_next];
+                g_step_next = (g_step_next + 1) % kStepGraphs;
+                if (e.used && e.exec != nullptr) {
+                    cudaDeviceSynchronize();  // the evicted graph may still run
+                    cudaGraphExecDestroy(e.exec);
+                }
+                e.used = true;
+                e.dev = dev;
+                e.key = key;
+                e.exec = exec;
+            }
+        }
+    }
+    if (exec != nullptr) {
+        if ((s = from_cuda(cudaGraphLaunch(exec, st))) != QX_OK) return s;
+    } else if ((s = issue_step(in, nin, groups, ngroups, batch, y_dtype, flags, ws, out, nout, st, d)) != QX_OK) {
+        return s;
+    }
+    return sync ? from_cuda(cudaStreamSynchronize(st)) : QX_OK;
+}
+
+}  // namespace
+
 QX_API qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups,
                                 int32_t batch, int32_t y_dtype, int32_t flags, const qx_copy *out, int32_t nout,
                                 int32_t sync, void *stream) {
@@ -421,16 +562,8 @@ QX_API qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_gr
     if (s != QX_OK) return s;
     DeviceInfo *d = nullptr;
     if ((s = device_info(&d)) != QX_OK) return s;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    for (int i = 0; i < nin; ++i)
-        if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
-            return s;
-    if ((s = run_chain(groups, ngroups, batch, y_dtype, flags, st, d)) != QX_OK) return s;
-    for (int i = 0; i < nout; ++i)
-        if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
-            QX_OK)
-            return s;
-    return sync ? from_cuda(cudaStreamSynchronize(st)) : QX_OK;
+    return run_step(in, nin, groups, ngroups, batch, y_dtype, flags, nullptr, out, nout, sync,
+                    static_cast<cudaStream_t>(stream), d);
 }
 
 namespace {
@@ -522,16 +655,8 @@ QX_API qx_status qx_decode_step_fused(const qx_copy *in, int32_t nin, const qx_g
     if (s != QX_OK) return s;
     DeviceInfo *d = nullptr;
     if ((s = device_info(&d)) != QX_OK) return s;
-    cudaStream_t st = static_cast<cudaStream_t>(stream);
-    for (int i = 0; i < nin; ++i)
-        if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
-            return s;
-    if ((s = run_chain_fused(groups, ngroups, batch, y_dtype, flags, workspace, st, d)) != QX_OK) return s;
-    for (int i = 0; i < nout; ++i)
-        if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
-            QX_OK)
-            return s;
-    return sync ? from_cuda(cudaStreamSynchronize(st)) : QX_OK;
+    return run_step(in, nin, groups, ngroups, batch, y_dtype, flags, workspace, out, nout, sync,
+                    static_cast<cudaStream_t>(stream), d);
 }
 
 namespace {

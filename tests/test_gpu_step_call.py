@@ -49,10 +49,32 @@ def test_decode_step_copies_in_and_out(qx, fused):
     dys = [torch.empty((2, P.n), dtype=torch.float16, device="cuda") for P in mats]
     hys = [torch.full((2, P.n), float("nan"), dtype=torch.float16).pin_memory() for P in mats]
     step = qx.DecodeStep([(mats, [dx, dx], dys)], h2d=[(dx, hx)], d2h=list(zip(hys, dys)), fused=fused)
-    step()
-    ref = qx.gemv_multi(mats, [hx.cuda(), hx.cuda()])
-    for h, r in zip(hys, ref):
-        assert torch.equal(h, r.cpu())
+    # the step is captured as a graph on its first call and replayed after: every
+    # call copies the host buffers' current contents in and the results out
+    for seed in (3, 4, 5):
+        hx.copy_(torch.from_numpy(synth.activations(2, 512, seed=seed, stream=3)))
+        for h in hys:
+            h.fill_(float("nan"))
+        step()
+        ref = qx.gemv_multi(mats, [hx.cuda(), hx.cuda()])
+        for h, r in zip(hys, ref):
+            assert torch.equal(h, r.cpu()), seed
+    assert qx.device_status() == 0
+
+
+def test_decode_step_with_pageable_host_memory(qx):
+    """Host buffers that are not pinned: the step is issued call by call (a
+    graph's copy nodes take pinned memory), with the same results."""
+    rec = qx.Recipe(3, 128, qx.LUT)
+    P = qx.quantize(torch.from_numpy(synth.student_t_weights(256, 512, 0.02, seed=1, stream=2)).cuda(), rec)
+    hx = torch.from_numpy(synth.activations(1, 512, seed=6, stream=3))
+    dx = torch.empty(hx.shape, dtype=hx.dtype, device="cuda")
+    dy = torch.empty((1, 256), dtype=torch.float16, device="cuda")
+    hy = torch.full((1, 256), float("nan"), dtype=torch.float16)
+    step = qx.DecodeStep([([P], [dx], [dy])], h2d=[(dx, hx)], d2h=[(hy, dy)])
+    for _ in range(2):
+        step()
+        assert torch.equal(hy, qx.gemv(P, hx.cuda()).cpu())
     assert qx.device_status() == 0
 
 
