@@ -27,13 +27,15 @@
 //     slot's group have released its previous fill (an mbarrier every lane
 //     arrives at); waits suspend in hardware rather than spin.
 //   * Partial sums of a row block stay in registers across its stages; at the
-//     end of the block each warp stores its partials and the last contributor
-//     adds them in a fixed order (deterministic) and writes y.
+//     end of the block each warp stores its partials in a shared-memory slot
+//     and arrives on the slot's barrier without waiting for anything.  A
+//     reducer warp adds them in a fixed order (deterministic), writes y and
+//     frees the slot, off the decoding warps' path.
 //   * x is read from global memory (L1/L2): no per-launch staging.
 //   * One launch may run several groups of matrices one after another
 //     (qx_gemv_fused): the producer streams the weights of every group without
-//     a break, and the consumers of group p + 1 read x only once every CTA has
-//     counted group p done in a device-side counter.
+//     a break, and the consumers of group p + 1 read x only once every CTA's
+//     reducer has counted group p done in a device-side counter.
 // Every wait is bounded in time and reports QX_ERR_TIMEOUT through the device
 // status.
 #include "qx_kernels.cuh"
@@ -45,7 +47,8 @@ namespace {
 constexpr int kWarps = 8;        // warps per group: warp w decodes superblock w of a stage
 constexpr int kGroups = 2;       // group g takes the stages q with q % kGroups == g
 constexpr int kProducer = kWarps * kGroups;  // the warp after the consumers issues the copies
-constexpr int kThreads = 32 * (kWarps * kGroups + 1);
+constexpr int kReducer = kProducer + 1;      // the last warp sums each block's partials and writes y
+constexpr int kThreads = 32 * (kWarps * kGroups + 2);
 constexpr int kRows = 32;        // rows per block: two 16-row MMA tiles
 constexpr int kSliceK = 1024;    // weights per row per stage: eight 128-weight superblocks
 constexpr int kBox = kRows * 128;  // one 32-row x 128-byte TMA box
@@ -109,36 +112,6 @@ __device__ __noinline__ bool mbar_wait(uint32_t b, uint32_t parity, uint64_t lim
         if (abort_flag != nullptr && *abort_flag) return false;
         if (globaltimer_ns() - t0 > limit_ns) return false;
     }
-}
-
-// Bounded wait for a shared-memory word to reach `want` (backing off between
-// reads, so that the waiting warp leaves the scheduler to the others).
-__device__ __noinline__ bool wait_equal(uint32_t *p, uint32_t want, uint64_t limit_ns,
-                                        volatile uint32_t *abort_flag) {
-    volatile uint32_t *v = p;
-    if (*v == want) return true;
-    const uint64_t t0 = globaltimer_ns();
-    for (;;) {
-        __nanosleep(64);
-        if (*v == want) {
-            __threadfence_block();
-            return true;
-        }
-        if (*abort_flag) return false;
-        if (globaltimer_ns() - t0 > limit_ns) return false;
-    }
-}
-
-// Shared-memory counter increment with acquire-release ordering at CTA scope:
-// the caller's earlier shared stores are visible to whoever sees the new count,
-// and the caller sees the stores of those that counted before it.
-__device__ __forceinline__ uint32_t atom_add_acq_rel(uint32_t *p, uint32_t v) {
-    uint32_t old;
-    asm volatile("atom.acq_rel.cta.shared::cta.add.u32 %0, [%1], %2;"
-                 : "=r"(old)
-                 : "r"(static_cast<uint32_t>(__cvta_generic_to_shared(p))), "r"(v)
-                 : "memory");
-    return old;
 }
 
 __device__ __forceinline__ void tma_2d(uint32_t dst, const CUtensorMap *map, uint32_t bar, int x, int y) {
@@ -231,8 +204,8 @@ struct MatS {
 struct Header {
     uint64_t full[kMaxRing];       // a stage's copies have landed
     uint64_t empty[kMaxRing];      // the eight warps of its group are done with it
-    uint32_t cnt[kMaxRbSlots];     // warps that stored their partials of a block
-    uint32_t gen[kMaxRbSlots];     // blocks finished in each partial-sum slot
+    uint64_t rfull[kMaxRbSlots];   // every consumer lane has stored its partials of the slot's block
+    uint64_t rempty[kMaxRbSlots];  // the reducer has summed the slot's block
     uint32_t abort_flag;
     int ph_q0[kMaxGemvPhases + 1];  // first CTA-local stage of each phase (multiples of kGroups)
     int ph_nst[kMaxGemvPhases];     // stages of each phase in this CTA (before the padding)
@@ -553,6 +526,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 mbar_init(smem_u32(&h.full[i]), 1);
                 mbar_init(smem_u32(&h.empty[i]), 32 * kWarps);
             }
+            for (int i = 0; i < a.rb_slots; ++i) {
+                mbar_init(smem_u32(&h.rfull[i]), 32 * kWarps * kGroups);
+                mbar_init(smem_u32(&h.rempty[i]), 32);
+            }
             h.abort_flag = 0;
             asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         }
@@ -599,10 +576,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             S.rbq0 = rbq;
         }
     } else if (warp == 1) {
-        if (lane < kMaxRbSlots) {
-            h.cnt[lane] = 0;
-            h.gen[lane] = 0;
-        }
         if (lane == 0) {
             int q = 0;
             for (int p = 0; p < a.nphase; ++p) {
@@ -666,13 +639,105 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         return;
     }
 
-    // ---- consumers: x is read, and y written, only after the previous kernel
-    // in the stream has finished
+    // x is read, and y written, only after the previous kernel in the stream
+    // has finished
     asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int nbs = partial_stride(nb, Dot<NT>::kCores);  // row stride (floats) of the partial sums
+
+    if (warp == kReducer) {
+        // ---- reducer: the CTA's row blocks in order; lane i sums row i of a
+        // block over the warps that worked on it, in a fixed order (group by the
+        // block's stage order, then superblock warp), and writes y.  In a fused
+        // launch it counts the CTA done with a phase once every y of the phase
+        // is written.
+        bool okr = true;
+        int rs = 0;
+        uint32_t use = 0;
+        for (int p = 0; p < a.nphase && okr; ++p) {
+            for (int m = a.phase_first[p]; m < a.phase_first[p + 1] && okr; ++m) {
+                const MatS &M = h.mats[m];
+                const int nks = M.nks, n = M.n;
+                const int ng = min(nks, kGroups);  // groups that worked on a block
+                for (int rbl = 0; rbl < M.nrb; ++rbl) {
+                    const uint32_t fb = smem_u32(&h.rfull[rs]);
+                    if (!mbar_try_wait(fb, use & 1u) && !mbar_wait(fb, use & 1u, a.wait_limit_ns, &h.abort_flag)) {
+                        okr = false;
+                        break;
+                    }
+                    const float *rp = red + (size_t)rs * (kGroups * kWarps * kRows * nbs);
+                    const int qb = M.q0 + rbl * nks;
+                    constexpr int VMAX = Dot<NT>::kCores ? 2 : 8 * NX;
+                    float v[VMAX];
+#pragma unroll
+                    for (int b = 0; b < VMAX; ++b) v[b] = 0.0f;
+                    for (int j = 0; j < ng; ++j) {
+                        const float *src = rp + (size_t)((qb + j) % kGroups * kWarps) * (kRows * nbs) + lane * nbs;
+#pragma unroll
+                        for (int w = 0; w < kWarps; ++w) {
+                            const float *sw = src + (size_t)w * (kRows * nbs);
+                            if (Dot<NT>::kCores) {
+#pragma unroll
+                                for (int b = 0; b < VMAX; ++b)
+                                    if (b < nb) v[b] += sw[b];
+                            } else {
+#pragma unroll
+                                for (int c4 = 0; c4 < VMAX / 4; ++c4) {
+                                    if (4 * c4 < nb) {
+                                        const float4 f = *reinterpret_cast<const float4 *>(sw + 4 * c4);
+                                        v[4 * c4] += f.x;
+                                        v[4 * c4 + 1] += f.y;
+                                        v[4 * c4 + 2] += f.z;
+                                        v[4 * c4 + 3] += f.w;
+                                    }
+                                }
+                            }
+                        }
+                    }
+                    // the slot is free once every lane has read it
+                    mbar_arrive(smem_u32(&h.rempty[rs]));
+                    const int row = (M.rb0 + rbl) * kRows + lane;
+                    if (row < n) {
+#pragma unroll
+                        for (int b = 0; b < VMAX; ++b) {
+                            if (b >= nb) break;
+                            if (a.y_f32)
+                                reinterpret_cast<float *>(M.y)[(int64_t)b * n + row] = v[b];
+                            else
+                                reinterpret_cast<__half *>(M.y)[(int64_t)b * n + row] = __float2half_rn(v[b]);
+                        }
+                    }
+                    if (++rs == a.rb_slots) {
+                        rs = 0;
+                        ++use;
+                    }
+                }
+            }
+            if (fused && okr) {
+                // every y of phase p written by this CTA is visible at gpu scope
+                // before the CTA is counted in
+                __threadfence();
+                __syncwarp();
+                if (lane == 0) {
+                    const uint32_t old = atom_add_release_gpu(a.phase_ctr + p, 1u);
+                    if (p == a.nphase - 1 && old == gridDim.x - 1) {
+                        // the last CTA of the launch: every other CTA has passed
+                        // every wait, so the counters go back to zero for the next launch
+                        for (int i = 0; i < a.nphase; ++i) a.phase_ctr[i] = 0u;
+                    }
+                }
+            }
+        }
+        if (!okr && lane == 0) {
+            h.abort_flag = 1u;
+            atomicOr(a.status, kStatusTimeout);
+        }
+        return;
+    }
+
+    // ---- consumers
     const int grp = warp / kWarps;   // stages q with q % kGroups == grp
     const int sb = warp % kWarps;    // superblock of each of those stages
     const int g = lane >> 2, t = lane & 3;
-    const int nbs = partial_stride(nb, Dot<NT>::kCores);  // row stride (floats) of the partial sums
     const int kunit = 128 * sb + 32 * t;  // the lane's 32-weight unit within a slice
     bool ok = true;
 
@@ -774,7 +839,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 }
                 const int qb = q0 + rbl * nks;  // the block's first stage
                 const int ks0 = (grp - qb % kGroups + kGroups) % kGroups;
-                if (ks0 >= nks) continue;  // this group has no stage of the block
+                // ks0 >= nks: this group has no stage of the block (it still hands
+                // the block on below)
                 const int row0 = (rb0 + rbl) * kRows + g;  // the lane's first row (of g, g + 8, g + 16, g + 24)
                 float acc[2][NX][4];
 #pragma unroll
@@ -836,106 +902,55 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     }
                 }
                 if (!ok) break;
-                // ---- partials of this block -> shared memory; the last contributor
-                // sums them in a fixed order and writes y
-                // the warp groups run independently: the slot's previous block must
-                // have been summed before this warp overwrites its partials
-                bool okf = true;
-                if (lane == 0 && *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) != use)
-                    okf = wait_equal(&h.gen[rs], use, a.wait_limit_ns, &h.abort_flag);
-                if (!__shfl_sync(0xffffffffu, okf, 0)) {
-                    ok = false;
-                    break;
+                // ---- partials of this block -> shared memory, then to the
+                // reducer warp; the slot's previous block must have been summed
+                // before its partials are overwritten (every consumer lane
+                // arrives for every block, with or without a stage of it)
+                if (use > 0) {
+                    const uint32_t eb = smem_u32(&h.rempty[rs]);
+                    const uint32_t ep = (use - 1u) & 1u;
+                    if (!mbar_try_wait(eb, ep) && !mbar_wait(eb, ep, a.wait_limit_ns, &h.abort_flag)) {
+                        ok = false;
+                        break;
+                    }
                 }
-                // slot layout: [group][superblock warp][32 rows][nbs]
-                float *rp = rp_base + (size_t)rs * (kGroups * kWarps * kRows * nbs);
-                float *mine = rp + (size_t)(grp * kWarps + sb) * (kRows * nbs);
-                if (Dot<NT>::kCores) {
-                    // CUDA cores: sum the four lanes of a row (units t = 0..3), then lane t
-                    // stores row of x t
+                if (ks0 < nks) {
+                    // slot layout: [group][superblock warp][32 rows][nbs]
+                    float *mine = rp_base + (size_t)rs * (kGroups * kWarps * kRows * nbs) +
+                                  (size_t)(grp * kWarps + sb) * (kRows * nbs);
+                    if (Dot<NT>::kCores) {
+                        // CUDA cores: sum the four lanes of a row (units t = 0..3), then lane t
+                        // stores row of x t
 #pragma unroll
-                    for (int rt = 0; rt < 2; ++rt)
+                        for (int rt = 0; rt < 2; ++rt)
 #pragma unroll
-                        for (int b = 0; b < NX; ++b)
+                            for (int b = 0; b < NX; ++b)
 #pragma unroll
-                            for (int r = 0; r < 2; ++r) {
-                                float v = acc[rt][b][r];
-                                v += __shfl_xor_sync(0xffffffffu, v, 1);
-                                v += __shfl_xor_sync(0xffffffffu, v, 2);
-                                if (t == b && b < nb) mine[(16 * rt + g + 8 * r) * nbs + b] = v;
-                            }
-                } else {
+                                for (int r = 0; r < 2; ++r) {
+                                    float v = acc[rt][b][r];
+                                    v += __shfl_xor_sync(0xffffffffu, v, 1);
+                                    v += __shfl_xor_sync(0xffffffffu, v, 2);
+                                    if (t == b && b < nb) mine[(16 * rt + g + 8 * r) * nbs + b] = v;
+                                }
+                    } else {
 #pragma unroll
-                    for (int rt = 0; rt < 2; ++rt)
+                        for (int rt = 0; rt < 2; ++rt)
 #pragma unroll
-                        for (int nt = 0; nt < NX; ++nt) {
-                            const int col = 8 * nt + 2 * t;
-                            const int r0 = 16 * rt + g;
-                            if (col < nb) {
-                                mine[r0 * nbs + col] = acc[rt][nt][0];
-                                mine[(r0 + 8) * nbs + col] = acc[rt][nt][2];
-                            }
-                            if (col + 1 < nb) {
-                                mine[r0 * nbs + col + 1] = acc[rt][nt][1];
-                                mine[(r0 + 8) * nbs + col + 1] = acc[rt][nt][3];
-                            }
-                        }
-                }
-                __syncwarp();
-                const int ng = min(nks, kGroups);  // groups that worked on this block
-                uint32_t fin = 0;
-                if (lane == 0) fin = atom_add_acq_rel(&h.cnt[rs], 1u) + 1u == (uint32_t)(ng * kWarps);
-                fin = __shfl_sync(0xffffffffu, fin, 0);
-                if (fin) {
-                    __syncwarp();  // lane 0's acquire orders the whole warp's reads below
-                    const int row = (rb0 + rbl) * kRows + lane;
-                    // the block's partials in a fixed order: group by the block's
-                    // stage order, then superblock warp
-                    constexpr int VMAX = Dot<NT>::kCores ? 2 : 8 * NX;
-                    float v[VMAX];
-#pragma unroll
-                    for (int b = 0; b < VMAX; ++b) v[b] = 0.0f;
-                    for (int j = 0; j < ng; ++j) {
-                        const float *src = rp + (size_t)((qb + j) % kGroups * kWarps) * (kRows * nbs) + lane * nbs;
-#pragma unroll
-                        for (int w = 0; w < kWarps; ++w) {
-                            const float *sw = src + (size_t)w * (kRows * nbs);
-                            if (Dot<NT>::kCores) {
-#pragma unroll
-                                for (int b = 0; b < VMAX; ++b)
-                                    if (b < nb) v[b] += sw[b];
-                            } else {
-#pragma unroll
-                                for (int c4 = 0; c4 < VMAX / 4; ++c4) {
-                                    if (4 * c4 < nb) {
-                                        const float4 f = *reinterpret_cast<const float4 *>(sw + 4 * c4);
-                                        v[4 * c4] += f.x;
-                                        v[4 * c4 + 1] += f.y;
-                                        v[4 * c4 + 2] += f.z;
-                                        v[4 * c4 + 3] += f.w;
-                                    }
+                            for (int nt = 0; nt < NX; ++nt) {
+                                const int col = 8 * nt + 2 * t;
+                                const int r0 = 16 * rt + g;
+                                if (col < nb) {
+                                    mine[r0 * nbs + col] = acc[rt][nt][0];
+                                    mine[(r0 + 8) * nbs + col] = acc[rt][nt][2];
+                                }
+                                if (col + 1 < nb) {
+                                    mine[r0 * nbs + col + 1] = acc[rt][nt][1];
+                                    mine[(r0 + 8) * nbs + col + 1] = acc[rt][nt][3];
                                 }
                             }
-                        }
-                    }
-                    // free the slot first: the fence must not wait for the y stores
-                    __syncwarp();
-                    if (lane == 0) {
-                        h.cnt[rs] = 0;
-                        __threadfence_block();
-                        *reinterpret_cast<volatile uint32_t *>(&h.gen[rs]) = use + 1u;
-                    }
-                    if (row < n) {
-#pragma unroll
-                        for (int b = 0; b < VMAX; ++b) {
-                            if (b >= nb) break;
-                            if (a.y_f32)
-                                reinterpret_cast<float *>(M.y)[(int64_t)b * n + row] = v[b];
-                            else
-                                reinterpret_cast<__half *>(M.y)[(int64_t)b * n + row] = __float2half_rn(v[b]);
-                        }
                     }
                 }
+                mbar_arrive(smem_u32(&h.rfull[rs]));
             }
         }
         // the padding stages of this phase that belong to this group
@@ -951,19 +966,6 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             if (slot >= ring) {
                 slot -= ring;
                 par ^= 1u;
-            }
-        }
-        if (fused) {
-            // every consumer warp of this CTA is done with phase p (partials
-            // summed, y written): count the CTA in
-            consumers_sync();
-            if (threadIdx.x == 0) {
-                const uint32_t old = atom_add_release_gpu(a.phase_ctr + p, 1u);
-                if (p == a.nphase - 1 && old == gridDim.x - 1) {
-                    // the last CTA of the launch: every other CTA has passed
-                    // every wait, so the counters go back to zero for the next launch
-                    for (int i = 0; i < a.nphase; ++i) a.phase_ctr[i] = 0u;
-                }
             }
         }
     }
