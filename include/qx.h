@@ -144,7 +144,12 @@ enum {
      * stream this call's weights, while the previous kernel in the stream is
      * still running; it waits for that kernel before reading x or writing y.
      * Set it only when the previous kernel does not write this call's weights. */
-    QX_GEMV_PDL = 1
+    QX_GEMV_PDL = 1,
+    /* qx_gemv_fused and qx_decode_step_fused only: launch each group on its
+     * own (one launch after another on the stream, with QX_GEMV_PDL as given)
+     * instead of all groups in one launch; each launch still balances its
+     * CTAs with the workspace. */
+    QX_GEMV_SEPARATE = 2
 };
 
 /* Several decode matmuls in one launch: y[i] = x[i] W_hat_i^T, i < count
@@ -200,7 +205,7 @@ qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_group *gr
                          int32_t sync, void *stream);
 
 /* Bytes of workspace qx_gemv_fused and qx_decode_step_fused need (host only;
- * a small constant). */
+ * a constant, about 1 MiB). */
 qx_status qx_gemv_fused_workspace(size_t *bytes);
 
 /* The groups of qx_gemv_chain (Section 2.4: decoding is memory-bound, so the
@@ -208,15 +213,22 @@ qx_status qx_gemv_fused_workspace(size_t *bytes);
  * persistent launch: one CTA per SM streams the weights of every group without
  * a break, and group i + 1 reads its x only once every CTA has finished group
  * i (its y written), so x of a later group may be the y of an earlier one.
- * The results equal qx_gemv_chain's bit for bit.  ngroups 1..64; the groups
- * run as one launch when there are at most 4 of them with at most 16 matrices
- * in all, sharing bits and kind (else as qx_gemv_chain runs them).
+ * ngroups 1..64; the groups run as one launch when there are at most 4 of them
+ * with at most 16 matrices in all, sharing bits and kind, and flags do not ask
+ * for QX_GEMV_SEPARATE (else one launch per group, one after another).
+ * Every launch splits its work between the CTAs at 1024-weight slices of a
+ * 32-row block rather than at whole blocks (qx_gemv_chain's unit), so that the
+ * CTAs finish together: the slices of a block split between CTAs are summed
+ * in fp32 per CTA and then in CTA order, so the results are deterministic and
+ * within fp32 rounding of qx_gemv_chain's, and equal bit for bit between the
+ * one-launch and the QX_GEMV_SEPARATE forms.
  * workspace: caller-owned device memory, 256-byte aligned, of at least
  * qx_gemv_fused_workspace() bytes, all zero before the first call: every
- * completed call leaves it zero (zero it again after QX_ERR_TIMEOUT).  Calls
- * that may run at the same time need separate workspaces.  flags: 0 or
- * QX_GEMV_PDL.  Errors: those of qx_gemv_chain; INVALID_ARG (workspace NULL
- * or too small), ALIGNMENT (workspace). */
+ * completed call leaves its counters zero (zero it again after
+ * QX_ERR_TIMEOUT).  Calls that may run at the same time need separate
+ * workspaces.  flags: 0, QX_GEMV_PDL, QX_GEMV_SEPARATE or both.  Errors: those
+ * of qx_gemv_chain; INVALID_ARG (workspace NULL or too small), ALIGNMENT
+ * (workspace). */
 qx_status qx_gemv_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
                         int32_t flags, void *workspace, size_t workspace_bytes, void *stream);
 

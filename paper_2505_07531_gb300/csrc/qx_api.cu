@@ -229,7 +229,7 @@ std::mutex g_plan_mu;
 bool same_inputs(const qx::GemvMulti &p, const qx::GemvMulti &a) {
     if (p.count != a.count || p.bits != a.bits || p.kind != a.kind || p.batch != a.batch || p.y_f32 != a.y_f32 ||
         p.status != a.status || p.wait_limit_ns != a.wait_limit_ns || p.nphase != a.nphase ||
-        p.phase_ctr != a.phase_ctr)
+        p.phase_ctr != a.phase_ctr || p.split_part != a.split_part || p.split_flag != a.split_flag)
         return false;
     for (int i = 0; i <= a.nphase; ++i)
         if (p.phase_first[i] != a.phase_first[i]) return false;
@@ -568,12 +568,19 @@ QX_API qx_status qx_decode_step(const qx_copy *in, int32_t nin, const qx_gemv_gr
 
 namespace {
 
-constexpr size_t kFusedWorkspaceBytes = 256;  // one phase counter per group, padded
+// Workspace of the fused calls: phase counters (one per group of a launch),
+// then the flags (one per CTA) and the fp32 partial sums (16 rows of x by 32
+// rows per CTA) of row blocks split between two CTAs.
+constexpr size_t kFusedFlagOffset = 256;
+constexpr size_t kFusedPartOffset = 2048;
+constexpr size_t kFusedWorkspaceBytes = kFusedPartOffset + (size_t)qx::kMaxGemvCtas * 16 * 32 * sizeof(float);
+static_assert(kFusedFlagOffset + qx::kMaxGemvCtas * sizeof(uint32_t) <= kFusedPartOffset, "workspace layout");
 
 // The groups of a decode step in one persistent launch (qx::GemvMulti with one
-// phase per group).  *launched is false, with nothing launched, when they
-// cannot share one: more groups or matrices than a launch holds, different
-// bits or kinds, or a plan that does not fit.
+// phase per group), its CTAs balanced stage by stage with the workspace.
+// *launched is false, with nothing launched, when they cannot share one: more
+// groups or matrices than a launch holds, different bits or kinds, or a plan
+// that does not fit.
 qx_status run_fused(const qx_gemv_group *groups, int ngroups, int batch, int y_dtype, int flags, void *ws,
                     cudaStream_t st, DeviceInfo *d, bool *launched) {
     *launched = false;
@@ -588,6 +595,8 @@ qx_status run_fused(const qx_gemv_group *groups, int ngroups, int batch, int y_d
     a.wait_limit_ns = wait_limit_ns();
     a.nphase = ngroups;
     a.phase_ctr = static_cast<uint32_t *>(ws);
+    a.split_flag = reinterpret_cast<uint32_t *>(static_cast<uint8_t *>(ws) + kFusedFlagOffset);
+    a.split_part = reinterpret_cast<float *>(static_cast<uint8_t *>(ws) + kFusedPartOffset);
     int count = 0;
     for (int gi = 0; gi < ngroups; ++gi) {
         const qx_gemv_group &g = groups[gi];
@@ -616,14 +625,24 @@ qx_status check_fused_ws(const void *ws, size_t bytes) {
     return QX_OK;
 }
 
+// All groups in one launch (unless QX_GEMV_SEPARATE), else group by group, each
+// launch balanced with the workspace; a group no balanced launch can take
+// runs as qx_gemv_multi runs it.
 qx_status run_chain_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
                           int32_t flags, void *ws, cudaStream_t st, DeviceInfo *d) {
-    if (ngroups > 1) {
+    const int lflags = flags & QX_GEMV_PDL;
+    if (ngroups > 1 && !(flags & QX_GEMV_SEPARATE)) {
         bool launched = false;
-        const qx_status s = run_fused(groups, ngroups, batch, y_dtype, flags, ws, st, d, &launched);
+        const qx_status s = run_fused(groups, ngroups, batch, y_dtype, lflags, ws, st, d, &launched);
         if (s != QX_OK || launched) return s;
     }
-    return run_chain(groups, ngroups, batch, y_dtype, flags, st, d);
+    for (int i = 0; i < ngroups; ++i) {
+        bool launched = false;
+        qx_status s = run_fused(groups + i, 1, batch, y_dtype, lflags, ws, st, d, &launched);
+        if (s == QX_OK && !launched) s = run_chain(groups + i, 1, batch, y_dtype, lflags, st, d);
+        if (s != QX_OK) return s;
+    }
+    return QX_OK;
 }
 
 }  // namespace
@@ -636,7 +655,7 @@ QX_API qx_status qx_gemv_fused_workspace(size_t *bytes) {
 
 QX_API qx_status qx_gemv_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t batch, int32_t y_dtype,
                                int32_t flags, void *workspace, size_t workspace_bytes, void *stream) {
-    qx_status s = check_chain(groups, ngroups, batch, y_dtype, flags);
+    qx_status s = check_chain(groups, ngroups, batch, y_dtype, flags & ~QX_GEMV_SEPARATE);
     if (s == QX_OK) s = check_fused_ws(workspace, workspace_bytes);
     if (s != QX_OK) return s;
     DeviceInfo *d = nullptr;
@@ -650,7 +669,7 @@ QX_API qx_status qx_decode_step_fused(const qx_copy *in, int32_t nin, const qx_g
                                       void *stream) {
     qx_status s = check_copies(in, nin);
     if (s == QX_OK) s = check_copies(out, nout);
-    if (s == QX_OK) s = check_chain(groups, ngroups, batch, y_dtype, flags);
+    if (s == QX_OK) s = check_chain(groups, ngroups, batch, y_dtype, flags & ~QX_GEMV_SEPARATE);
     if (s == QX_OK) s = check_fused_ws(workspace, workspace_bytes);
     if (s != QX_OK) return s;
     DeviceInfo *d = nullptr;

@@ -168,11 +168,12 @@ __device__ __forceinline__ void mma16816(float (&d)[4], uint32_t a0, uint32_t a1
 }
 
 // 16 bytes of x: through the read-only path, or (fused launches, whose x may
-// be written by an earlier phase of the same launch) from L2.
-__device__ __forceinline__ uint4 ldg_x(const __half *p, bool l2) {
+// be written by an earlier phase of the same launch) as a plain load, which
+// the phase handoff's acquire orders after those writes.
+__device__ __forceinline__ uint4 ldg_x(const __half *p, bool written) {
     uint4 v;
-    if (l2)
-        asm volatile("ld.global.cg.v4.u32 {%0, %1, %2, %3}, [%4];"
+    if (written)
+        asm volatile("ld.global.v4.u32 {%0, %1, %2, %3}, [%4];"
                      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
                      : "l"(p));
     else
@@ -196,10 +197,20 @@ struct MatS {
     void *y;
     int n, K, G, zbytes, log2g, nks, nlb;
     int q0;     // first CTA-local stage of this matrix
-    int rbq0;   // first CTA-local row block of this matrix
     int rb0;    // first matrix-local row block of this CTA
-    int nrb;    // row blocks of this CTA in this matrix
+    int nrb;    // row blocks this CTA has stages of
+    int ks_f;   // first slice of the first of them
+    int ks_e;   // end slice of the last of them
+    int st_off; // first stage of the matrix in its phase's list
 };
+
+// Slices [blo, bhi) this CTA takes of its row block rbl of M, and the
+// CTA-local index qb of the first of them.
+__device__ __forceinline__ void block_slices(const MatS &M, int rbl, int &blo, int &bhi, int &qb) {
+    blo = rbl == 0 ? M.ks_f : 0;
+    bhi = rbl == M.nrb - 1 ? M.ks_e : M.nks;
+    qb = M.q0 + (rbl == 0 ? 0 : (M.nks - M.ks_f) + (rbl - 1) * M.nks);
+}
 
 struct Header {
     uint64_t full[kMaxRing];       // a stage's copies have landed
@@ -302,9 +313,12 @@ __device__ __forceinline__ Meta load_meta(const MatS &M, int row0, int k0) {
     return t;
 }
 
-// Row blocks of matrix m in this CTA's range [lo, hi) of its phase's list.
-__device__ __forceinline__ int cta_nrb(const GemvMulti &a, int m, int lo, int hi) {
-    const int f = max(lo, a.mat[m].rb_off), e = min(hi, a.mat[m].rb_off + a.mat[m].nrb);
+// Stages [f, f + return) of matrix m in this CTA's range [lo, hi) of its
+// phase's list.
+__device__ __forceinline__ int cta_mat_stages(const GemvMulti &a, int m, int lo, int hi, int &f) {
+    const GemvMat &G = a.mat[m];
+    f = max(lo, G.st_off);
+    const int e = min(hi, G.st_off + G.nrb * G.nks);
     return e > f ? e - f : 0;
 }
 
@@ -314,12 +328,9 @@ __device__ __forceinline__ int phase_of(const GemvMulti &a, int m) {
     return p;
 }
 
-// This CTA's stages of phase p (its row blocks times their slices).
+// This CTA's stages of phase p.
 __device__ __forceinline__ int phase_stages(const GemvMulti &a, int p) {
-    const int lo = a.cta_rb[p][blockIdx.x], hi = a.cta_rb[p][blockIdx.x + 1];
-    int q = 0;
-    for (int m = a.phase_first[p]; m < a.phase_first[p + 1]; ++m) q += cta_nrb(a, m, lo, hi) * a.mat[m].nks;
-    return q;
+    return a.cta_st[p][blockIdx.x + 1] - a.cta_st[p][blockIdx.x];
 }
 
 // Pull the activations of phase p into L2 (lane i: matrix i of the phase).
@@ -351,7 +362,70 @@ __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
     return v;
 }
 
-// Named barrier of the consumer warps (the producer warp does not take part).
+__device__ __forceinline__ void st_release_gpu(uint32_t *p, uint32_t v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// y[b][row] of a block's 32 rows (lane = row within the block).
+template <int VMAX>
+__device__ __forceinline__ void store_y(const GemvMulti &a, const MatS &M, int row, const float (&v)[VMAX], int nb) {
+    if (row >= M.n) return;
+#pragma unroll
+    for (int b = 0; b < VMAX; ++b) {
+        if (b >= nb) break;
+        if (a.y_f32)
+            reinterpret_cast<float *>(M.y)[(int64_t)b * M.n + row] = v[b];
+        else
+            reinterpret_cast<__half *>(M.y)[(int64_t)b * M.n + row] = __float2half_rn(v[b]);
+    }
+}
+
+// A row block whose slices are split between two consecutive CTAs (the plan
+// never gives a block more than two).  The tail holder, for which the block is
+// the first of its range and so among the first it finishes, stores its fp32
+// sums and raises the block's flag (release); the head holder, for which the
+// block is the last, fetches them (acquire, bounded wait) before its own part
+// is summed, adds them after its own (slice order) and writes y.  Flags and
+// sums are indexed by the tail holder's CTA; the head holder clears the flag.
+constexpr int kSplitSlot = 16 * kRows;  // floats per CTA: [rows of x][32 rows]
+
+template <int VMAX>
+__device__ __forceinline__ void split_publish(const GemvMulti &a, const float (&v)[VMAX], int lane, int nb) {
+    float *mine = a.split_part + (size_t)blockIdx.x * kSplitSlot + lane;
+#pragma unroll
+    for (int b = 0; b < VMAX; ++b)
+        if (b < nb) __stcg(mine + b * kRows, v[b]);
+    __syncwarp();
+    if (lane == 0) st_release_gpu(a.split_flag + blockIdx.x, 1u);
+}
+
+template <int VMAX>
+__device__ __forceinline__ bool split_fetch(const GemvMulti &a, float (&w)[VMAX], int lane, int nb,
+                                            volatile uint32_t *abort_flag) {
+    const int partner = blockIdx.x + 1;
+    uint32_t ok = 1;
+    if (lane == 0 && ld_acquire_gpu(a.split_flag + partner) == 0u) {
+        const uint64_t t0 = globaltimer_ns();
+        while (ld_acquire_gpu(a.split_flag + partner) == 0u) {
+            __nanosleep(100);
+            if (*abort_flag || globaltimer_ns() - t0 > a.wait_limit_ns) {
+                ok = 0;
+                break;
+            }
+        }
+    }
+    if (!__shfl_sync(0xffffffffu, ok, 0)) return false;
+    __syncwarp();  // lane 0's acquire orders every lane's reads below
+    const float *src = a.split_part + (size_t)partner * kSplitSlot + lane;
+#pragma unroll
+    for (int b = 0; b < VMAX; ++b) w[b] = b < nb ? __ldcg(src + b * kRows) : 0.0f;
+    __syncwarp();
+    if (lane == 0) a.split_flag[partner] = 0u;  // for the next launch (or phase)
+    return true;
+}
+
+// Named barrier of the consumer warps (the producer and reducer warps do not
+// take part).
 __device__ __forceinline__ void consumers_sync() {
     asm volatile("bar.sync 1, %0;" ::"n"(32 * kWarps * kGroups) : "memory");
 }
@@ -542,10 +616,11 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         if (lane < count) {  // matrix `lane`: this CTA's row blocks and stage numbering
             const int t = lane;
             const int p = phase_of(a, t);
-            const int lo = a.cta_rb[p][blockIdx.x], hi = a.cta_rb[p][blockIdx.x + 1];
+            const int lo = a.cta_st[p][blockIdx.x], hi = a.cta_st[p][blockIdx.x + 1];
             const GemvMat &G = a.mat[t];
             MatS &S = h.mats[t];
-            const int f = max(lo, G.rb_off);
+            int f;
+            const int ns = cta_mat_stages(a, t, lo, hi, f);
             S.zeros = G.zeros;
             S.scales = G.scales;
             S.x = G.x;
@@ -557,23 +632,25 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
             S.log2g = G.log2g;
             S.nks = G.nks;
             S.nlb = G.nlb;
-            S.rb0 = f - G.rb_off;
-            S.nrb = cta_nrb(a, t, lo, hi);
-            // stages and blocks before this matrix: earlier phases (their stage
-            // counts padded to a multiple of kGroups), then this phase's earlier matrices
-            int q = 0, rbq = 0;
-            for (int pp = 0; pp < p; ++pp) {
-                q += round_groups(phase_stages(a, pp));
-                const int l2 = a.cta_rb[pp][blockIdx.x], h2 = a.cta_rb[pp][blockIdx.x + 1];
-                for (int m = a.phase_first[pp]; m < a.phase_first[pp + 1]; ++m) rbq += cta_nrb(a, m, l2, h2);
+            S.st_off = G.st_off;
+            if (ns > 0) {
+                const int r = f - G.st_off, l = f + ns - 1 - G.st_off;
+                S.rb0 = r / G.nks;
+                S.ks_f = r % G.nks;
+                S.nrb = l / G.nks - S.rb0 + 1;
+                S.ks_e = l % G.nks + 1;
+            } else {
+                S.rb0 = S.nrb = S.ks_f = S.ks_e = 0;
             }
+            // stages before this matrix: earlier phases (their stage counts
+            // padded to a multiple of kGroups), then this phase's earlier matrices
+            int q = 0;
+            for (int pp = 0; pp < p; ++pp) q += round_groups(phase_stages(a, pp));
             for (int m = a.phase_first[p]; m < t; ++m) {
-                const int nr = cta_nrb(a, m, lo, hi);
-                q += nr * a.mat[m].nks;
-                rbq += nr;
+                int fm;
+                q += cta_mat_stages(a, m, lo, hi, fm);
             }
             S.q0 = q;
-            S.rbq0 = rbq;
         }
     } else if (warp == 1) {
         if (lane == 0) {
@@ -602,6 +679,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 const int qend = h.ph_q0[p + 1];
                 int m = a.phase_first[p], rbl = 0, ks = 0;
                 while (m < a.phase_first[p + 1] && h.mats[m].nrb == 0) ++m;
+                if (m < a.phase_first[p + 1]) ks = h.mats[m].ks_f;
                 for (; q < qend; ++q) {
                     const int slot = q % ring;
                     if (q >= ring) {
@@ -614,12 +692,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                         continue;
                     }
                     issue_at<BITS, KIND>(a, h, ring_s, m, h.mats[m].rb0 + rbl, ks, slot);
-                    if (++ks == h.mats[m].nks) {
+                    const int nrb = h.mats[m].nrb;
+                    if (++ks == (rbl == nrb - 1 ? h.mats[m].ks_e : h.mats[m].nks)) {
                         ks = 0;
-                        if (++rbl == h.mats[m].nrb) {
+                        if (++rbl == nrb) {
                             rbl = 0;
                             ++m;
                             while (m < a.phase_first[p + 1] && h.mats[m].nrb == 0) ++m;
+                            if (m < a.phase_first[p + 1]) ks = h.mats[m].ks_f;
                         }
                     }
                 }
@@ -656,17 +736,24 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
         for (int p = 0; p < a.nphase && okr; ++p) {
             for (int m = a.phase_first[p]; m < a.phase_first[p + 1] && okr; ++m) {
                 const MatS &M = h.mats[m];
-                const int nks = M.nks, n = M.n;
-                const int ng = min(nks, kGroups);  // groups that worked on a block
                 for (int rbl = 0; rbl < M.nrb; ++rbl) {
+                    int blo, bhi, qb;
+                    block_slices(M, rbl, blo, bhi, qb);
+                    constexpr int VMAX = Dot<NT>::kCores ? 2 : 8 * NX;
+                    // a block that goes on in the next CTA: fetch that CTA's sums
+                    // while this CTA's warps still decode its own part
+                    float w[VMAX];
+                    if (bhi < M.nks && !split_fetch(a, w, lane, nb, &h.abort_flag)) {
+                        okr = false;
+                        break;
+                    }
                     const uint32_t fb = smem_u32(&h.rfull[rs]);
                     if (!mbar_try_wait(fb, use & 1u) && !mbar_wait(fb, use & 1u, a.wait_limit_ns, &h.abort_flag)) {
                         okr = false;
                         break;
                     }
                     const float *rp = red + (size_t)rs * (kGroups * kWarps * kRows * nbs);
-                    const int qb = M.q0 + rbl * nks;
-                    constexpr int VMAX = Dot<NT>::kCores ? 2 : 8 * NX;
+                    const int ng = min(bhi - blo, kGroups);  // groups that worked on the block
                     float v[VMAX];
 #pragma unroll
                     for (int b = 0; b < VMAX; ++b) v[b] = 0.0f;
@@ -695,16 +782,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     }
                     // the slot is free once every lane has read it
                     mbar_arrive(smem_u32(&h.rempty[rs]));
-                    const int row = (M.rb0 + rbl) * kRows + lane;
-                    if (row < n) {
+                    if (blo > 0) {
+                        split_publish(a, v, lane, nb);
+                    } else {
+                        if (bhi < M.nks) {
 #pragma unroll
-                        for (int b = 0; b < VMAX; ++b) {
-                            if (b >= nb) break;
-                            if (a.y_f32)
-                                reinterpret_cast<float *>(M.y)[(int64_t)b * n + row] = v[b];
-                            else
-                                reinterpret_cast<__half *>(M.y)[(int64_t)b * n + row] = __float2half_rn(v[b]);
+                            for (int b = 0; b < VMAX; ++b) v[b] += w[b];
                         }
+                        store_y(a, M, (M.rb0 + rbl) * kRows + lane, v, nb);
                     }
                     if (++rs == a.rb_slots) {
                         rs = 0;
@@ -837,9 +922,10 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                     blk_slot = 0;
                     ++blk_use;
                 }
-                const int qb = q0 + rbl * nks;  // the block's first stage
-                const int ks0 = (grp - qb % kGroups + kGroups) % kGroups;
-                // ks0 >= nks: this group has no stage of the block (it still hands
+                int blo, bhi, qb;  // the CTA's slices of the block, the first one's stage
+                block_slices(M, rbl, blo, bhi, qb);
+                const int ks0 = blo + (grp - qb % kGroups + kGroups) % kGroups;
+                // ks0 >= bhi: this group has no stage of the block (it still hands
                 // the block on below)
                 const int row0 = (rb0 + rbl) * kRows + g;  // the lane's first row (of g, g + 8, g + 16, g + 24)
                 float acc[2][NX][4];
@@ -851,9 +937,9 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                         for (int i = 0; i < 4; ++i) acc[rt][nt][i] = 0.0f;
                 Meta cur{};
                 if (KIND == 0) cur = load_meta(M, row0, ks0 * kSliceK + kunit);
-                for (int ks = ks0; ks < nks; ks += kGroups) {
+                for (int ks = ks0; ks < bhi; ks += kGroups) {
                     Meta nxt{};
-                    if (KIND == 0 && ks + kGroups < nks) nxt = load_meta(M, row0, (ks + kGroups) * kSliceK + kunit);
+                    if (KIND == 0 && ks + kGroups < bhi) nxt = load_meta(M, row0, (ks + kGroups) * kSliceK + kunit);
                     const bool live = ks * kSliceK + 128 * sb < K;  // K is a multiple of 128
                     uint32_t xw[NX][16];
                     load_x(ks, xw);
@@ -914,7 +1000,7 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                         break;
                     }
                 }
-                if (ks0 < nks) {
+                if (ks0 < bhi) {
                     // slot layout: [group][superblock warp][32 rows][nbs]
                     float *mine = rp_base + (size_t)rs * (kGroups * kWarps * kRows * nbs) +
                                   (size_t)(grp * kWarps + sb) * (kRows * nbs);
@@ -993,8 +1079,9 @@ cudaError_t launch_one(const GemvMulti &a, cudaStream_t st, bool pdl) {
         attr[na].val.programmaticStreamSerializationAllowed = 1;
         ++na;
     }
-    if (a.nphase > 1) {
-        // the phases wait on one another across CTAs: every CTA must be resident
+    if (a.nphase > 1 || a.has_split) {
+        // the phases, or the two halves of a split row block, wait on one
+        // another across CTAs: every CTA must be resident
         attr[na].id = cudaLaunchAttributeCooperative;
         attr[na].val.cooperative = 1;
         ++na;
@@ -1053,44 +1140,89 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
     }
     a.total_bytes = 0;
     a.grid = 1;
+    const bool split_ok = a.split_part != nullptr && a.split_flag != nullptr;
+    a.has_split = 0;
     int grids[kMaxGemvPhases];
     for (int p = 0; p < a.nphase; ++p) {
         const int m0 = a.phase_first[p], m1 = a.phase_first[p + 1];
         if (m1 <= m0) return false;
-        int64_t rbs = 0, total = 0;
+        int64_t rbs = 0, nst = 0, total = 0;
         int64_t rb_bytes[kMaxGemvTotal];  // bytes per row block (balancing only)
         for (int m = m0; m < m1; ++m) {
             GemvMat &M = a.mat[m];
             M.rb_off = (int)rbs;
+            M.st_off = (int)nst;
             rbs += M.nrb;
+            nst += (int64_t)M.nrb * M.nks;
             const int64_t row = M.k * a.bits / 8 + (a.kind == 1 ? (int64_t)M.G * 16 : (int64_t)M.G * 2 + M.zbytes);
             rb_bytes[m] = row * kRows;
             total += rb_bytes[m] * M.nrb;
         }
-        if (rbs > (int64_t)1 << 30) return false;
+        if (nst > (int64_t)1 << 30) return false;
         a.total_bytes += total;
-        const int grid = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), rbs);
+        // CTA c's first stage: the first unit (a whole row block, or a stage)
+        // that starts at or after byte c T / grid of the phase, in one pass
+        auto partition = [&](bool by_stage, int grid, int32_t *cst) {
+            cst[0] = 0;
+            int c = 1;
+            int64_t base = 0, st = 0;  // bytes before the current block, its first stage
+            for (int m = m0; m < m1 && c < grid; ++m) {
+                const GemvMat &M = a.mat[m];
+                for (int rb = 0; rb < M.nrb && c < grid; ++rb, base += rb_bytes[m]) {
+                    for (int ks = 0; ks < M.nks; ++ks, ++st) {
+                        if (ks > 0 && !by_stage) continue;
+                        // the stage's first byte (exact at block starts)
+                        const int64_t off = base + rb_bytes[m] * ks * kSliceK / M.k;
+                        while (c < grid && off >= (int64_t)((__int128)c * total / grid)) cst[c++] = (int32_t)st;
+                    }
+                }
+            }
+            while (c < grid) cst[c++] = (int32_t)nst;
+            cst[grid] = (int32_t)nst;
+        };
+        int grid = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), rbs);
+        int32_t *cst = a.cta_st[p];
+        partition(false, grid, cst);
+        if (split_ok) {
+            // by stages (a block's slices may go to two consecutive CTAs) when
+            // that lowers the most stages a CTA has and no block would go to
+            // three or more CTAs
+            int32_t alt[kMaxGemvCtas + 1];
+            const int g2 = (int)std::min<int64_t>(std::min(num_sms, kMaxGemvCtas), nst);
+            partition(true, g2, alt);
+            for (int i = 1; i < g2; ++i) alt[i] = std::max(alt[i], alt[i - 1] + 1);  // no empty CTA
+            for (int i = g2 - 1; i >= 1; --i) alt[i] = std::min(alt[i], alt[i + 1] - 1);
+            int most_w = 0, most_s = 0;
+            for (int c = 0; c < grid; ++c) most_w = std::max(most_w, cst[c + 1] - cst[c]);
+            for (int c = 0; c < g2; ++c) most_s = std::max(most_s, alt[c + 1] - alt[c]);
+            // a CTA whose range starts and ends inside one block (not at its
+            // edges) would make that block's third contributor
+            bool two = true, any = false;
+            for (int m = m0; m < m1 && two; ++m) {
+                const GemvMat &M = a.mat[m];
+                for (int c = 0; c < g2; ++c) {
+                    const int lo = std::max(alt[c], M.st_off), hi = std::min(alt[c + 1], M.st_off + M.nrb * M.nks);
+                    if (lo >= hi) continue;
+                    const bool cut_lo = (lo - M.st_off) % M.nks != 0, cut_hi = (hi - M.st_off) % M.nks != 0;
+                    any = any || cut_lo || cut_hi;
+                    if (cut_lo && cut_hi && (lo - M.st_off) / M.nks == (hi - 1 - M.st_off) / M.nks) {
+                        two = false;
+                        break;
+                    }
+                }
+            }
+            if (two && most_s < most_w) {
+                grid = g2;
+                std::copy(alt, alt + g2 + 1, cst);
+                a.has_split = a.has_split || any;
+            }
+        }
         grids[p] = grid;
         a.grid = std::max(a.grid, grid);
-        // CTA c owns the row blocks whose first byte lies in [c T / grid, (c+1) T / grid)
-        for (int c = 0; c <= grid; ++c) {
-            const int64_t b = (int64_t)((__int128)c * total / grid);
-            int64_t acc = 0, r = rbs;
-            for (int m = m0; m < m1; ++m) {
-                const GemvMat &M = a.mat[m];
-                const int64_t mb = rb_bytes[m] * M.nrb;
-                if (b < acc + mb) {
-                    r = M.rb_off + std::min<int64_t>((b - acc + rb_bytes[m] - 1) / rb_bytes[m], M.nrb);
-                    break;
-                }
-                acc += mb;
-            }
-            a.cta_rb[p][c] = (int32_t)r;
-        }
     }
-    // CTAs beyond a phase's own grid have no row block of that phase
+    // CTAs beyond a phase's own grid have no stage of that phase
     for (int p = 0; p < a.nphase; ++p)
-        for (int c = grids[p] + 1; c <= a.grid; ++c) a.cta_rb[p][c] = a.cta_rb[p][grids[p]];
+        for (int c = grids[p] + 1; c <= a.grid; ++c) a.cta_st[p][c] = a.cta_st[p][grids[p]];
     a.stage_bytes = (a.bits == 3 ? 3 * kBox : 4 * kBox) + (a.kind == 1 ? nlb_max * kBox : 0);
     // The ring is a multiple of the number of warp groups, so that every
     // slot is only ever used by one group: a warp then never waits on a

@@ -55,6 +55,7 @@ struct GemvMat {
     int nlb;         // LUT boxes (32 rows x 8 groups) per slice
     int nrb;         // 32-row blocks
     int rb_off;      // first row-block of this matrix in its phase's list
+    int st_off;      // first stage (row block x slice) of this matrix in its phase's list
 };
 
 // A decode launch: one phase (qx_gemv_multi), or several phases run one after
@@ -69,11 +70,20 @@ struct GemvMulti {
     int64_t total_bytes;
     uint32_t *status;
     uint32_t *phase_ctr;                   // nphase counters (nphase > 1): zero between launches
+    // Row blocks split between two CTAs (allowed when split_part is set; the
+    // plan sets has_split when it uses that): the CTA with the block's later
+    // slices stores their fp32 sums to split_part [CTA][16][32] and raises
+    // split_flag[CTA] (zero between launches); the CTA with the earlier slices
+    // adds them to its own and writes y
+    float *split_part;
+    uint32_t *split_flag;
+    int has_split;
     uint64_t wait_limit_ns;
     GemvMat mat[kMaxGemvTotal];
-    // per phase, the first row-block of every CTA in the phase's list
-    // (byte-balanced, computed on the host); cta_rb[p][grid] = the phase's row-blocks
-    int32_t cta_rb[kMaxGemvPhases][kMaxGemvCtas + 1];
+    // per phase, the first stage (row block x 1024-weight slice) of every CTA
+    // in the phase's list, byte-balanced on the host; at whole row blocks
+    // unless split_part is set.  cta_st[p][grid] = the phase's stages
+    int32_t cta_st[kMaxGemvPhases][kMaxGemvCtas + 1];
     CUtensorMap tm_codes[kMaxGemvTotal];  // packed codes, 32-row x 128-byte boxes
     CUtensorMap tm_luts[kMaxGemvTotal];   // LUTs, 32-row x 128-byte boxes (LUT kind)
 };

@@ -18,6 +18,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "lib", "lib
 UNIFORM, LUT, Q4X = 0, 1, 2
 F16, F32 = 0, 1
 GEMV_PDL = 1
+GEMV_SEPARATE = 2  # fused calls: one launch per group, each balanced with the workspace
 GEMM_PDL = 1
 
 STATUS = {
@@ -317,10 +318,13 @@ class GemvChain:
     dtype throughout); the ctypes arguments are built here once, so calling
     the object costs one library call.  Build a new chain if any of the
     tensors is replaced.  With `fused`, the groups run as ONE persistent launch
-    (qx_gemv_fused; same results), on a workspace the object owns: do not call
-    one fused object on two streams at the same time."""
+    (qx_gemv_fused: its CTAs balanced slice by slice, so the results are within
+    fp32 rounding of the chain's), on a workspace the object owns: do not call
+    one fused object on two streams at the same time.  With `separate` (which
+    implies the workspace) every group is a balanced launch of its own."""
 
-    def __init__(self, groups, pdl: bool = True, fused: bool = False):
+    def __init__(self, groups, pdl: bool = True, fused: bool = False, separate: bool = False):
+        fused = fused or separate
         self._keep, built = [], []
         batch, dt, dev = None, None, None
         for mats, xs, outs in groups:
@@ -349,7 +353,7 @@ class GemvChain:
             raise ValueError("no groups")
         self._groups = (_GemvGroup * len(built))(*built)
         self._args = (self._groups, len(built), batch, F32 if dt == torch.float32 else F16,
-                      GEMV_PDL if pdl else 0)
+                      (GEMV_PDL if pdl else 0) | (GEMV_SEPARATE if separate else 0))
         self._dev = dev
         self._ws = None
         if fused:
@@ -374,8 +378,9 @@ class DecodeStep(GemvChain):
     synchronization of the stream.  Host tensors should be pinned.  Arguments
     are bound once; build a new step if a tensor is replaced."""
 
-    def __init__(self, groups, h2d=(), d2h=(), pdl: bool = True, sync: bool = True, fused: bool = False):
-        super().__init__(groups, pdl, fused)
+    def __init__(self, groups, h2d=(), d2h=(), pdl: bool = True, sync: bool = True, fused: bool = False,
+                 separate: bool = False):
+        super().__init__(groups, pdl, fused, separate)
 
         def copies(pairs, to_device):
             arr = []

@@ -268,7 +268,7 @@ struct Pool {
             }
         }
     }
-    void launch_block(int nthreads, dim3 b, Block *blk, const std::function<void()> &f) {
+    void start_block(int nthreads, dim3 b, Block *blk, const std::function<void()> &f) {
         {
             std::lock_guard<std::mutex> l(mu);
             job = f;
@@ -279,8 +279,14 @@ struct Pool {
             ++gen;
         }
         cv.notify_all();
+    }
+    void wait_block() {
         std::unique_lock<std::mutex> l(mu);
         done_cv.wait(l, [&] { return remaining == 0; });
+    }
+    void launch_block(int nthreads, dim3 b, Block *blk, const std::function<void()> &f) {
+        start_block(nthreads, b, blk, f);
+        wait_block();
     }
 };
 
@@ -289,23 +295,48 @@ inline Pool &pool() {
     return p;
 }
 
-inline void launch(const Cfg &c, const std::function<void()> &f) {
+struct DynSmem {
+    uint8_t *p;
+    explicit DynSmem(size_t n) : p(n ? new (std::align_val_t(16)) uint8_t[n] : nullptr) {}
+    ~DynSmem() { if (p) ::operator delete[](p, std::align_val_t(16)); }
+};
+
+inline void init_block(Block &blk, const DynSmem &dyn, size_t smem, int nt) {
+    blk.dyn = dyn.p;
+    blk.dyn_bytes = smem;
+    blk.bar = std::make_unique<std::barrier<>>(nt);
+    const int nw = (nt + 31) / 32;
+    blk.warps.resize(nw);
+    for (int w = 0; w < nw; ++w) blk.warps[w].bar = std::make_unique<std::barrier<>>(std::min(32, nt - 32 * w));
+}
+
+// Blocks one after another (a normal launch), or all at once, each on a thread
+// pool of its own (a cooperative launch: its blocks may wait on one another).
+inline void launch(const Cfg &c, const std::function<void()> &f, bool concurrent = false) {
     const int nt = (int)(c.block.x * c.block.y * c.block.z);
     g_grid = c.grid;
     g_blockdim = c.block;
+    if (concurrent) {
+        const int nb = (int)(c.grid.x * c.grid.y);
+        std::vector<std::unique_ptr<Block>> blks;
+        std::vector<std::unique_ptr<DynSmem>> dyns;
+        std::vector<std::unique_ptr<Pool>> pools;
+        for (int i = 0; i < nb; ++i) {
+            blks.push_back(std::make_unique<Block>());
+            dyns.push_back(std::make_unique<DynSmem>(c.smem));
+            init_block(*blks.back(), *dyns.back(), c.smem, nt);
+            pools.push_back(std::make_unique<Pool>(nt));
+        }
+        for (int i = 0; i < nb; ++i)
+            pools[i]->start_block(nt, dim3((unsigned)(i % c.grid.x), (unsigned)(i / c.grid.x), 0), blks[i].get(), f);
+        for (auto &p : pools) p->wait_block();
+        return;
+    }
     for (unsigned by = 0; by < c.grid.y; ++by)
         for (unsigned bx = 0; bx < c.grid.x; ++bx) {
             Block blk;
-            struct Dyn {
-                uint8_t *p;
-                ~Dyn() { if (p) ::operator delete[](p, std::align_val_t(16)); }
-            } dyn{c.smem ? new (std::align_val_t(16)) uint8_t[c.smem] : nullptr};
-            blk.dyn = dyn.p;
-            blk.dyn_bytes = c.smem;
-            blk.bar = std::make_unique<std::barrier<>>(nt);
-            const int nw = (nt + 31) / 32;
-            blk.warps.resize(nw);
-            for (int w = 0; w < nw; ++w) blk.warps[w].bar = std::make_unique<std::barrier<>>(std::min(32, nt - 32 * w));
+            DynSmem dyn(c.smem);
+            init_block(blk, dyn, c.smem, nt);
             pool().launch_block(nt, dim3(bx, by, 0), &blk, f);
         }
 }
@@ -600,8 +631,9 @@ inline void emu_tma_load(uint32_t dst, const void *map, uint32_t bar, const int 
     emu_mbar_complete_tx(bar, (uint32_t)bytes);
 }
 
-// cudaLaunchKernelEx with its configuration (launch attributes are ignored:
-// kernels run one after another).
+// cudaLaunchKernelEx with its configuration (kernels run one after another;
+// of the launch attributes only the cooperative one counts: its blocks run at
+// the same time).
 enum cudaLaunchAttributeID { cudaLaunchAttributeProgrammaticStreamSerialization = 1, cudaLaunchAttributeCooperative = 2 };
 struct cudaLaunchAttributeValue {
     int programmaticStreamSerializationAllowed;
@@ -620,7 +652,10 @@ struct cudaLaunchConfig_t {
 };
 template <class K, class... A>
 inline cudaError_t cudaLaunchKernelEx(const cudaLaunchConfig_t *c, K k, A... args) {
-    emu::launch(emu::Cfg{c->gridDim, c->blockDim, c->dynamicSmemBytes, c->stream}, [&] { k(args...); });
+    bool coop = false;
+    for (unsigned i = 0; i < c->numAttrs; ++i)
+        coop = coop || (c->attrs[i].id == cudaLaunchAttributeCooperative && c->attrs[i].val.cooperative);
+    emu::launch(emu::Cfg{c->gridDim, c->blockDim, c->dynamicSmemBytes, c->stream}, [&] { k(args...); }, coop);
     return cudaSuccess;
 }
 
@@ -633,6 +668,8 @@ inline float __uint_as_float(uint32_t u) {
 inline __half2 __float2half2_rn(float x) { return __half2{__float2half_rn(x), __float2half_rn(x)}; }
 template <class T>
 inline T __ldcg(const T *p) { return *p; }
+template <class T>
+inline void __stcg(T *p, T v) { *p = v; }
 inline uint32_t emu_lds32(uint32_t a) {
     if (a & 3u) emu_fail("misaligned 4-byte shared load");
     uint32_t v;

@@ -200,13 +200,24 @@ int main(int argc, char **argv) {
             const int batch = extra;
             __half *x = alloc<__half>(2 * batch * k);
             if (!get(fi, x, 2 * batch * k)) return 2;
-            float *y0 = alloc<float>(4 * batch * n), *y1 = alloc<float>(4 * batch * n),
-                  *y2 = alloc<float>(4 * batch * n);
+            // launches: one matrix; the matrix twice (PDL); then twice more the
+            // matrix twice with the CTAs balanced stage by stage (row blocks
+            // split between CTAs, their partial sums in a workspace)
+            float *ys[7];
+            for (auto &y : ys) y = alloc<float>(4 * batch * n);
+            float *part = alloc<float>(4 * 2 * qx::kMaxGemvCtas * 16 * 32);
+            uint32_t *tick = alloc<uint32_t>(4 * qx::kMaxGemvCtas);
+            std::memset(tick, 0, 4 * qx::kMaxGemvCtas);  // the workspace starts at zero
             int l = 0;
             while ((1 << l) < g) ++l;
-            for (int launch = 0; launch < 2; ++launch) {
+            int has_split = 0;
+            for (int launch = 0; launch < 4; ++launch) {
                 qx::GemvMulti m{};
                 m.count = launch == 0 ? 1 : 2;
+                if (launch >= 2) {
+                    m.split_part = part;
+                    m.split_flag = tick;
+                }
                 m.nphase = 1;
                 m.phase_first[0] = 0;
                 m.phase_first[1] = m.count;
@@ -223,7 +234,7 @@ int main(int argc, char **argv) {
                     M.zeros = zeros;
                     M.luts = luts;
                     M.x = x;
-                    M.y = launch == 0 ? y0 : (i == 0 ? y1 : y2);
+                    M.y = launch == 0 ? ys[0] : ys[2 * launch - 1 + i];
                     M.n = n;
                     M.k = k;
                     M.G = G;
@@ -231,11 +242,14 @@ int main(int argc, char **argv) {
                     M.log2g = l;
                 }
                 if (!qx::plan_gemv(m, sms)) return 3;
+                has_split = m.has_split;
                 qx::launch_gemv_multi(m, nullptr, launch == 1);
             }
-            put(fo, y0, 4 * batch * n);
-            put(fo, y1, 4 * batch * n);
-            put(fo, y2, 4 * batch * n);
+            for (auto &y : ys) put(fo, y, 4 * batch * n);
+            put(fo, &has_split, 4);  // whether the balanced plan split a block
+            uint32_t left = 0;  // flags not back at zero
+            for (int i = 0; i < qx::kMaxGemvCtas; ++i) left += tick[i] != 0;
+            put(fo, &left, 4);
         } else if (cmd == "quant") {
             __half *Wh = alloc<__half>(2 * n * k);
             qx::DequantArgs d{codes, scales, zeros, luts, n, k, bits, g, kind, G, zb, Wh};

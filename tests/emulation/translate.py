@@ -39,10 +39,13 @@ BY_INSTRUCTION = [
     ("ldmatrix.sync.aligned.m8n8.x2", "emu_ldsm({i0}, 2, &{o0}, &{o1}, nullptr, nullptr);"),
     ("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32",
      "emu_mma16816({o0}, {o1}, {o2}, {o3}, {i0}, {i1}, {i2}, {i3}, {i4}, {i5});"),
+    ("ld.global.v4.u32",
+     "{{ uint4 t_; std::memcpy(&t_, (const void *)({i0}), 16); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
     ("ld.global.cg.v4.u32",
      "{{ uint4 t_; std::memcpy(&t_, (const void *)({i0}), 16); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
     ("bar.sync 1", "emu_named_bar({i0});"),
     ("atom.add.release.gpu.global.u32", "{o0} = std::atomic_ref<uint32_t>(*({i0})).fetch_add({i1});"),
+    ("st.release.gpu.global.u32", "std::atomic_ref<uint32_t>(*({i0})).store({i1});"),
     ("ld.acquire.gpu.global.u32", "{o0} = std::atomic_ref<uint32_t>(*const_cast<uint32_t *>({i0})).load();"),
     ("ld.global.nc.v4.u32",
      "{{ uint4 t_; std::memcpy(&t_, (const void *)({i0}), 16); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),

@@ -111,19 +111,28 @@ def test_int8_activations_and_w_a8_matmul(harness, n, k, bits, g, batch):
     assert np.all(oracle.max_abs_err(y, oracle.gemv_a8(ref, rec, x, k)) <= tol)
 
 
-@pytest.mark.parametrize("n,k,bits,g,kind,batch,sms", [  # 1..16 rows of x, ragged row blocks
-    (37, 384, 4, 64, 0, 1, 2), (130, 640, 3, 64, 0, 4, 3), (33, 256, 4, 32, 0, 8, 2),
-    (20, 512, 3, 128, 1, 3, 2), (5, 4096, 4, 128, 0, 2, 4), (70, 1152, 3, 128, 0, 1, 3),
-    (40, 512, 3, 128, 1, 16, 2), (33, 384, 4, 64, 0, 11, 2), (24, 768, 3, 32, 1, 5, 2)])
-def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms):
+@pytest.mark.parametrize("n,k,bits,g,kind,batch,sms,split", [  # 1..16 rows of x, ragged row blocks
+    (37, 384, 4, 64, 0, 1, 2, 0), (130, 640, 3, 64, 0, 4, 3, 0), (33, 256, 4, 32, 0, 8, 2, 0),
+    (20, 512, 3, 128, 1, 3, 2, 0), (5, 4096, 4, 128, 0, 2, 4, 1), (70, 1152, 3, 128, 0, 1, 3, 0),
+    (40, 512, 3, 128, 1, 16, 2, 0), (33, 384, 4, 64, 0, 11, 2, 0), (24, 768, 3, 32, 1, 5, 2, 0),
+    # the balanced plan: blocks split between two CTAs (1), or kept whole
+    # because a block would get three CTAs or no CTA would get fewer stages (0)
+    (5, 4096, 4, 128, 0, 2, 3, 1), (5, 4096, 3, 128, 1, 1, 8, 0), (130, 2048, 3, 64, 0, 4, 3, 1),
+    (40, 3072, 3, 128, 1, 9, 5, 0)])
+def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms, split):
     """qx_gemv's kernel and host plan (tensor maps, byte-balanced CTA slices):
-    one matrix, and the same matrix twice in one launch (with PDL set)."""
+    one matrix, the same matrix twice in one launch (with PDL set), and twice
+    more the pair with the CTAs balanced stage by stage (row blocks split
+    between CTAs through the workspace): within tolerance, the balanced
+    launches deterministic, their flags back at zero."""
     W = _weights(n, k, seed=n + g)
     x = synth.activations(batch, k, seed=batch, stream=n)
     rd = _run(harness, ["gemv", n, k, bits, g, kind, batch, sms], W, x)
     G = k // g
     rd.take(n * k * bits // 8 + (2 * n * G + n * ((G + 1) // 2) if kind == 0 else 2 * n * G * 8), np.uint8)
-    ys = [rd.take(batch * n, np.float32).reshape(batch, n) for _ in range(3)]
+    ys = [rd.take(batch * n, np.float32).reshape(batch, n) for _ in range(7)]
+    assert rd.take(1, np.int32)[0] == split
+    assert rd.take(1, np.uint32)[0] == 0  # every split flag back at zero
     assert rd.take(1, np.uint32)[0] == 0  # no bounded wait gave up
     rec = ORecipe(bits, g, "lut" if kind else "uniform", 25)
     ref = oracle.quantize(W, rec)
@@ -132,6 +141,7 @@ def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms):
     for y in ys:
         assert np.all(oracle.max_abs_err(y, y_ref) <= tol)
     assert np.array_equal(ys[0], ys[1]) and np.array_equal(ys[1], ys[2])
+    assert np.array_equal(ys[3], ys[5]) and np.array_equal(ys[4], ys[6])
 
 
 @pytest.mark.parametrize("n,k,bits,g,kind,m,sms", [  # 16-, 64- and 256-token tiles, 1..4 k splits

@@ -8,7 +8,8 @@ matmul within max_n |y - y_ref| <= 2e-3 ||x_b||_2 max_n ||w_hat_n||_2.
 * The Llama-7B-shaped layer with 4-bit uniform g128 and 3-bit uniform g64
   weights through the decode chain q,k,v | o | gate,up | down (four
   qx_gemv_multi launches with PDL in one CUDA graph) at batch 1, 4 and 16, and
-  through the same chain as one fused launch (qx_gemv_fused).
+  through the same chain with its CTAs balanced slice by slice (qx_gemv_fused:
+  one launch, and one launch per group).
 * One LLaVA-v1.6-7B-shaped language layer with the mixed per-matrix recipe of
   the recipe table (q, k: 3-bit LUT g128; v, o, gate, up, down: 4-bit uniform
   g64) through its five-launch chain.
@@ -94,16 +95,21 @@ def test_llama_layer_uniform_decode_chain(qx, bits, g):
         g_.replay()
         torch.cuda.synchronize()
         assert qx.device_status() == 0
-        yf = {nm: torch.full((batch, n), float("nan"), dtype=torch.float16, device="cuda") for nm, n, _, _ in LLAMA}
-        fused = qx.GemvChain([([mats[nm][0] for nm in names], [xs[nm] for nm in names], [yf[nm] for nm in names])
-                              for names in LLAMA_CHAIN], fused=True)
-        fused()
+        # the same chain with its CTAs balanced slice by slice: one launch, and
+        # one balanced launch per group (bit for bit the same)
+        yb = {}
+        for mode in ("fused", "separate"):
+            yb[mode] = {nm: torch.full((batch, n), float("nan"), dtype=torch.float16, device="cuda")
+                        for nm, n, _, _ in LLAMA}
+            qx.GemvChain([([mats[nm][0] for nm in names], [xs[nm] for nm in names], [yb[mode][nm] for nm in names])
+                          for names in LLAMA_CHAIN], **{mode: True})()
         torch.cuda.synchronize()
         assert qx.device_status() == 0
         for nm, n, k, _ in LLAMA:
             P, rows, ref, orec, Wh = mats[nm]
-            assert torch.equal(ys[nm], yf[nm]), nm  # the fused launch: the chain's results bit for bit
-            _check(ys[nm].float().cpu().numpy()[:, rows], ref, orec, xk[k], k, Wh)
+            assert torch.equal(yb["fused"][nm], yb["separate"][nm]), nm
+            for y in (ys[nm], yb["fused"][nm]):
+                _check(y.float().cpu().numpy()[:, rows], ref, orec, xk[k], k, Wh)
 
 
 def test_llava_language_layer_mixed_recipe_decode(qx):

@@ -81,12 +81,15 @@ def test_decode_step_with_pageable_host_memory(qx):
 @pytest.mark.parametrize("bits,g,kind", [(3, 128, 1), (4, 64, 0)])
 @pytest.mark.parametrize("batch", [1, 2, 5, 16])
 def test_fused_launch_equals_the_chain(qx, bits, g, kind, batch):
-    """qx_gemv_fused: the groups of a chain in one persistent launch, bit for
-    bit the chain's results.  With fp16 outputs the third group reads the first
-    group's output as its x, which the launch may read only once every CTA has
-    finished the first group (the outputs start as NaN, so an early read
-    shows).  Three calls in a row share one workspace: each launch leaves its
-    phase counters zero for the next."""
+    """qx_gemv_fused: the groups of a chain in one persistent launch, its CTAs
+    balanced slice by slice (blocks split between CTAs summed through the
+    workspace): bit for bit the same as the balanced launches one group at a
+    time (QX_GEMV_SEPARATE), and within fp32 summation order (fp16 outputs:
+    one rounding) of the chain, whose CTAs take whole blocks.  With fp16
+    outputs the third group reads the first group's output as its x, which the
+    launch may read only once every CTA has finished the first group (the
+    outputs start as NaN, so an early read shows).  Three calls in a row share
+    one workspace: each launch leaves its counters zero for the next."""
     rec = qx.Recipe(bits, g, kind)
     shapes = {"q": (256, 512), "k": (96, 512), "up": (1000, 512), "o": (512, 256), "down": (384, 1024)}
     mats = {nm: qx.quantize(torch.from_numpy(synth.student_t_weights(n, k, 0.02, seed=i, stream=n)).cuda(), rec)
@@ -95,19 +98,31 @@ def test_fused_launch_equals_the_chain(qx, bits, g, kind, batch):
     xd = torch.from_numpy(synth.activations(batch, 1024, seed=2, stream=2)).cuda()
     for dt in (torch.float16, torch.float32):
         ys = {nm: torch.empty((batch, P.n), dtype=dt, device="cuda") for nm, P in mats.items()}
+        yss = {nm: torch.empty((batch, P.n), dtype=dt, device="cuda") for nm, P in mats.items()}
         handoff = dt == torch.float16
-        xo = ys["q"] if handoff else torch.from_numpy(synth.activations(batch, 256, seed=3, stream=3)).cuda()
-        groups = [(["q", "k"], [xa, xa]), (["up"], [xa]), (["o"], [xo]), (["down"], [xd])]
-        fused = qx.GemvChain([([mats[nm] for nm in names], xs, [ys[nm] for nm in names]) for names, xs in groups],
-                             fused=True)
+        xo_ref = torch.from_numpy(synth.activations(batch, 256, seed=3, stream=3)).cuda()
+
+        def groups_for(out):
+            xo = out["q"] if handoff else xo_ref
+            return [(["q", "k"], [xa, xa]), (["up"], [xa]), (["o"], [xo]), (["down"], [xd])]
+
+        def chain(out, **kw):
+            return qx.GemvChain([([mats[nm] for nm in names], xs, [out[nm] for nm in names])
+                                 for names, xs in groups_for(out)], **kw)
+
+        fused, separate = chain(ys, fused=True), chain(yss, separate=True)
         for rep in range(3):
-            for y in ys.values():
+            for y in list(ys.values()) + list(yss.values()):
                 y.fill_(float("nan"))
             fused()
+            separate()
             ref = {}
-            for names, xs in groups:
+            for names, xs in groups_for(ys):
                 xs_ref = [ref["q"] if handoff and x is ys["q"] else x for x in xs]
                 ref.update(zip(names, qx.gemv_multi([mats[nm] for nm in names], xs_ref, out_dtype=dt, pdl=True)))
             for nm in mats:
-                assert torch.equal(ys[nm], ref[nm]), (nm, rep)
+                assert torch.equal(ys[nm], yss[nm]), (nm, rep)
+                r = ref[nm].float()
+                tol = 4e-5 * r.abs().amax(dim=1, keepdim=True) + (r.abs() * 2.0 ** -10 if handoff else 0.0)
+                assert torch.all((ys[nm].float() - r).abs() <= tol), (nm, rep)
         assert qx.device_status() == 0
