@@ -356,6 +356,10 @@ __device__ __forceinline__ uint32_t atom_add_release_gpu(uint32_t *p, uint32_t v
     return old;
 }
 
+__device__ __forceinline__ void red_add_release_gpu(uint32_t *p, uint32_t v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
 __device__ __forceinline__ uint32_t ld_acquire_gpu(const uint32_t *p) {
     uint32_t v;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
@@ -798,15 +802,18 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 }
             }
             if (fused && okr) {
-                // every y of phase p written by this CTA is visible at gpu scope
-                // before the CTA is counted in
-                __threadfence();
+                // count the CTA in with a release (the warp barrier orders every
+                // lane's y stores before it): whoever acquires the count sees them.
+                // Before the last phase a reduction, which the warp does not wait
+                // for; in the last one an atomic, whose old value tells the last
+                // CTA of the launch
                 __syncwarp();
                 if (lane == 0) {
-                    const uint32_t old = atom_add_release_gpu(a.phase_ctr + p, 1u);
-                    if (p == a.nphase - 1 && old == gridDim.x - 1) {
-                        // the last CTA of the launch: every other CTA has passed
-                        // every wait, so the counters go back to zero for the next launch
+                    if (p < a.nphase - 1) {
+                        red_add_release_gpu(a.phase_ctr + p, 1u);
+                    } else if (atom_add_release_gpu(a.phase_ctr + p, 1u) == gridDim.x - 1) {
+                        // every other CTA has passed every wait, so the counters
+                        // go back to zero for the next launch
                         for (int i = 0; i < a.nphase; ++i) a.phase_ctr[i] = 0u;
                     }
                 }

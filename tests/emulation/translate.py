@@ -46,6 +46,7 @@ BY_INSTRUCTION = [
     ("bar.sync 1", "emu_named_bar({i0});"),
     ("atom.add.release.gpu.global.u32", "{o0} = std::atomic_ref<uint32_t>(*({i0})).fetch_add({i1});"),
     ("st.release.gpu.global.u32", "std::atomic_ref<uint32_t>(*({i0})).store({i1});"),
+    ("red.release.gpu.global.add.u32", "std::atomic_ref<uint32_t>(*({i0})).fetch_add({i1});"),
     ("ld.acquire.gpu.global.u32", "{o0} = std::atomic_ref<uint32_t>(*const_cast<uint32_t *>({i0})).load();"),
     ("ld.global.nc.v4.u32",
      "{{ uint4 t_; std::memcpy(&t_, (const void *)({i0}), 16); {o0} = t_.x; {o1} = t_.y; {o2} = t_.z; {o3} = t_.w; }}"),
