@@ -5,8 +5,11 @@ gate, up 11008x4096; down 4096x11008), Student-t(4) weights with sigma 0.01
 (q, k), 0.02 (v, o), 0.04 (MLP), quantized to 3-bit non-uniform codes with a
 per-group 8-entry fp16 LUT (Lloyd-Max, group 128 along k).  One step = one
 decode token through all seven matrices: the decode dependency chain
-q,k,v | o | gate,up | down as four qx_gemv_multi launches at batch 1 (PDL,
-one CUDA graph).  Metric: HBM GB/s of the packed weights (+ x, y) per step.
+q,k,v | o | gate,up | down at batch 1 as the four phases of one persistent
+qx_gemv_fused launch (each phase reads its x once every CTA has written the
+previous phase's y; one CUDA graph).  Metric: HBM GB/s of the packed weights
+(+ x, y) per step.  The same step as four qx_gemv_multi launches (PDL) is
+reported beside it.
 
 Also reported on the same line: the prefill GEMM (M = 2048 tokens against the
 11008x4096 and 4096x11008 3-bit LUT matrices, tcgen05), the same layer with
@@ -362,6 +365,7 @@ def _summary(line, hbm, tf_burst):
         return d
 
     out = {"decode_L3g128_b1_GBps": line["value"], "frac_of_measured_hbm": line["value"] / hbm,
+           "decode_L3g128_b1_4_launches_GBps": get(line, "chain_4_launches", "GBps"),
            "e2e_GBps": get(line, "e2e", "value"),
            "prefill_TFLOPs": get(line, "gemm", "value"), "prefill_frac_of_bf16_burst": get(line, "gemm", "roofline", "frac")}
     for rec in ("U4g128", "U3g64"):
@@ -421,9 +425,18 @@ def run_ours(args):
         names, x = CHAIN[j]
         qx.gemv_multi([layers[c][nm] for nm in names], [x] * len(names), outs=[ys[nm] for nm in names], pdl=True)
 
-    def step(c):
+    def chain_step(c):
         for j in range(len(CHAIN)):
             launch(c, j)
+
+    # the timed step: the four groups as phases of ONE persistent launch
+    # (qx_gemv_fused, CTAs balanced slice by slice, a group's x read once every
+    # CTA has written the previous group's y), one workspace per weight copy
+    fsteps = [qx.GemvChain([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
+                            for names, x in CHAIN], fused=True) for c in range(copies)]
+
+    def step(c):
+        fsteps[c]()
 
     with torch.cuda.stream(stream):
         for c in range(copies):
@@ -474,10 +487,10 @@ def run_ours(args):
     ms = _max_over_ranks(dist, ms, dev)
     value = _job_rate(step_bytes, ws, ms) / 1e9
 
-    # The timed region holds only gemv_kernel<3,LUT,1> launches (four per step),
-    # so its average launch duration is ms / 4 and the algorithmic bytes of an
-    # average launch are step_bytes / 4: achieved = step_bytes / ms.
-    launch_us = ms * 1e3 / len(CHAIN)
+    # The timed region holds only gemv_kernel<3,LUT,-1> launches, one per step,
+    # so the launch duration is ms and its algorithmic bytes are step_bytes:
+    # achieved = step_bytes / ms.
+    launch_us = ms * 1e3
     achieved = step_bytes / (ms * 1e-3) / 1e9
     # steady-state duration of each launch of the chain: one graph per launch
     # kind, `copies` back-to-back launches (PDL) over rotating weight copies
@@ -516,37 +529,40 @@ def run_ours(args):
     torch.cuda.synchronize(dev)
     one_launch_ms = e0.elapsed_time(e1) / reps
 
-    # the same chain as ONE persistent launch (qx_gemv_fused): the four groups
-    # hand off through device-side counters instead of kernel boundaries
-    fused_us = None
-    try:
-        fsteps = [qx.GemvChain([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
-                                for names, x in CHAIN], fused=True) for c in range(copies)]
-        with torch.cuda.stream(stream):
-            for fs in fsteps:
-                fs()
-        torch.cuda.synchronize(dev)
-        gf = torch.cuda.CUDAGraph()
-        with torch.cuda.graph(gf, stream=stream):
-            for fs in fsteps:
-                fs()
-        fused_us = _time_graph(torch, stream, gf, 20) / copies * 1e3
-        del gf, fsteps
-    except Exception as e:  # noqa: BLE001
-        fused_us = f"unavailable: {type(e).__name__}: {e}"[:160]
+    # the same step as four qx_gemv_multi launches (PDL), whole row blocks per
+    # CTA, and as four balanced launches (qx_gemv_fused with QX_GEMV_SEPARATE)
+    alt_us = {}
+    sep = [qx.GemvChain([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
+                         for names, x in CHAIN], separate=True) for c in range(copies)]
+    for nm_, fn in (("chain_4_launches", chain_step), ("balanced_4_launches", lambda c: sep[c]())):
+        try:
+            with torch.cuda.stream(stream):
+                for c in range(copies):
+                    fn(c)
+            torch.cuda.synchronize(dev)
+            ga = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(ga, stream=stream):
+                for c in range(copies):
+                    fn(c)
+            us = _time_graph(torch, stream, ga, 20) / copies * 1e3
+            alt_us[nm_] = {"us": us, "GBps": step_bytes / (us * 1e-6) / 1e9}
+            del ga
+        except Exception as e:  # noqa: BLE001
+            alt_us[nm_] = f"unavailable: {type(e).__name__}: {e}"[:160]
+    del sep
 
     # end to end through the public API with host buffers: the step's activations
     # in from pinned host memory (one copy), the four decode calls, the outputs
     # back (one copy), then a stream synchronisation, per step
     hx = x_flat.cpu().pin_memory()
     hy = torch.empty(y_flat.shape, dtype=y_flat.dtype).pin_memory()
-    # a step is one qx_decode_step call (copy in, the four launches, copy out,
-    # synchronize; arguments bound once per weight copy); if it cannot be built
-    # or run, the step is the torch copies around the four qx_gemv_multi calls
-    e2e_call, e2e_path = None, "torch copies + 4 qx_gemv_multi calls + synchronize per step"
+    # a step is one qx_decode_step_fused call (copy in, the one launch, copy
+    # out, synchronize; arguments bound once per weight copy); if it cannot be
+    # built or run, the step is the torch copies around the fused call
+    e2e_call, e2e_path = None, "torch copies + 1 qx_gemv_fused call + synchronize per step"
     try:
         dsteps = [qx.DecodeStep([([layers[c][nm] for nm in names], [x] * len(names), [ys[nm] for nm in names])
-                                 for names, x in CHAIN], h2d=[(x_flat, hx)], d2h=[(hy, y_flat)])
+                                 for names, x in CHAIN], h2d=[(x_flat, hx)], d2h=[(hy, y_flat)], fused=True)
                   for c in range(copies)]
         with torch.cuda.stream(stream):
             for ds in dsteps:
@@ -554,7 +570,7 @@ def run_ours(args):
         if qx.device_status(stream) != 0:
             raise RuntimeError("device status after the decode step")
         e2e_call = lambda c: dsteps[c]()  # noqa: E731
-        e2e_path = "1 qx_decode_step call per step: copy in, 4 PDL launches, copy out, synchronize"
+        e2e_path = "1 qx_decode_step_fused call per step: copy in, 1 launch, copy out, synchronize"
     except Exception as e:  # noqa: BLE001
         e2e_path += f" (decode step unavailable: {type(e).__name__}: {e})"[:200]
     e2e_steps = max(3, min(args.steps, 2000))
@@ -577,7 +593,7 @@ def run_ours(args):
 
     section = lambda fn, *a: _section(torch, fn, *a)  # noqa: E731
     gemm = section(run_gemm_part, qx, torch, dev, stream, tf_burst, peak_src) if not args.skip_gemm else None
-    del layers, graphs, g_all
+    del layers, graphs, g_all, fsteps
     extra = {}
     if not args.skip_configs:
         extra["config3"] = section(run_config3, qx, torch, dev, stream, l2, hbm)
@@ -596,27 +612,26 @@ def run_ours(args):
                        "matrices": {nm: [n, k] for nm, n, k, _, _ in LAYER},
                        "recipe": "3-bit LUT (8 fp16 levels, Lloyd-Max) group 128",
                        "batch": 1, "bytes_per_step": step_bytes,
-                       "step": "qkv | o | gate+up | down: 4 qx_gemv_multi launches (PDL); CUDA graphs of one "
-                               "step on every weight copy in turn",
+                       "step": "qkv | o | gate+up | down as the 4 phases of one qx_gemv_fused launch (PDL "
+                               "between steps); CUDA graphs of one step on every weight copy in turn",
                        "l2": f"{copies} rotating weight copies ({copies * layer_bytes / 1e6:.0f} MB) > "
                              f"4x L2 ({l2 / 1e6:.0f} MB)"},
             # the long sections first: the record keeps the end of the line
             **extra,
-            "per_launch_us": per_launch_us,
+            "chain_per_launch_us": per_launch_us,
             "one_launch_7_matrices": {"us": one_launch_ms * 1e3,
                                       "GBps": step_bytes / (one_launch_ms * 1e-3) / 1e9},
-            "fused_one_launch_4_groups": ({"us": fused_us, "GBps": step_bytes / (fused_us * 1e-6) / 1e9}
-                                          if isinstance(fused_us, float) else fused_us),
+            **alt_us,
             "cpu_baseline": cpu,
             "clocks": clocks,
             "e2e": {"value": e2e_value, "unit": "GB/s", "ms_per_step": e2e_ms,
                     "h2d_bytes_per_step": hx.numel() * hx.element_size(),
                     "d2h_bytes_per_step": hy.numel() * hy.element_size(), "path": e2e_path},
-            "gpu_launches": args.steps * len(CHAIN),
+            "gpu_launches": args.steps,
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
                          "frac": achieved / hbm, "peak_source": f"{peak_src} hbm_gbs",
-                         "kernel": "gemv_kernel<3,LUT,-1>", "launches_per_step": len(CHAIN),
-                         "launch_us": launch_us, "bytes_per_launch": step_bytes / len(CHAIN),
+                         "kernel": "gemv_kernel<3,LUT,-1> (4 phases)", "launches_per_step": 1,
+                         "launch_us": launch_us, "bytes_per_launch": step_bytes,
                          "traffic": _traffic("qx_gemv.cu", "gemv_L3g128_b1")},
             "gemm": gemm,
         }
