@@ -373,9 +373,10 @@ def _summary(line, hbm, tf_burst):
             v = get(line, "config3", f"llama7b_layer_decode_{rec}_b{b}", "GBps")
             if v is not None:
                 out[f"decode_{rec}_b{b}_GBps"] = v
-    v = get(line, "q4x", "llama7b_layer_decode_Q4X_b1", "GBps")
-    if v is not None:
-        out["decode_Q4X_b1_GBps"] = v
+    for b in (1, 4, 16):
+        v = get(line, "q4x", f"llama7b_layer_decode_Q4X_b{b}", "GBps")
+        if v is not None:
+            out[f"decode_Q4X_b{b}_GBps"] = v
     return out
 
 
@@ -852,7 +853,7 @@ def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
     """Q4X shared codebooks (groups of 64 with an fp16 scale and a 2-bit book
     index, 4-bit codes, four 16-level codebooks learned per matrix): the
     learner's device time per Llama-7B layer matrix, and the decode matmul over
-    the layer at batch 1 and 4 (q,k,v | o | gate,up | down: four
+    the layer at batch 1, 4 and 16 (q,k,v | o | gate,up | down: four
     qx_q4x_gemv_multi launches per layer copy in one CUDA graph, weights
     rotated over copies larger than 4x L2), and the tensor-core prefill
     (qx_q4x_gemm) at M = 2048 against the two MLP shapes."""
@@ -882,7 +883,7 @@ def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
     layers = [base] + [{nm: dup(P) for nm, P in base.items()} for _ in range(copies - 1)]
     out = {"learn_ms": learn_ms, "weight_bytes": layer_bytes,
            "bits_per_weight": 8.0 * layer_bytes / sum(n * k for _, n, k, _, _ in LAYER)}
-    for batch in (1, 4):
+    for batch in (1, 4, 16):
         xs = {k: synth.activations_torch(batch, k, seed=batch, stream=70 + i, device=dev)
               for i, k in enumerate((4096, 11008))}
         ys = {nm: torch.empty((batch, n), dtype=torch.float16, device=dev) for nm, n, *_ in LAYER}
@@ -907,7 +908,8 @@ def run_q4x(qx, torch, dev, stream, l2, hbm, tf_burst):
         gbps = (layer_bytes + io) / (ms * 1e-3) / 1e9
         out[f"llama7b_layer_decode_Q4X_b{batch}"] = {
             "us_per_layer": ms * 1e3, "GBps": gbps, "frac_of_measured_hbm": gbps / hbm,
-            "path": "4 qx_q4x_gemv_multi launches (persistent warps over the rows, codebooks in shared memory)"}
+            "path": "4 qx_q4x_gemv_multi launches: weights dequantized in registers from TMA-staged codes, "
+                    "the codebooks as pair tables in shared memory"}
     if qx.device_status(stream) != 0:
         raise RuntimeError("q4x decode reported a device error")
     # prefill on the tensor cores (qx_q4x_gemm): M = 2048 tokens against the two

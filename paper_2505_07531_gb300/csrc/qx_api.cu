@@ -1086,6 +1086,50 @@ QX_API qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream) {
                                             static_cast<cudaStream_t>(stream)));
 }
 
+namespace {
+
+// Q4X decode on the register-dequant kernel (csrc/qx_gemv.cu, kind 2: the
+// books in `zeros`, the codebooks in `luts`), which works in 128-weight
+// superblocks.  A matrix's results do not depend on the launch it is in.
+bool q4x_ring_fits(const qx::Q4xMat &m) { return m.k % 128 == 0 && m.k <= 32768; }
+
+// *launched stays false, with nothing launched, when the plan does not fit.
+qx_status run_q4x_ring(const qx::Q4xGemvMulti &q, cudaStream_t st, DeviceInfo *d, bool *launched) {
+    *launched = false;
+    qx::GemvMulti a{};
+    a.bits = 4;
+    a.kind = 2;
+    a.batch = q.batch;
+    a.y_f32 = q.y_f32;
+    a.status = d->status;
+    a.wait_limit_ns = wait_limit_ns();
+    a.nphase = 1;
+    a.count = q.count;
+    a.phase_first[0] = 0;
+    a.phase_first[1] = q.count;
+    for (int i = 0; i < q.count; ++i) {
+        const qx::Q4xMat &m = q.mat[i];
+        if (!q4x_ring_fits(m)) return QX_OK;
+        qx::GemvMat &M = a.mat[i];
+        M.codes = m.codes;
+        M.scales = m.scales;
+        M.zeros = m.books;
+        M.luts = m.codebooks;
+        M.x = q.x[i];
+        M.y = q.y[i];
+        M.n = m.n;
+        M.k = m.k;
+        M.G = m.G;
+        M.zbytes = m.bbytes;
+        M.log2g = 6;
+    }
+    if (!plan_cached(a, d)) return QX_OK;
+    *launched = true;
+    return from_cuda(qx::launch_gemv_multi(a, st, false));
+}
+
+}  // namespace
+
 QX_API qx_status qx_q4x_gemv_multi(const qx_q4x *mats, int32_t count, const void *const *x, int32_t batch,
                                    void *const *y, int32_t y_dtype, void *stream) {
     if (mats == nullptr || x == nullptr || y == nullptr) return QX_ERR_INVALID_ARG;
@@ -1111,7 +1155,31 @@ QX_API qx_status qx_q4x_gemv_multi(const qx_q4x *mats, int32_t count, const void
     DeviceInfo *d = nullptr;
     qx_status s = device_info(&d);
     if (s != QX_OK) return s;
-    return from_cuda(qx::launch_q4x_gemv(a, d->num_sms, static_cast<cudaStream_t>(stream)));
+    // the matrices the register-dequant kernel takes in one launch, the rest
+    // (k not a multiple of 128) in one launch of the row-per-warp kernel
+    const cudaStream_t st = static_cast<cudaStream_t>(stream);
+    qx::Q4xGemvMulti part[2]{};
+    for (int j = 0; j < 2; ++j) {
+        part[j].batch = batch;
+        part[j].y_f32 = a.y_f32;
+    }
+    for (int i = 0; i < count; ++i) {
+        qx::Q4xGemvMulti &p = part[q4x_ring_fits(a.mat[i]) ? 0 : 1];
+        p.mat[p.count] = a.mat[i];
+        p.x[p.count] = a.x[i];
+        p.y[p.count] = a.y[i];
+        p.row_off[p.count + 1] = p.row_off[p.count] + a.mat[i].n;
+        ++p.count;
+    }
+    if (part[0].count > 0) {
+        bool launched = false;
+        s = run_q4x_ring(part[0], st, d, &launched);
+        if (s != QX_OK) return s;
+        if (!launched) s = from_cuda(qx::launch_q4x_gemv(part[0], d->num_sms, st));
+        if (s != QX_OK) return s;
+    }
+    if (part[1].count > 0) s = from_cuda(qx::launch_q4x_gemv(part[1], d->num_sms, st));
+    return s;
 }
 
 QX_API qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream) {

@@ -57,6 +57,7 @@ constexpr int kMaxRbSlots = 8;
 constexpr int kHeader = 2048;    // barriers, counters, per-matrix and per-phase CTA plan
 constexpr int kSmemBudget = 220 * 1024;
 constexpr int kCoreBatch = 2;    // batches up to this take the CUDA-core products
+constexpr int kQ4xTableBytes = 4 * 256 * 4;  // Q4X: a matrix's four books as 256-entry pair tables
 
 __device__ __forceinline__ uint32_t smem_u32(const void *p) {
     return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -288,14 +289,16 @@ __device__ __forceinline__ void issue_at(const GemvMulti &a, Header &h, uint32_t
                            ring_s + (uint32_t)(slot * a.stage_bytes), rb, ks);
 }
 
-// Uniform scales and zero-points of a lane's four rows (tile rows g, g + 8 of
-// both 16-row tiles) for its 32-weight unit of a stage: scales as half2
-// pairs (rows g, g + 8) per tile, zero-points in nibbles 0..3.
+// Uniform scales and zero-points (Q4X: scales and codebook indices) of a
+// lane's four rows (tile rows g, g + 8 of both 16-row tiles) for its 32-weight
+// unit of a stage: scales as half2 pairs (rows g, g + 8) per tile,
+// zero-points (book indices) in nibbles 0..3.
 struct Meta {
     uint32_t s[2];
     uint32_t z;
 };
 
+template <int KIND>
 __device__ __forceinline__ Meta load_meta(const MatS &M, int row0, int k0) {
     Meta t{{0u, 0u}, 0u};
     if (k0 >= M.K) return t;
@@ -306,8 +309,13 @@ __device__ __forceinline__ Meta load_meta(const MatS &M, int row0, int k0) {
         const int row = row0 + 8 * i;  // g, g + 8, 16 + g, 24 + g
         if (row < M.n) {
             t.s[i >> 1] |= (uint32_t)__ldg(sp + (int64_t)row * M.G + grp) << ((i & 1) * 16);
-            const uint32_t zb = __ldg(M.zeros + (int64_t)row * M.zbytes + (grp >> 1));
-            t.z |= ((zb >> ((grp & 1) * 4)) & 15u) << (4 * i);
+            if (KIND == 2) {  // 2-bit book index of group grp: bits 2 (grp % 4) of byte grp / 4
+                const uint32_t bb = __ldg(M.zeros + (int64_t)row * M.zbytes + (grp >> 2));
+                t.z |= ((bb >> ((grp & 3) * 2)) & 3u) << (4 * i);
+            } else {
+                const uint32_t zb = __ldg(M.zeros + (int64_t)row * M.zbytes + (grp >> 1));
+                t.z |= ((zb >> ((grp & 1) * 4)) & 15u) << (4 * i);
+            }
         }
     }
     return t;
@@ -559,6 +567,76 @@ __device__ __forceinline__ void tile4(const uint4 &c0, const uint4 &c1, uint32_t
     d.finish(nb, __low2float(s0), __low2float(s1), acc);
 }
 
+// Q4X (paper Section 3.2).  Byte j of code word w (k = 8t .. 8t + 7) holds the
+// codes of a pair of k two apart: (8t, 8t + 2), (8t + 4, 8t + 6), (8t + 1,
+// 8t + 3), (8t + 5, 8t + 7) for j = 0..3.  Each byte indexes the book's pair
+// table (entry v holds CB[v % 16] and CB[v / 16]; tables are 1 KB-aligned, so
+// the address is the table's OR'd with 4 v), and one fp16 multiply by the
+// group's scale gives w_hat = fp16(s CB[b][q]) with the dequantization's single
+// rounding.  x is re-paired the same way (x_pairs_q4x): the order of a dot
+// product's terms, and of an MMA's contraction, is free as long as both
+// operands follow it.
+__device__ __forceinline__ uint32_t lds32(uint32_t a) {
+    uint32_t v;
+    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
+    return v;
+}
+
+template <bool SCALED>
+__device__ __forceinline__ void pairs_q4x(uint32_t w, uint32_t tab, __half2 s, __half2 (&o)[4]) {
+    o[0] = u2h2(lds32(tab | ((w << 2) & 0x3FCu)));
+    o[1] = u2h2(lds32(tab | (shr_fma(w, 6) & 0x3FCu)));
+    o[2] = u2h2(lds32(tab | (shr_fma(w, 14) & 0x3FCu)));
+    o[3] = u2h2(lds32(tab | (shr_fma(w, 22) & 0x3FCu)));
+    if (SCALED) {
+#pragma unroll
+        for (int i = 0; i < 4; ++i) o[i] = __hmul2(o[i], s);
+    }
+}
+
+// x words (x[k], x[k + 1]) of 8 k re-paired as the code bytes pair the
+// weights: (x0, x2), (x4, x6), (x1, x3), (x5, x7).
+template <int NX>
+__device__ __forceinline__ void x_pairs_q4x(uint32_t (&xv)[NX][16]) {
+#pragma unroll
+    for (int nt = 0; nt < NX; ++nt)
+#pragma unroll
+        for (int wd = 0; wd < 4; ++wd) {
+            const uint32_t x01 = xv[nt][4 * wd], x23 = xv[nt][4 * wd + 1];
+            const uint32_t x45 = xv[nt][4 * wd + 2], x67 = xv[nt][4 * wd + 3];
+            xv[nt][4 * wd] = prmt(x01, x23, 0x5410u);
+            xv[nt][4 * wd + 1] = prmt(x45, x67, 0x5410u);
+            xv[nt][4 * wd + 2] = prmt(x01, x23, 0x7632u);
+            xv[nt][4 * wd + 3] = prmt(x45, x67, 0x7632u);
+        }
+}
+
+// One 16-row tile, Q4X codes: the lane's 16 code bytes of rows g (c0) and
+// g + 8 (c1), the shared addresses of their groups' pair tables and their
+// scales.  Tensor cores: products with x of the dequantized weights
+// themselves.  CUDA cores: products of the codebook levels (in [-1, 1]) with
+// x, and the group's scale applied to their fp32 sum (a 32-weight unit lies in
+// one 64-weight group), as the uniform kind does.
+template <int NT>
+__device__ __forceinline__ void tile4q(const uint4 &c0, const uint4 &c1, uint32_t tab0, uint32_t tab1, __half2 s0,
+                                       __half2 s1, const uint32_t (&xw)[Dot<NT>::NX][16], int nb,
+                                       float (&acc)[Dot<NT>::NX][4]) {
+    const uint32_t w0[4] = {c0.x, c0.y, c0.z, c0.w};
+    const uint32_t w1[4] = {c1.x, c1.y, c1.z, c1.w};
+    Dot<NT> d;
+    d.start();
+#pragma unroll
+    for (int wd = 0; wd < 4; ++wd) {  // codes m = 8 wd .. 8 wd + 7: steps 2 wd, 2 wd + 1
+        __half2 o0[4], o1[4];
+        pairs_q4x<!Dot<NT>::kCores>(w0[wd], tab0, s0, o0);
+        pairs_q4x<!Dot<NT>::kCores>(w1[wd], tab1, s1, o1);
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh)
+            d.step(2 * wd + hh, o0[2 * hh], o0[2 * hh + 1], o1[2 * hh], o1[2 * hh + 1], xw, nb, acc);
+    }
+    d.finish(nb, __low2float(s0), __low2float(s1), acc);
+}
+
 // Row stride (floats) of a block's partial sums in shared memory.  CUDA-core
 // path (one or two rows of x, scalar reads): odd, so that the finisher's
 // lane-strided reads hit 32 different banks.  Tensor-core path (16-byte
@@ -584,7 +662,8 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
     uint8_t *base = smem_raw + (base_s - raw_s);
     Header &h = *reinterpret_cast<Header *>(base);
     float *red = reinterpret_cast<float *>(base + kHeader);
-    const uint32_t ring_s = base_s + (uint32_t)(kHeader + a.red_bytes);
+    const uint32_t tab_s = base_s + (uint32_t)(kHeader + a.red_bytes);  // Q4X pair tables
+    const uint32_t ring_s = tab_s + (uint32_t)a.tab_bytes;
 
     const int warp = threadIdx.x >> 5;
     const int lane = threadIdx.x & 31;
@@ -665,6 +744,16 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                 q += round_groups(h.ph_nst[p]);
             }
             h.ph_q0[a.nphase] = q;
+        }
+    }
+    if (KIND == 2) {
+        // every matrix's four books as pair tables: entry q0 + 16 q1 of book b
+        // holds CB[b][q0] (low half) and CB[b][q1] (high half)
+        uint32_t *tab = reinterpret_cast<uint32_t *>(base + kHeader + a.red_bytes);
+        for (int e = threadIdx.x; e < count * (kQ4xTableBytes / 4); e += kThreads) {
+            const unsigned short *cb =
+                reinterpret_cast<const unsigned short *>(a.mat[e >> 10].luts) + ((e >> 8) & 3) * 16;
+            tab[e] = (uint32_t)__ldg(cb + (e & 15)) | ((uint32_t)__ldg(cb + ((e >> 4) & 15)) << 16);
         }
     }
     __syncthreads();
@@ -943,13 +1032,14 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
 #pragma unroll
                         for (int i = 0; i < 4; ++i) acc[rt][nt][i] = 0.0f;
                 Meta cur{};
-                if (KIND == 0) cur = load_meta(M, row0, ks0 * kSliceK + kunit);
+                if (KIND != 1) cur = load_meta<KIND>(M, row0, ks0 * kSliceK + kunit);
                 for (int ks = ks0; ks < bhi; ks += kGroups) {
                     Meta nxt{};
-                    if (KIND == 0 && ks + kGroups < bhi) nxt = load_meta(M, row0, (ks + kGroups) * kSliceK + kunit);
+                    if (KIND != 1 && ks + kGroups < bhi) nxt = load_meta<KIND>(M, row0, (ks + kGroups) * kSliceK + kunit);
                     const bool live = ks * kSliceK + 128 * sb < K;  // K is a multiple of 128
                     uint32_t xw[NX][16];
                     load_x(ks, xw);
+                    if (KIND == 2) x_pairs_q4x<NX>(xw);
                     const uint32_t fb = smem_u32(&h.full[slot]);
                     if (!mbar_try_wait(fb, par) && !mbar_wait(fb, par, a.wait_limit_ns, &h.abort_flag)) {
                         ok = false;
@@ -980,14 +1070,22 @@ __global__ void __launch_bounds__(kThreads, 1) gemv_kernel(const __grid_constant
                             } else {
                                 const uint4 c0 = lds128(sbase + co[rt][0]);
                                 const uint4 c1 = lds128(sbase + co[rt][1]);
-                                tile4<NT>(c0, c1, (cur.z >> (8 * rt)) & 15u, (cur.z >> (8 * rt + 4)) & 15u,
-                                          half2_of(cur.s[rt], 0), half2_of(cur.s[rt], 1), xw, nb, acc[rt]);
+                                if (KIND == 2) {
+                                    // the pair tables of this matrix's books for rows g, g + 8
+                                    const uint32_t tb = tab_s + (uint32_t)m * kQ4xTableBytes;
+                                    tile4q<NT>(c0, c1, tb + ((cur.z >> (8 * rt)) & 3u) * 1024u,
+                                               tb + ((cur.z >> (8 * rt + 4)) & 3u) * 1024u, half2_of(cur.s[rt], 0),
+                                               half2_of(cur.s[rt], 1), xw, nb, acc[rt]);
+                                } else {
+                                    tile4<NT>(c0, c1, (cur.z >> (8 * rt)) & 15u, (cur.z >> (8 * rt + 4)) & 15u,
+                                              half2_of(cur.s[rt], 0), half2_of(cur.s[rt], 1), xw, nb, acc[rt]);
+                                }
                             }
                         }
                     }
                     // release the slot (every lane arrives: no warp-level sync needed)
                     mbar_arrive(smem_u32(&h.empty[slot]));
-                    if (KIND == 0) cur = nxt;
+                    if (KIND != 1) cur = nxt;
                     slot += kGroups;
                     if (slot >= ring) {
                         slot -= ring;
@@ -1116,6 +1214,7 @@ bool encode(CUtensorMap *map, const void *base, int rank, const cuuint64_t *dims
 bool plan_gemv(GemvMulti &a, int num_sms) {
     if (a.nphase < 1 || a.nphase > kMaxGemvPhases || a.count < 1 || a.count > kMaxGemvTotal) return false;
     if (a.phase_first[0] != 0 || a.phase_first[a.nphase] != a.count) return false;
+    if (a.kind == 2 && (a.bits != 4 || a.count > kMaxGemvMats)) return false;
     int nks_min = 1 << 30, nlb_max = 1;
     for (int m = 0; m < a.count; ++m) {
         GemvMat &M = a.mat[m];
@@ -1231,6 +1330,7 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
     for (int p = 0; p < a.nphase; ++p)
         for (int c = grids[p] + 1; c <= a.grid; ++c) a.cta_st[p][c] = a.cta_st[p][grids[p]];
     a.stage_bytes = (a.bits == 3 ? 3 * kBox : 4 * kBox) + (a.kind == 1 ? nlb_max * kBox : 0);
+    a.tab_bytes = a.kind == 2 ? a.count * kQ4xTableBytes : 0;
     // The ring is a multiple of the number of warp groups, so that every
     // slot is only ever used by one group: a warp then never waits on a
     // barrier phase more than one ahead of the slot's current one.
@@ -1242,7 +1342,7 @@ bool plan_gemv(GemvMulti &a, int num_sms) {
         int slots = std::min(kMaxRbSlots, (ring + nks_min - 1) / nks_min + 2);
         while (slots > 2 && slots * slot_bytes > 48 * 1024) --slots;
         const int red = (slots * slot_bytes + 1023) / 1024 * 1024;
-        const int smem = 1024 + kHeader + red + ring * a.stage_bytes;
+        const int smem = 1024 + kHeader + red + a.tab_bytes + ring * a.stage_bytes;
         if (smem <= kSmemBudget || ring == kGroups) {
             a.ring = ring;
             a.rb_slots = slots;
@@ -1286,6 +1386,7 @@ cudaError_t launch_wait_selftest(uint64_t limit_ns, uint32_t *status, cudaStream
 }
 
 cudaError_t launch_gemv_multi(GemvMulti &a, cudaStream_t st, bool pdl) {
+    if (a.kind == 2) return launch_nt<4, 2>(a, st, pdl);
     if (a.bits == 4) return launch_nt<4, 0>(a, st, pdl);
     if (a.kind == 1) return launch_nt<3, 1>(a, st, pdl);
     return launch_nt<3, 0>(a, st, pdl);

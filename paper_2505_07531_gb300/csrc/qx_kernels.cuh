@@ -66,7 +66,7 @@ struct GemvMulti {
     int count, bits, kind, batch, y_f32;   // count: matrices over all phases
     int nphase;
     int phase_first[kMaxGemvPhases + 1];   // first matrix of each phase; [nphase] = count
-    int grid, ring, rb_slots, stage_bytes, red_bytes, smem_bytes;
+    int grid, ring, rb_slots, stage_bytes, red_bytes, tab_bytes, smem_bytes;
     int64_t total_bytes;
     uint32_t *status;
     uint32_t *phase_ctr;                   // nphase counters (nphase > 1): zero between launches

@@ -149,6 +149,42 @@ int main(int argc, char **argv) {
         g.y_f32 = 0;
         g.y[0] = yh;
         qx::launch_q4x_gemv(g, sms, nullptr);
+        // the same decodes on the register-dequant kernel (kind 2; k a multiple
+        // of 128): the matrix twice in fp32, then once in fp16
+        float *y2 = alloc<float>(4 * batch * n), *y3 = alloc<float>(4 * batch * n);
+        __half *yh2 = alloc<__half>(2 * batch * n);
+        int ring = 0;
+        if (k % 128 == 0) {
+            for (int launch = 0; launch < 2; ++launch) {
+                qx::GemvMulti r{};
+                r.bits = 4;
+                r.kind = 2;
+                r.batch = batch;
+                r.y_f32 = launch == 0;
+                r.status = status;
+                r.wait_limit_ns = 60000000000ull;
+                r.nphase = 1;
+                r.count = launch == 0 ? 2 : 1;
+                r.phase_first[1] = r.count;
+                for (int i = 0; i < r.count; ++i) {
+                    qx::GemvMat &M = r.mat[i];
+                    M.codes = codes;
+                    M.scales = scales;
+                    M.zeros = books;
+                    M.luts = cbs;
+                    M.x = x;
+                    M.y = launch == 1 ? static_cast<void *>(yh2) : static_cast<void *>(i == 0 ? y2 : y3);
+                    M.n = n;
+                    M.k = k;
+                    M.G = G;
+                    M.zbytes = bb;
+                    M.log2g = 6;
+                }
+                if (!qx::plan_gemv(r, sms)) return 3;
+                qx::launch_gemv_multi(r, nullptr, false);
+            }
+            ring = 1;
+        }
         put(fo, codes, n * k / 2);
         put(fo, scales, 2 * n * G);
         put(fo, books, n * bb);
@@ -157,6 +193,10 @@ int main(int argc, char **argv) {
         put(fo, y0, 4 * batch * n);
         put(fo, y1, 4 * batch * n);
         put(fo, yh, 2 * batch * n);
+        put(fo, &ring, 4);
+        put(fo, y2, 4 * batch * n);
+        put(fo, y3, 4 * batch * n);
+        put(fo, yh2, 2 * batch * n);
     } else {
         const int bits = atoi(argv[4]), g = atoi(argv[5]);
         const bool three = cmd == "quant" || cmd == "gemv" || cmd == "gemm";  // commands that take a kind

@@ -203,6 +203,7 @@ def _q4x_cases():
         "all_zero": (np.zeros((8, 256), np.float16), 3, 2, 2),
         "few_distinct": (np.tile(np.array([-1, 0, 0.5, 1], np.float16), (8, 64)), 3, 2, 4),
         "nonfinite": (nan, 3, 2, 1),
+        "three_slices": (_weights(40, 2176, seed=4), 3, 3, 2),
     }
 
 
@@ -233,10 +234,22 @@ def test_q4x_learner_dequant_and_multi_matrix_decode(harness, name):
     y0 = rd.take(batch * n, np.float32).reshape(batch, n)
     y1 = rd.take(batch * n, np.float32).reshape(batch, n)
     yh = rd.take(batch * n, np.float16).reshape(batch, n).astype(np.float64)
+    # the register-dequant kernel (run when k is a multiple of 128)
+    ring = rd.take(1, np.int32)[0] == 1
+    assert ring == (k % 128 == 0)
+    y2 = rd.take(batch * n, np.float32).reshape(batch, n)
+    y3 = rd.take(batch * n, np.float32).reshape(batch, n)
+    yh2 = rd.take(batch * n, np.float16).reshape(batch, n).astype(np.float64)
     assert np.array_equal(y0, y1)  # both entries of the two-matrix launch
+    if ring:
+        assert np.array_equal(y2, y3)
     if not bad.any():
         y_ref = oracle.gemv_q4x(ref, x)
         tol = oracle.tolerance(x, Wh)
+        fp16_out = np.abs(y_ref).max(axis=1) * 2.0 ** -11
         assert np.all(oracle.max_abs_err(y0, y_ref) <= tol)
-        assert np.all(oracle.max_abs_err(yh, y_ref) <= tol + np.abs(y_ref).max(axis=1) * 2.0 ** -11)
+        assert np.all(oracle.max_abs_err(yh, y_ref) <= tol + fp16_out)
+        if ring:
+            assert np.all(oracle.max_abs_err(y2, y_ref) <= tol)
+            assert np.all(oracle.max_abs_err(yh2, y_ref) <= tol + fp16_out)
     assert rd.take(1, np.uint32)[0] == (1 if bad.any() else 0)  # the non-finite status bit
