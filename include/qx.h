@@ -410,14 +410,16 @@ qx_status qx_q4x_dequant(const qx_q4x *p, void *W_out, void *stream);
 /* Decode matmul y = x W_hat^T for a Q4X matrix: x device fp16 [batch][k],
  * 16-byte aligned; y device [batch][n] of y_dtype, 4-byte aligned; batch
  * 1..16.  w_hat exactly as above.  When k is a multiple of 128 (and at most
- * 32768) the weights are dequantized in registers from TMA-staged codes, as
- * qx_gemv does (Section 2.4): for one or two rows of x the products and their
- * sums over 8 consecutive weight pairs are formed in fp16 (so they must stay
- * within its range, |.| < 65504), then summed in fp32; for 3..16 rows the
- * products are summed in fp32 on the tensor cores.  Otherwise the products and
- * their sums over 16 consecutive pairs are formed in fp16, then summed in
- * fp32.  A matrix's results do not depend on the other matrices of a
- * qx_q4x_gemv_multi call. */
+ * 32768) the codes are decoded in registers from TMA-staged tiles, as qx_gemv
+ * does (Section 2.4): for one or two rows of x the products of the codebook
+ * levels (in [-1, 1]) with x and their sums over 8 weight pairs are formed in
+ * fp16, then summed in fp32 and multiplied by the group's scale (s * sum
+ * CB[q] x, not sum w_hat x: they differ by the rounding of w_hat); for 3..16
+ * rows the products of w_hat itself are summed in fp32 on the tensor cores.
+ * Otherwise the products of w_hat and their sums over 16 consecutive pairs are
+ * formed in fp16, then summed in fp32.  fp16 intermediates must stay within
+ * its range (|.| < 65504).  A matrix's results do not depend on the other
+ * matrices of a qx_q4x_gemv_multi call. */
 qx_status qx_q4x_gemv(const qx_q4x *p, const void *x, int32_t batch, void *y, int32_t y_dtype, void *stream);
 
 /* Several Q4X decode matmuls in one launch: y[i] = x[i] W_hat_i^T, i < count
