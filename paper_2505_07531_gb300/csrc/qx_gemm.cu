@@ -789,9 +789,12 @@ GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_spli
     p.tiles = ((m + p.bn - 1) / p.bn) * nt;
     if (allow_split && num_sms > 0) {
         // Time ~ rounds of units per CTA x (superblocks per unit + about two
-        // for pipeline fill and epilogue), plus the last split's reduction
-        // (one L2 round trip, about half a superblock, per split and 32
-        // columns).  Decode sizes take 16-token tiles; longer inputs choose
+        // for pipeline fill and epilogue), plus the last split's reduction:
+        // per 32 columns about two superblocks of fixed cost (the counter's
+        // round trip, the partial tiles' stores and loads) and half a
+        // superblock per split -- fitted to 64-token tiles at 576 tokens,
+        // where a 1024 x 1024 matrix took 9.9 us unsplit and 11.8 us in two
+        // splits.  Decode sizes take 16-token tiles; longer inputs choose
         // between 64-token tiles, which may split k, and 256-token tiles.
         const int cands[2] = {m <= 16 ? 16 : 64, 256};
         double best = -1.0;
@@ -802,7 +805,7 @@ GemmPlan plan_gemm(int64_t n, int64_t k, int64_t m, int num_sms, bool allow_spli
             for (int sp = 1; sp <= smax; ++sp) {
                 const int64_t rounds = (tiles * sp + num_sms - 1) / num_sms;
                 const double cost = (double)rounds * ((nsb + sp - 1) / sp + 2) +
-                                    (sp > 1 ? 0.5 * sp * ((bn + 31) / 32) : 0.0);
+                                    (sp > 1 ? (2.0 + 0.5 * sp) * ((bn + 31) / 32) : 0.0);
                 if (best < 0 || cost < best) {
                     best = cost;
                     p.bn = bn;

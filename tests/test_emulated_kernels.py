@@ -146,7 +146,8 @@ def test_tma_pipelined_decode_gemv(harness, n, k, bits, g, kind, batch, sms, spl
 
 @pytest.mark.parametrize("n,k,bits,g,kind,m,sms", [  # 16-, 64- and 256-token tiles, 1..4 k splits
     (37, 384, 4, 64, 0, 5, 2), (128, 2048, 4, 128, 0, 16, 4), (200, 1024, 3, 64, 0, 40, 4),
-    (64, 1152, 4, 32, 0, 1, 8), (130, 256, 4, 256, 0, 300, 2), (40, 256, 3, 128, 1, 3, 2)])
+    (64, 1152, 4, 32, 0, 1, 8), (130, 256, 4, 256, 0, 300, 2), (40, 256, 3, 128, 1, 3, 2),
+    (128, 2048, 3, 128, 1, 40, 4)])  # 64-token tiles split four ways
 def test_tensor_core_matmul(harness, n, k, bits, g, kind, m, sms):
     """qx_gemm (one CTA per tile), then qx_gemm_splitk twice on one workspace,
     the second with PDL: each within tolerance (fp16 output), and the split

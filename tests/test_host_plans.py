@@ -16,9 +16,9 @@ def qx():
     (4096, 4096, 1, (16, 4)),
     (11008, 4096, 16, (16, 3)),
     (4096, 11008, 16, (16, 4)),
-    (1024, 1024, 576, (64, 2)),    # vision prefill: 64-token tiles, two splits
+    (1024, 1024, 576, (64, 1)),    # vision prefill: 64-token tiles fill 72 SMs; a split costs more
     (4096, 1024, 576, (256, 1)),   # enough 256-token tiles already
-    (1024, 4096, 576, (64, 2)),
+    (1024, 4096, 576, (64, 2)),    # 64-token tiles, two splits
     (11008, 4096, 2048, (256, 1)),  # full prefill: no split
 ])
 def test_plans_of_the_benchmark_shapes(qx, n, k, m, want):

@@ -92,8 +92,8 @@ def test_noalloc_allocates_nothing(qx):
 
 @pytest.mark.gpu
 def test_noalloc_refuses_plans_larger_than_its_scratch(qx):
-    # 21632 x 1152 at m = 1 splits into 507 units: 4.2 MB of workspace > 4 MiB
-    n, k = 21632, 1152
+    # 21632 x 1920 at m = 1 splits into 507 units: 4.2 MB of workspace > 4 MiB
+    n, k = 21632, 1920
     rec = qx.Recipe(4, 128, 0)
     assert qx.gemm_splitk_workspace_bytes(n, k, 1, rec) > 4 << 20
     P = qx.PackedMatrix.empty(n, k, rec, torch.device("cuda"))
