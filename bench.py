@@ -571,7 +571,8 @@ def run_ours(args):
         if qx.device_status(stream) != 0:
             raise RuntimeError("device status after the decode step")
         e2e_call = lambda c: dsteps[c]()  # noqa: E731
-        e2e_path = "1 qx_decode_step_fused call per step: copy in, 1 launch, copy out, synchronize"
+        e2e_path = ("1 qx_decode_step_fused call per step: copy in (copy kernel reading the pinned host x), "
+                    "1 launch, copy out (copy kernel writing the pinned host y), synchronize")
     except Exception as e:  # noqa: BLE001
         e2e_path += f" (decode step unavailable: {type(e).__name__}: {e})"[:200]
     e2e_steps = max(3, min(args.steps, 2000))

@@ -194,6 +194,13 @@ typedef struct qx_copy {
  * non-zero, a synchronization of the stream (the outputs are then in host
  * memory).  nin, nout 0..16.  Every group is validated before the first copy;
  * a failing argument returns its status and nothing is issued.
+ * When every host buffer of a direction is pinned (mapped into the device's
+ * address space), every device buffer is device memory and they total at
+ * most 4 MiB, that direction's copies are made by one small kernel of the
+ * library that reads or writes the host buffers through their device
+ * addresses (the copy out starts early under programmatic dependent launch
+ * and waits in the kernel for the groups to finish); otherwise by
+ * cudaMemcpyAsync, one per buffer.  Either way the bytes are the same.
  * When every host buffer is pinned and `stream` is not being captured, the
  * first call with a given set of arguments captures the copies and launches
  * as a CUDA graph (on a stream of the library's own) and every later call

@@ -420,20 +420,61 @@ qx_status run_chain_fused(const qx_gemv_group *groups, int32_t ngroups, int32_t 
 
 // The copies and launches of one decode step, issued on `st` (ws non-null: the
 // groups as one fused launch).
+// The copies of one direction as one copy kernel (qx_copy.cu) when every
+// host buffer is pinned and mapped, every device buffer is device memory and
+// they are small (a decode step's x and y): a copy engine's start-up costs
+// more than such copies take.  False leaves them to cudaMemcpyAsync.
+bool kernel_copies(const qx_copy *c, int32_t n, bool h2d, qx::CopyList &l) {
+    if (n < 1 || n > qx::kMaxCopies) return false;
+    int64_t total = 0;
+    l.n = n;
+    for (int i = 0; i < n; ++i) {
+        const void *host = h2d ? c[i].src : c[i].dst;
+        const void *dev = h2d ? c[i].dst : c[i].src;
+        cudaPointerAttributes ah, ad;
+        if (cudaPointerGetAttributes(&ah, host) != cudaSuccess || cudaPointerGetAttributes(&ad, dev) != cudaSuccess) {
+            cudaGetLastError();
+            return false;
+        }
+        if (ah.type != cudaMemoryTypeHost || ah.devicePointer == nullptr || ad.type != cudaMemoryTypeDevice)
+            return false;
+        total += (int64_t)c[i].bytes;
+        uint8_t *hd = static_cast<uint8_t *>(ah.devicePointer);  // the host buffer's device address
+        uint8_t *dd = static_cast<uint8_t *>(const_cast<void *>(dev));
+        l.src[i] = h2d ? hd : dd;
+        l.dst[i] = h2d ? dd : hd;
+        l.bytes[i] = (int64_t)c[i].bytes;
+    }
+    return total <= ((int64_t)4 << 20);
+}
+
 qx_status issue_step(const qx_copy *in, int32_t nin, const qx_gemv_group *groups, int32_t ngroups, int32_t batch,
                      int32_t y_dtype, int32_t flags, void *ws, const qx_copy *out, int32_t nout, cudaStream_t st,
                      DeviceInfo *d) {
     qx_status s = QX_OK;
-    for (int i = 0; i < nin; ++i)
-        if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) != QX_OK)
-            return s;
+    qx::CopyList cl{};
+    // in: stream-ordered after whatever may still read the device buffers
+    if (kernel_copies(in, nin, true, cl)) {
+        if ((s = from_cuda(qx::launch_copies(cl, d->num_sms, false, st))) != QX_OK) return s;
+    } else {
+        for (int i = 0; i < nin; ++i)
+            if ((s = from_cuda(cudaMemcpyAsync(in[i].dst, in[i].src, in[i].bytes, cudaMemcpyHostToDevice, st))) !=
+                QX_OK)
+                return s;
+    }
     s = ws != nullptr ? run_chain_fused(groups, ngroups, batch, y_dtype, flags, ws, st, d)
                       : run_chain(groups, ngroups, batch, y_dtype, flags, st, d);
     if (s != QX_OK) return s;
-    for (int i = 0; i < nout; ++i)
-        if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
-            QX_OK)
-            return s;
+    // out: under PDL the copy kernel starts early and waits in the kernel for
+    // the matmuls to finish
+    if (kernel_copies(out, nout, false, cl)) {
+        if ((s = from_cuda(qx::launch_copies(cl, d->num_sms, true, st))) != QX_OK) return s;
+    } else {
+        for (int i = 0; i < nout; ++i)
+            if ((s = from_cuda(cudaMemcpyAsync(out[i].dst, out[i].src, out[i].bytes, cudaMemcpyDeviceToHost, st))) !=
+                QX_OK)
+                return s;
+    }
     return QX_OK;
 }
 

@@ -232,6 +232,20 @@ bool plan_gemv(GemvMulti &a, int num_sms);
 cudaError_t launch_gemv_multi(GemvMulti &a, cudaStream_t st, bool pdl);
 cudaError_t launch_gemm(const GemmArgs &a, int num_sms, cudaStream_t st);
 
+// Copies of a decode step done by a kernel (qx_copy.cu): src and dst are
+// device-accessible addresses (a pinned host buffer's mapped device address
+// on the host side); `bytes` each.  pdl: launched with programmatic dependent
+// launch, so that it waits for the previous kernel in the stream inside the
+// kernel rather than before it starts.
+constexpr int kMaxCopies = 16;
+struct CopyList {
+    int n;
+    const uint8_t *src[kMaxCopies];
+    uint8_t *dst[kMaxCopies];
+    int64_t bytes[kMaxCopies];
+};
+cudaError_t launch_copies(const CopyList &c, int num_sms, bool pdl, cudaStream_t st);
+
 // cuTensorMapEncodeTiled, fetched once through the runtime's driver entry
 // point (null if the driver does not provide it).
 using EncodeTiledFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,

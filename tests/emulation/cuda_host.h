@@ -787,10 +787,11 @@ inline cudaError_t cudaDeviceSynchronize() { return cudaSuccess; }
 // captured (no stream reports capturing, no host memory counts as pinned).
 enum cudaStreamCaptureStatus { cudaStreamCaptureStatusNone = 0, cudaStreamCaptureStatusActive = 1 };
 enum cudaStreamCaptureMode { cudaStreamCaptureModeThreadLocal = 1 };
-enum cudaMemoryType { cudaMemoryTypeUnregistered = 0, cudaMemoryTypeHost = 1 };
+enum cudaMemoryType { cudaMemoryTypeUnregistered = 0, cudaMemoryTypeHost = 1, cudaMemoryTypeDevice = 2 };
 enum { cudaStreamNonBlocking = 1 };
 struct cudaPointerAttributes {
     cudaMemoryType type;
+    void *devicePointer;
 };
 typedef struct EmuGraph *cudaGraph_t;
 typedef struct EmuGraphExec *cudaGraphExec_t;
@@ -800,6 +801,7 @@ inline cudaError_t cudaStreamIsCapturing(cudaStream_t, cudaStreamCaptureStatus *
 }
 inline cudaError_t cudaPointerGetAttributes(cudaPointerAttributes *a, const void *) {
     a->type = cudaMemoryTypeUnregistered;
+    a->devicePointer = nullptr;
     return cudaSuccess;
 }
 inline cudaError_t cudaStreamCreateWithFlags(cudaStream_t *s, unsigned) {

@@ -17,7 +17,7 @@ import re
 CSRC = os.path.join(os.path.dirname(os.path.dirname(os.path.dirname(os.path.abspath(__file__)))),
                     "paper_2505_07531_gb300", "csrc")
 FILES = ["qx_common.cuh", "qx_kernels.cuh", "qx_quant.cu", "qx_act8.cu", "qx_select.cu", "qx_q4x.cu",
-         "qx_gemv.cu", "qx_gemm.cu", "qx_api.cu"]
+         "qx_gemv.cu", "qx_gemm.cu", "qx_copy.cu", "qx_api.cu"]
 
 # first match wins: longer instruction names before their prefixes
 BY_INSTRUCTION = [

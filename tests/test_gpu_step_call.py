@@ -62,6 +62,35 @@ def test_decode_step_copies_in_and_out(qx, fused):
     assert qx.device_status() == 0
 
 
+def test_decode_step_copies_of_any_alignment(qx):
+    """Pinned host buffers are copied by the library's copy kernel: two copies
+    each way, a host x starting 2 bytes past a 16-byte boundary, a y of 400
+    bytes and a host y at an odd element offset; the host outputs equal the
+    separate calls, call after call."""
+    rec = qx.Recipe(4, 128, qx.UNIFORM)
+    mats = [qx.quantize(torch.from_numpy(synth.student_t_weights(n, 512, 0.02, seed=n, stream=4)).cuda(), rec)
+            for n in (200, 384)]
+    hbuf = torch.empty(1 + 512, dtype=torch.float16).pin_memory()
+    hx = hbuf[1:].view(1, 512)  # 2 bytes past the pinned buffer's start
+    hx2 = torch.empty((1, 512), dtype=torch.float16).pin_memory()
+    dx = torch.empty((1, 512), dtype=torch.float16, device="cuda")
+    dx2 = torch.empty((1, 512), dtype=torch.float16, device="cuda")
+    dys = [torch.empty((1, P.n), dtype=torch.float16, device="cuda") for P in mats]
+    ybuf = torch.empty(1 + 200, dtype=torch.float16).pin_memory()
+    hys = [ybuf[1:].view(1, 200), torch.empty((1, 384), dtype=torch.float16).pin_memory()]
+    step = qx.DecodeStep([(mats, [dx, dx2], dys)], h2d=[(dx, hx), (dx2, hx2)], d2h=list(zip(hys, dys)))
+    for seed in (7, 8, 9):
+        hx.copy_(torch.from_numpy(synth.activations(1, 512, seed=seed, stream=1)))
+        hx2.copy_(torch.from_numpy(synth.activations(1, 512, seed=seed, stream=2)))
+        for h in hys:
+            h.fill_(float("nan"))
+        step()
+        ref = qx.gemv_multi(mats, [hx.cuda(), hx2.cuda()])
+        for h, r in zip(hys, ref):
+            assert torch.equal(h, r.cpu()), seed
+    assert qx.device_status() == 0
+
+
 def test_decode_step_with_pageable_host_memory(qx):
     """Host buffers that are not pinned: the step is issued call by call (a
     graph's copy nodes take pinned memory), with the same results."""
